@@ -1,0 +1,236 @@
+"""Pins of the oracle's whole-network forward/backward (CPU only):
+
+* an independent torch-fp64 autograd evaluation of the same parareal network
+  (loss, every gradient, and dL/dy_j = D_j of Algorithm 2);
+* central finite differences of the loss;
+* N = 1 reproduces the untorn network (Section 4.2: Parareal ResNet-1);
+* delta mode with F^j := g^{j+1} reproduces the untorn nonlinear network;
+* Prop:equiv -- residual mode with F^j := g^{j+1} on a linear body
+  reproduces the untorn network;
+* the parameter count of ResNet-1001 printed in Table errorrate.
+"""
+import copy
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import workloads as W
+from oracle import pnn_oracle as O
+import torch_ref as T
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def small_bottleneck_net(correction="residual"):
+    B = W.bottleneck
+    return {
+        "name": "small_bottleneck", "batch": 3, "in_c": 3, "in_h": 16, "in_w": 16, "classes": 5,
+        "precision": "fp32", "correction": correction,
+        "stem": [W.conv(8)],
+        "body": [B(16, 4), B(16, 4), B(32, 8, 2), B(32, 8), B(64, 16, 2), B(64, 16)],
+        "segments": [2, 2, 2],
+        "coarse": [[B(32, 8, 2), B(32, 8)], [B(64, 16, 2), B(64, 16)]],
+        "cj_post": "none", "head": {"kind": "bn_relu_gap_fc", "hidden": []},
+    }
+
+
+def small_vgg_net(correction="residual"):
+    C = W.conv_bn_relu
+    return {
+        "name": "small_vgg", "batch": 4, "in_c": 3, "in_h": 16, "in_w": 16, "classes": 6,
+        "precision": "fp32", "correction": correction,
+        "stem": [C(8)],
+        "body": [C(8, pool=2), C(16), C(16, pool=2), C(32, pool=2)],
+        "segments": [1, 2, 1],
+        "coarse": [[C(16, pool=2)], [C(32, pool=2)]],
+        "cj_post": "bn_relu", "head": {"kind": "gap_mlp", "hidden": [20]},
+    }
+
+
+def tiny(correction="residual", batch=3, hw=16):
+    d = W.tiny_resnet(batch=batch, correction=correction)
+    d["in_h"] = d["in_w"] = hw
+    return d
+
+
+NETS = {
+    "tiny": tiny,
+    "bottleneck": small_bottleneck_net,
+    "vgg": small_vgg_net,
+}
+
+
+def _setup(desc, seed=3):
+    net = O.ParaNet(desc)
+    theta = W.init_params(net.spec, seed=seed).astype(np.float64)
+    # perturb BN affine parameters so that gamma != 1, beta != 0 are exercised
+    r = np.random.default_rng(seed + 1)
+    i = 0
+    for kind, shape in net.spec:
+        n = int(np.prod(shape))
+        if kind in (O.KIND_BN_G, O.KIND_BN_B, O.KIND_FC_B):
+            theta[i:i + n] += 0.1 * r.standard_normal(n)
+        i += n
+    x, labels = W.make_batch(desc, seed=seed)
+    return net, theta, x.astype(np.float64), labels
+
+
+@pytest.mark.parametrize("name", list(NETS))
+@pytest.mark.parametrize("mode", ["residual", "delta"])
+def test_matches_torch_autograd(name, mode):
+    desc = NETS[name](mode)
+    net, theta, x, labels = _setup(desc)
+    res = O.train_step(desc, theta, x, labels)
+    tl, tg = T.grad_of(desc, theta, x, labels)
+    assert np.isclose(res["loss"], tl, rtol=1e-12)
+    np.testing.assert_allclose(res["grad"], tg, rtol=1e-8, atol=1e-11 * np.abs(tg).max())
+
+
+@pytest.mark.parametrize("name", ["tiny", "bottleneck"])
+def test_D_j_is_dL_dy_j(name):
+    """Algorithm 2: the seed of subnetwork j is dL/dy_j = D_j."""
+    desc = NETS[name]()
+    net, theta, x, labels = _setup(desc)
+    loss, st = net.forward(theta, x, labels)
+    net.backward(st)
+    t = torch.tensor(theta, requires_grad=True)
+    tl, parts = T.parareal_loss(desc, t, x, labels, return_parts=True)
+    for y in parts["ys"]:
+        y.retain_grad()
+    tl.backward()
+    for j in range(net.N):
+        g = parts["ys"][j].grad.numpy()
+        np.testing.assert_allclose(st["D"][j], g, rtol=1e-8, atol=1e-12 * np.abs(g).max())
+        np.testing.assert_allclose(st["ys"][j], parts["ys"][j].detach().numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_finite_differences_every_parameter_kind():
+    desc = tiny(batch=2, hw=8)
+    net, theta, x, labels = _setup(desc)
+    res = O.train_step(desc, theta, x, labels)
+    g = res["grad"]
+    r = np.random.default_rng(11)
+    # pick entries from every block (pre, fine, coarse, head)
+    offs, i = [], 0
+    for name, j, sp in net.blocks:
+        n = sum(int(np.prod(s)) for _, s in sp)
+        offs += list(i + r.choice(n, size=min(n, 4), replace=False))
+        i += n
+    h = 1e-6
+    for k in offs:
+        e = np.zeros_like(theta)
+        e[k] = h
+        lp, _ = net.forward(theta + e, x, labels)
+        lm, _ = net.forward(theta - e, x, labels)
+        fd = (lp - lm) / (2 * h)
+        assert abs(fd - g[k]) <= 1e-6 * max(1e-3, abs(fd)), (k, fd, g[k])
+
+
+@pytest.mark.parametrize("name", list(NETS))
+def test_n1_is_untorn_network(name):
+    desc = NETS[name]()
+    d1 = copy.deepcopy(desc)
+    d1["segments"] = [len(desc["body"])]
+    d1["coarse"] = []
+    net, theta, x, labels = _setup(d1)
+    res = O.train_step(d1, theta, x, labels)
+    t = torch.tensor(theta, requires_grad=True)
+    sl, _ = T.sequential_loss(d1, t, x, labels)
+    sl.backward()
+    assert np.isclose(res["loss"], float(sl), rtol=1e-12)
+    np.testing.assert_allclose(res["grad"], t.grad.numpy(), rtol=1e-8, atol=1e-11 * np.abs(t.grad.numpy()).max())
+    # eq:correct with N = 1: ytilde = y_1
+    np.testing.assert_array_equal(res["state"]["ytilde"], res["state"]["ys"][0])
+
+
+def _coarse_is_fine(desc):
+    """Description and parameter map with F^j := g^{j+1} (same layers, same weights)."""
+    d = copy.deepcopy(desc)
+    segs = d["segments"]
+    starts = np.cumsum([0] + segs)
+    d["coarse"] = [copy.deepcopy(d["body"][starts[j + 1]:starts[j + 2]]) for j in range(len(segs) - 1)]
+    return d
+
+
+def _copy_fine_into_coarse(net, theta):
+    P = net.unflatten(theta)
+    for j in range(net.N - 1):
+        for a, b in zip(P[("coarse", j)], P[("fine", j + 1)]):
+            a[...] = b
+    return net.flatten(P)
+
+
+def _sequential_theta(net, theta):
+    P = net.unflatten(theta)
+    parts = P[("pre", 0)] + [a for j in range(net.N) for a in P[("fine", j)]] + P[("head", 0)]
+    return np.concatenate([a.ravel() for a in parts])
+
+
+@pytest.mark.parametrize("name", list(NETS))
+def test_delta_mode_with_fine_coarse_is_sequential(name):
+    """The benchmark spec's consistency check, exact for the nonlinear network in the
+    delta form: state_{j} = x_{j+1} + rt_j equals g^j(...g^1(C x)) when
+    F^j = g^{j+1}."""
+    desc = _coarse_is_fine(NETS[name]("delta"))
+    net, theta, x, labels = _setup(desc)
+    theta = _copy_fine_into_coarse(net, theta)
+    loss, st = net.forward(theta, x, labels)
+    grad = net.backward(st)
+    ts = torch.tensor(_sequential_theta(net, theta), requires_grad=True)
+    sl, z = T.sequential_loss(desc, ts, x, labels)
+    sl.backward()
+    assert np.isclose(loss, float(sl), rtol=1e-10)
+    np.testing.assert_allclose(st["logits"], z.detach().numpy(), rtol=1e-8, atol=1e-10)
+    # d/d(phi_{j+1}) + d/d(eta_j) of the parareal loss = sequential gradient of segment j+1
+    G = net.unflatten(grad)
+    gs = ts.grad.numpy()
+    off = sum(int(np.prod(s)) for _, s in net.stem.spec) + sum(int(np.prod(s)) for _, s in net.fine[0].spec)
+    for j in range(1, net.N):
+        n = sum(int(np.prod(s)) for _, s in net.fine[j].spec)
+        total = np.concatenate([(a + b).ravel() for a, b in zip(G[("fine", j)], G[("coarse", j - 1)])])
+        np.testing.assert_allclose(total, gs[off:off + n], rtol=1e-6, atol=1e-9 * np.abs(gs).max())
+        off += n
+
+
+@pytest.mark.parametrize("name", ["tiny", "bottleneck"])
+def test_prop_equiv_linear_residual_mode(name):
+    """Prop:equiv: f linear in its body and F^j = g^{j+1} give f-bar = f, for
+    arbitrary (here nonlinear) C^j and h."""
+    desc = _coarse_is_fine(NETS[name]("residual"))
+    net = O.ParaNet(desc, linear_body=True)
+    _, theta, x, labels = _setup(desc)
+    theta = _copy_fine_into_coarse(net, theta)
+    loss, st = net.forward(theta, x, labels)
+    ts = torch.tensor(_sequential_theta(net, theta))
+    sl, z = T.sequential_loss(desc, ts, x, labels, linear_body=True)
+    np.testing.assert_allclose(st["logits"], z.numpy(), rtol=1e-9, atol=1e-9 * np.abs(z.numpy()).max())
+    assert np.isclose(loss, float(sl), rtol=1e-10)
+    # and it is NOT the identity for the nonlinear body (the proposition needs linearity)
+    net_nl = O.ParaNet(desc)
+    l_nl, _ = net_nl.forward(theta, x, labels)
+    sl_nl, _ = T.sequential_loss(desc, ts, x, labels)
+    assert abs(l_nl - float(sl_nl)) > 1e-6
+
+
+def test_resnet1001_parameter_count():
+    g = json.load(open(os.path.join(GOLDEN, "param_counts.json")))["resnet1001_cifar10"]
+    d = W.parareal_resnet1001(n_seg=4)
+    d["segments"] = [333]
+    d["coarse"] = []
+    n = O.ParaNet(d).num_params()
+    assert n == 10_327_706
+    assert f"{n / 1e6:.1f}M" == g["printed"]
+
+
+@pytest.mark.parametrize("idx,shapes", [
+    (0, [(16, 32, 32), (16, 32, 32), (16, 32, 32)]),
+    (1, [(64, 32, 32), (128, 8, 8), (256, 4, 4), (512, 2, 2), (512, 1, 1)]),
+    (2, [(16, 32, 32), (64, 32, 32), (128, 16, 16), (256, 8, 8), (256, 8, 8)]),
+    (4, [(16, 32, 32)] + [(64, 32, 32)] * 2 + [(128, 16, 16)] * 3 + [(256, 8, 8)] * 3),
+])
+def test_config_interfaces(idx, shapes):
+    net = O.ParaNet(W.config(idx))
+    assert [tuple(s) for s in net.X] == shapes
