@@ -1,0 +1,302 @@
+#!/usr/bin/env python
+"""Training-throughput benchmark of the parareal network on GB300.
+
+Workload (default): parareal pre-activation ResNet-1001 torn into N=8 fine
+subnetworks, batch 256, 3x64x64 synthetic N(0,1) images (stride-2 stem),
+200 classes, bf16 -- the headline configuration.  A step is one whole
+training iteration (Algorithm 1 forward, Algorithm 2 backward, SGD update).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config I]
+
+Prints one JSON line (rank 0).  For N > 1 (launched by torchrun) every rank
+trains an independent replica on its own batch (the path is single-GPU by
+design): value = images of all ranks / max over ranks of the timed region.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import workloads as W  # noqa: E402
+
+METRIC = "parareal-net training images/sec on 1 GB300; conv TFLOP/s as % of bf16 dense peak"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# CUDA-core fp32 peak: 152 SMs x 128 FP32 lanes x 2 FLOP (FMA) x 2.07 GHz max SM clock
+FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+CONV_KINDS = ("conv_fwd", "conv_dgrad", "conv_wgrad", "conv_fwd_tc", "conv_dgrad_tc", "conv_wgrad_tc")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", type=int, default=4)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample-batch", type=int, default=1)
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return PEAKS_FALLBACK, "fallback"
+
+
+# ---------------------------------------------------------------- clocks
+class Clocks:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.p = None
+
+    def __enter__(self):
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                       "--format=csv,noheader,nounits", "-lms", "200"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+        return self
+
+    def __exit__(self, *a):
+        if self.p:
+            self.p.terminate()
+            self.p.wait(timeout=10)
+
+    def summary(self):
+        self.f.flush()
+        rows = []
+        with open(self.f.name) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.f.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------- distributed
+def dist_setup(gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("gloo")
+    return rank, local, world, dist
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+def max_over_ranks(dist, v):
+    if dist is None:
+        return v
+    import torch
+    t = torch.tensor([v], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t[0])
+
+
+# ---------------------------------------------------------------- CPU oracle
+def oracle_sample(desc, batch):
+    """One oracle training step on `batch` images of the same network."""
+    from oracle import pnn_oracle as O
+    d = W.with_batch(desc, batch)
+    net = O.ParaNet(d)
+    theta = W.init_params(net.spec, seed=0, bf16=d["precision"] == "bf16")
+    x, labels = W.make_batch(d)
+    prec = "bf16" if d["precision"] == "bf16" else "fp64"
+    t0 = time.perf_counter()
+    O.train_step(d, theta, x, labels, precision=prec)
+    return time.perf_counter() - t0
+
+
+def cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def reference_arm(args, desc, rank):
+    if rank != 0:
+        return
+    b = args.cpu_sample_batch
+    for _ in range(args.warmup):
+        oracle_sample(desc, b)
+    ts = [oracle_sample(desc, b) for _ in range(args.steps)]
+    total = sum(ts)
+    value = b * args.steps / total
+    sample = f"{b} image(s) of the same network per step (CPU fp64 oracle, one forward+backward+SGD)"
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": desc["name"] + "_b%d" % desc["batch"], "batch": desc["batch"]},
+        "cpu_baseline": {"value": value, "unit": "images/s", "cores": cores(), "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+# ---------------------------------------------------------------- our arm
+def our_arm(args, desc, rank, local, world, dist):
+    import torch
+    from paper_2103_08802_gb300 import build, pnn
+
+    build.build()
+    torch.cuda.set_device(local)
+    stream = torch.cuda.Stream()
+    net = pnn.ParaNet(desc, seed=0, stream=stream)
+    B = desc["batch"]
+    x, labels = W.make_batch(desc, seed=1000 + desc.get("config_index", 0) + rank)
+    xd = torch.from_numpy(x).cuda()
+    ld = torch.from_numpy(labels).cuda()
+    loss = torch.zeros(1, device="cuda")
+    torch.cuda.synchronize()
+
+    for _ in range(max(3, args.warmup)):
+        net.train_step(xd, ld, loss)
+    net.sync()
+
+    # ------------------------------------------------ timed region (device events)
+    with Clocks(local) as clk:
+        barrier(dist)
+        torch.cuda.synchronize()
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for _ in range(args.steps):
+            net.train_step(xd, ld, loss)
+        end.record(stream)
+        torch.cuda.synchronize()
+        ms = start.elapsed_time(end)
+        barrier(dist)
+    ms = max_over_ranks(dist, ms)
+    clocks = clk.summary()
+    net.sync()
+    final_loss = float(loss.cpu())
+    value = B * args.steps * world / (ms / 1e3)
+
+    # ------------------------------------------------ per-kernel profile (eager steps)
+    net.profile(True)
+    for _ in range(args.steps):
+        net.forward(xd, ld, loss)
+        net.backward()
+        net.sgd_step()
+    prof = net.profile_read()
+    net.profile(False)
+    fw, bw, up = net.launch_counts()
+    launches_per_step = fw + bw + up
+    phases = net.timings()
+
+    # ------------------------------------------------ end to end through the host API
+    xh = torch.from_numpy(x).pin_memory()
+    lh = torch.from_numpy(labels).pin_memory()
+    net.train_step_host(xh, lh)  # captures the host-staged step graph
+    barrier(dist)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        net.train_step_host(xh, lh)
+    e2e_s = max_over_ranks(dist, time.perf_counter() - t0)
+    e2e = {"value": B * args.steps * world / e2e_s, "unit": "images/s",
+           "h2d_bytes_per_step": int(x.nbytes + labels.nbytes), "d2h_bytes_per_step": 4}
+
+    if rank != 0:
+        return
+    pk, src = peaks()
+    conv_ms = sum(prof[k][0] for k in CONV_KINDS if k in prof)
+    conv_flops = sum(prof[k][2] for k in CONV_KINDS if k in prof)
+    total_prof_ms = sum(v[0] for v in prof.values())
+    # dominant kernel kind by device time
+    dom = max(prof.items(), key=lambda kv: kv[1][0])
+    name, (kms, kn, kfl, kby) = dom
+    per_launch_ms = kms / kn
+    if name.endswith("_tc"):
+        bound, peak, unit = "tensor", pk["bf16_tflops_sustained"], "TFLOP/s"
+        achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
+    elif name.startswith("conv"):
+        bound, peak, unit = "alu", FP32_ALU_TFLOPS, "TFLOP/s"
+        achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
+    else:
+        bound, peak, unit = "hbm", pk["hbm_gbs"], "GB/s"
+        achieved = kby / kn / (per_launch_ms / 1e3) / 1e9
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        b = args.cpu_sample_batch
+        t = oracle_sample(desc, b)
+        cpu = {"value": b / t, "unit": "images/s", "cores": cores(), "kind": "oracle",
+               "sample": f"{b} image(s) of the same network, one forward+backward+SGD step of the CPU "
+                         f"fp64 oracle ({t:.1f} s)"}
+    out = {
+        "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world, "steps": args.steps,
+        "warmup": max(3, args.warmup), "ms_per_step": ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if desc["precision"] == "bf16" else "fp32",
+        "data": "synthetic",
+        "config": {"workload": desc["name"] + "_b%d_%dpx_c%d" % (B, desc["in_h"], desc["classes"]),
+                   "batch": B, "input": "3x%dx%d" % (desc["in_h"], desc["in_w"]), "classes": desc["classes"],
+                   "subnetworks": len(desc["segments"]), "correction": desc.get("correction", "residual"),
+                   "l2": "inputs larger than L2 (%.1f GB workspace per step)" % (net.workspace_bytes / 1e9),
+                   "parallelism": "replicas" if world > 1 else "single-gpu"},
+        "conv_tflops": conv_flops / (conv_ms / 1e3) / 1e12 if conv_ms else None,
+        "conv_frac_of_bf16_peak": (conv_flops / (conv_ms / 1e3) / 1e12) / pk["bf16_tflops_sustained"] if conv_ms else None,
+        "conv_share_of_device_time": conv_ms / total_prof_ms if total_prof_ms else None,
+        "roofline": {"kernel": name, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+                     "frac": achieved / peak, "traffic": None, "peak_source": src if bound != "alu" else
+                     "derived: 152 SM x 128 FP32 lanes x 2 x 2.07 GHz", "launches_per_step": kn / args.steps},
+        "kernels": {k: {"ms_per_step": v[0] / args.steps, "launches_per_step": v[1] / args.steps,
+                        "gflop_per_step": v[2] / args.steps / 1e9, "gb_per_step": v[3] / args.steps / 1e9}
+                    for k, v in sorted(prof.items(), key=lambda kv: -kv[1][0])},
+        "phases_ms": phases,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks,
+        "loss_after": final_loss,
+    }
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse()
+    rank, local, world, dist = dist_setup(args.gpus)
+    desc = W.config(args.config)
+    if args.impl == "reference":
+        reference_arm(args, desc, rank)
+    else:
+        our_arm(args, desc, rank, local, world, dist)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

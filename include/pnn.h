@@ -1,0 +1,219 @@
+/*
+ * pnn.h -- C ABI of the GB300 parareal neural network training library.
+ *
+ * The library trains the parareal network f-bar of Lee, Lee & Park,
+ * "Parareal Neural Networks Emulating a Parallel-in-time Algorithm"
+ * (Section 3, eq:barf): a feed-forward CNN f = h o g o C is torn into N
+ * consecutive subnetworks g^j (Section 3.1); all N run at once on one GPU
+ * (Algorithm 1's parallel loop becomes grouped kernel launches), and the
+ * coarse network F^j joins them through the parareal correction eq:correct.
+ * The gradient follows Algorithm 2 (Section 3.2) and the update is SGD with
+ * Nesterov momentum and weight decay (Section 4).
+ *
+ * Conventions shared by every call:
+ *   - Every call returns a pnn_status; the library never aborts or exits.
+ *     pnn_last_error() returns a human-readable message for the last failure.
+ *   - Device pointers are CUDA device addresses of the current device; host
+ *     pointers are ordinary (pageable or pinned) host memory.
+ *   - All GPU work is enqueued on the stream given in pnn_options (NULL = the
+ *     legacy default stream).  Calls marked "synchronises" wait for it.
+ *   - The library owns the plan; the caller owns the workspace (one device
+ *     allocation, see pnn_workspace_bytes / pnn_bind_workspace), which holds
+ *     every parameter, gradient, momentum buffer, activation and table.
+ *   - Tensors at the boundary are NCHW float32.  Inside, activations are NHWC.
+ *   - A handle is not thread-safe.
+ */
+#ifndef PNN_H_
+#define PNN_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct pnn_net pnn_net; /* opaque, library-owned */
+
+typedef enum {
+  PNN_OK = 0,
+  PNN_EINVAL = 1,     /* bad argument or description */
+  PNN_ENOMEM = 2,     /* workspace too small */
+  PNN_ECUDA = 3,      /* a CUDA runtime call failed (message in pnn_last_error) */
+  PNN_ESTATE = 4,     /* call out of order (e.g. backward before forward) */
+  PNN_ETIMEOUT = 5,   /* a device-side bounded wait gave up */
+  PNN_ENONFINITE = 6, /* loss is NaN/Inf or a label is out of range */
+  PNN_ENOTBOUND = 7   /* no workspace bound yet */
+} pnn_status;
+
+typedef enum { PNN_BF16 = 0, PNN_FP32_CHECK = 1 } pnn_precision;
+
+/* Section 3.1 eq:correct (default) or the classic parareal update of
+ * Section 2 written for the residual: rt_{j+1} = r_{j+1} + F^j(x_{j+1}+rt_j) - F^j(x_{j+1}). */
+typedef enum { PNN_CORR_RESIDUAL = 0, PNN_CORR_DELTA = 1 } pnn_correction;
+
+/* Layer kinds of a description (Section 4, Tables vgg and resnet).  Every
+ * conv is bias-free, k x k with zero padding k/2.
+ *   PNN_CONV            bare conv (cout, k, stride)
+ *   PNN_CONV_BN_RELU    conv -> BN -> ReLU, then a 2x2/s2 maxpool if pool != 0
+ *   PNN_BASIC           post-activation basic block: ReLU(BN(conv(ReLU(BN(conv x)))) + x)
+ *   PNN_BOTTLENECK      pre-activation bottleneck (cout, mid, stride on the 3x3
+ *                       conv, 1x1 projection shortcut when the shape changes) */
+typedef enum { PNN_CONV = 0, PNN_CONV_BN_RELU = 1, PNN_BASIC = 2, PNN_BOTTLENECK = 3 } pnn_layer_op;
+
+/* Postprocessing h (eq:barf's epsilon part) */
+typedef enum { PNN_HEAD_GAP_FC = 0, PNN_HEAD_BN_RELU_GAP_FC = 1, PNN_HEAD_GAP_MLP = 2 } pnn_head_kind;
+
+/* What follows the 1x1 conv of C^j for j > 1 (Section 4.1 / 4.2: maxpools
+ * 3x3/s2 down to the size of X_{j-1}, then a 1x1 conv). */
+typedef enum { PNN_CJ_NONE = 0, PNN_CJ_BN_RELU = 1 } pnn_cj_post;
+
+typedef struct {
+  int32_t op;     /* pnn_layer_op */
+  int32_t cout;   /* output channels */
+  int32_t mid;    /* bottleneck width (PNN_BOTTLENECK only) */
+  int32_t k;      /* kernel size (PNN_CONV, PNN_CONV_BN_RELU): 1 or 3 */
+  int32_t stride; /* 1 or 2 */
+  int32_t pool;   /* PNN_CONV_BN_RELU: non-zero appends a 2x2/s2 maxpool */
+} pnn_layer;
+
+/* A network description (Section 3.1):
+ *   stem     the preprocessing operator C_delta = C^1
+ *   body     the block-repetitive part g, torn into n_seg consecutive segments
+ *            of segments[j] layers each (g^1 .. g^N)
+ *   coarse   F^1 .. F^{N-1} concatenated; coarse_len[j] layers each
+ *   head     h; head_hidden lists hidden FC widths for PNN_HEAD_GAP_MLP.
+ * Arrays are read during pnn_create only. */
+typedef struct {
+  int32_t batch, in_c, in_h, in_w, classes;
+  const pnn_layer* stem;
+  int32_t n_stem;
+  const pnn_layer* body;
+  int32_t n_body;
+  const int32_t* segments;
+  int32_t n_seg;
+  const pnn_layer* coarse;
+  const int32_t* coarse_len; /* n_seg - 1 entries */
+  int32_t cj_post;           /* pnn_cj_post */
+  int32_t head_kind;         /* pnn_head_kind */
+  const int32_t* head_hidden;
+  int32_t n_hidden;
+} pnn_desc;
+
+typedef struct {
+  int32_t precision;     /* pnn_precision */
+  int32_t correction;    /* pnn_correction */
+  uint64_t seed;         /* He-normal initialisation seed */
+  float lr, momentum, weight_decay;
+  int32_t nesterov;
+  int32_t stream_fp32;   /* bf16 mode: keep the residual stream (block outputs,
+                            correction tensors) in fp32 storage */
+  int32_t conv_impl;     /* 0 = best available, 1 = force CUDA-core kernels */
+  void* stream;          /* cudaStream_t; NULL = legacy default stream */
+} pnn_options;
+
+/* Fill o with the defaults: bf16, residual correction, seed 0, lr 0.1,
+ * momentum 0.9, weight decay 5e-4, Nesterov (Section 4), stream_fp32 1. */
+void pnn_default_options(pnn_options* o);
+
+/* Plan the network from a description.  Host only: no GPU work, no device
+ * allocation.  *out receives a handle that must be released with pnn_destroy. */
+int pnn_create(const pnn_desc* desc, const pnn_options* opts, pnn_net** out);
+
+/* Bytes of device memory the caller must provide. */
+int pnn_workspace_bytes(const pnn_net* net, size_t* bytes);
+
+/* Bind a device allocation of at least pnn_workspace_bytes bytes (256-byte
+ * aligned).  The caller keeps it alive until pnn_destroy.  Uploads the launch
+ * tables and initialises the parameters (He-normal from opts.seed: std
+ * sqrt(2/fan_in) for conv and FC weights, BN gamma 1, beta 0, FC bias 0).
+ * Synchronises. */
+int pnn_bind_workspace(pnn_net* net, void* dev, size_t bytes);
+
+/* Algorithm 1: x (device, batch x in_c x in_h x in_w float32 NCHW), labels
+ * (device, batch int32 in [0, classes)).  Writes the mean softmax
+ * cross-entropy to loss_dev (device, 1 float; may be NULL).  x and labels
+ * must stay valid until pnn_backward returns. */
+int pnn_forward(pnn_net* net, const float* x_dev, const int32_t* labels_dev, float* loss_dev);
+
+/* Algorithm 2: gradients of the loss of the preceding pnn_forward with
+ * respect to every parameter (eq:etak, eq:phij, eq:deltaj). */
+int pnn_backward(pnn_net* net);
+
+/* One SGD step with the gradients of the preceding pnn_backward:
+ * d = g + wd*w; v = d (first step) or mu*v + d; w -= lr*(d + mu*v) (Nesterov)
+ * or lr*v.  lr <= 0 uses opts.lr. */
+int pnn_sgd_step(pnn_net* net, float lr);
+
+/* One whole training step (forward + backward + SGD) replayed from a CUDA
+ * graph captured on first use; x_dev/labels_dev as in pnn_forward and must be
+ * the same pointers on every call (the graph records them). */
+int pnn_train_step(pnn_net* net, const float* x_dev, const int32_t* labels_dev, float* loss_dev);
+
+/* The same step from HOST buffers: copies x and labels to the workspace,
+ * runs the step and copies the loss back to *loss_host.  Synchronises. */
+int pnn_train_step_host(pnn_net* net, const float* x_host, const int32_t* labels_host, float* loss_host);
+
+/* Wait for the stream and report device-side status words (PNN_ENONFINITE,
+ * PNN_ETIMEOUT).  Synchronises. */
+int pnn_sync(pnn_net* net);
+
+/* NULL-safe. Does not free the caller's workspace. */
+void pnn_destroy(pnn_net* net);
+
+/* ---- parameters (flat vector theta-bar in eq:barf order:
+ *      (delta_1, phi_1, ..., delta_N, phi_N, eta_1, ..., eta_{N-1}, eps);
+ *      conv weights in (K, C, R, S) order, FC weights (out, in)) ---- */
+int pnn_num_params(const pnn_net* net, size_t* n);
+int pnn_num_param_tensors(const pnn_net* net, int32_t* n);
+/* kind: 0 conv weight, 1 BN gamma, 2 BN beta, 3 FC weight, 4 FC bias;
+ * dims[4] (unused trailing dims are 1); offset into theta-bar. */
+int pnn_param_tensor_info(const pnn_net* net, int32_t i, int32_t* kind, int32_t dims[4], size_t* offset);
+/* Copies of length n (must equal pnn_num_params).  Synchronise. */
+int pnn_get_params(pnn_net* net, float* host, size_t n);
+int pnn_set_params(pnn_net* net, const float* host, size_t n);
+int pnn_get_grads(pnn_net* net, float* host, size_t n);
+int pnn_get_momentum(pnn_net* net, float* host, size_t n);
+
+/* ---- interface tensors of the last forward/backward, NCHW float32 ---- */
+typedef enum {
+  PNN_T_X = 0,      /* x_j = C^j(x), j = 1..N (eq:xjyj) */
+  PNN_T_Y = 1,      /* y_j = g^j(x_j), j = 1..N */
+  PNN_T_R = 2,      /* r_j = y_j - x_{j+1}, j = 1..N-1 (eq:rk) */
+  PNN_T_RTILDE = 3, /* rt_j, j = 1..N (eq:tilderk) */
+  PNN_T_YTILDE = 4, /* ytilde (eq:tildey); j ignored */
+  PNN_T_D = 5,      /* D_j = dL/drt_j, j = 1..N (Algorithm 2) */
+  PNN_T_LOGITS = 6  /* batch x classes; j ignored */
+} pnn_tensor;
+/* Number of floats of tensor (which, j), or 0 if it does not exist. */
+int pnn_tensor_size(const pnn_net* net, int32_t which, int32_t j, size_t* n);
+int pnn_get_tensor(pnn_net* net, int32_t which, int32_t j, float* host, size_t n);
+
+/* Per-phase device time of the last eager forward/backward/update in ms,
+ * in the paper's column order (Tables gradvgg and grad): pre, fine, coarse,
+ * post for forward, the same four for backward, then the SGD update and the
+ * total: ms[10]. */
+int pnn_get_timings(pnn_net* net, float ms[10]);
+/* Counts of the step's kernel launches: forward, backward, update. */
+int pnn_launch_counts(const pnn_net* net, int32_t counts[3]);
+
+/* ---- profiling: with enable != 0 every kernel launch of eager calls
+ * (pnn_forward / pnn_backward / pnn_sgd_step) is bracketed by CUDA events on
+ * the library stream; pnn_profile_read synchronises, folds the recorded
+ * launches into per-kind totals and returns, for one kernel kind, the summed
+ * device time (ms), the launch count and the algorithmic FLOPs and bytes of
+ * those launches (conv FLOPs = 2 * B*P*Q*K*C*R*S; bytes = each operand read
+ * once and each result written once).  Enabling or disabling resets totals
+ * and drops a captured step graph.  Kinds are 0 .. pnn_num_kernel_kinds()-1. */
+int pnn_profile(pnn_net* net, int32_t enable);
+int pnn_profile_read(pnn_net* net, int32_t kind, double* ms, int64_t* launches, double* flops, double* bytes);
+int32_t pnn_num_kernel_kinds(void);
+const char* pnn_kernel_kind_name(int32_t kind); /* NULL for a bad kind */
+
+const char* pnn_last_error(const pnn_net* net);
+const char* pnn_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PNN_H_ */

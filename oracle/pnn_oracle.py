@@ -27,6 +27,15 @@ definition written out; numpy's tensordot (a library matmul) serves as the
 inner contraction of the convolution.  Readings of points the paper leaves
 open (BN eps, pooling padding, block layout, loss) are the module constants
 and the layer classes below.
+
+Precision model.  The paper fixes no precision.  By default everything is
+float64.  With precision="bf16" the forward pass rounds to bfloat16 exactly
+the values a bf16 tensor-core implementation holds in bf16: every
+convolution operand (input activation and weight) and every stored
+convolution / pooling output that is not followed by a residual add.  This
+makes the floating-point decisions of the forward pass (ReLU masks, maxpool
+argmax) use the kernel's precision; all arithmetic stays float64 and no
+gradient is rounded.
 """
 from __future__ import annotations
 
@@ -38,6 +47,18 @@ KIND_CONV_W, KIND_BN_G, KIND_BN_B, KIND_FC_W, KIND_FC_B = 0, 1, 2, 3, 4
 
 
 # ====================================================================== ops
+def round_bf16(a):
+    """Round float64 values to the nearest bfloat16 value (8 significant bits,
+    ties to even), returned as float64.  Operates on the float64 bit pattern:
+    drop the low 45 of the 52 mantissa bits with round-half-to-even."""
+    a = np.asarray(a, dtype=np.float64)
+    u = a.view(np.uint64)
+    lsb = (u >> np.uint64(45)) & np.uint64(1)
+    r = (u + np.uint64((1 << 44) - 1) + lsb) & ~np.uint64((1 << 45) - 1)
+    out = r.view(np.float64)
+    return np.where(np.isfinite(a), out, a)
+
+
 def conv2d(x, w, stride, pad):
     """y[b,k,p,q] = sum_{c,r,s} x[b,c,p*stride+r-pad,q*stride+s-pad] w[k,c,r,s]
     with zero padding."""
@@ -186,6 +207,11 @@ class _Layer:
     (kind, shape) and implements forward / backward on numpy arrays."""
 
     linear = False
+    bf16 = False      # precision model (see the module docstring)
+    store_q = True    # this conv's output is stored (rounded) on its own
+
+    def _q(self, a):
+        return round_bf16(a) if self.bf16 else a
 
     def _bn(self, h, g, b):
         if self.linear:
@@ -212,10 +238,12 @@ class Conv(_Layer):
         self.spec = [(KIND_CONV_W, (cout, cin, k, k))]
 
     def forward(self, x, P):
-        return conv2d(x, P[0], self.stride, self.pad), x
+        xq = self._q(x)
+        y = conv2d(xq, self._q(P[0]), self.stride, self.pad)
+        return (self._q(y) if self.store_q else y), xq
 
     def backward(self, dy, P, cache, need_dx=True):
-        dx, dw = conv2d_backward(cache, P[0], self.stride, self.pad, dy, need_dx)
+        dx, dw = conv2d_backward(cache, self._q(P[0]), self.stride, self.pad, dy, need_dx)
         return dx, [dw]
 
 
@@ -238,6 +266,7 @@ class ConvBnRelu(_Layer):
                 out, arg = avgpool(a, 2, 2, 0), None
             else:
                 out, arg = maxpool(a, 2, 2, 0)
+                out = self._q(out)
         else:
             out, arg = a, None
         return out, (cc, z, bc, a.shape, arg)
@@ -301,6 +330,7 @@ class Bottleneck(_Layer):
         _, ho, wo = self.c2.out_shape
         self.c3 = Conv(mid, ho, wo, cout, 1, 1)
         self.cp = Conv(cin, h, w, cout, 1, stride) if self.proj else None
+        self.c3.store_q = False   # its output goes straight into the residual sum
         self.out_shape = (cout, ho, wo)
         self.spec = ([(KIND_BN_G, (cin,)), (KIND_BN_B, (cin,))] + self.c1.spec
                      + [(KIND_BN_G, (mid,)), (KIND_BN_B, (mid,))] + self.c2.spec
@@ -341,7 +371,7 @@ class Bottleneck(_Layer):
         return dx, [dg1, db1, dw1, dg2, db2, dw2, dg3, db3, dw3] + grads_p
 
 
-def make_layer(spec, shape, linear=False):
+def make_layer(spec, shape, linear=False, bf16=False):
     c, h, w = shape
     op = spec["op"]
     if op == "conv":
@@ -355,20 +385,22 @@ def make_layer(spec, shape, linear=False):
     else:
         raise ValueError(op)
     L.linear = linear
+    L.bf16 = bf16
     for sub in ("conv", "c1", "c2", "c3", "cp"):
         if getattr(L, sub, None) is not None:
             getattr(L, sub).linear = linear
+            getattr(L, sub).bf16 = bf16
     return L
 
 
 class Stack:
     """A sequence of layers with a contiguous slice of the parameter vector."""
 
-    def __init__(self, specs, shape, linear=False):
+    def __init__(self, specs, shape, linear=False, bf16=False):
         self.layers = []
         self.in_shape = tuple(shape)
         for s in specs:
-            L = make_layer(s, shape, linear)
+            L = make_layer(s, shape, linear, bf16)
             self.layers.append(L)
             shape = L.out_shape
         self.out_shape = tuple(shape)
@@ -401,13 +433,14 @@ class Preprocess:
     image down to the size of X_{j-1}, then a bias-free 1x1 conv to its
     channel count, optionally followed by BN + ReLU."""
 
-    def __init__(self, in_shape, target, post):
+    def __init__(self, in_shape, target, post, bf16=False):
         c, h, w = in_shape
         ct, ht, wt = target
         k = int(round(math.log2(h / ht)))
         assert h == ht << k and w == wt << k, (in_shape, target)
         self.k, self.post = k, post
         self.conv = Conv(c, ht, wt, ct, 1, 1)
+        self.conv.bf16 = bf16
         self.spec = self.conv.spec + ([(KIND_BN_G, (ct,)), (KIND_BN_B, (ct,))] if post == "bn_relu" else [])
         self.out_shape = tuple(target)
 
@@ -497,11 +530,12 @@ class Head:
 class ParaNet:
     """The parareal network f-bar of eq:barf built from a description."""
 
-    def __init__(self, desc, linear_body=False):
+    def __init__(self, desc, linear_body=False, precision="fp64"):
         self.desc = desc
         self.mode = desc.get("correction", "residual")
+        q = precision == "bf16"
         x_shape = (desc["in_c"], desc["in_h"], desc["in_w"])
-        self.stem = Stack(desc["stem"], x_shape)
+        self.stem = Stack(desc["stem"], x_shape, bf16=q)
         segs = desc["segments"]
         assert sum(segs) == len(desc["body"]) and all(s > 0 for s in segs)
         self.N = len(segs)
@@ -509,17 +543,17 @@ class ParaNet:
         shape = self.stem.out_shape
         start = 0
         for n in segs:
-            st = Stack(desc["body"][start:start + n], shape, linear_body)
+            st = Stack(desc["body"][start:start + n], shape, linear_body, q)
             self.fine.append(st)
             shape = st.out_shape
             start += n
         # X_0 .. X_N
         self.X = [self.stem.out_shape] + [st.out_shape for st in self.fine]
-        self.pre = [None] + [Preprocess(x_shape, self.X[j], desc["cj_post"]) for j in range(1, self.N)]
+        self.pre = [None] + [Preprocess(x_shape, self.X[j], desc["cj_post"], q) for j in range(1, self.N)]
         assert len(desc["coarse"]) == self.N - 1
         self.coarse = []
         for j in range(self.N - 1):
-            st = Stack(desc["coarse"][j], self.X[j + 1], linear_body)
+            st = Stack(desc["coarse"][j], self.X[j + 1], linear_body, q)
             assert st.out_shape == self.X[j + 2], (j, st.out_shape, self.X[j + 2])
             self.coarse.append(st)
         self.head = Head(desc["head"], self.X[self.N], desc["classes"])
@@ -634,10 +668,10 @@ class ParaNet:
 
 
 def train_step(desc, theta, x, labels, lr=0.1, momentum=0.9, weight_decay=5e-4,
-               nesterov=True, momentum_buf=None, linear_body=False):
+               nesterov=True, momentum_buf=None, linear_body=False, precision="fp64"):
     """Forward, backward and one SGD step.  Returns a dict with loss, grad,
     theta_new, buf_new and the forward state."""
-    net = ParaNet(desc, linear_body)
+    net = ParaNet(desc, linear_body, precision)
     loss, st = net.forward(theta, x, labels)
     grad = net.backward(st)
     theta_new, buf = sgd_step(np.asarray(theta, np.float64), grad, momentum_buf, lr, momentum,

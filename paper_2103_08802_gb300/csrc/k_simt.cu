@@ -1,0 +1,831 @@
+// CUDA-core kernels of the parareal training step: implicit-GEMM convolution
+// (forward, data gradient, weight gradient) used in fp32 check mode, and every
+// non-convolution op of the step (BN statistics and backward, elementwise
+// correction/residual ops, pooling, head, loss, SGD) used in both precisions.
+//
+// Every kernel is "grouped": one launch covers a list of independent problem
+// instances (typically the same layer position of all N fine subnetworks,
+// Algorithm 1's parallel loop), each CTA finds its instance from a tile prefix.
+// All reductions run in a fixed order so that results are bit-reproducible.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "pnn_internal.h"
+
+namespace pnn {
+
+// ---------------------------------------------------------------- helpers
+__device__ __forceinline__ float ldv(const void* p, int dt, int64_t i) {
+  return dt == DT_F32 ? __ldg(reinterpret_cast<const float*>(p) + i)
+                      : __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(p)[i]);
+}
+__device__ __forceinline__ float rnd(int dt, float v) {
+  return dt == DT_BF16 ? __bfloat162float(__float2bfloat16_rn(v)) : v;
+}
+__device__ __forceinline__ void stv(void* p, int dt, int64_t i, float v) {
+  if (dt == DT_F32) reinterpret_cast<float*>(p)[i] = v;
+  else reinterpret_cast<__nv_bfloat16*>(p)[i] = __float2bfloat16_rn(v);
+}
+__device__ __forceinline__ float ld_src(const Src& s, int64_t i, int c) {
+  float v = ldv(s.ptr, s.dt, i);
+  if (s.scale) {
+    v = fmaf(__ldg(s.scale + c), v, __ldg(s.shift + c));
+    if (s.relu) v = fmaxf(v, 0.f);
+  }
+  return v;
+}
+// index of the instance that owns CTA b: the largest i with tstart[i] <= b
+__device__ __forceinline__ int find_instance(const int* tstart, int n, int b) {
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (__ldg(tstart + mid) <= b) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// ---------------------------------------------------------------- conv fwd
+// Y[m][k] = sum_{r,s,c} act(X)[n, p*st+r-pad, q*st+s-pad, c] * W[k][r][s][c] (+ res[m][k])
+template <int BM, int BN>
+__global__ void __launch_bounds__(256) k_conv_fwd(const ConvDesc* __restrict__ tab,
+                                                  const int* __restrict__ tstart, int n) {
+  constexpr int BK = 16, TM = BM / 16, TN = BN / 16;
+  __shared__ float As[BK][BM + 4];
+  __shared__ float Bs[BK][BN + 4];
+  __shared__ float red[16][BN][2];
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const ConvDesc& d = tab[inst];
+  const int t = blockIdx.x - tstart[inst];
+  const int tm = t % d.mtiles, tn = t / d.mtiles;
+  const int M = d.B * d.P * d.Q, Kt = d.R * d.S * d.C;
+  const int m0 = tm * BM, n0 = tn * BN;
+  const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+  float acc[TM][TN];
+#pragma unroll
+  for (int i = 0; i < TM; ++i)
+#pragma unroll
+    for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
+
+  for (int k0 = 0; k0 < Kt; k0 += BK) {
+    for (int e = tid; e < BM * BK; e += 256) {
+      const int kk = e % BK, mm = e / BK;
+      const int m = m0 + mm, k = k0 + kk;
+      float v = 0.f;
+      if (m < M && k < Kt) {
+        const int c = k % d.C, rs = k / d.C, s = rs % d.S, r = rs / d.S;
+        const int q = m % d.Q, tmp = m / d.Q, p = tmp % d.P, nb = tmp / d.P;
+        const int h = p * d.stride + r - d.pad, w = q * d.stride + s - d.pad;
+        if (h >= 0 && h < d.H && w >= 0 && w < d.W)
+          v = ld_src(d.x, ((int64_t)(nb * d.H + h) * d.W + w) * d.C + c, c);
+      }
+      As[kk][mm] = d.op_bf16 ? rnd(DT_BF16, v) : v;
+    }
+    for (int e = tid; e < BN * BK; e += 256) {
+      const int kk = e % BK, nn = e / BK;
+      const int k = k0 + kk, co = n0 + nn;
+      Bs[kk][nn] = (k < Kt && co < d.K) ? ldv(d.w, d.w_dt, (int64_t)co * Kt + k) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < BK; ++kk) {
+      float a[TM], b[TN];
+#pragma unroll
+      for (int i = 0; i < TM; ++i) a[i] = As[kk][ty + 16 * i];
+#pragma unroll
+      for (int j = 0; j < TN; ++j) b[j] = Bs[kk][tx + 16 * j];
+#pragma unroll
+      for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+  // epilogue: residual, store, BN partials of the stored value
+#pragma unroll
+  for (int j = 0; j < TN; ++j) {
+    const int co = n0 + tx + 16 * j;
+    float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+    for (int i = 0; i < TM; ++i) {
+      const int m = m0 + ty + 16 * i;
+      if (m < M && co < d.K) {
+        const int64_t o = (int64_t)m * d.K + co;
+        float v = acc[i][j];
+        if (d.res) v += ldv(d.res, d.res_dt, o);
+        v = rnd(d.y_dt, v);
+        stv(d.y, d.y_dt, o, v);
+        s1 += v;
+        s2 += v * v;
+      }
+    }
+    red[ty][tx + 16 * j][0] = s1;
+    red[ty][tx + 16 * j][1] = s2;
+  }
+  if (d.stats) {
+    __syncthreads();
+    for (int nn = tid; nn < BN; nn += 256) {
+      const int co = n0 + nn;
+      if (co < d.K) {
+        float s1 = 0.f, s2 = 0.f;
+        for (int r = 0; r < 16; ++r) { s1 += red[r][nn][0]; s2 += red[r][nn][1]; }
+        d.stats[((int64_t)tm * d.K + co) * 2 + 0] = s1;
+        d.stats[((int64_t)tm * d.K + co) * 2 + 1] = s2;
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------- conv dgrad
+// dX[m=(n,h,w)][c] (+)= sum_{r,s,k} dY[n, (h+pad-r)/st, (w+pad-s)/st, k] * W[k][r][s][c]
+// (terms whose division is inexact or out of range are zero)
+template <int BM, int BN>
+__global__ void __launch_bounds__(256) k_conv_dgrad(const ConvDesc* __restrict__ tab,
+                                                    const int* __restrict__ tstart, int n) {
+  constexpr int BK = 16, TM = BM / 16, TN = BN / 16;
+  __shared__ float As[BK][BM + 4];
+  __shared__ float Bs[BK][BN + 4];
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const ConvDesc& d = tab[inst];
+  const int t = blockIdx.x - tstart[inst];
+  const int tm = t % d.mtiles, tn = t / d.mtiles;
+  const int M = d.B * d.H * d.W, Kt = d.R * d.S * d.K;
+  const int m0 = tm * BM, n0 = tn * BN;
+  const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+  float acc[TM][TN];
+#pragma unroll
+  for (int i = 0; i < TM; ++i)
+#pragma unroll
+    for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
+  for (int k0 = 0; k0 < Kt; k0 += BK) {
+    for (int e = tid; e < BM * BK; e += 256) {
+      const int kk = e % BK, mm = e / BK;
+      const int m = m0 + mm, k = k0 + kk;
+      float v = 0.f;
+      if (m < M && k < Kt) {
+        const int ko = k % d.K, rs = k / d.K, s = rs % d.S, r = rs / d.S;
+        const int w = m % d.W, tmp = m / d.W, h = tmp % d.H, nb = tmp / d.H;
+        const int pn = h + d.pad - r, qn = w + d.pad - s;
+        if (pn >= 0 && qn >= 0 && pn % d.stride == 0 && qn % d.stride == 0) {
+          const int p = pn / d.stride, q = qn / d.stride;
+          if (p < d.P && q < d.Q) v = __ldg(d.dy + ((int64_t)(nb * d.P + p) * d.Q + q) * d.K + ko);
+        }
+      }
+      As[kk][mm] = d.op_bf16 ? rnd(DT_BF16, v) : v;
+    }
+    for (int e = tid; e < BN * BK; e += 256) {
+      const int nn = e % BN, kk = e / BN;
+      const int k = k0 + kk, c = n0 + nn;
+      float v = 0.f;
+      if (k < Kt && c < d.C) {
+        const int ko = k % d.K, rs = k / d.K;
+        v = ldv(d.w, d.w_dt, ((int64_t)ko * d.R * d.S + rs) * d.C + c);
+      }
+      Bs[kk][nn] = v;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < BK; ++kk) {
+      float a[TM], b[TN];
+#pragma unroll
+      for (int i = 0; i < TM; ++i) a[i] = As[kk][ty + 16 * i];
+#pragma unroll
+      for (int j = 0; j < TN; ++j) b[j] = Bs[kk][tx + 16 * j];
+#pragma unroll
+      for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < TM; ++i) {
+    const int m = m0 + ty + 16 * i;
+#pragma unroll
+    for (int j = 0; j < TN; ++j) {
+      const int c = n0 + tx + 16 * j;
+      if (m < M && c < d.C) {
+        const int64_t o = (int64_t)m * d.C + c;
+        d.dx[o] = d.accumulate ? d.dx[o] + acc[i][j] : acc[i][j];
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------- conv wgrad
+// part[split][k][(r,s,c)] = sum_{m in split} dY[m][k] * act(X)[n, p*st+r-pad, q*st+s-pad, c]
+__global__ void __launch_bounds__(256) k_conv_wgrad(const ConvDesc* __restrict__ tab,
+                                                    const int* __restrict__ tstart, int n) {
+  constexpr int BM = kWgradBM, BN = kWgradBN, BK = kWgradBK, TM = BM / 16, TN = BN / 16;
+  __shared__ float As[BK][BM + 4];
+  __shared__ float Bs[BK][BN + 4];
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const ConvDesc& d = tab[inst];
+  int t = blockIdx.x - tstart[inst];
+  const int tm = t % d.mtiles;
+  t /= d.mtiles;
+  const int tn = t % d.ntiles, split = t / d.ntiles;
+  const int RSC = d.R * d.S * d.C, Mp = d.B * d.P * d.Q;
+  const int m0 = tm * BM, n0 = tn * BN;
+  const int p_begin = split * d.pix_per_split;
+  const int p_end = min(Mp, p_begin + d.pix_per_split);
+  const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+  float acc[TM][TN];
+#pragma unroll
+  for (int i = 0; i < TM; ++i)
+#pragma unroll
+    for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
+  for (int k0 = p_begin; k0 < p_end; k0 += BK) {
+    for (int e = tid; e < BM * BK; e += 256) {
+      const int mm = e % BM, kk = e / BM;
+      const int ko = m0 + mm, pix = k0 + kk;
+      const float v = (ko < d.K && pix < p_end) ? __ldg(d.dy + (int64_t)pix * d.K + ko) : 0.f;
+      As[kk][mm] = d.op_bf16 ? rnd(DT_BF16, v) : v;
+    }
+    for (int e = tid; e < BN * BK; e += 256) {
+      const int nn = e % BN, kk = e / BN;
+      const int j = n0 + nn, pix = k0 + kk;
+      float v = 0.f;
+      if (j < RSC && pix < p_end) {
+        const int c = j % d.C, rs = j / d.C, s = rs % d.S, r = rs / d.S;
+        const int q = pix % d.Q, tmp = pix / d.Q, p = tmp % d.P, nb = tmp / d.P;
+        const int h = p * d.stride + r - d.pad, w = q * d.stride + s - d.pad;
+        if (h >= 0 && h < d.H && w >= 0 && w < d.W)
+          v = ld_src(d.x, ((int64_t)(nb * d.H + h) * d.W + w) * d.C + c, c);
+      }
+      Bs[kk][nn] = d.op_bf16 ? rnd(DT_BF16, v) : v;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < BK; ++kk) {
+      float a[TM], b[TN];
+#pragma unroll
+      for (int i = 0; i < TM; ++i) a[i] = As[kk][ty + 16 * i];
+#pragma unroll
+      for (int j = 0; j < TN; ++j) b[j] = Bs[kk][tx + 16 * j];
+#pragma unroll
+      for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+  float* out = d.dw_part + (int64_t)split * d.K * RSC;
+#pragma unroll
+  for (int i = 0; i < TM; ++i) {
+    const int ko = m0 + ty + 16 * i;
+#pragma unroll
+    for (int j = 0; j < TN; ++j) {
+      const int jj = n0 + tx + 16 * j;
+      if (ko < d.K && jj < RSC) out[(int64_t)ko * RSC + jj] = acc[i][j];
+    }
+  }
+}
+
+__global__ void k_wreduce(const WReduceDesc* __restrict__ tab, const int* __restrict__ tstart, int n) {
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const WReduceDesc& d = tab[inst];
+  const int64_t i = (int64_t)(blockIdx.x - tstart[inst]) * blockDim.x + threadIdx.x;
+  if (i >= d.n) return;
+  float s = 0.f;
+  for (int k = 0; k < d.splits; ++k) s += d.part[(int64_t)k * d.n + i];
+  d.dw[i] = d.accumulate ? d.dw[i] + s : s;
+}
+
+// ---------------------------------------------------------------- row-tile geometry
+// A tile is rows_per_tile rows x all C channels.  For C <= 256 (a power of
+// two) thread t owns channel t % C and rows t / C + g * (256 / C); for
+// C > 256 it owns channels t + 256 i and all rows.
+struct RowTile {
+  int G, cpt, c0, g;
+  __device__ RowTile(int C, int tid) {
+    if (C <= 256) {
+      G = 256 / C; cpt = 1; c0 = tid % C; g = tid / C;
+      if (g >= G) c0 = C;  // idle thread (C does not divide 256)
+    } else { G = 1; cpt = (C + 255) / 256; c0 = tid; g = 0; }
+  }
+};
+
+__global__ void __launch_bounds__(256) k_ew(const EwDesc* __restrict__ tab, const int* __restrict__ tstart, int n) {
+  __shared__ float red[256][2];
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const EwDesc& d = tab[inst];
+  const int tile = blockIdx.x - tstart[inst];
+  const int C = d.C;
+  const RowTile rt(C, threadIdx.x);
+  const int64_t r0 = (int64_t)tile * d.rows_per_tile;
+  const int64_t r1 = min((int64_t)d.M, r0 + d.rows_per_tile);
+  for (int ci = 0; ci < rt.cpt; ++ci) {
+    const int c = rt.c0 + 256 * ci;
+    float s1 = 0.f, s2 = 0.f;
+    if (c < C) {
+      for (int64_t r = r0 + rt.g; r < r1; r += rt.G) {
+        const int64_t o = r * C + c;
+        float v = 0.f;
+        for (int i = 0; i < d.nin; ++i) v = fmaf(d.coef[i], ld_src(d.in[i], o, c), v);
+        if (d.relu) v = fmaxf(v, 0.f);
+        if (d.out) {
+          v = rnd(d.out_dt, v);
+          stv(d.out, d.out_dt, o, v);
+        }
+        s1 += v;
+        s2 += v * v;
+      }
+    }
+    if (d.stats) {
+      if (rt.G == 1) {
+        if (c < C) {
+          d.stats[((int64_t)tile * C + c) * 2] = s1;
+          d.stats[((int64_t)tile * C + c) * 2 + 1] = s2;
+        }
+      } else {
+        red[threadIdx.x][0] = s1;
+        red[threadIdx.x][1] = s2;
+        __syncthreads();
+        if ((int)threadIdx.x < C) {
+          float a = 0.f, b = 0.f;
+          for (int g = 0; g < rt.G; ++g) { a += red[g * C + threadIdx.x][0]; b += red[g * C + threadIdx.x][1]; }
+          d.stats[((int64_t)tile * C + threadIdx.x) * 2] = a;
+          d.stats[((int64_t)tile * C + threadIdx.x) * 2 + 1] = b;
+        }
+        __syncthreads();
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) k_ew_bwd(const EwBwdDesc* __restrict__ tab, const int* __restrict__ tstart,
+                                                int n) {
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const EwBwdDesc& d = tab[inst];
+  const int tile = blockIdx.x - tstart[inst];
+  const int64_t base = (int64_t)tile * d.rows_per_tile * d.C;
+  const int64_t end = min((int64_t)d.M * d.C, base + (int64_t)d.rows_per_tile * d.C);
+  for (int64_t o = base + threadIdx.x; o < end; o += blockDim.x) {
+    float g = d.dout[o];
+    if (d.relu && !(ldv(d.out, d.out_dt, o) > 0.f)) g = 0.f;
+    for (int i = 0; i < d.nin; ++i) {
+      float v = d.coef[i] * g;
+      d.gin[i][o] = d.acc[i] ? d.gin[i][o] + v : v;
+    }
+  }
+}
+
+// ---------------------------------------------------------------- BN
+__global__ void __launch_bounds__(256) k_bn_fin(const BnFinDesc* __restrict__ tab, const int* __restrict__ tstart,
+                                                int n) {
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const BnFinDesc& d = tab[inst];
+  const int c = (blockIdx.x - tstart[inst]) * 8 + threadIdx.x / 32;
+  const int lane = threadIdx.x % 32;
+  if (c >= d.C) return;
+  double s1 = 0.0, s2 = 0.0;
+  for (int t = lane; t < d.tiles; t += 32) {
+    s1 += (double)d.part[((int64_t)t * d.C + c) * 2];
+    s2 += (double)d.part[((int64_t)t * d.C + c) * 2 + 1];
+  }
+  for (int off = 16; off > 0; off >>= 1) {
+    s1 += __shfl_xor_sync(0xffffffffu, s1, off);
+    s2 += __shfl_xor_sync(0xffffffffu, s2, off);
+  }
+  if (lane == 0) {
+    const double mean = s1 / (double)d.count;
+    double var = s2 / (double)d.count - mean * mean;
+    if (var < 0.0) var = 0.0;
+    const double rstd = 1.0 / sqrt(var + 1e-5);
+    const double sc = (double)d.gamma[c] * rstd;
+    d.mean[c] = (float)mean;
+    d.rstd[c] = (float)rstd;
+    d.scale[c] = (float)sc;
+    d.shift[c] = (float)((double)d.beta[c] - mean * sc);
+  }
+}
+
+__global__ void __launch_bounds__(256) k_bnb_reduce(const BnBwdDesc* __restrict__ tab,
+                                                    const int* __restrict__ tstart, int n) {
+  __shared__ float red[256][2];
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const BnBwdDesc& d = tab[inst];
+  const int tile = blockIdx.x - tstart[inst];
+  const int C = d.C;
+  const RowTile rt(C, threadIdx.x);
+  const int64_t r0 = (int64_t)tile * d.rows_per_tile;
+  const int64_t r1 = min((int64_t)d.M, r0 + d.rows_per_tile);
+  for (int ci = 0; ci < rt.cpt; ++ci) {
+    const int c = rt.c0 + 256 * ci;
+    float s1 = 0.f, s2 = 0.f;
+    if (c < C) {
+      const float mean = d.mean[c], rstd = d.rstd[c], sc = d.scale[c], sh = d.shift[c];
+      for (int64_t r = r0 + rt.g; r < r1; r += rt.G) {
+        const int64_t o = r * C + c;
+        const float h = ldv(d.h, d.h_dt, o);
+        float dz = d.da[o];
+        if (d.relu && !(fmaf(sc, h, sh) > 0.f)) dz = 0.f;
+        s1 += dz;
+        s2 += dz * ((h - mean) * rstd);
+      }
+    }
+    if (rt.G == 1) {
+      if (c < C) {
+        d.part[((int64_t)tile * C + c) * 2] = s1;
+        d.part[((int64_t)tile * C + c) * 2 + 1] = s2;
+      }
+    } else {
+      red[threadIdx.x][0] = s1;
+      red[threadIdx.x][1] = s2;
+      __syncthreads();
+      if ((int)threadIdx.x < C) {
+        float a = 0.f, b = 0.f;
+        for (int g = 0; g < rt.G; ++g) { a += red[g * C + threadIdx.x][0]; b += red[g * C + threadIdx.x][1]; }
+        d.part[((int64_t)tile * C + threadIdx.x) * 2] = a;
+        d.part[((int64_t)tile * C + threadIdx.x) * 2 + 1] = b;
+      }
+      __syncthreads();
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) k_bnb_fin(const BnBwdDesc* __restrict__ tab, const int* __restrict__ tstart,
+                                                 int n) {
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const BnBwdDesc& d = tab[inst];
+  const int c = (blockIdx.x - tstart[inst]) * 8 + threadIdx.x / 32;
+  const int lane = threadIdx.x % 32;
+  if (c >= d.C) return;
+  double s1 = 0.0, s2 = 0.0;
+  for (int t = lane; t < d.tiles; t += 32) {
+    s1 += (double)d.part[((int64_t)t * d.C + c) * 2];
+    s2 += (double)d.part[((int64_t)t * d.C + c) * 2 + 1];
+  }
+  for (int off = 16; off > 0; off >>= 1) {
+    s1 += __shfl_xor_sync(0xffffffffu, s1, off);
+    s2 += __shfl_xor_sync(0xffffffffu, s2, off);
+  }
+  if (lane == 0) {
+    d.dbeta[c] = d.accumulate ? d.dbeta[c] + (float)s1 : (float)s1;
+    d.dgamma[c] = d.accumulate ? d.dgamma[c] + (float)s2 : (float)s2;
+    d.coef[c * 3 + 0] = d.gamma[c] * d.rstd[c];
+    d.coef[c * 3 + 1] = (float)(s1 / (double)d.M);
+    d.coef[c * 3 + 2] = (float)(s2 / (double)d.M);
+  }
+}
+
+__global__ void __launch_bounds__(256) k_bnb_apply(const BnBwdDesc* __restrict__ tab,
+                                                   const int* __restrict__ tstart, int n) {
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const BnBwdDesc& d = tab[inst];
+  const int tile = blockIdx.x - tstart[inst];
+  const int C = d.C;
+  const int64_t base = (int64_t)tile * d.rows_per_tile * C;
+  const int64_t end = min((int64_t)d.M * C, base + (int64_t)d.rows_per_tile * C);
+  for (int64_t o = base + threadIdx.x; o < end; o += blockDim.x) {
+    const int c = (int)(o % C);
+    const float h = ldv(d.h, d.h_dt, o);
+    float dz = d.da[o];
+    if (d.relu && !(fmaf(d.scale[c], h, d.shift[c]) > 0.f)) dz = 0.f;
+    const float xhat = (h - d.mean[c]) * d.rstd[c];
+    float v = d.coef[c * 3] * (dz - d.coef[c * 3 + 1] - xhat * d.coef[c * 3 + 2]);
+    if (d.add0) v += d.add0[o];
+    if (d.add1) v += d.add1[o];
+    d.dh[o] = d.accumulate ? d.dh[o] + v : v;
+  }
+}
+
+// ---------------------------------------------------------------- pooling
+__global__ void __launch_bounds__(256) k_pool_fwd(const PoolDesc* __restrict__ tab, const int* __restrict__ tstart,
+                                                  int n) {
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const PoolDesc& d = tab[inst];
+  const int64_t i = (int64_t)(blockIdx.x - tstart[inst]) * 256 + threadIdx.x;
+  const int64_t total = (int64_t)d.B * d.P * d.Q * d.C;
+  if (i >= total) return;
+  const int c = (int)(i % d.C);
+  int64_t t = i / d.C;
+  const int q = (int)(t % d.Q); t /= d.Q;
+  const int p = (int)(t % d.P);
+  const int nb = (int)(t / d.P);
+  float best = -INFINITY;
+  for (int r = 0; r < d.k; ++r)
+    for (int s = 0; s < d.k; ++s) {
+      const int h = p * d.stride + r - d.pad, w = q * d.stride + s - d.pad;
+      if (h < 0 || h >= d.H || w < 0 || w >= d.W) continue;
+      const float v = ld_src(d.x, ((int64_t)(nb * d.H + h) * d.W + w) * d.C + c, c);
+      if (v > best) best = v;
+    }
+  stv(d.y, d.y_dt, i, best);
+}
+
+// dx[n,h,w,c] (+)= sum over windows whose first maximum sits at (h,w) of dy
+__global__ void __launch_bounds__(256) k_pool_bwd(const PoolDesc* __restrict__ tab, const int* __restrict__ tstart,
+                                                  int n) {
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const PoolDesc& d = tab[inst];
+  const int64_t i = (int64_t)(blockIdx.x - tstart[inst]) * 256 + threadIdx.x;
+  const int64_t total = (int64_t)d.B * d.H * d.W * d.C;
+  if (i >= total) return;
+  const int c = (int)(i % d.C);
+  int64_t t = i / d.C;
+  const int w = (int)(t % d.W); t /= d.W;
+  const int h = (int)(t % d.H);
+  const int nb = (int)(t / d.H);
+  float g = 0.f;
+  const int p_lo = max(0, (h + d.pad - d.k + d.stride) / d.stride), p_hi = min(d.P - 1, (h + d.pad) / d.stride);
+  const int q_lo = max(0, (w + d.pad - d.k + d.stride) / d.stride), q_hi = min(d.Q - 1, (w + d.pad) / d.stride);
+  for (int p = p_lo; p <= p_hi; ++p)
+    for (int q = q_lo; q <= q_hi; ++q) {
+      if (h + d.pad - p * d.stride >= d.k || w + d.pad - q * d.stride >= d.k) continue;
+      float best = -INFINITY;
+      int bh = -1, bw = -1;
+      for (int r = 0; r < d.k; ++r)
+        for (int s = 0; s < d.k; ++s) {
+          const int hh = p * d.stride + r - d.pad, ww = q * d.stride + s - d.pad;
+          if (hh < 0 || hh >= d.H || ww < 0 || ww >= d.W) continue;
+          const float v = ld_src(d.x, ((int64_t)(nb * d.H + hh) * d.W + ww) * d.C + c, c);
+          if (v > best) { best = v; bh = hh; bw = ww; }
+        }
+      if (bh == h && bw == w) g += d.dy[((int64_t)(nb * d.P + p) * d.Q + q) * d.C + c];
+    }
+  d.dx[i] = d.accumulate ? d.dx[i] + g : g;
+}
+
+// ---------------------------------------------------------------- GEMM (head)
+__global__ void __launch_bounds__(256) k_gemm(const GemmDesc* __restrict__ tab, const int* __restrict__ tstart,
+                                              int n) {
+  constexpr int BM = 64, BN = 64, BK = 16;
+  __shared__ float As[BK][BM + 4];
+  __shared__ float Bs[BK][BN + 4];
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const GemmDesc& d = tab[inst];
+  const int t = blockIdx.x - tstart[inst];
+  const int tm = t % d.mtiles, tn = t / d.mtiles;
+  const int m0 = tm * BM, n0 = tn * BN;
+  const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+  float acc[4][4] = {};
+  for (int k0 = 0; k0 < d.K; k0 += BK) {
+    for (int e = tid; e < BM * BK; e += 256) {
+      const int kk = e % BK, mm = e / BK;
+      const int m = m0 + mm, k = k0 + kk;
+      As[kk][mm] = (m < d.M && k < d.K) ? d.A[m * d.sam + k * d.sak] : 0.f;
+    }
+    for (int e = tid; e < BN * BK; e += 256) {
+      const int nn = e % BN, kk = e / BN;
+      const int nc = n0 + nn, k = k0 + kk;
+      Bs[kk][nn] = (nc < d.N && k < d.K) ? d.Bm[k * d.sbk + nc * d.sbn] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < BK; ++kk)
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(As[kk][ty + 16 * i], Bs[kk][tx + 16 * j], acc[i][j]);
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int m = m0 + ty + 16 * i, nc = n0 + tx + 16 * j;
+      if (m < d.M && nc < d.N) {
+        float v = acc[i][j];
+        if (d.bias) v += d.bias[nc];
+        if (d.beta != 0.f) v += d.beta * d.Cm[m * d.scm + nc];
+        if (d.relu) v = fmaxf(v, 0.f);
+        d.Cm[m * d.scm + nc] = v;
+      }
+    }
+}
+
+// ---------------------------------------------------------------- head + misc
+__global__ void k_gap(Src x, float* feat, int B, int HW, int C) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= B * C) return;
+  const int b = i / C, c = i % C;
+  float s = 0.f;
+  for (int k = 0; k < HW; ++k) s += ld_src(x, ((int64_t)b * HW + k) * C + c, c);
+  feat[i] = s / (float)HW;
+}
+
+__global__ void k_gap_bwd(const float* dfeat, float* dx, int B, int HW, int C) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (int64_t)B * HW * C) return;
+  const int c = (int)(i % C);
+  const int b = (int)(i / ((int64_t)HW * C));
+  dx[i] = dfeat[b * C + c] / (float)HW;
+}
+
+// one CTA: per-sample log-sum-exp loss, mean over the batch in a fixed order
+__global__ void __launch_bounds__(256) k_softmax_ce(const float* logits, const int32_t* labels, int B, int m,
+                                                    float* loss, float* dlogits, int32_t* status) {
+  __shared__ float per[1024];
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  for (int b = warp; b < B; b += 8) {
+    const float* z = logits + (int64_t)b * m;
+    float mx = -INFINITY;
+    for (int i = lane; i < m; i += 32) mx = fmaxf(mx, z[i]);
+    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    float se = 0.f;
+    for (int i = lane; i < m; i += 32) se += expf(z[i] - mx);
+    for (int off = 16; off > 0; off >>= 1) se += __shfl_xor_sync(0xffffffffu, se, off);
+    const int lab = labels[b];
+    const float lse = logf(se) + mx;
+    for (int i = lane; i < m; i += 32) {
+      const float p = expf(z[i] - mx) / se;
+      dlogits[(int64_t)b * m + i] = (p - (i == lab ? 1.f : 0.f)) / (float)B;
+    }
+    if (lane == 0) per[b] = lse - ((lab >= 0 && lab < m) ? z[lab] : 0.f);
+    if (lane == 0 && (lab < 0 || lab >= m)) atomicExch(status, 1);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    for (int b = 0; b < B; ++b) s += per[b];
+    const float l = (float)(s / B);
+    *loss = l;
+    if (!isfinite(l)) atomicExch(status, 2);
+  }
+}
+
+__global__ void k_colsum(const float* A, int rows, int cols, float* out) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= cols) return;
+  float s = 0.f;
+  for (int r = 0; r < rows; ++r) s += A[(int64_t)r * cols + c];
+  out[c] = s;
+}
+
+__global__ void k_relu_mask(float* g, const float* pre, int64_t n) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n && !(pre[i] > 0.f)) g[i] = 0.f;
+}
+
+__global__ void k_sgd(float* __restrict__ w, const float* __restrict__ g, float* __restrict__ v, void* shadow,
+                      int32_t shadow_dt, int64_t n, float lr, float mu, float wd, int nesterov, int first) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const float wi = w[i];
+    const float di = fmaf(wd, wi, g[i]);
+    const float vi = first ? di : fmaf(mu, v[i], di);
+    v[i] = vi;
+    const float step = nesterov ? fmaf(mu, vi, di) : vi;
+    const float wn = fmaf(-lr, step, wi);
+    w[i] = wn;
+    if (shadow) stv(shadow, shadow_dt, i, wn);
+  }
+}
+
+__global__ void k_pack_input(const float* x, void* out, int32_t dt, int B, int C, int H, int W) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = (int64_t)B * C * H * W;
+  if (i >= total) return;
+  const int c = (int)(i % C);
+  int64_t t = i / C;
+  const int w = (int)(t % W); t /= W;
+  const int h = (int)(t % H);
+  const int b = (int)(t / H);
+  stv(out, dt, i, x[(((int64_t)b * C + c) * H + h) * W + w]);
+}
+
+__global__ void k_export(Src x, int B, int H, int W, int C, float* out) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = (int64_t)B * C * H * W;
+  if (i >= total) return;
+  const int c = (int)(i % C);
+  int64_t t = i / C;
+  const int w = (int)(t % W); t /= W;
+  const int h = (int)(t % H);
+  const int b = (int)(t / H);
+  out[(((int64_t)b * C + c) * H + h) * W + w] = ld_src(x, i, c);
+}
+
+__global__ void k_copy_cast(const float* in, void* out, int32_t dt, int64_t n) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) stv(out, dt, i, in[i]);
+}
+
+// ---------------------------------------------------------------- launchers
+static inline int cdiv64(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
+
+cudaError_t launch_conv_fwd_simt(const ConvDesc* tab, const int* tstart, int n, int total, int variant,
+                                 cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  if (variant == 0) k_conv_fwd<64, 64><<<total, 256, 0, st>>>(tab, tstart, n);
+  else if (variant == 1) k_conv_fwd<128, 32><<<total, 256, 0, st>>>(tab, tstart, n);
+  else k_conv_fwd<256, 16><<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_conv_dgrad_simt(const ConvDesc* tab, const int* tstart, int n, int total, int variant,
+                                   cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  if (variant == 0) k_conv_dgrad<64, 64><<<total, 256, 0, st>>>(tab, tstart, n);
+  else if (variant == 1) k_conv_dgrad<128, 32><<<total, 256, 0, st>>>(tab, tstart, n);
+  else k_conv_dgrad<256, 16><<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_conv_wgrad_simt(const ConvDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_conv_wgrad<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_wreduce(const WReduceDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_wreduce<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_ew(const EwDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_ew<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_ew_bwd(const EwBwdDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_ew_bwd<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_bn_fin(const BnFinDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_bn_fin<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_bnb_reduce(const BnBwdDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_bnb_reduce<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_bnb_fin(const BnBwdDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_bnb_fin<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_bnb_apply(const BnBwdDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_bnb_apply<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_pool_fwd(const PoolDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_pool_fwd<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_pool_bwd(const PoolDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_pool_bwd<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_gemm(const GemmDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_gemm<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_pack_input(const float* x, void* out, int32_t dt, int B, int C, int H, int W, cudaStream_t st) {
+  const int64_t total = (int64_t)B * C * H * W;
+  k_pack_input<<<cdiv64(total, 256), 256, 0, st>>>(x, out, dt, B, C, H, W);
+  return cudaGetLastError();
+}
+cudaError_t launch_gap(Src x, float* feat, int B, int HW, int C, cudaStream_t st) {
+  k_gap<<<cdiv64((int64_t)B * C, 256), 256, 0, st>>>(x, feat, B, HW, C);
+  return cudaGetLastError();
+}
+cudaError_t launch_gap_bwd(const float* dfeat, float* dx, int B, int HW, int C, cudaStream_t st) {
+  k_gap_bwd<<<cdiv64((int64_t)B * HW * C, 256), 256, 0, st>>>(dfeat, dx, B, HW, C);
+  return cudaGetLastError();
+}
+cudaError_t launch_softmax_ce(const float* logits, const int32_t* labels, int B, int m, float* loss,
+                              float* dlogits, int32_t* status, cudaStream_t st) {
+  if (B > 1024) return cudaErrorInvalidValue;
+  k_softmax_ce<<<1, 256, 0, st>>>(logits, labels, B, m, loss, dlogits, status);
+  return cudaGetLastError();
+}
+cudaError_t launch_colsum(const float* A, int rows, int cols, float* out, cudaStream_t st) {
+  k_colsum<<<cdiv64(cols, 128), 128, 0, st>>>(A, rows, cols, out);
+  return cudaGetLastError();
+}
+cudaError_t launch_relu_mask(float* g, const float* pre, int64_t n, cudaStream_t st) {
+  k_relu_mask<<<cdiv64(n, 256), 256, 0, st>>>(g, pre, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_sgd(float* w, const float* g, float* v, void* shadow, int32_t shadow_dt, int64_t n, float lr,
+                       float mu, float wd, int nesterov, int first, cudaStream_t st) {
+  int blocks = cdiv64(n, 256);
+  if (blocks > 152 * 16) blocks = 152 * 16;
+  if (blocks < 1) blocks = 1;
+  k_sgd<<<blocks, 256, 0, st>>>(w, g, v, shadow, shadow_dt, n, lr, mu, wd, nesterov, first);
+  return cudaGetLastError();
+}
+cudaError_t launch_export(Src x, int B, int H, int W, int C, float* out, cudaStream_t st) {
+  const int64_t total = (int64_t)B * C * H * W;
+  k_export<<<cdiv64(total, 256), 256, 0, st>>>(x, B, H, W, C, out);
+  return cudaGetLastError();
+}
+cudaError_t launch_copy_cast(const float* in, void* out, int32_t dt, int64_t n, cudaStream_t st) {
+  int blocks = cdiv64(n, 256);
+  if (blocks > 152 * 16) blocks = 152 * 16;
+  if (blocks < 1) blocks = 1;
+  k_copy_cast<<<blocks, 256, 0, st>>>(in, out, dt, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_weight_cast(const float* in, void* out, int32_t dt, int64_t n, cudaStream_t st) {
+  return launch_copy_cast(in, out, dt, n, st);
+}
+
+}  // namespace pnn

@@ -1,0 +1,172 @@
+// Internal descriptors shared by the host runtime and the CUDA kernels.
+// Every grouped launch receives a device table of per-instance descriptors
+// plus a prefix array of tile counts; CTA b belongs to the instance i with
+// tile_start[i] <= b < tile_start[i+1].  Tensors are NHWC with the batch
+// folded into the row index (row m = (n*H + h)*W + w).
+#pragma once
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace pnn {
+
+enum DType : int32_t { DT_F32 = 0, DT_BF16 = 1 };
+
+// A tensor operand.  When scale != nullptr the value read is the "virtual"
+// BN(+ReLU) output  v = act(scale[c] * src + shift[c]); zero padding of a
+// convolution applies to v, not to src.
+struct Src {
+  const void* ptr;
+  const float* scale;
+  const float* shift;
+  int32_t dt;
+  int32_t relu;
+};
+
+struct ConvDesc {
+  Src x;                 // forward / wgrad: conv input (maybe virtual)
+  const void* w;         // weights [K][R][S][C], dtype w_dt
+  int32_t w_dt;
+  int32_t B, H, W, C;    // input geometry
+  int32_t P, Q, K;       // output geometry
+  int32_t R, S, stride, pad;
+  // forward epilogue
+  void* y; int32_t y_dt;
+  const void* res; int32_t res_dt;   // residual added to the output (or null)
+  float* stats;                       // per-tile BN partials [mtiles][K][2] or null
+  // dgrad: dx[B*H*W][C] (fp32) = (accumulate ? dx : 0) + W^T * dy
+  float* dx; int32_t accumulate;
+  // dgrad / wgrad operand dy[B*P*Q][K] (fp32)
+  const float* dy;
+  // wgrad: partial sums [splits][K][R*S*C]
+  float* dw_part;
+  int32_t splits, pix_per_split;
+  int32_t mtiles, ntiles;             // tile grid of this instance
+  int32_t op_bf16;                    // round both contraction operands to bf16 (bf16 mode)
+};
+
+// out = act( sum_i coef_i * in_i ), optional BN partials of out, NHWC [M][C].
+struct EwDesc {
+  Src in[3];
+  float coef[3];
+  int32_t nin;
+  void* out; int32_t out_dt;
+  int32_t relu;
+  float* stats;          // [tiles][C][2] or null
+  int64_t M;
+  int32_t C;
+  int32_t rows_per_tile;
+  int32_t tiles;
+};
+
+// backward of EW: g = dout * [out > 0 if relu]; grad_i (+)= coef_i * g
+struct EwBwdDesc {
+  const float* dout;
+  const void* out; int32_t out_dt; int32_t relu;
+  float* gin[3]; float coef[3]; int32_t acc[3];
+  int32_t nin;
+  int64_t M; int32_t C;
+  int32_t rows_per_tile, tiles;
+};
+
+// BN statistics finalisation: partials[tiles][C][2] -> mean, rstd, scale, shift
+struct BnFinDesc {
+  const float* part;
+  int32_t tiles, C;
+  int64_t count;         // number of rows M
+  const float* gamma; const float* beta;
+  float* mean; float* rstd; float* scale; float* shift;
+};
+
+// BN backward: dz = da * [z > 0 if relu], z = scale*h + shift, xhat = (h-mean)*rstd
+//   reduce: part[tile][c] = (sum dz, sum dz*xhat)
+//   fin:    dbeta = sum dz, dgamma = sum dz*xhat, coef[c] = (gamma*rstd, dbeta/M, dgamma/M)
+//   apply:  dh (+)= gamma*rstd * (dz - dbeta/M - xhat*dgamma/M)
+struct BnBwdDesc {
+  const float* da;
+  const void* h; int32_t h_dt;
+  const float* mean; const float* rstd; const float* scale; const float* shift;
+  const float* gamma;
+  int32_t relu;
+  float* part;           // [tiles][C][2]
+  float* dgamma; float* dbeta;
+  float* coef;           // [C][3]
+  float* dh; int32_t accumulate;     // apply: accumulate into dh; fin: into dgamma/dbeta
+  const float* add0; const float* add1;  // apply: extra gradients added into dh (residual paths)
+  int64_t M; int32_t C;
+  int32_t rows_per_tile, tiles;
+};
+
+struct PoolDesc {
+  Src x;                 // input (maybe virtual)
+  void* y; int32_t y_dt; // output
+  int32_t B, H, W, C, P, Q, k, stride, pad;
+  // backward: dx (+)= route(dy)
+  const float* dy; float* dx; int32_t accumulate;
+  int32_t tiles;
+};
+
+// wgrad split reduction: dw[K*RSC] = sum_s part[s][K*RSC]
+struct WReduceDesc {
+  const float* part;
+  float* dw;
+  int32_t splits;
+  int32_t accumulate;
+  int64_t n;
+  int32_t tiles;
+};
+
+// generic strided fp32 GEMM: C[m][n] = beta*C + sum_k A[m*sam + k*sak] * B[k*sbk + n*sbn] (+ bias[n]) (relu)
+struct GemmDesc {
+  const float* A; const float* Bm; float* Cm;
+  const float* bias;
+  int32_t M, N, K;
+  int64_t sam, sak, sbk, sbn, scm;
+  float beta;
+  int32_t relu;
+  int32_t mtiles, ntiles;
+};
+
+// ------------------------------------------------------------ launchers
+// All launchers enqueue on `st` and return cudaGetLastError().
+cudaError_t launch_conv_fwd_simt(const ConvDesc* tab, const int* tstart, int n, int total_tiles,
+                                 int variant, cudaStream_t st);
+cudaError_t launch_conv_dgrad_simt(const ConvDesc* tab, const int* tstart, int n, int total_tiles,
+                                   int variant, cudaStream_t st);
+cudaError_t launch_conv_wgrad_simt(const ConvDesc* tab, const int* tstart, int n, int total_tiles,
+                                   cudaStream_t st);
+cudaError_t launch_wreduce(const WReduceDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+cudaError_t launch_ew(const EwDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+cudaError_t launch_ew_bwd(const EwBwdDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+cudaError_t launch_bn_fin(const BnFinDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+cudaError_t launch_bnb_reduce(const BnBwdDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+cudaError_t launch_bnb_fin(const BnBwdDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+cudaError_t launch_bnb_apply(const BnBwdDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+cudaError_t launch_pool_fwd(const PoolDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+cudaError_t launch_pool_bwd(const PoolDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+cudaError_t launch_gemm(const GemmDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+
+// single-instance helpers
+cudaError_t launch_pack_input(const float* x_nchw, void* out, int32_t out_dt, int B, int C, int H, int W,
+                              cudaStream_t st);
+cudaError_t launch_gap(Src x, float* feat, int B, int HW, int C, cudaStream_t st);
+cudaError_t launch_gap_bwd(const float* dfeat, float* dx, int B, int HW, int C, cudaStream_t st);
+cudaError_t launch_softmax_ce(const float* logits, const int32_t* labels, int B, int m, float* loss,
+                              float* dlogits, int32_t* status, cudaStream_t st);
+cudaError_t launch_colsum(const float* A, int rows, int cols, float* out, cudaStream_t st);
+cudaError_t launch_relu_mask(float* g, const float* pre, int64_t n, cudaStream_t st);
+cudaError_t launch_sgd(float* w, const float* g, float* v, void* shadow, int32_t shadow_dt, int64_t n,
+                       float lr, float mu, float wd, int nesterov, int first, cudaStream_t st);
+cudaError_t launch_export(Src x, int B, int H, int W, int C, float* out_nchw, cudaStream_t st);
+cudaError_t launch_copy_cast(const float* in, void* out, int32_t out_dt, int64_t n, cudaStream_t st);
+cudaError_t launch_weight_cast(const float* in, void* out, int32_t out_dt, int64_t n, cudaStream_t st);
+
+// tile geometry helpers shared by runtime and kernels
+constexpr int kEwRowsPerTile = 64;
+struct ConvTile { int BM, BN; };
+inline ConvTile simt_tile(int variant) {
+  return variant == 0 ? ConvTile{64, 64} : (variant == 1 ? ConvTile{128, 32} : ConvTile{256, 16});
+}
+constexpr int kWgradBM = 64, kWgradBN = 64, kWgradBK = 16;
+
+}  // namespace pnn

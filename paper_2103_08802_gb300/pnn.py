@@ -1,0 +1,283 @@
+"""Thin Python binding of libpnn.so (include/pnn.h).
+
+Argument marshalling only: every step of the training path runs in the
+library's CUDA kernels.  PyTorch provides the device workspace and streams.
+If the library has not been built this module raises; there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libpnn.so")
+
+PNN_OK = 0
+PRECISION = {"bf16": 0, "fp32": 1}
+CORRECTION = {"residual": 0, "delta": 1}
+LAYER_OP = {"conv": 0, "conv_bn_relu": 1, "basic": 2, "bottleneck": 3}
+HEAD = {"gap_fc": 0, "bn_relu_gap_fc": 1, "gap_mlp": 2}
+CJ_POST = {"none": 0, "bn_relu": 1}
+TENSOR = {"x": 0, "y": 1, "r": 2, "rtilde": 3, "ytilde": 4, "D": 5, "logits": 6}
+
+
+class PnnError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__(f"pnn status {status}: {msg}")
+        self.status = status
+
+
+class Layer(C.Structure):
+    _fields_ = [("op", C.c_int32), ("cout", C.c_int32), ("mid", C.c_int32), ("k", C.c_int32),
+                ("stride", C.c_int32), ("pool", C.c_int32)]
+
+
+class Desc(C.Structure):
+    _fields_ = [("batch", C.c_int32), ("in_c", C.c_int32), ("in_h", C.c_int32), ("in_w", C.c_int32),
+                ("classes", C.c_int32),
+                ("stem", C.POINTER(Layer)), ("n_stem", C.c_int32),
+                ("body", C.POINTER(Layer)), ("n_body", C.c_int32),
+                ("segments", C.POINTER(C.c_int32)), ("n_seg", C.c_int32),
+                ("coarse", C.POINTER(Layer)), ("coarse_len", C.POINTER(C.c_int32)),
+                ("cj_post", C.c_int32), ("head_kind", C.c_int32),
+                ("head_hidden", C.POINTER(C.c_int32)), ("n_hidden", C.c_int32)]
+
+
+class Options(C.Structure):
+    _fields_ = [("precision", C.c_int32), ("correction", C.c_int32), ("seed", C.c_uint64),
+                ("lr", C.c_float), ("momentum", C.c_float), ("weight_decay", C.c_float),
+                ("nesterov", C.c_int32), ("stream_fp32", C.c_int32), ("conv_impl", C.c_int32),
+                ("stream", C.c_void_p)]
+
+
+_lib = None
+
+
+def load():
+    """Load libpnn.so; raises if it is missing (run build() first)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is not built; call __graft_entry__.build() or "
+                          "paper_2103_08802_gb300.build.build()")
+    lib = C.CDLL(LIB_PATH)
+    P, I32, SZ = C.c_void_p, C.c_int32, C.c_size_t
+    sig = {
+        "pnn_default_options": (None, [C.POINTER(Options)]),
+        "pnn_create": (C.c_int, [C.POINTER(Desc), C.POINTER(Options), C.POINTER(P)]),
+        "pnn_workspace_bytes": (C.c_int, [P, C.POINTER(SZ)]),
+        "pnn_bind_workspace": (C.c_int, [P, P, SZ]),
+        "pnn_forward": (C.c_int, [P, P, P, P]),
+        "pnn_backward": (C.c_int, [P]),
+        "pnn_sgd_step": (C.c_int, [P, C.c_float]),
+        "pnn_train_step": (C.c_int, [P, P, P, P]),
+        "pnn_train_step_host": (C.c_int, [P, P, P, P]),
+        "pnn_sync": (C.c_int, [P]),
+        "pnn_destroy": (None, [P]),
+        "pnn_num_params": (C.c_int, [P, C.POINTER(SZ)]),
+        "pnn_num_param_tensors": (C.c_int, [P, C.POINTER(I32)]),
+        "pnn_param_tensor_info": (C.c_int, [P, I32, C.POINTER(I32), C.POINTER(I32), C.POINTER(SZ)]),
+        "pnn_get_params": (C.c_int, [P, P, SZ]),
+        "pnn_set_params": (C.c_int, [P, P, SZ]),
+        "pnn_get_grads": (C.c_int, [P, P, SZ]),
+        "pnn_get_momentum": (C.c_int, [P, P, SZ]),
+        "pnn_tensor_size": (C.c_int, [P, I32, I32, C.POINTER(SZ)]),
+        "pnn_get_tensor": (C.c_int, [P, I32, I32, P, SZ]),
+        "pnn_get_timings": (C.c_int, [P, C.POINTER(C.c_float)]),
+        "pnn_launch_counts": (C.c_int, [P, C.POINTER(I32)]),
+        "pnn_profile": (C.c_int, [P, I32]),
+        "pnn_profile_read": (C.c_int, [P, I32, C.POINTER(C.c_double), C.POINTER(C.c_int64),
+                                       C.POINTER(C.c_double), C.POINTER(C.c_double)]),
+        "pnn_num_kernel_kinds": (I32, []),
+        "pnn_kernel_kind_name": (C.c_char_p, [I32]),
+        "pnn_last_error": (C.c_char_p, [P]),
+        "pnn_status_string": (C.c_char_p, [C.c_int]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _layers(specs):
+    arr = (Layer * max(1, len(specs)))()
+    for i, s in enumerate(specs):
+        arr[i] = Layer(LAYER_OP[s["op"]], s["cout"], s.get("mid", 0), s.get("k", 3), s.get("stride", 1),
+                       s.get("pool", 0))
+    return arr
+
+
+class ParaNet:
+    """A parareal network planned and trained by libpnn.
+
+    desc: a description dict (see workloads).  The workspace is one torch
+    uint8 tensor on `device`."""
+
+    def __init__(self, desc, precision=None, correction=None, seed=0, lr=0.1, momentum=0.9,
+                 weight_decay=5e-4, nesterov=True, stream_fp32=True, conv_impl=0, stream=None,
+                 device="cuda", bind=True):
+        self.lib = load()
+        self.desc = desc
+        self._keep = []
+        d = Desc()
+        d.batch, d.in_c, d.in_h, d.in_w = desc["batch"], desc["in_c"], desc["in_h"], desc["in_w"]
+        d.classes = desc["classes"]
+        stem, body = _layers(desc["stem"]), _layers(desc["body"])
+        segs = (C.c_int32 * len(desc["segments"]))(*desc["segments"])
+        flat = [l for F in desc["coarse"] for l in F]
+        coarse = _layers(flat)
+        clen = (C.c_int32 * max(1, len(desc["coarse"])))(*[len(F) for F in desc["coarse"]])
+        hidden = list(desc["head"].get("hidden", []))
+        hid = (C.c_int32 * max(1, len(hidden)))(*hidden)
+        self._keep += [stem, body, segs, coarse, clen, hid]
+        d.stem, d.n_stem = stem, len(desc["stem"])
+        d.body, d.n_body = body, len(desc["body"])
+        d.segments, d.n_seg = segs, len(desc["segments"])
+        d.coarse, d.coarse_len = coarse, clen
+        d.cj_post = CJ_POST[desc["cj_post"]]
+        d.head_kind = HEAD[desc["head"]["kind"]]
+        d.head_hidden, d.n_hidden = hid, len(hidden)
+        o = Options()
+        self.lib.pnn_default_options(C.byref(o))
+        o.precision = PRECISION[precision or desc["precision"]]
+        o.correction = CORRECTION[correction or desc.get("correction", "residual")]
+        o.seed, o.lr, o.momentum, o.weight_decay = seed, lr, momentum, weight_decay
+        o.nesterov, o.stream_fp32, o.conv_impl = int(nesterov), int(stream_fp32), int(conv_impl)
+        self.stream = stream
+        o.stream = None if stream is None else C.c_void_p(stream.cuda_stream)
+        self.h = C.c_void_p()
+        self._check(self.lib.pnn_create(C.byref(d), C.byref(o), C.byref(self.h)), global_err=True)
+        sz = C.c_size_t()
+        self._check(self.lib.pnn_workspace_bytes(self.h, C.byref(sz)))
+        self.workspace_bytes = sz.value
+        self.device = device
+        self.ws = None
+        if bind:
+            self.bind()
+
+    # ------------------------------------------------------------ plumbing
+    def _check(self, status, global_err=False):
+        if status != PNN_OK:
+            msg = self.lib.pnn_last_error(None if global_err else self.h)
+            raise PnnError(status, msg.decode() if msg else "")
+
+    def bind(self):
+        import torch
+        self.ws = torch.empty(self.workspace_bytes, dtype=torch.uint8, device=self.device)
+        self._check(self.lib.pnn_bind_workspace(self.h, C.c_void_p(self.ws.data_ptr()), self.workspace_bytes))
+
+    def close(self):
+        if getattr(self, "h", None):
+            self.lib.pnn_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # ------------------------------------------------------------ step
+    def forward(self, x, labels, loss=None):
+        self._check(self.lib.pnn_forward(self.h, C.c_void_p(x.data_ptr()), C.c_void_p(labels.data_ptr()),
+                                         None if loss is None else C.c_void_p(loss.data_ptr())))
+
+    def backward(self):
+        self._check(self.lib.pnn_backward(self.h))
+
+    def sgd_step(self, lr=0.0):
+        self._check(self.lib.pnn_sgd_step(self.h, lr))
+
+    def train_step(self, x, labels, loss=None):
+        self._check(self.lib.pnn_train_step(self.h, C.c_void_p(x.data_ptr()), C.c_void_p(labels.data_ptr()),
+                                            None if loss is None else C.c_void_p(loss.data_ptr())))
+
+    def train_step_host(self, x, labels):
+        """x: float32 NCHW host array (ideally pinned), labels int32."""
+        out = C.c_float()
+        xp = x.data_ptr() if hasattr(x, "data_ptr") else x.ctypes.data
+        lp = labels.data_ptr() if hasattr(labels, "data_ptr") else labels.ctypes.data
+        self._check(self.lib.pnn_train_step_host(self.h, C.c_void_p(xp), C.c_void_p(lp), C.byref(out)))
+        return out.value
+
+    def sync(self):
+        self._check(self.lib.pnn_sync(self.h))
+
+    # ------------------------------------------------------------ parameters
+    @property
+    def num_params(self):
+        n = C.c_size_t()
+        self._check(self.lib.pnn_num_params(self.h, C.byref(n)))
+        return n.value
+
+    def param_spec(self):
+        """[(kind, dims, offset)] in theta-bar order."""
+        n = C.c_int32()
+        self._check(self.lib.pnn_num_param_tensors(self.h, C.byref(n)))
+        out = []
+        for i in range(n.value):
+            k, dims, off = C.c_int32(), (C.c_int32 * 4)(), C.c_size_t()
+            self._check(self.lib.pnn_param_tensor_info(self.h, i, C.byref(k), dims, C.byref(off)))
+            out.append((k.value, tuple(dims), off.value))
+        return out
+
+    def _vec(self, fn):
+        a = np.empty(self.num_params, dtype=np.float32)
+        self._check(fn(self.h, C.c_void_p(a.ctypes.data), a.size))
+        return a
+
+    def get_params(self):
+        return self._vec(self.lib.pnn_get_params)
+
+    def get_grads(self):
+        return self._vec(self.lib.pnn_get_grads)
+
+    def get_momentum(self):
+        return self._vec(self.lib.pnn_get_momentum)
+
+    def set_params(self, theta):
+        a = np.ascontiguousarray(theta, dtype=np.float32)
+        self._check(self.lib.pnn_set_params(self.h, C.c_void_p(a.ctypes.data), a.size))
+
+    # ------------------------------------------------------------ tensors
+    def tensor_size(self, which, j=0):
+        n = C.c_size_t()
+        self._check(self.lib.pnn_tensor_size(self.h, TENSOR[which], j, C.byref(n)))
+        return n.value
+
+    def get_tensor(self, which, j=0):
+        n = self.tensor_size(which, j)
+        if n == 0:
+            raise KeyError((which, j))
+        a = np.empty(n, dtype=np.float32)
+        self._check(self.lib.pnn_get_tensor(self.h, TENSOR[which], j, C.c_void_p(a.ctypes.data), n))
+        return a
+
+    def timings(self):
+        ms = (C.c_float * 10)()
+        self._check(self.lib.pnn_get_timings(self.h, ms))
+        keys = ["pre_f", "fine_f", "coarse_f", "post_f", "pre_b", "fine_b", "coarse_b", "post_b", "update", "total"]
+        return dict(zip(keys, list(ms)))
+
+    def profile(self, enable=True):
+        self._check(self.lib.pnn_profile(self.h, int(enable)))
+
+    def profile_read(self):
+        """{kind name: (ms, launches, flops, bytes)} accumulated since profile()."""
+        out = {}
+        for k in range(self.lib.pnn_num_kernel_kinds()):
+            ms, n, fl, by = C.c_double(), C.c_int64(), C.c_double(), C.c_double()
+            self._check(self.lib.pnn_profile_read(self.h, k, C.byref(ms), C.byref(n), C.byref(fl), C.byref(by)))
+            if n.value:
+                out[self.lib.pnn_kernel_kind_name(k).decode()] = (ms.value, n.value, fl.value, by.value)
+        return out
+
+    def launch_counts(self):
+        c = (C.c_int32 * 3)()
+        self._check(self.lib.pnn_launch_counts(self.h, c))
+        return list(c)

@@ -1,0 +1,90 @@
+"""Host-side checks of the C-ABI library (no GPU needed): it loads, exports
+every function include/pnn.h declares, plans the five workloads with the
+parameter table of the oracle (eq:barf order and shapes) and rejects bad
+descriptions with PNN_EINVAL."""
+import copy
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+import workloads as W
+from oracle import pnn_oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def pnn():
+    from paper_2103_08802_gb300 import build, pnn as P
+    build.build()
+    P.load()
+    return P
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "pnn.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(pnn_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_symbol(pnn):
+    lib = C.CDLL(pnn.LIB_PATH)
+    names = declared_functions()
+    assert len(names) >= 20
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+@pytest.mark.parametrize("idx", range(5))
+def test_plan_matches_oracle_parameter_table(pnn, idx):
+    d = W.config(idx)
+    net = pnn.ParaNet(d, bind=False)
+    spec = net.param_spec()
+    ospec = O.ParaNet(d).spec
+    assert len(spec) == len(ospec)
+    off = 0
+    for (kind, dims, o), (okind, shape) in zip(spec, ospec):
+        assert kind == okind
+        assert tuple(dims[:len(shape)]) == tuple(shape) and all(x == 1 for x in dims[len(shape):])
+        assert o == off
+        off += int(np.prod(shape))
+    assert net.num_params == off
+    assert net.workspace_bytes > 0
+
+
+@pytest.mark.parametrize("mode", ["residual", "delta"])
+def test_plan_delta_and_n1(pnn, mode):
+    d = W.config(2)
+    d["correction"] = mode
+    net = pnn.ParaNet(d, bind=False)
+    assert net.num_params == O.ParaNet(d).num_params()
+    d1 = copy.deepcopy(d)
+    d1["segments"] = [333]
+    d1["coarse"] = []
+    assert pnn.ParaNet(d1, bind=False).num_params == O.ParaNet(d1).num_params() == 10_327_706
+
+
+def test_bad_descriptions_are_rejected(pnn):
+    base = W.config(0)
+    bad = []
+    d = copy.deepcopy(base); d["segments"] = [1, 2]; bad.append(d)            # does not sum to body
+    d = copy.deepcopy(base); d["batch"] = 0; bad.append(d)
+    d = copy.deepcopy(base); d["coarse"] = [[W.conv_bn_relu(32)]]; bad.append(d)  # F^1 output is not X_2
+    d = copy.deepcopy(base); d["body"][0] = W.basic(16) | {"cout": 0}; bad.append(d)
+    d = copy.deepcopy(base); d["stem"] = [W.conv(16, k=5)]; bad.append(d)
+    for d in bad:
+        with pytest.raises(pnn.PnnError) as e:
+            pnn.ParaNet(d, bind=False)
+        assert e.value.status == 1
+
+
+def test_calls_without_workspace_fail_cleanly(pnn):
+    net = pnn.ParaNet(W.config(0), bind=False)
+    lib = net.lib
+    assert lib.pnn_backward(net.h) == 7          # PNN_ENOTBOUND
+    assert lib.pnn_sgd_step(net.h, 0.1) == 7
+    assert lib.pnn_backward(None) == 1            # null handle
+    assert lib.pnn_status_string(5) == b"device wait timed out"

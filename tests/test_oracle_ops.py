@@ -150,3 +150,41 @@ def test_sgd_nesterov_hand_example():
     th2, b2 = O.sgd_step(th1, np.array(g["grad2"]), b1, g["lr"], g["momentum"], g["weight_decay"], True)
     np.testing.assert_allclose(th2, g["theta2"], rtol=1e-10)
     np.testing.assert_allclose(b2, g["buf2"], rtol=1e-10, atol=1e-15)
+
+
+def test_round_bf16_matches_torch_and_ties_to_even():
+    x = (rng.standard_normal(20000) * 10.0 ** rng.integers(-6, 6, 20000)).astype(np.float32)
+    ref = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(O.round_bf16(x.astype(np.float64)), ref)
+    # exact halfway cases round to the even neighbour
+    assert O.round_bf16(1 + 2.0 ** -8) == 1.0
+    assert O.round_bf16(1 + 3 * 2.0 ** -8) == 1 + 2.0 ** -6
+    assert O.round_bf16(-(1 + 2.0 ** -8)) == -1.0
+    assert O.round_bf16(np.inf) == np.inf
+
+
+def test_bf16_precision_model_rounds_conv_operands():
+    """With precision='bf16' every convolution input the oracle contracts is
+    bf16-representable; with the default precision nothing is rounded."""
+    import workloads as W
+    d = W.tiny_resnet(batch=2)
+    d["in_h"] = d["in_w"] = 8
+    seen = []
+    orig = O.conv2d
+
+    def spy(x, w, stride, pad):
+        seen.append(np.array_equal(O.round_bf16(x), x) and np.array_equal(O.round_bf16(w), w))
+        return orig(x, w, stride, pad)
+
+    O.conv2d = spy
+    try:
+        net = O.ParaNet(d, precision="bf16")
+        theta = W.init_params(net.spec, seed=1, bf16=True)
+        x, labels = W.make_batch(d, seed=2)
+        net.forward(theta, x, labels)
+        assert seen and all(seen)
+        seen.clear()
+        O.ParaNet(d).forward(theta, x.astype(np.float64) + 1e-3, labels)
+        assert not all(seen)
+    finally:
+        O.conv2d = orig

@@ -92,30 +92,36 @@ def parareal_vgg16(batch=128, precision="bf16", correction="residual", classes=1
     }
 
 
-def _resnet_stage(block_index):
-    return min(block_index // 111, 2)
+def _resnet_stage(block_index, per_stage=111):
+    return min(block_index // per_stage, 2)
 
 
 def parareal_resnet1001(n_seg=4, batch=128, classes=10, hw=32, precision="bf16",
-                        correction="residual", coarse_blocks=2):
+                        correction="residual", coarse_blocks=2, per_stage=111, segments=None):
     """Parareal pre-activation ResNet-1001 (Section 4.2): 333 bottleneck
     blocks in three stages (widths 64/128/256, bottleneck 16/32/64, stride 2
     at the first block of stages 2 and 3), torn into n_seg consecutive
     segments of ceil(333/n_seg) blocks (the last takes the remainder).  Each
     coarse block F^j is `coarse_blocks` pre-activation bottlenecks at the
     width of X_{j+1}; the first one is strided and projected when the shape
-    changes.  hw=64 adds a stride-2 conv to the stem."""
+    changes.  hw=64 adds a stride-2 conv to the stem.
+
+    per_stage < 111 gives the same family with fewer blocks per stage (a
+    depth-reduced variant with the same stages, strides, projections and
+    interface kinds); `segments` then overrides the tearing."""
+    nb = 3 * per_stage
     body = []
-    for b in range(333):
-        s = _resnet_stage(b)
-        first = b in (111, 222)
+    for b in range(nb):
+        s = _resnet_stage(b, per_stage)
+        first = b in (per_stage, 2 * per_stage)
         body.append(bottleneck(64 << s, 16 << s, 2 if first else 1))
-    per = -(-333 // n_seg)
-    segments = [per] * (n_seg - 1) + [333 - per * (n_seg - 1)]
-    assert segments[-1] > 0
+    if segments is None:
+        per = -(-nb // n_seg)
+        segments = [per] * (n_seg - 1) + [nb - per * (n_seg - 1)]
+    assert len(segments) == n_seg and sum(segments) == nb and min(segments) > 0
     # shape of X_j: output of the last block of segment j
-    ends = np.cumsum(segments) - 1
-    shapes = [(64 << _resnet_stage(e), 32 >> _resnet_stage(e)) for e in ends]
+    ends = [int(e) for e in np.cumsum(segments) - 1]
+    shapes = [(64 << _resnet_stage(e, per_stage), 32 >> _resnet_stage(e, per_stage)) for e in ends]
     coarse = []
     for j in range(n_seg - 1):
         (c0, h0), (c1, h1) = shapes[j], shapes[j + 1]
@@ -126,7 +132,7 @@ def parareal_resnet1001(n_seg=4, batch=128, classes=10, hw=32, precision="bf16",
     stem = [conv(16)] if hw == 32 else [conv_bn_relu(16), conv(16, stride=2)]
     assert hw in (32, 64)
     return {
-        "name": f"parareal_resnet1001_n{n_seg}", "batch": batch, "in_c": 3,
+        "name": f"parareal_resnet{9 * per_stage + 2}_n{n_seg}", "batch": batch, "in_c": 3,
         "in_h": hw, "in_w": hw, "classes": classes, "precision": precision,
         "correction": correction,
         "stem": stem, "body": body, "segments": segments, "coarse": coarse,
