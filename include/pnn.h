@@ -109,6 +109,8 @@ typedef struct {
   int32_t stream_fp32;   /* bf16 mode: keep the residual stream (block outputs,
                             correction tensors) in fp32 storage */
   int32_t conv_impl;     /* 0 = best available, 1 = force CUDA-core kernels */
+  int32_t grad_fp32;     /* bf16 mode: contract gradients (dgrad, wgrad) with fp32
+                            operands instead of bf16 ones */
   void* stream;          /* cudaStream_t; NULL = legacy default stream */
 } pnn_options;
 

@@ -145,6 +145,11 @@ cudaError_t launch_bnb_apply(const BnBwdDesc* tab, const int* tstart, int n, int
 cudaError_t launch_pool_fwd(const PoolDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
 cudaError_t launch_pool_bwd(const PoolDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
 cudaError_t launch_gemm(const GemmDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+// tcgen05 implicit-GEMM convolution (bf16 operands, fp32 accumulate in TMEM);
+// instances need C % 8 == 0; bnmax = largest N tile (multiple of 16, <= 256)
+cudaError_t launch_conv_fwd_tc(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int bnmax,
+                               int32_t* status, cudaStream_t st);
+constexpr int kTcBM = 128;
 
 // single-instance helpers
 cudaError_t launch_pack_input(const float* x_nchw, void* out, int32_t out_dt, int B, int C, int H, int W,

@@ -92,6 +92,7 @@ struct Launch {
   size_t table_off, tstart_off;
   int count, total;
   int phase;
+  int aux;  // tcgen05 conv: largest N tile of the group
   double flops, bytes;  // algorithmic work of this launch
 };
 
@@ -252,10 +253,18 @@ struct pnn_net {
     c.in = in; c.out = out; c.res = res; c.w = w; c.k = k; c.stride = stride; c.pad = k / 2;
     c.key[0] = key0; c.key[1] = slot;
     int M = B * P * Q;
-    c.variant = cout <= 16 ? 2 : (cout <= 32 ? 1 : 0);
-    ConvTile t = simt_tile(c.variant);
-    c.mtiles = cdiv(M, t.BM);
-    c.ntiles = cdiv(cout, t.BN);
+    if (act_dt == DT_BF16 && opt.conv_impl != 1 && iv.C % 8 == 0 && cout % 8 == 0) {
+      // tcgen05 path: 128-pixel tiles, all output channels (<= 256) per tile
+      c.kind = K_CONV_FWD_TC;
+      c.variant = 0;
+      c.mtiles = cdiv(M, kTcBM);
+      c.ntiles = cdiv(cout, 256);
+    } else {
+      c.variant = cout <= 16 ? 2 : (cout <= 32 ? 1 : 0);
+      ConvTile t = simt_tile(c.variant);
+      c.mtiles = cdiv(M, t.BM);
+      c.ntiles = cdiv(cout, t.BN);
+    }
     c.tiles = c.mtiles;  // stats partial rows
     int id = new_op(list, c);
     vals[out].producer = id;
@@ -407,7 +416,8 @@ struct pnn_net {
     }
     auto key = [&](POp& o, int sub) { o.key[0] = k0; o.key[1] = k1; o.key[2] = sub; };
     switch (f.kind) {
-      case K_CONV_FWD: {
+      case K_CONV_FWD:
+      case K_CONV_FWD_TC: {
         const Value& ov = vals[f.out];
         if (f.res >= 0 && vals[f.res].need_grad) vals[f.res].pending.push_back(f.out);
         POp wg;
@@ -699,7 +709,19 @@ int pnn_net::plan(const pnn_desc* d) {
     if (order.size() != params.size()) return fail(PNN_EINVAL, "internal: parameter order");
     size_t o = 0;
     for (int id : order) { params[id].off = o; o += params[id].n; }
-    // keep ids stable but sort the info table by offset for pnn_param_tensor_info
+  }
+  // the tcgen05 conv reads weight rows with 16-byte loads: a weight that does
+  // not start on an 8-element boundary falls back to the CUDA-core kernel
+  for (auto& c : ops) {
+    if (c.kind != K_CONV_FWD_TC || params[c.w].off % 8 == 0) continue;
+    c.kind = K_CONV_FWD;
+    const int cout = vals[c.out].C;
+    c.variant = cout <= 16 ? 2 : (cout <= 32 ? 1 : 0);
+    const ConvTile t = simt_tile(c.variant);
+    c.mtiles = cdiv(rows(c.out), t.BM);
+    c.ntiles = cdiv(cout, t.BN);
+    c.tiles = c.mtiles;
+    if (c.stats_norm >= 0) norms[c.stats_norm].tiles = c.tiles;
   }
   // backward lists (Algorithm 2): head, coarse chain, fine wave, pre wave
   backward_list(head_f, head_b);
@@ -857,6 +879,7 @@ int pnn_net::build_tables() {
         const POp& o = ops[id];
         switch (o.kind) {
           case K_CONV_FWD:
+          case K_CONV_FWD_TC:
           case K_DGRAD:
           case K_WGRAD: {
             ConvDesc c{};
@@ -867,8 +890,8 @@ int pnn_net::build_tables() {
             c.B = B; c.H = iv.H; c.W = iv.W; c.C = iv.C; c.P = ov.H; c.Q = ov.W; c.K = ov.C;
             c.R = o.k; c.S = o.k; c.stride = o.stride; c.pad = o.pad;
             c.mtiles = o.mtiles; c.ntiles = o.ntiles;
-            c.op_bf16 = act_dt == DT_BF16;
-            if (o.kind == K_CONV_FWD) {
+            c.op_bf16 = act_dt == DT_BF16 && ((o.kind != K_DGRAD && o.kind != K_WGRAD) || !opt.grad_fp32);
+            if (o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC) {
               c.y = ws + ov.off; c.y_dt = ov.dt;
               if (o.res >= 0) { c.res = ws + vals[o.res].off; c.res_dt = vals[o.res].dt; }
               if (o.stats_norm >= 0) c.stats = P<float>(norms[o.stats_norm].part);
@@ -989,19 +1012,24 @@ int pnn_net::build_tables() {
       }
       Launch L;
       L.kind = g.kind; L.variant = g.variant; L.count = (int)g.ops.size(); L.total = total; L.phase = p;
-      L.flops = 0; L.bytes = 0;
+      L.flops = 0; L.bytes = 0; L.aux = 16;
+      for (int id : g.ops)
+        if (ops[id].kind == K_CONV_FWD_TC) {
+          const int K = vals[ops[id].out].C;
+          L.aux = std::max(L.aux, ops[id].ntiles == 1 ? ((K + 15) & ~15) : 256);
+        }
       for (int id : g.ops) {
         const POp& o = ops[id];
         auto esz = [&](int v) { return vals[v].virt ? (vals[vals[v].src].dt == DT_F32 ? 4.0 : 2.0) : (vals[v].dt == DT_F32 ? 4.0 : 2.0); };
         auto elems = [&](int v) { return (double)B * vals[v].H * vals[v].W * vals[v].C; };
         const double wsz = act_dt == DT_BF16 ? 2.0 : 4.0;
         switch (o.kind) {
-          case K_CONV_FWD: case K_DGRAD: case K_WGRAD: {
+          case K_CONV_FWD: case K_CONV_FWD_TC: case K_DGRAD: case K_WGRAD: {
             const Value& iv = vals[o.in]; const Value& ov = vals[o.out];
             const double macs = (double)B * ov.H * ov.W * ov.C * iv.C * o.k * o.k;
             L.flops += 2 * macs;
             const double wbytes = (double)ov.C * iv.C * o.k * o.k * wsz;
-            if (o.kind == K_CONV_FWD)
+            if (o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC)
               L.bytes += elems(o.in) * esz(o.in) + wbytes + elems(o.out) * esz(o.out) + (o.res >= 0 ? elems(o.res) * esz(o.res) : 0);
             else if (o.kind == K_DGRAD)
               L.bytes += elems(o.out) * 4 + wbytes + elems(o.in) * 4 * (o.acc ? 2 : 1);
@@ -1135,6 +1163,9 @@ int pnn_net::run_phase(int p) {
     }
     switch (L.kind) {
       case K_CONV_FWD: e = launch_conv_fwd_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, stream); break;
+      case K_CONV_FWD_TC:
+        e = launch_conv_fwd_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
+        break;
       case K_DGRAD: e = launch_conv_dgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, stream); break;
       case K_WGRAD: e = launch_conv_wgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, stream); break;
       case K_WREDUCE: e = launch_wreduce((const WReduceDesc*)tab, ts, L.count, L.total, stream); break;

@@ -49,6 +49,7 @@ class Options(C.Structure):
     _fields_ = [("precision", C.c_int32), ("correction", C.c_int32), ("seed", C.c_uint64),
                 ("lr", C.c_float), ("momentum", C.c_float), ("weight_decay", C.c_float),
                 ("nesterov", C.c_int32), ("stream_fp32", C.c_int32), ("conv_impl", C.c_int32),
+                ("grad_fp32", C.c_int32),
                 ("stream", C.c_void_p)]
 
 
@@ -119,7 +120,7 @@ class ParaNet:
     uint8 tensor on `device`."""
 
     def __init__(self, desc, precision=None, correction=None, seed=0, lr=0.1, momentum=0.9,
-                 weight_decay=5e-4, nesterov=True, stream_fp32=True, conv_impl=0, stream=None,
+                 weight_decay=5e-4, nesterov=True, stream_fp32=True, conv_impl=0, grad_fp32=False, stream=None,
                  device="cuda", bind=True):
         self.lib = load()
         self.desc = desc
@@ -148,6 +149,7 @@ class ParaNet:
         o.correction = CORRECTION[correction or desc.get("correction", "residual")]
         o.seed, o.lr, o.momentum, o.weight_decay = seed, lr, momentum, weight_decay
         o.nesterov, o.stream_fp32, o.conv_impl = int(nesterov), int(stream_fp32), int(conv_impl)
+        o.grad_fp32 = int(grad_fp32)
         self.stream = stream
         o.stream = None if stream is None else C.c_void_p(stream.cuda_stream)
         self.h = C.c_void_p()
@@ -183,7 +185,19 @@ class ParaNet:
             pass
 
     # ------------------------------------------------------------ step
+    def _args(self, x, labels, loss):
+        import torch
+        d = self.desc
+        if x.dtype != torch.float32 or not x.is_cuda or not x.is_contiguous() \
+                or tuple(x.shape) != (d["batch"], d["in_c"], d["in_h"], d["in_w"]):
+            raise TypeError("x must be a contiguous float32 CUDA tensor of shape (batch, C, H, W)")
+        if labels.dtype != torch.int32 or not labels.is_cuda or labels.numel() != d["batch"]:
+            raise TypeError("labels must be an int32 CUDA tensor of length batch")
+        if loss is not None and (loss.dtype != torch.float32 or not loss.is_cuda):
+            raise TypeError("loss must be a float32 CUDA tensor")
+
     def forward(self, x, labels, loss=None):
+        self._args(x, labels, loss)
         self._check(self.lib.pnn_forward(self.h, C.c_void_p(x.data_ptr()), C.c_void_p(labels.data_ptr()),
                                          None if loss is None else C.c_void_p(loss.data_ptr())))
 
@@ -194,6 +208,7 @@ class ParaNet:
         self._check(self.lib.pnn_sgd_step(self.h, lr))
 
     def train_step(self, x, labels, loss=None):
+        self._args(x, labels, loss)
         self._check(self.lib.pnn_train_step(self.h, C.c_void_p(x.data_ptr()), C.c_void_p(labels.data_ptr()),
                                             None if loss is None else C.c_void_p(loss.data_ptr())))
 

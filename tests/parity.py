@@ -41,7 +41,7 @@ def run_gpu(desc, theta, x, labels, **kw):
     net.set_params(theta)
     xd = torch.from_numpy(x).cuda()
     ld = torch.from_numpy(labels).cuda()
-    loss = torch.zeros(1, device="cuda")
+    loss = torch.zeros(1, dtype=torch.float32, device="cuda")
     net.forward(xd, ld, loss)
     net.backward()
     net.sync()
@@ -60,6 +60,7 @@ def run_gpu(desc, theta, x, labels, **kw):
     out["theta_new"] = net.get_params()
     out["momentum"] = net.get_momentum()
     out["net"] = net
+    out["onet"] = O.ParaNet(desc)
     return out
 
 
@@ -105,7 +106,9 @@ def compare(desc, g, o, tol=None):
     report["loss"] = le
     if not le <= tol["fwd"]:
         fails.append(("loss", le))
-    onet = o["onet"]
+    onet = o.get("onet") or g.get("onet")
+    if onet is None:  # two GPU runs: no parameter table at hand
+        return report, fails
     off = 0
     worst = 0.0
     for i, (kind, shape) in enumerate(onet.spec):

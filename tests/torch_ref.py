@@ -8,7 +8,7 @@ import math
 import torch
 import torch.nn.functional as F
 
-torch.set_default_dtype(torch.float64)
+F64 = torch.float64
 
 
 class _Params:
@@ -103,7 +103,7 @@ def head(desc, y, p):
 def _shapes(desc, x):
     """Output shapes X_0..X_N found by a dry run with zero parameters."""
     with torch.no_grad():
-        p = _Params(torch.zeros(10 ** 8))
+        p = _Params(torch.zeros(10 ** 8, dtype=F64))
         h = stack(desc["stem"], x[:2], p)
         out = [tuple(h.shape[1:])]
         i = 0
