@@ -108,7 +108,8 @@ typedef struct {
   int32_t nesterov;
   int32_t stream_fp32;   /* bf16 mode: keep the residual stream (block outputs,
                             correction tensors) in fp32 storage */
-  int32_t conv_impl;     /* 0 = best available, 1 = force CUDA-core kernels */
+  int32_t conv_impl;     /* 0 = tensor cores wherever the shape allows, 1 = CUDA-core
+                            kernels only, 2 = CUDA-core forward + tensor-core gradients */
   int32_t grad_fp32;     /* bf16 mode: contract gradients (dgrad, wgrad) with fp32
                             operands instead of bf16 ones */
   void* stream;          /* cudaStream_t; NULL = legacy default stream */
@@ -211,6 +212,11 @@ int pnn_profile(pnn_net* net, int32_t enable);
 int pnn_profile_read(pnn_net* net, int32_t kind, double* ms, int64_t* launches, double* flops, double* bytes);
 int32_t pnn_num_kernel_kinds(void);
 const char* pnn_kernel_kind_name(int32_t kind); /* NULL for a bad kind */
+
+/* Debug builds (compiled with PNN_DEBUG_CHECKS): the first misaligned vector
+ * access a tensor-core kernel detected and skipped, as (source line << 40 |
+ * address low 40 bits); 0 if none or in release builds. */
+uint64_t pnn_debug_word(void);
 
 const char* pnn_last_error(const pnn_net* net);
 const char* pnn_status_string(int status);

@@ -19,7 +19,7 @@ CUDA = os.environ.get("CUDA_HOME", "/usr/local/cuda")
 NVCC = os.path.join(CUDA, "bin", "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
-CU_SOURCES = ["k_simt.cu", "k_tc.cu"]
+CU_SOURCES = ["k_simt.cu", "k_tc_conv.cu"]
 CPP_SOURCES = ["pnn_runtime.cpp"]
 
 
@@ -50,12 +50,14 @@ def _run(cmd, verbose):
     return r.stdout + r.stderr
 
 
-def build(force=False, verbose=False, ptxas_verbose=False):
-    """Compile every CUDA/C++ source of the library and link libpnn.so."""
-    if not force and up_to_date():
+def build(force=False, verbose=False, ptxas_verbose=False, defines=()):
+    """Compile every CUDA/C++ source of the library and link libpnn.so.
+    defines: extra preprocessor symbols (e.g. PNN_DEBUG_CHECKS for the
+    self-checking debug build)."""
+    if not force and not defines and up_to_date():
         return LIB
     os.makedirs(BUILD, exist_ok=True)
-    inc = ["-I", os.path.join(ROOT, "include"), "-I", CSRC]
+    inc = ["-I", os.path.join(ROOT, "include"), "-I", CSRC] + [f"-D{d}" for d in defines]
     jobs = []
     objs = []
     for src in _sources():

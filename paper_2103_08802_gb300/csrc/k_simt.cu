@@ -287,9 +287,24 @@ __global__ void k_wreduce(const WReduceDesc* __restrict__ tab, const int* __rest
   const WReduceDesc& d = tab[inst];
   const int64_t i = (int64_t)(blockIdx.x - tstart[inst]) * blockDim.x + threadIdx.x;
   if (i >= d.n) return;
+  // i indexes dw[k_out][j]; transposed partials are stored [s][j][k_out]
+  const int64_t src = d.transposed ? (int64_t)(i % d.rsc) * d.kout + i / d.rsc : i;
   float s = 0.f;
-  for (int k = 0; k < d.splits; ++k) s += d.part[(int64_t)k * d.n + i];
+  for (int k = 0; k < d.splits; ++k) s += d.part[(int64_t)k * d.n + src];
   d.dw[i] = d.accumulate ? d.dw[i] + s : s;
+}
+
+__global__ void k_wtrans(const WtDesc* __restrict__ tab, const int* __restrict__ tstart, int n) {
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const WtDesc& d = tab[inst];
+  const int64_t i = (int64_t)(blockIdx.x - tstart[inst]) * blockDim.x + threadIdx.x;
+  if (i >= d.n) return;
+  const int k = (int)(i % d.K);
+  const int64_t t = i / d.K;
+  const int rs = (int)(t % d.RS);
+  const int c = (int)(t / d.RS);
+  reinterpret_cast<__nv_bfloat16*>(d.dst)[i] =
+      reinterpret_cast<const __nv_bfloat16*>(d.src)[((int64_t)k * d.RS + rs) * d.C + c];
 }
 
 // ---------------------------------------------------------------- row-tile geometry
@@ -730,6 +745,11 @@ cudaError_t launch_conv_wgrad_simt(const ConvDesc* tab, const int* tstart, int n
 cudaError_t launch_wreduce(const WReduceDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
   if (total <= 0) return cudaSuccess;
   k_wreduce<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_wtrans(const WtDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_wtrans<<<total, 256, 0, st>>>(tab, tstart, n);
   return cudaGetLastError();
 }
 cudaError_t launch_ew(const EwDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {

@@ -107,6 +107,8 @@ struct PoolDesc {
 };
 
 // wgrad split reduction: dw[K*RSC] = sum_s part[s][K*RSC]
+// wgrad split reduction: dw[K*RSC] = sum_s part[s][...]; partials are laid out
+// [s][K][RSC] (CUDA-core wgrad) or [s][RSC][K] (tensor-core wgrad, transposed = 1)
 struct WReduceDesc {
   const float* part;
   float* dw;
@@ -114,6 +116,15 @@ struct WReduceDesc {
   int32_t accumulate;
   int64_t n;
   int32_t tiles;
+  int32_t transposed, kout, rsc;
+};
+
+// bf16 weight transpose for the tensor-core data gradient: dst[c][r][s][k] = src[k][r][s][c]
+struct WtDesc {
+  const void* src;
+  void* dst;
+  int32_t K, RS, C;
+  int64_t n;
 };
 
 // generic strided fp32 GEMM: C[m][n] = beta*C + sum_k A[m*sam + k*sak] * B[k*sbk + n*sbn] (+ bias[n]) (relu)
@@ -149,6 +160,13 @@ cudaError_t launch_gemm(const GemmDesc* tab, const int* tstart, int n, int total
 // instances need C % 8 == 0; bnmax = largest N tile (multiple of 16, <= 256)
 cudaError_t launch_conv_fwd_tc(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int bnmax,
                                int32_t* status, cudaStream_t st);
+cudaError_t launch_conv_dgrad_tc(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int bnmax,
+                                 int32_t* status, cudaStream_t st);
+cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int bnmax,
+                                 int32_t* status, cudaStream_t st);
+// debug builds: first misaligned vector access of the tensor-core kernels (0 = none)
+unsigned long long conv_tc_debug_word();
+cudaError_t launch_wtrans(const WtDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
 constexpr int kTcBM = 128;
 
 // single-instance helpers

@@ -139,7 +139,10 @@ struct pnn_net {
   size_t labels_stage = 0, x_stage = 0, export_off = 0;
   size_t export_bytes = 0;
   // memory
-  size_t off_master = 0, off_grad = 0, off_mom = 0, off_shadow = 0;
+  size_t off_master = 0, off_grad = 0, off_mom = 0, off_shadow = 0, off_wt = 0;
+  // weight transpose launch (bf16 mode): Wt[c][r][s][k] for the tensor-core data gradient
+  size_t wt_tab = 0, wt_ts = 0;
+  int wt_count = 0, wt_total = 0;
   size_t ws_bytes = 0, cursor = 0;
   size_t tables_off = 0, tables_bytes = 0;
   char* ws = nullptr;
@@ -245,7 +248,7 @@ struct pnn_net {
   }
   int conv(std::vector<int>& list, int in, int w, int cout, int k, int stride, int res, int out_dt, int key0,
            int slot) {
-    const Value& iv = vals[in];
+    const Value iv = vals[in];  // a copy: new_value() below may reallocate vals
     int P = (iv.H + 2 * (k / 2) - k) / stride + 1, Q = (iv.W + 2 * (k / 2) - k) / stride + 1;
     int out = new_value(cout, P, Q, out_dt, true);
     POp c;
@@ -253,7 +256,7 @@ struct pnn_net {
     c.in = in; c.out = out; c.res = res; c.w = w; c.k = k; c.stride = stride; c.pad = k / 2;
     c.key[0] = key0; c.key[1] = slot;
     int M = B * P * Q;
-    if (act_dt == DT_BF16 && opt.conv_impl != 1 && iv.C % 8 == 0 && cout % 8 == 0) {
+    if (act_dt == DT_BF16 && opt.conv_impl == 0 && iv.C % 8 == 0 && cout % 8 == 0) {
       // tcgen05 path: 128-pixel tiles, all output channels (<= 256) per tile
       c.kind = K_CONV_FWD_TC;
       c.variant = 0;
@@ -272,7 +275,7 @@ struct pnn_net {
   }
   int ew(std::vector<int>& list, std::vector<int> ins, std::vector<float> coef, bool relu, int out_dt, int key0,
          int slot) {
-    const Value& a = vals[ins[0]];
+    const Value a = vals[ins[0]];  // a copy: new_value() below may reallocate vals
     bool ng = false;
     for (int i : ins) ng = ng || vals[i].need_grad;
     int out = new_value(a.C, a.H, a.W, out_dt, ng);
@@ -288,7 +291,7 @@ struct pnn_net {
     return out;
   }
   int pool(std::vector<int>& list, int in, int k, int s, int p, int key0, int slot) {
-    const Value& iv = vals[in];
+    const Value iv = vals[in];  // a copy: new_value() below may reallocate vals
     int P = (iv.H + 2 * p - k) / s + 1, Q = (iv.W + 2 * p - k) / s + 1;
     int out = new_value(iv.C, P, Q, iv.virt ? act_dt : iv.dt, iv.need_grad);
     POp o;
@@ -424,18 +427,28 @@ struct pnn_net {
         wg.kind = K_WGRAD; wg.in = f.in; wg.out = f.out; wg.w = f.w; wg.k = f.k; wg.stride = f.stride; wg.pad = f.pad;
         const int RSC = f.k * f.k * vals[f.in].C;
         const int64_t Mp = (int64_t)B * ov.H * ov.W;
-        wg.mtiles = cdiv(ov.C, kWgradBM);
-        wg.ntiles = cdiv(RSC, kWgradBN);
+        const bool tc_ok = act_dt == DT_BF16 && opt.conv_impl != 1 && vals[f.in].C % 8 == 0 && ov.C % 8 == 0;
+        int pix_align = kWgradBK;
+        if (tc_ok) {
+          // tensor cores: rows (r,s,c) in 128-row tiles, all k_out per tile, pixels split across CTAs
+          wg.kind = K_WGRAD_TC;
+          wg.mtiles = cdiv(RSC, kTcBM);
+          wg.ntiles = cdiv(ov.C, 256);
+          pix_align = 64;
+        } else {
+          wg.mtiles = cdiv(ov.C, kWgradBM);
+          wg.ntiles = cdiv(RSC, kWgradBN);
+        }
         int base = wg.mtiles * wg.ntiles;
         int splits = std::max(1, std::min(cdiv(Mp, 256), cdiv(2 * 152, base)));
-        wg.pix_per_split = cdiv(cdiv(Mp, splits), kWgradBK) * kWgradBK;
+        wg.pix_per_split = cdiv(cdiv(Mp, splits), pix_align) * pix_align;
         wg.splits = cdiv(Mp, wg.pix_per_split);
         wg.tiles = base * wg.splits;
         key(wg, 0);
         new_op(L, wg);
         POp rd;
         rd.kind = K_WREDUCE; rd.w = f.w; rd.splits = wg.splits; rd.out = f.out; rd.in = f.in; rd.k = f.k;
-        rd.acc = params[f.w].kind == 99 ? 1 : 0;
+        rd.variant = tc_ok ? 1 : 0;  // partial layout of the matching wgrad
         rd.tiles = cdiv((int64_t)ov.C * RSC, 256);
         key(rd, 1);
         new_op(L, rd);
@@ -444,10 +457,16 @@ struct pnn_net {
           POp dg;
           dg.kind = K_DGRAD; dg.in = f.in; dg.out = f.out; dg.w = f.w; dg.k = f.k; dg.stride = f.stride; dg.pad = f.pad;
           const Value& iv = vals[f.in];
-          dg.variant = iv.C <= 16 ? 2 : (iv.C <= 32 ? 1 : 0);
-          ConvTile t = simt_tile(dg.variant);
-          dg.mtiles = cdiv((int64_t)B * iv.H * iv.W, t.BM);
-          dg.ntiles = cdiv(iv.C, t.BN);
+          if (act_dt == DT_BF16 && opt.conv_impl != 1 && iv.C % 8 == 0 && ov.C % 8 == 0 && params[f.w].off % 8 == 0) {
+            dg.kind = K_DGRAD_TC;
+            dg.mtiles = cdiv((int64_t)B * iv.H * iv.W, kTcBM);
+            dg.ntiles = cdiv(iv.C, 256);
+          } else {
+            dg.variant = iv.C <= 16 ? 2 : (iv.C <= 32 ? 1 : 0);
+            ConvTile t = simt_tile(dg.variant);
+            dg.mtiles = cdiv((int64_t)B * iv.H * iv.W, t.BM);
+            dg.ntiles = cdiv(iv.C, t.BN);
+          }
           dg.tiles = dg.mtiles * dg.ntiles;
           dg.acc = grad_acc(f.in);
           key(dg, 2);
@@ -556,6 +575,7 @@ struct pnn_net {
   int do_forward(bool timed);
   int do_backward(bool timed);
   int do_sgd(float lr, bool timed);
+  cudaError_t refresh_wt();
   int fail(int code, const std::string& m) {
     err = m;
     return code;
@@ -759,6 +779,7 @@ int pnn_net::plan(const pnn_desc* d) {
   off_grad = alloc(nparams * 4);
   off_mom = alloc(nparams * 4);
   off_shadow = act_dt == DT_BF16 ? alloc(nparams * 2) : 0;
+  off_wt = act_dt == DT_BF16 ? alloc(nparams * 2) : 0;
   for (auto& v : vals) {
     if (!v.virt) v.off = alloc((size_t)B * v.H * v.W * v.C * (v.dt == DT_F32 ? 4 : 2));
     if (v.need_grad) v.goff = alloc((size_t)B * v.H * v.W * v.C * 4);
@@ -772,7 +793,7 @@ int pnn_net::plan(const pnn_desc* d) {
   }
   // wgrad scratch: one region per op (sized per op)
   for (auto& o : ops)
-    if (o.kind == K_WGRAD) o.scratch = alloc((size_t)o.splits * vals[o.out].C * o.k * o.k * vals[o.in].C * 4);
+    if (o.kind == K_WGRAD || o.kind == K_WGRAD_TC) o.scratch = alloc((size_t)o.splits * vals[o.out].C * o.k * o.k * vals[o.in].C * 4);
   for (size_t l = 0; l < fc_width.size(); ++l) {
     feat.push_back(alloc((size_t)B * fc_width[l] * 4));
     dfeat.push_back(alloc((size_t)B * fc_width[l] * 4));
@@ -881,7 +902,9 @@ int pnn_net::build_tables() {
           case K_CONV_FWD:
           case K_CONV_FWD_TC:
           case K_DGRAD:
-          case K_WGRAD: {
+          case K_DGRAD_TC:
+          case K_WGRAD:
+          case K_WGRAD_TC: {
             ConvDesc c{};
             const Value& iv = vals[o.in];
             const Value& ov = vals[o.out];
@@ -891,12 +914,13 @@ int pnn_net::build_tables() {
             c.R = o.k; c.S = o.k; c.stride = o.stride; c.pad = o.pad;
             c.mtiles = o.mtiles; c.ntiles = o.ntiles;
             c.op_bf16 = act_dt == DT_BF16 && ((o.kind != K_DGRAD && o.kind != K_WGRAD) || !opt.grad_fp32);
+            if (o.kind == K_DGRAD_TC) c.w = (const char*)(ws + off_wt) + params[o.w].off * 2;
             if (o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC) {
               c.y = ws + ov.off; c.y_dt = ov.dt;
               if (o.res >= 0) { c.res = ws + vals[o.res].off; c.res_dt = vals[o.res].dt; }
               if (o.stats_norm >= 0) c.stats = P<float>(norms[o.stats_norm].part);
               add(&c, sizeof c, o.mtiles * o.ntiles);
-            } else if (o.kind == K_DGRAD) {
+            } else if (o.kind == K_DGRAD || o.kind == K_DGRAD_TC) {
               c.dy = P<float>(gptr(o.out));
               c.dx = P<float>(gptr(o.in)); c.accumulate = o.acc;
               add(&c, sizeof c, o.tiles);
@@ -913,11 +937,17 @@ int pnn_net::build_tables() {
             WReduceDesc r{};
             const POp* wg = nullptr;
             for (int q = id - 1; q >= 0; --q)
-              if (ops[q].kind == K_WGRAD && ops[q].w == o.w && ops[q].out == o.out) { wg = &ops[q]; break; }
+              if ((ops[q].kind == K_WGRAD || ops[q].kind == K_WGRAD_TC) && ops[q].w == o.w && ops[q].out == o.out) {
+                wg = &ops[q];
+                break;
+              }
             r.part = P<float>(wg->scratch);
             r.dw = grad + params[o.w].off;
             r.splits = o.splits;
             r.accumulate = o.acc;
+            r.transposed = wg->kind == K_WGRAD_TC;
+            r.kout = vals[o.out].C;
+            r.rsc = o.k * o.k * vals[o.in].C;
             r.n = (int64_t)params[o.w].n;
             r.tiles = o.tiles;
             add(&r, sizeof r, o.tiles);
@@ -1014,8 +1044,8 @@ int pnn_net::build_tables() {
       L.kind = g.kind; L.variant = g.variant; L.count = (int)g.ops.size(); L.total = total; L.phase = p;
       L.flops = 0; L.bytes = 0; L.aux = 16;
       for (int id : g.ops)
-        if (ops[id].kind == K_CONV_FWD_TC) {
-          const int K = vals[ops[id].out].C;
+        if (ops[id].kind == K_CONV_FWD_TC || ops[id].kind == K_DGRAD_TC || ops[id].kind == K_WGRAD_TC) {
+          const int K = ops[id].kind == K_DGRAD_TC ? vals[ops[id].in].C : vals[ops[id].out].C;
           L.aux = std::max(L.aux, ops[id].ntiles == 1 ? ((K + 15) & ~15) : 256);
         }
       for (int id : g.ops) {
@@ -1024,14 +1054,14 @@ int pnn_net::build_tables() {
         auto elems = [&](int v) { return (double)B * vals[v].H * vals[v].W * vals[v].C; };
         const double wsz = act_dt == DT_BF16 ? 2.0 : 4.0;
         switch (o.kind) {
-          case K_CONV_FWD: case K_CONV_FWD_TC: case K_DGRAD: case K_WGRAD: {
+          case K_CONV_FWD: case K_CONV_FWD_TC: case K_DGRAD: case K_DGRAD_TC: case K_WGRAD: case K_WGRAD_TC: {
             const Value& iv = vals[o.in]; const Value& ov = vals[o.out];
             const double macs = (double)B * ov.H * ov.W * ov.C * iv.C * o.k * o.k;
             L.flops += 2 * macs;
             const double wbytes = (double)ov.C * iv.C * o.k * o.k * wsz;
             if (o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC)
               L.bytes += elems(o.in) * esz(o.in) + wbytes + elems(o.out) * esz(o.out) + (o.res >= 0 ? elems(o.res) * esz(o.res) : 0);
-            else if (o.kind == K_DGRAD)
+            else if (o.kind == K_DGRAD || o.kind == K_DGRAD_TC)
               L.bytes += elems(o.out) * 4 + wbytes + elems(o.in) * 4 * (o.acc ? 2 : 1);
             else
               L.bytes += elems(o.in) * esz(o.in) + elems(o.out) * 4 + (double)o.splits * ov.C * iv.C * o.k * o.k * 4;
@@ -1061,10 +1091,31 @@ int pnn_net::build_tables() {
     }
   }
   build_head_tables();
+  {
+    std::vector<WtDesc> wt;
+    std::vector<int> ts;
+    wt_total = 0;
+    if (act_dt == DT_BF16)
+      for (const ParamT& p : params) {
+        if (p.kind != 0) continue;
+        WtDesc w{};
+        w.src = ws + off_shadow + p.off * 2;
+        w.dst = ws + off_wt + p.off * 2;
+        w.K = p.dims[0]; w.C = p.dims[1]; w.RS = p.dims[2] * p.dims[3];
+        w.n = (int64_t)p.n;
+        wt.push_back(w);
+        ts.push_back(wt_total);
+        wt_total += cdiv(w.n, 256);
+      }
+    ts.push_back(wt_total);
+    wt_count = (int)wt.size();
+    wt_tab = put_table(wt.data(), wt.size() * sizeof(WtDesc));
+    wt_ts = put_table(ts.data(), ts.size() * sizeof(int));
+  }
   counts[0] = counts[1] = 0;
   for (int p = 0; p < 4; ++p) counts[0] += (int)ph[p].launches.size();
   for (int p = 4; p < 9; ++p) counts[1] += (int)ph[p].launches.size();
-  counts[2] = 1;
+  counts[2] = act_dt == DT_BF16 && wt_count ? 2 : 1;
   return PNN_OK;
 }
 
@@ -1166,6 +1217,12 @@ int pnn_net::run_phase(int p) {
       case K_CONV_FWD_TC:
         e = launch_conv_fwd_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
         break;
+      case K_DGRAD_TC:
+        e = launch_conv_dgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
+        break;
+      case K_WGRAD_TC:
+        e = launch_conv_wgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
+        break;
       case K_DGRAD: e = launch_conv_dgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, stream); break;
       case K_WGRAD: e = launch_conv_wgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, stream); break;
       case K_WREDUCE: e = launch_wreduce((const WReduceDesc*)tab, ts, L.count, L.total, stream); break;
@@ -1213,12 +1270,20 @@ int pnn_net::do_backward(bool timed) {
   return PNN_OK;
 }
 
+cudaError_t pnn_net::refresh_wt() {
+  if (act_dt != DT_BF16 || wt_count == 0) return cudaSuccess;
+  const char* tb = ws + tables_off;
+  return launch_wtrans(reinterpret_cast<const WtDesc*>(tb + wt_tab), reinterpret_cast<const int*>(tb + wt_ts), wt_count,
+                       wt_total, stream);
+}
+
 int pnn_net::do_sgd(float lr, bool timed) {
   if (timed) cudaEventRecord(ev[10], stream);
   if (lr <= 0.f) lr = opt.lr;
   cudaError_t e = launch_sgd(P<float>(off_master), P<float>(off_grad), P<float>(off_mom),
                              act_dt == DT_BF16 ? (void*)(ws + off_shadow) : nullptr, DT_BF16, (int64_t)nparams, lr,
                              opt.momentum, opt.weight_decay, opt.nesterov, first_step ? 1 : 0, stream);
+  if (e == cudaSuccess) e = refresh_wt();
   if (timed) cudaEventRecord(ev[11], stream);
   first_step = false;
   return cuda_check(e, "sgd");
@@ -1297,6 +1362,7 @@ int pnn_net::bind(void* dev, size_t bytes) {
   if (e == cudaSuccess) e = cudaMemset(ws + status_off, 0, 64);
   if (e == cudaSuccess && act_dt == DT_BF16)
     e = launch_copy_cast(P<float>(off_master), ws + off_shadow, DT_BF16, (int64_t)nparams, stream);
+  if (e == cudaSuccess) e = refresh_wt();
   if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return cuda_check(e, "initialise parameters");
   for (auto& v : ev)
@@ -1551,6 +1617,7 @@ int pnn_set_params(pnn_net* n, const float* host, size_t count) {
   if (e == cudaSuccess) e = cudaMemcpy(n->ws + n->off_master, tmp.data(), n->nparams * 4, cudaMemcpyHostToDevice);
   if (e == cudaSuccess && n->act_dt == DT_BF16)
     e = launch_copy_cast(n->P<float>(n->off_master), n->ws + n->off_shadow, DT_BF16, (int64_t)n->nparams, n->stream);
+  if (e == cudaSuccess) e = n->refresh_wt();
   if (e == cudaSuccess) e = cudaStreamSynchronize(n->stream);
   return n->cuda_check(e, "set parameters");
 }
@@ -1638,7 +1705,7 @@ int pnn_launch_counts(const pnn_net* n, int32_t counts[3]) {
   extra_head = 2 + nfc;  // gap, gemms, softmax
   counts[0] = n->counts[0] - 1 + extra_head + 1;  // + pack input
   counts[1] = n->counts[1] - 1 + 3 * nfc + (nfc - 1) + 1;
-  counts[2] = 1;
+  counts[2] = n->counts[2];
   return PNN_OK;
 }
 
@@ -1684,6 +1751,8 @@ const char* pnn_kernel_kind_name(int32_t kind) {
 }
 
 int32_t pnn_num_kernel_kinds(void) { return K_NKINDS; }
+
+uint64_t pnn_debug_word(void) { return conv_tc_debug_word(); }
 
 const char* pnn_last_error(const pnn_net* n) { return n ? n->err.c_str() : g_err.c_str(); }
 

@@ -93,6 +93,7 @@ def load():
         "pnn_profile_read": (C.c_int, [P, I32, C.POINTER(C.c_double), C.POINTER(C.c_int64),
                                        C.POINTER(C.c_double), C.POINTER(C.c_double)]),
         "pnn_num_kernel_kinds": (I32, []),
+        "pnn_debug_word": (C.c_uint64, []),
         "pnn_kernel_kind_name": (C.c_char_p, [I32]),
         "pnn_last_error": (C.c_char_p, [P]),
         "pnn_status_string": (C.c_char_p, [C.c_int]),
