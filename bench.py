@@ -46,6 +46,8 @@ def parse():
     ap.add_argument("--config", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-batch", type=int, default=1)
+    ap.add_argument("--batch", type=int, default=None,
+                    help="override the workload's batch (profiling a small case of the same network)")
     return ap.parse_args()
 
 
@@ -289,7 +291,7 @@ def our_arm(args, desc, rank, local, world, dist):
 def main():
     args = parse()
     rank, local, world, dist = dist_setup(args.gpus)
-    desc = W.config(args.config)
+    desc = W.config(args.config, batch=args.batch)
     if args.impl == "reference":
         reference_arm(args, desc, rank)
     else:

@@ -282,16 +282,25 @@ __global__ void __launch_bounds__(256) k_conv_wgrad(const ConvDesc* __restrict__
   }
 }
 
-__global__ void k_wreduce(const WReduceDesc* __restrict__ tab, const int* __restrict__ tstart, int n) {
+// 32 elements per CTA, 8 lanes per element: lane l sums splits l, l+8, ...
+// in order, then a fixed xor-shuffle tree combines the 8 lanes.
+__global__ void __launch_bounds__(256) k_wreduce(const WReduceDesc* __restrict__ tab, const int* __restrict__ tstart,
+                                                 int n) {
   const int inst = find_instance(tstart, n, blockIdx.x);
   const WReduceDesc& d = tab[inst];
-  const int64_t i = (int64_t)(blockIdx.x - tstart[inst]) * blockDim.x + threadIdx.x;
-  if (i >= d.n) return;
-  // i indexes dw[k_out][j]; transposed partials are stored [s][j][k_out]
-  const int64_t src = d.transposed ? (int64_t)(i % d.rsc) * d.kout + i / d.rsc : i;
+  const int64_t i = (int64_t)(blockIdx.x - tstart[inst]) * 32 + threadIdx.x / 8;
+  const int l = threadIdx.x % 8;
   float s = 0.f;
-  for (int k = 0; k < d.splits; ++k) s += d.part[(int64_t)k * d.n + src];
-  d.dw[i] = d.accumulate ? d.dw[i] + s : s;
+  int64_t src = 0;
+  if (i < d.n) {
+    // i indexes dw[k_out][j]; transposed partials are stored [s][j][k_out]
+    src = d.transposed ? (int64_t)(i % d.rsc) * d.kout + i / d.rsc : i;
+    for (int k = l; k < d.splits; k += 8) s += d.part[(int64_t)k * d.n + src];
+  }
+  s += __shfl_xor_sync(0xffffffffu, s, 4);
+  s += __shfl_xor_sync(0xffffffffu, s, 2);
+  s += __shfl_xor_sync(0xffffffffu, s, 1);
+  if (i < d.n && l == 0) d.dw[i] = d.accumulate ? d.dw[i] + s : s;
 }
 
 __global__ void k_wtrans(const WtDesc* __restrict__ tab, const int* __restrict__ tstart, int n) {
@@ -387,23 +396,36 @@ __global__ void __launch_bounds__(256) k_ew_bwd(const EwBwdDesc* __restrict__ ta
 }
 
 // ---------------------------------------------------------------- BN
+// one CTA per channel: thread t sums tiles t, t+256, ... in double, then a
+// fixed shared-memory tree combines the 256 partial sums
+__device__ __forceinline__ void block_sum2(double& a, double& b) {
+  __shared__ double ra[256], rb[256];
+  ra[threadIdx.x] = a;
+  rb[threadIdx.x] = b;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if ((int)threadIdx.x < w) {
+      ra[threadIdx.x] += ra[threadIdx.x + w];
+      rb[threadIdx.x] += rb[threadIdx.x + w];
+    }
+    __syncthreads();
+  }
+  a = ra[0];
+  b = rb[0];
+}
+
 __global__ void __launch_bounds__(256) k_bn_fin(const BnFinDesc* __restrict__ tab, const int* __restrict__ tstart,
                                                 int n) {
   const int inst = find_instance(tstart, n, blockIdx.x);
   const BnFinDesc& d = tab[inst];
-  const int c = (blockIdx.x - tstart[inst]) * 8 + threadIdx.x / 32;
-  const int lane = threadIdx.x % 32;
-  if (c >= d.C) return;
+  const int c = blockIdx.x - tstart[inst];
   double s1 = 0.0, s2 = 0.0;
-  for (int t = lane; t < d.tiles; t += 32) {
+  for (int t = threadIdx.x; t < d.tiles; t += 256) {
     s1 += (double)d.part[((int64_t)t * d.C + c) * 2];
     s2 += (double)d.part[((int64_t)t * d.C + c) * 2 + 1];
   }
-  for (int off = 16; off > 0; off >>= 1) {
-    s1 += __shfl_xor_sync(0xffffffffu, s1, off);
-    s2 += __shfl_xor_sync(0xffffffffu, s2, off);
-  }
-  if (lane == 0) {
+  block_sum2(s1, s2);
+  if (threadIdx.x == 0) {
     const double mean = s1 / (double)d.count;
     double var = s2 / (double)d.count - mean * mean;
     if (var < 0.0) var = 0.0;
@@ -464,19 +486,14 @@ __global__ void __launch_bounds__(256) k_bnb_fin(const BnBwdDesc* __restrict__ t
                                                  int n) {
   const int inst = find_instance(tstart, n, blockIdx.x);
   const BnBwdDesc& d = tab[inst];
-  const int c = (blockIdx.x - tstart[inst]) * 8 + threadIdx.x / 32;
-  const int lane = threadIdx.x % 32;
-  if (c >= d.C) return;
+  const int c = blockIdx.x - tstart[inst];
   double s1 = 0.0, s2 = 0.0;
-  for (int t = lane; t < d.tiles; t += 32) {
+  for (int t = threadIdx.x; t < d.tiles; t += 256) {
     s1 += (double)d.part[((int64_t)t * d.C + c) * 2];
     s2 += (double)d.part[((int64_t)t * d.C + c) * 2 + 1];
   }
-  for (int off = 16; off > 0; off >>= 1) {
-    s1 += __shfl_xor_sync(0xffffffffu, s1, off);
-    s2 += __shfl_xor_sync(0xffffffffu, s2, off);
-  }
-  if (lane == 0) {
+  block_sum2(s1, s2);
+  if (threadIdx.x == 0) {
     d.dbeta[c] = d.accumulate ? d.dbeta[c] + (float)s1 : (float)s1;
     d.dgamma[c] = d.accumulate ? d.dgamma[c] + (float)s2 : (float)s2;
     d.coef[c * 3 + 0] = d.gamma[c] * d.rstd[c];
@@ -503,6 +520,129 @@ __global__ void __launch_bounds__(256) k_bnb_apply(const BnBwdDesc* __restrict__
     if (d.add0) v += d.add0[o];
     if (d.add1) v += d.add1[o];
     d.dh[o] = d.accumulate ? d.dh[o] + v : v;
+  }
+}
+
+// ---------------------------------------------------------------- BN backward, 8 channels per thread
+// Used when C % 8 == 0: each thread moves 8 consecutive channels of one row
+// with 16/32-byte accesses.
+__device__ __forceinline__ void ld8f(const float* p, float* v) {
+  const float4 a = *reinterpret_cast<const float4*>(p), b = *reinterpret_cast<const float4*>(p + 4);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void st8f(float* p, const float* v) {
+  *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
+}
+__device__ __forceinline__ void ld8any(const void* base, int dt, int64_t i, float* v) {
+  if (dt == DT_F32) {
+    ld8f(reinterpret_cast<const float*>(base) + i, v);
+  } else {
+    const uint4 u = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(base) + i);
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 f = __bfloat1622float2(h[k]);
+      v[2 * k] = f.x;
+      v[2 * k + 1] = f.y;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) k_bnb_reduce8(const BnBwdDesc* __restrict__ tab,
+                                                     const int* __restrict__ tstart, int n) {
+  __shared__ float red[256][16];
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const BnBwdDesc& d = tab[inst];
+  const int tile = blockIdx.x - tstart[inst];
+  const int C = d.C, CG = C / 8;
+  const int G = 256 / CG;  // row groups (CG <= 256)
+  const int cg = threadIdx.x % CG, g = threadIdx.x / CG;
+  const int64_t r0 = (int64_t)tile * d.rows_per_tile;
+  const int64_t r1 = min((int64_t)d.M, r0 + d.rows_per_tile);
+  float s1[8], s2[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) { s1[k] = 0.f; s2[k] = 0.f; }
+  if (g < G) {
+    const int c0 = cg * 8;
+    float mean[8], rstd[8], sc[8], sh[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      mean[k] = d.mean[c0 + k]; rstd[k] = d.rstd[c0 + k]; sc[k] = d.scale[c0 + k]; sh[k] = d.shift[c0 + k];
+    }
+    for (int64_t r = r0 + g; r < r1; r += G) {
+      const int64_t o = r * C + c0;
+      float h[8], dz[8];
+      ld8any(d.h, d.h_dt, o, h);
+      ld8f(d.da + o, dz);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (d.relu && !(fmaf(sc[k], h[k], sh[k]) > 0.f)) dz[k] = 0.f;
+        s1[k] += dz[k];
+        s2[k] += dz[k] * ((h[k] - mean[k]) * rstd[k]);
+      }
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 8; ++k) { red[threadIdx.x][k] = s1[k]; red[threadIdx.x][8 + k] = s2[k]; }
+  __syncthreads();
+  if ((int)threadIdx.x < CG) {
+    float a[8], b[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) { a[k] = 0.f; b[k] = 0.f; }
+    for (int gg = 0; gg < G; ++gg)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) { a[k] += red[gg * CG + threadIdx.x][k]; b[k] += red[gg * CG + threadIdx.x][8 + k]; }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      d.part[((int64_t)tile * C + threadIdx.x * 8 + k) * 2] = a[k];
+      d.part[((int64_t)tile * C + threadIdx.x * 8 + k) * 2 + 1] = b[k];
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) k_bnb_apply8(const BnBwdDesc* __restrict__ tab,
+                                                    const int* __restrict__ tstart, int n) {
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const BnBwdDesc& d = tab[inst];
+  const int tile = blockIdx.x - tstart[inst];
+  const int C = d.C, CG = C / 8;
+  const int64_t r0 = (int64_t)tile * d.rows_per_tile;
+  const int64_t r1 = min((int64_t)d.M, r0 + d.rows_per_tile);
+  const int64_t groups = (r1 - r0) * CG;
+  for (int64_t e = threadIdx.x; e < groups; e += blockDim.x) {
+    const int64_t r = r0 + e / CG;
+    const int c0 = (int)(e % CG) * 8;
+    const int64_t o = r * C + c0;
+    float h[8], dz[8], out[8];
+    ld8any(d.h, d.h_dt, o, h);
+    ld8f(d.da + o, dz);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int c = c0 + k;
+      if (d.relu && !(fmaf(d.scale[c], h[k], d.shift[c]) > 0.f)) dz[k] = 0.f;
+      const float xhat = (h[k] - d.mean[c]) * d.rstd[c];
+      out[k] = d.coef[c * 3] * (dz[k] - d.coef[c * 3 + 1] - xhat * d.coef[c * 3 + 2]);
+    }
+    if (d.add0) {
+      float a[8];
+      ld8f(d.add0 + o, a);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) out[k] += a[k];
+    }
+    if (d.add1) {
+      float a[8];
+      ld8f(d.add1 + o, a);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) out[k] += a[k];
+    }
+    if (d.accumulate) {
+      float a[8];
+      ld8f(d.dh + o, a);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) out[k] += a[k];
+    }
+    st8f(d.dh + o, out);
   }
 }
 
@@ -772,6 +912,11 @@ cudaError_t launch_bnb_reduce(const BnBwdDesc* tab, const int* tstart, int n, in
   k_bnb_reduce<<<total, 256, 0, st>>>(tab, tstart, n);
   return cudaGetLastError();
 }
+cudaError_t launch_bnb_reduce8(const BnBwdDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_bnb_reduce8<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
 cudaError_t launch_bnb_fin(const BnBwdDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
   if (total <= 0) return cudaSuccess;
   k_bnb_fin<<<total, 256, 0, st>>>(tab, tstart, n);
@@ -780,6 +925,11 @@ cudaError_t launch_bnb_fin(const BnBwdDesc* tab, const int* tstart, int n, int t
 cudaError_t launch_bnb_apply(const BnBwdDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
   if (total <= 0) return cudaSuccess;
   k_bnb_apply<<<total, 256, 0, st>>>(tab, tstart, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_bnb_apply8(const BnBwdDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  k_bnb_apply8<<<total, 256, 0, st>>>(tab, tstart, n);
   return cudaGetLastError();
 }
 cudaError_t launch_pool_fwd(const PoolDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {

@@ -153,6 +153,9 @@ cudaError_t launch_bn_fin(const BnFinDesc* tab, const int* tstart, int n, int to
 cudaError_t launch_bnb_reduce(const BnBwdDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
 cudaError_t launch_bnb_fin(const BnBwdDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
 cudaError_t launch_bnb_apply(const BnBwdDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+// 8 channels per thread; every instance needs C % 8 == 0 and C <= 2048
+cudaError_t launch_bnb_reduce8(const BnBwdDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
+cudaError_t launch_bnb_apply8(const BnBwdDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
 cudaError_t launch_pool_fwd(const PoolDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
 cudaError_t launch_pool_bwd(const PoolDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
 cudaError_t launch_gemm(const GemmDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
@@ -186,6 +189,7 @@ cudaError_t launch_weight_cast(const float* in, void* out, int32_t out_dt, int64
 
 // tile geometry helpers shared by runtime and kernels
 constexpr int kEwRowsPerTile = 64;
+constexpr int kBnbRowsPerTile = 256;  // BN backward reduce/apply tiles
 struct ConvTile { int BM, BN; };
 inline ConvTile simt_tile(int variant) {
   return variant == 0 ? ConvTile{64, 64} : (variant == 1 ? ConvTile{128, 32} : ConvTile{256, 16});

@@ -449,7 +449,7 @@ struct pnn_net {
         POp rd;
         rd.kind = K_WREDUCE; rd.w = f.w; rd.splits = wg.splits; rd.out = f.out; rd.in = f.in; rd.k = f.k;
         rd.variant = tc_ok ? 1 : 0;  // partial layout of the matching wgrad
-        rd.tiles = cdiv((int64_t)ov.C * RSC, 256);
+        rd.tiles = cdiv((int64_t)ov.C * RSC, 32);  // 32 elements per CTA
         key(rd, 1);
         new_op(L, rd);
         if (vals[f.in].need_grad) {
@@ -513,17 +513,18 @@ struct pnn_net {
         if (vv < 0 || !vals[vv].grad_written) break;
         POp r;
         r.kind = K_BNB_RED; r.norm = f.norm; r.in = vv;
-        r.tiles = cdiv(n.count, kEwRowsPerTile);
+        r.variant = (n.C % 8 == 0 && n.C <= 2048) ? 1 : 0;  // 1: 8 channels per thread
+        r.tiles = cdiv(n.count, kBnbRowsPerTile);
         key(r, 0);
         new_op(L, r);
         POp fi = r;
         fi.kind = K_BNB_FIN;
-        fi.tiles = cdiv(n.C, 8);
+        fi.tiles = n.C;  // one CTA per channel
         key(fi, 1);
         new_op(L, fi);
         POp ap = r;
         ap.kind = K_BNB_APPLY;
-        ap.tiles = cdiv(n.count, kEwRowsPerTile);
+        ap.tiles = cdiv(n.count, kBnbRowsPerTile);
         if (vals[n.h].need_grad) {
           ap.acc = grad_acc(n.h);
           ap.out = n.h;
@@ -787,7 +788,7 @@ int pnn_net::plan(const pnn_desc* d) {
   for (auto& n : norms) {
     n.part = alloc((size_t)n.tiles * n.C * 8);
     n.mean = alloc(n.C * 4); n.rstd = alloc(n.C * 4); n.scale = alloc(n.C * 4); n.shift = alloc(n.C * 4);
-    n.btiles = cdiv(n.count, kEwRowsPerTile);
+    n.btiles = cdiv(n.count, kBnbRowsPerTile);
     n.bpart = alloc((size_t)n.btiles * n.C * 8);
     n.coef = alloc((size_t)n.C * 12);
   }
@@ -988,7 +989,7 @@ int pnn_net::build_tables() {
             f.part = P<float>(n.part); f.tiles = n.tiles; f.C = n.C; f.count = n.count;
             f.gamma = master + params[n.gamma].off; f.beta = master + params[n.beta].off;
             f.mean = P<float>(n.mean); f.rstd = P<float>(n.rstd); f.scale = P<float>(n.scale); f.shift = P<float>(n.shift);
-            add(&f, sizeof f, cdiv(n.C, 8));
+            add(&f, sizeof f, n.C);  // one CTA per channel
             break;
           }
           case K_BNB_RED:
@@ -1006,7 +1007,7 @@ int pnn_net::build_tables() {
             b.dgamma = grad + params[n.gamma].off; b.dbeta = grad + params[n.beta].off;
             b.coef = P<float>(n.coef);
             b.M = n.count; b.C = n.C;
-            b.rows_per_tile = kEwRowsPerTile; b.tiles = n.btiles;
+            b.rows_per_tile = kBnbRowsPerTile; b.tiles = n.btiles;
             if (o.kind == K_BNB_FIN) b.accumulate = o.acc_in[0];
             if (o.kind == K_BNB_APPLY) {
               b.dh = P<float>(gptr(n.h));
@@ -1229,9 +1230,15 @@ int pnn_net::run_phase(int p) {
       case K_EW: e = launch_ew((const EwDesc*)tab, ts, L.count, L.total, stream); break;
       case K_EW_BWD: e = launch_ew_bwd((const EwBwdDesc*)tab, ts, L.count, L.total, stream); break;
       case K_BN_FIN: e = launch_bn_fin((const BnFinDesc*)tab, ts, L.count, L.total, stream); break;
-      case K_BNB_RED: e = launch_bnb_reduce((const BnBwdDesc*)tab, ts, L.count, L.total, stream); break;
+      case K_BNB_RED:
+        e = L.variant ? launch_bnb_reduce8((const BnBwdDesc*)tab, ts, L.count, L.total, stream)
+                      : launch_bnb_reduce((const BnBwdDesc*)tab, ts, L.count, L.total, stream);
+        break;
       case K_BNB_FIN: e = launch_bnb_fin((const BnBwdDesc*)tab, ts, L.count, L.total, stream); break;
-      case K_BNB_APPLY: e = launch_bnb_apply((const BnBwdDesc*)tab, ts, L.count, L.total, stream); break;
+      case K_BNB_APPLY:
+        e = L.variant ? launch_bnb_apply8((const BnBwdDesc*)tab, ts, L.count, L.total, stream)
+                      : launch_bnb_apply((const BnBwdDesc*)tab, ts, L.count, L.total, stream);
+        break;
       case K_POOL_FWD: e = launch_pool_fwd((const PoolDesc*)tab, ts, L.count, L.total, stream); break;
       case K_POOL_BWD: e = launch_pool_bwd((const PoolDesc*)tab, ts, L.count, L.total, stream); break;
       case K_HEAD_FWD: { int r = run_head_fwd(); if (r) return r; break; }
