@@ -243,11 +243,15 @@ def our_arm(args, desc, rank, local, world, dist):
     dom = max(prof.items(), key=lambda kv: kv[1][0])
     name, (kms, kn, kfl, kby) = dom
     per_launch_ms = kms / kn
-    if name.endswith("_tc"):
-        bound, peak, unit = "tensor", pk["bf16_tflops_sustained"], "TFLOP/s"
-        achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
-    elif name.startswith("conv"):
+    # the bound follows the kernel's algorithmic intensity: below the ridge point
+    # (peak FLOP/s / peak B/s) the roof is HBM bandwidth
+    ridge = pk["bf16_tflops_sustained"] * 1e12 / (pk["hbm_gbs"] * 1e9)
+    intensity = kfl / kby if kby else float("inf")
+    if name.startswith("conv") and not name.endswith("_tc") and intensity >= FP32_ALU_TFLOPS * 1e3 / pk["hbm_gbs"]:
         bound, peak, unit = "alu", FP32_ALU_TFLOPS, "TFLOP/s"
+        achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
+    elif name.endswith("_tc") and intensity >= ridge:
+        bound, peak, unit = "tensor", pk["bf16_tflops_sustained"], "TFLOP/s"
         achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
     else:
         bound, peak, unit = "hbm", pk["hbm_gbs"], "GB/s"
@@ -273,8 +277,11 @@ def our_arm(args, desc, rank, local, world, dist):
         "conv_frac_of_bf16_peak": (conv_flops / (conv_ms / 1e3) / 1e12) / pk["bf16_tflops_sustained"] if conv_ms else None,
         "conv_share_of_device_time": conv_ms / total_prof_ms if total_prof_ms else None,
         "roofline": {"kernel": name, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                     "frac": achieved / peak, "traffic": None, "peak_source": src if bound != "alu" else
-                     "derived: 152 SM x 128 FP32 lanes x 2 x 2.07 GHz", "launches_per_step": kn / args.steps},
+                     "frac": achieved / peak, "traffic": None,
+                     "intensity_flop_per_byte": intensity,
+                     "peak_source": (src + (" (hbm_gbs)" if bound == "hbm" else " (bf16_tflops_sustained)"))
+                     if bound != "alu" else "derived: 152 SM x 128 FP32 lanes x 2 x 2.07 GHz",
+                     "launches_per_step": kn / args.steps},
         "kernels": {k: {"ms_per_step": v[0] / args.steps, "launches_per_step": v[1] / args.steps,
                         "gflop_per_step": v[2] / args.steps / 1e9, "gb_per_step": v[3] / args.steps / 1e9}
                     for k, v in sorted(prof.items(), key=lambda kv: -kv[1][0])},
