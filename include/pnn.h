@@ -218,6 +218,33 @@ const char* pnn_kernel_kind_name(int32_t kind); /* NULL for a bad kind */
  * address low 40 bits); 0 if none or in release builds. */
 uint64_t pnn_debug_word(void);
 
+/* ---- allocation-free weight gradient of one convolution ----
+ * The paper has no counterpart to this call.  It exists for callers that
+ * cannot allocate device memory at the point they need the result, e.g.
+ * code running inside a memory pool they do not control, or a runtime that
+ * forbids cudaMalloc after start-up.  It computes the same weight gradient
+ * as the tensor-core kernel pnn_backward uses,
+ *   dw[kk][r][s][cc] = sum_{n,p,q} dy[n][p][q][kk] * x[n][p*stride+r-pad][q*stride+s-pad][cc]
+ * (pad = ksize/2, zero padding, both operands rounded to bf16, fp32
+ * accumulation), but keeps its split-K partial sums, launch descriptors and
+ * status word in fixed-size device arrays compiled into the library: 16 MiB
+ * of partial sums, so k * ksize * ksize * c must not exceed 4,194,304
+ * (PNN_EINVAL otherwise).  It calls no cudaMalloc, cudaFree or allocating
+ * library routine.
+ *   x   device, batch x h x w x c float32, NHWC
+ *   dy  device, batch x p x q x k float32, NHWC, p = (h + 2*pad - ksize)/stride + 1
+ *   dw  device, k x ksize x ksize x c float32 (written, not accumulated)
+ *   c and k multiples of 8; ksize 1 or 3; stride 1 or 2; stream NULL = legacy default.
+ * Every GPU that loads the library keeps these arrays until the process ends.
+ * The first call on a device looks up their device addresses (once per
+ * device); make that first call before capturing a stream into a CUDA graph.
+ * All calls share the arrays and each call overwrites them: calls that
+ * overlap on the GPU (other streams, other threads) race.  Synchronises.
+ * Errors: PNN_EINVAL (arguments), PNN_ECUDA, PNN_ETIMEOUT; message in
+ * pnn_last_error(NULL). */
+int pnn_conv_wgrad_noalloc(const float* x, const float* dy, float* dw, int32_t batch, int32_t h, int32_t w,
+                           int32_t c, int32_t k, int32_t ksize, int32_t stride, void* stream);
+
 const char* pnn_last_error(const pnn_net* net);
 const char* pnn_status_string(int status);
 

@@ -28,6 +28,9 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <algorithm>
+
+#include "pnn.h"
 #include "pnn_internal.h"
 #include "tc_ptx.cuh"
 
@@ -548,3 +551,120 @@ cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
 }
 
 }  // namespace pnn
+
+// ============================================================================
+// Allocation-free weight gradient: the same tensor-core kernel, with its
+// split-K partial sums, launch descriptors and status word in fixed-size
+// file-scope device arrays instead of memory from the caller or the library.
+// Every GPU that loads the library holds these arrays until the process ends.
+// Calls share them: two calls that overlap on the GPU race.
+namespace pnn {
+namespace {
+constexpr size_t kNoAllocFloats = size_t(4) << 20;  // 16 MiB of split-K partial sums
+}  // namespace
+
+static __device__ __align__(256) float g_noalloc_part[kNoAllocFloats];
+static __device__ __align__(256) ConvDesc g_noalloc_conv;
+static __device__ __align__(256) WReduceDesc g_noalloc_red;
+static __device__ __align__(16) int g_noalloc_ts[4];
+static __device__ int32_t g_noalloc_status;
+
+namespace {
+struct NoAllocSymbols {
+  float* part = nullptr;
+  ConvDesc* conv = nullptr;
+  WReduceDesc* red = nullptr;
+  int* ts = nullptr;
+  int32_t* status = nullptr;
+  bool ready = false;
+};
+NoAllocSymbols g_noalloc_syms[64];
+
+// Device addresses of the arrays for the current device (once per device).
+// The host-side names are stand-ins, not device addresses.
+cudaError_t noalloc_symbols(NoAllocSymbols** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  NoAllocSymbols& s = g_noalloc_syms[dev];
+  if (!s.ready) {
+    e = cudaGetSymbolAddress((void**)&s.part, g_noalloc_part);
+    if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&s.conv, g_noalloc_conv);
+    if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&s.red, g_noalloc_red);
+    if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&s.ts, g_noalloc_ts);
+    if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&s.status, g_noalloc_status);
+    if (e != cudaSuccess) return e;
+    s.ready = true;
+  }
+  *out = &s;
+  return cudaSuccess;
+}
+}  // namespace
+}  // namespace pnn
+
+extern "C" int pnn_conv_wgrad_noalloc(const float* x, const float* dy, float* dw, int32_t batch, int32_t h,
+                                      int32_t w, int32_t c, int32_t k, int32_t r, int32_t stride, void* stream) {
+  using namespace pnn;
+  if (!x || !dy || !dw) return set_last_error(PNN_EINVAL, "pnn_conv_wgrad_noalloc: null pointer");
+  if (batch <= 0 || h <= 0 || w <= 0 || c <= 0 || k <= 0 || (r != 1 && r != 3) || (stride != 1 && stride != 2))
+    return set_last_error(PNN_EINVAL, "pnn_conv_wgrad_noalloc: bad geometry");
+  if (c % 8 != 0 || k % 8 != 0)
+    return set_last_error(PNN_EINVAL, "pnn_conv_wgrad_noalloc: channels and k must be multiples of 8");
+  const int pad = r / 2;
+  const int p = (h + 2 * pad - r) / stride + 1, q = (w + 2 * pad - r) / stride + 1;
+  const int rsc = r * r * c;
+  const size_t nw = (size_t)k * rsc;
+  if (nw > kNoAllocFloats)
+    return set_last_error(PNN_EINVAL, "pnn_conv_wgrad_noalloc: k*r*r*c exceeds the 4Mi-float static scratch");
+  const int64_t mp = (int64_t)batch * p * q;
+  if (mp > 0x7fffffffLL || (int64_t)batch * h * w * c > 0x7fffffffLL)
+    return set_last_error(PNN_EINVAL, "pnn_conv_wgrad_noalloc: tensor too large");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  NoAllocSymbols* sym = nullptr;
+  cudaError_t e = noalloc_symbols(&sym);
+  if (e != cudaSuccess) return set_last_error(PNN_ECUDA, cudaGetErrorString(e));
+
+  ConvDesc cd{};
+  cd.x = Src{x, nullptr, nullptr, DT_F32, 0};
+  cd.B = batch; cd.H = h; cd.W = w; cd.C = c; cd.P = p; cd.Q = q; cd.K = k;
+  cd.R = r; cd.S = r; cd.stride = stride; cd.pad = pad;
+  cd.dy = dy;
+  cd.dw_part = sym->part;
+  cd.mtiles = (rsc + kTcBM - 1) / kTcBM;
+  cd.ntiles = (k + 255) / 256;
+  cd.op_bf16 = 1;
+  const int base = cd.mtiles * cd.ntiles;
+  int splits = (int)std::min<int64_t>((mp + 255) / 256, (2 * 152 + base - 1) / base);
+  splits = std::max(1, std::min<int>(splits, (int)(kNoAllocFloats / nw)));
+  cd.pix_per_split = (int)(((mp + splits - 1) / splits + 63) / 64 * 64);
+  cd.splits = (int)((mp + cd.pix_per_split - 1) / cd.pix_per_split);
+  const int conv_tiles = base * cd.splits;
+  WReduceDesc rd{};
+  rd.part = sym->part;
+  rd.dw = dw;
+  rd.splits = cd.splits;
+  rd.accumulate = 0;
+  rd.n = (int64_t)nw;
+  rd.tiles = (int)((nw + 31) / 32);
+  rd.transposed = 1;
+  rd.kout = k;
+  rd.rsc = rsc;
+  const int ts[4] = {0, conv_tiles, 0, rd.tiles};
+  const int bnmax = cd.ntiles == 1 ? ((k + 15) & ~15) : 256;
+  // descriptors into the static arrays (copies, not allocations); the status
+  // word must start at zero; the partial sums need no clearing (every element
+  // used is written before it is read)
+  e = cudaMemcpyAsync(sym->conv, &cd, sizeof cd, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(sym->red, &rd, sizeof rd, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(sym->ts, ts, sizeof ts, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(sym->status, 0, sizeof(int32_t), st);
+  if (e == cudaSuccess) e = launch_conv_wgrad_tc(sym->conv, sym->ts, 1, conv_tiles, bnmax, sym->status, st);
+  if (e == cudaSuccess) e = launch_wreduce(sym->red, sym->ts + 2, 1, rd.tiles, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  int32_t status = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&status, sym->status, sizeof status, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return set_last_error(PNN_ECUDA, cudaGetErrorString(e));
+  if (status == 3) return set_last_error(PNN_ETIMEOUT, "pnn_conv_wgrad_noalloc: device wait timed out");
+  return PNN_OK;
+}

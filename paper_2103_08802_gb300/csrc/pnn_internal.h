@@ -167,6 +167,9 @@ cudaError_t launch_conv_dgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
                                  int32_t* status, cudaStream_t st);
 cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int bnmax,
                                  int32_t* status, cudaStream_t st);
+// record a message for pnn_last_error(NULL) and return `code`
+int set_last_error(int code, const char* msg);
+
 // debug builds: first misaligned vector access of the tensor-core kernels (0 = none)
 unsigned long long conv_tc_debug_word();
 cudaError_t launch_wtrans(const WtDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);

@@ -1384,6 +1384,14 @@ int set_global(int code, const std::string& m) {
   g_err = m;
   return code;
 }
+}  // namespace
+
+int pnn::set_last_error(int code, const char* msg) {
+  g_err = msg ? msg : "";
+  return code;
+}
+
+namespace {
 #define NET_OR_FAIL(n) \
   if (!(n)) return set_global(PNN_EINVAL, "null handle");
 #define BOUND_OR_FAIL(n)  \
