@@ -46,6 +46,8 @@ def parse():
     ap.add_argument("--config", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-batch", type=int, default=1)
+    ap.add_argument("--stream-fp32", type=int, default=1, choices=[0, 1],
+                    help="keep the residual stream and correction tensors in fp32 (1) or bf16 (0)")
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch (profiling a small case of the same network)")
     return ap.parse_args()
@@ -179,7 +181,7 @@ def our_arm(args, desc, rank, local, world, dist):
     build.build()
     torch.cuda.set_device(local)
     stream = torch.cuda.Stream()
-    net = pnn.ParaNet(desc, seed=0, stream=stream)
+    net = pnn.ParaNet(desc, seed=0, stream=stream, stream_fp32=bool(args.stream_fp32))
     B = desc["batch"]
     x, labels = W.make_batch(desc, seed=1000 + desc.get("config_index", 0) + rank)
     xd = torch.from_numpy(x).cuda()
@@ -271,6 +273,7 @@ def our_arm(args, desc, rank, local, world, dist):
         "config": {"workload": desc["name"] + "_b%d_%dpx_c%d" % (B, desc["in_h"], desc["classes"]),
                    "batch": B, "input": "3x%dx%d" % (desc["in_h"], desc["in_w"]), "classes": desc["classes"],
                    "subnetworks": len(desc["segments"]), "correction": desc.get("correction", "residual"),
+                   "residual_stream": "fp32" if args.stream_fp32 else "bf16",
                    "l2": "inputs larger than L2 (%.1f GB workspace per step)" % (net.workspace_bytes / 1e9),
                    "parallelism": "replicas" if world > 1 else "single-gpu"},
         "conv_tflops": conv_flops / (conv_ms / 1e3) / 1e12 if conv_ms else None,

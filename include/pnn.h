@@ -210,6 +210,25 @@ int pnn_launch_counts(const pnn_net* net, int32_t counts[3]);
  * and drops a captured step graph.  Kinds are 0 .. pnn_num_kernel_kinds()-1. */
 int pnn_profile(pnn_net* net, int32_t enable);
 int pnn_profile_read(pnn_net* net, int32_t kind, double* ms, int64_t* launches, double* flops, double* bytes);
+
+/* One record per kernel launch bracketed since pnn_profile(net, 1), in launch
+ * order: kind (as for pnn_kernel_kind_name), step phase (0 preprocessing
+ * forward, 1 fine forward, 2 coarse forward, 3 head forward, 4 head backward,
+ * 5 coarse backward, 6 correction backward, 7 fine backward, 8
+ * preprocessing backward), the number of layer instances grouped in the
+ * launch and its work items (tiles or rows), the first instance's shape
+ * (convolutions: C_in, C_out, kernel size, stride, H_out, W_out; other kinds:
+ * C, H, W of the tensor read, then zeros), device time and algorithmic
+ * FLOPs and bytes as for pnn_profile_read.  Writes min(max, recorded)
+ * records to out (caller-owned host memory) and the number recorded to
+ * *count; synchronises the library stream.  Records stay until the next
+ * pnn_profile call. */
+typedef struct pnn_trace {
+  int32_t kind, phase, instances, tiles;
+  int32_t shape[6];
+  double ms, flops, bytes;
+} pnn_trace;
+int pnn_profile_trace(pnn_net* net, int32_t max, pnn_trace* out, int32_t* count);
 int32_t pnn_num_kernel_kinds(void);
 const char* pnn_kernel_kind_name(int32_t kind); /* NULL for a bad kind */
 

@@ -94,6 +94,7 @@ struct Launch {
   int phase;
   int aux;  // tcgen05 conv: largest N tile of the group
   double flops, bytes;  // algorithmic work of this launch
+  int shape[6];         // first op: conv (C_in, C_out, k, stride, H_out, W_out); else (C, H, W, 0, 0, 0)
 };
 
 const char* kKindName[K_NKINDS] = {"conv_fwd", "conv_dgrad", "conv_wgrad", "wgrad_reduce", "elementwise",
@@ -171,9 +172,8 @@ struct pnn_net {
   // profiling: events around every launch, accumulated per kind
   bool prof = false;
   std::vector<cudaEvent_t> pev;
-  std::vector<int> pkind;
-  std::vector<double> pflops, pbytes;
-  size_t pnext = 0;
+  std::vector<const Launch*> plaunch;
+  size_t pnext = 0, pfold = 0;
   double kms[K_NKINDS + 1] = {}, kflops[K_NKINDS + 1] = {}, kbytes[K_NKINDS + 1] = {};
   int64_t klaunch[K_NKINDS + 1] = {};
 
@@ -1044,6 +1044,19 @@ int pnn_net::build_tables() {
       Launch L;
       L.kind = g.kind; L.variant = g.variant; L.count = (int)g.ops.size(); L.total = total; L.phase = p;
       L.flops = 0; L.bytes = 0; L.aux = 16;
+      {
+        const POp& o = ops[g.ops[0]];
+        const bool conv = o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC || o.kind == K_DGRAD ||
+                          o.kind == K_DGRAD_TC || o.kind == K_WGRAD || o.kind == K_WGRAD_TC;
+        const int v = o.in >= 0 ? o.in : (o.out >= 0 ? o.out : o.ins[0]);
+        for (int& x : L.shape) x = 0;
+        if (conv) {
+          const int sh[6] = {vals[o.in].C, vals[o.out].C, o.k, o.stride, vals[o.out].H, vals[o.out].W};
+          for (int i = 0; i < 6; ++i) L.shape[i] = sh[i];
+        } else if (v >= 0 && v < (int)vals.size()) {
+          L.shape[0] = vals[v].C; L.shape[1] = vals[v].H; L.shape[2] = vals[v].W;
+        }
+      }
       for (int id : g.ops)
         if (ops[id].kind == K_CONV_FWD_TC || ops[id].kind == K_DGRAD_TC || ops[id].kind == K_WGRAD_TC) {
           const int K = ops[id].kind == K_DGRAD_TC ? vals[ops[id].in].C : vals[ops[id].out].C;
@@ -1204,13 +1217,9 @@ int pnn_net::run_phase(int p) {
         size_t old = pev.size();
         pev.resize(std::max<size_t>(2 * old, 4096));
         for (size_t i = old; i < pev.size(); ++i) cudaEventCreate(&pev[i]);
-        pkind.resize(pev.size() / 2);
-        pflops.resize(pev.size() / 2);
-        pbytes.resize(pev.size() / 2);
+        plaunch.resize(pev.size() / 2);
       }
-      pkind[pnext / 2] = L.kind;
-      pflops[pnext / 2] = L.flops;
-      pbytes[pnext / 2] = L.bytes;
+      plaunch[pnext / 2] = &L;
       cudaEventRecord(pev[pnext], stream);
     }
     switch (L.kind) {
@@ -1734,6 +1743,7 @@ int pnn_profile(pnn_net* n, int32_t enable) {
   }
   n->prof = enable != 0;
   n->pnext = 0;
+  n->pfold = 0;
   for (int k = 0; k <= K_NKINDS; ++k) { n->kms[k] = 0; n->kflops[k] = 0; n->kbytes[k] = 0; n->klaunch[k] = 0; }
   return PNN_OK;
 }
@@ -1743,21 +1753,40 @@ int pnn_profile_read(pnn_net* n, int32_t kind, double* ms, int64_t* launches, do
   if (kind < 0 || kind >= K_NKINDS) return n->fail(PNN_EINVAL, "bad kernel kind");
   cudaError_t e = cudaStreamSynchronize(n->stream);
   if (e != cudaSuccess) return n->cuda_check(e, "synchronise");
-  // fold recorded launches into the per-kind totals
-  for (size_t i = 0; i + 1 < n->pnext; i += 2) {
+  // fold launches recorded since the last read into the per-kind totals
+  for (size_t i = n->pfold; i + 1 < n->pnext; i += 2) {
     float t = 0.f;
     cudaEventElapsedTime(&t, n->pev[i], n->pev[i + 1]);
-    const int k = n->pkind[i / 2];
-    n->kms[k] += t;
-    n->kflops[k] += n->pflops[i / 2];
-    n->kbytes[k] += n->pbytes[i / 2];
-    n->klaunch[k] += 1;
+    const Launch& L = *n->plaunch[i / 2];
+    n->kms[L.kind] += t;
+    n->kflops[L.kind] += L.flops;
+    n->kbytes[L.kind] += L.bytes;
+    n->klaunch[L.kind] += 1;
   }
-  n->pnext = 0;
+  n->pfold = n->pnext;
   if (ms) *ms = n->kms[kind];
   if (launches) *launches = n->klaunch[kind];
   if (flops) *flops = n->kflops[kind];
   if (bytes) *bytes = n->kbytes[kind];
+  return PNN_OK;
+}
+
+int pnn_profile_trace(pnn_net* n, int32_t max, pnn_trace* out, int32_t* count) {
+  BOUND_OR_FAIL(n);
+  if (max < 0 || (max > 0 && !out) || !count) return n->fail(PNN_EINVAL, "bad trace buffer");
+  cudaError_t e = cudaStreamSynchronize(n->stream);
+  if (e != cudaSuccess) return n->cuda_check(e, "synchronise");
+  const int32_t have = (int32_t)(n->pnext / 2);
+  for (int32_t i = 0; i < std::min(have, max); ++i) {
+    const Launch& L = *n->plaunch[i];
+    pnn_trace& r = out[i];
+    float t = 0.f;
+    cudaEventElapsedTime(&t, n->pev[2 * i], n->pev[2 * i + 1]);
+    r.kind = L.kind; r.phase = L.phase; r.instances = L.count; r.tiles = L.total;
+    for (int j = 0; j < 6; ++j) r.shape[j] = L.shape[j];
+    r.ms = t; r.flops = L.flops; r.bytes = L.bytes;
+  }
+  *count = have;
   return PNN_OK;
 }
 

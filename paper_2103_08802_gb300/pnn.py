@@ -53,6 +53,11 @@ class Options(C.Structure):
                 ("stream", C.c_void_p)]
 
 
+class Trace(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("phase", C.c_int32), ("instances", C.c_int32), ("tiles", C.c_int32),
+                ("shape", C.c_int32 * 6), ("ms", C.c_double), ("flops", C.c_double), ("bytes", C.c_double)]
+
+
 _lib = None
 
 
@@ -92,6 +97,7 @@ def load():
         "pnn_profile": (C.c_int, [P, I32]),
         "pnn_profile_read": (C.c_int, [P, I32, C.POINTER(C.c_double), C.POINTER(C.c_int64),
                                        C.POINTER(C.c_double), C.POINTER(C.c_double)]),
+        "pnn_profile_trace": (C.c_int, [P, I32, C.POINTER(Trace), C.POINTER(I32)]),
         "pnn_num_kernel_kinds": (I32, []),
         "pnn_debug_word": (C.c_uint64, []),
         "pnn_kernel_kind_name": (C.c_char_p, [I32]),
@@ -293,6 +299,16 @@ class ParaNet:
             if n.value:
                 out[self.lib.pnn_kernel_kind_name(k).decode()] = (ms.value, n.value, fl.value, by.value)
         return out
+
+    def profile_trace(self):
+        """Per-launch records since profile(): list of dicts in launch order."""
+        n = C.c_int32()
+        self._check(self.lib.pnn_profile_trace(self.h, 0, None, C.byref(n)))
+        buf = (Trace * max(1, n.value))()
+        self._check(self.lib.pnn_profile_trace(self.h, n.value, buf, C.byref(n)))
+        return [{"kind": self.lib.pnn_kernel_kind_name(r.kind).decode(), "phase": r.phase,
+                 "instances": r.instances, "tiles": r.tiles, "shape": tuple(r.shape),
+                 "ms": r.ms, "flops": r.flops, "bytes": r.bytes} for r in buf[:n.value]]
 
     def launch_counts(self):
         c = (C.c_int32 * 3)()
