@@ -44,11 +44,23 @@ constexpr int kStages = 4;
 constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr int kABytes = kBM * kBK * 2;
-constexpr int kProd = 256;                  // gather threads (warps 0-7)
 constexpr int kGroup = 128;                 // two gather groups fill alternating stages
 constexpr int kMmaWarp = 8;
 constexpr int kThreads = 13 * 32;
 enum { FWD = 0, DGRAD = 1, WGRAD = 2 };
+
+#ifdef PNN_ROLE_TIMING
+// Diagnostic build only: SM cycles each role spends waiting and working,
+// summed over CTAs, per mode: [0] gather wait for a free stage, [1] gather
+// work, [2] stages gathered (both counted for thread 0 of each group), [3]
+// MMA wait for a free accumulator, [4] MMA wait for a full stage, [5] MMA
+// issue, [6] epilogue wait, [7] epilogue work, [8] tiles, [9] CTA lifetime,
+// [10] CTAs.
+__device__ unsigned long long g_role_cycles[3][12];
+#define RT(...) __VA_ARGS__
+#else
+#define RT(...)
+#endif
 
 struct Shared {
   uint64_t full[kStages];
@@ -106,141 +118,281 @@ __device__ __forceinline__ void act8(float* v, const float* sc, const float* sf,
 
 // ---------------------------------------------------------------- gather one stage
 // The gatherers form two groups of 128 threads that fill alternating stages.
-// Rows of the A operand handled by group thread p: chunk cc = p & 7 of rows
-// rg + 16 i (i = 0..7), rg = p >> 3.
-template <int MODE>
-__device__ __forceinline__ void gather_stage(const Tile& T, int kt, uint8_t* A, uint8_t* Bt, int p) {
+// Each stage issues all of its global loads before it consumes any, so that a
+// thread waits for memory once per stage, not once per row.
+
+// Forward and data gradient: group thread p handles chunk cc = p & 7 (8
+// consecutive K elements) of rows rg + 16 i (i = 0..7), rg = p >> 3.  Every
+// row is loaded unconditionally (a row in the zero padding or past the end
+// reads the tensor's first elements and is masked afterwards).  XBF: the
+// source rows are bf16, else fp32.
+template <int MODE, bool XBF>
+__device__ __forceinline__ void gather_fd(const Tile& T, int kt, uint8_t* A, uint8_t* Bt, int p) {
   const ConvDesc& d = *T.d;
   const int cc = p & 7, rg = p >> 3;
-  if (MODE == FWD || MODE == DGRAD) {
-    const int k = kt * kBK + cc * 8;
-    const bool kin = k < T.Kt;
-    int c0 = 0, r_ = 0, s_ = 0;
-    if (kin) {
-      const int cdim = MODE == FWD ? d.C : d.K;
-      c0 = k % cdim;
-      const int rs = k / cdim;
-      s_ = rs % d.S;
-      r_ = rs / d.S;
-    }
-    float sc[8], sf[8];
-    const bool tr = MODE == FWD && kin && d.x.scale != nullptr;
-    if (tr) {
+  const int k = kt * kBK + cc * 8;
+  const bool kin = k < T.Kt;
+  int c0 = 0, r_ = 0, s_ = 0;
+  if (kin) {
+    const int cdim = MODE == FWD ? d.C : d.K;
+    c0 = k % cdim;
+    const int rs = k / cdim;
+    s_ = rs % d.S;
+    r_ = rs / d.S;
+  }
+  const bool tr = MODE == FWD && kin && d.x.scale != nullptr;
+  const void* base = MODE == FWD ? d.x.ptr : static_cast<const void*>(d.dy);
+  // phase 1: addresses and loads
+  uint4 raw[8][XBF ? 1 : 2];
+  unsigned have = 0;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) { sc[i] = __ldg(d.x.scale + c0 + i); sf[i] = __ldg(d.x.shift + c0 + i); }
+  for (int i = 0; i < 8; ++i) {
+    const int m = T.m0 + rg + 16 * i;
+    int64_t e = 0;
+    bool ok = false;
+    if (MODE == FWD) {
+      const int q = m % d.Q, tmp = m / d.Q, pp = tmp % d.P, nb = tmp / d.P;
+      const int h = pp * d.stride - d.pad + r_, w = q * d.stride - d.pad + s_;
+      ok = h >= 0 && h < d.H && w >= 0 && w < d.W;
+      e = ((int64_t)(nb * d.H + h) * d.W + w) * d.C + c0;
+    } else {
+      const int w = m % d.W, tmp = m / d.W, h = tmp % d.H, nb = tmp / d.H;
+      const int pn = h + d.pad - r_, qn = w + d.pad - s_;
+      const int pp = pn / d.stride, q = qn / d.stride;
+      ok = pn >= 0 && qn >= 0 && pn % d.stride == 0 && qn % d.stride == 0 && pp < d.P && q < d.Q;
+      e = ((int64_t)(nb * d.P + pp) * d.Q + q) * d.K + c0;
     }
-    // issue all row loads first (8 in flight), then convert and store
-    float v[8][8];
-    bool have[8];
+    ok = ok && kin && m < T.Mrows;
+    if (!ok) e = 0;
+    have |= (ok ? 1u : 0u) << i;
+    const uint4* src = XBF ? reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(base) + e)
+                           : reinterpret_cast<const uint4*>(reinterpret_cast<const float*>(base) + e);
+    raw[i][0] = __ldg(src);
+    if (!XBF) raw[i][XBF ? 0 : 1] = __ldg(src + 1);
+  }
+  float sc[8], sf[8];
+  if (tr) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) { sc[i] = __ldg(d.x.scale + c0 + i); sf[i] = __ldg(d.x.shift + c0 + i); }
+  }
+  // B: weight rows (forward W[n][k], dgrad Wt[c][k]), K-contiguous bf16,
+  // copied asynchronously straight into their swizzled slots (zero-filled
+  // outside the matrix)
+  const uint32_t bt = smem_u32(Bt);
+  for (int idx = p; idx < T.BN * 8; idx += kGroup) {
+    const int n = idx >> 3, ch = idx & 7;
+    const int kk = kt * kBK + ch * 8;
+    const __nv_bfloat16* q = reinterpret_cast<const __nv_bfloat16*>(d.w);
+    int nbytes = 0;
+    if (T.n0 + n < T.Ncols && kk < T.Kt) {
+      q += (int64_t)(T.n0 + n) * T.Kt + kk;
+      nbytes = PNN_ALIGNED(q, 16) ? 16 : 0;
+    }
+    cp_async16(bt + swz(n, ch), q, nbytes);
+  }
+  // phase 2: BN scale/shift + ReLU of the producing layer, bf16, mask, store
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    float v[8];
+    if (XBF) {
+      const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&raw[i][0]);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float2 f = __bfloat1622float2(hh[j]);
+        v[2 * j] = f.x;
+        v[2 * j + 1] = f.y;
+      }
+    } else {
+      const float* f0 = reinterpret_cast<const float*>(&raw[i][0]);
+      const float* f1 = reinterpret_cast<const float*>(&raw[i][XBF ? 0 : 1]);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) { v[j] = f0[j]; v[4 + j] = f1[j]; }
+    }
+    if (tr) act8(v, sc, sf, d.x.relu);
+    const uint4 out = (have >> i) & 1 ? pack8(v) : make_uint4(0, 0, 0, 0);
+    *reinterpret_cast<uint4*>(A + swz(rg + 16 * i, cc)) = out;
+  }
+  cp_async_wait_all();
+}
+
+// wgrad B operand: dY[pix][ko0 .. ko0+8) (fp32) for the 4 pixels pixa ..
+// pixa+3, loaded but not consumed; returns the mask of pixels inside the split
+__device__ __forceinline__ unsigned load_dy_half(const Tile& T, int pixa, int ko0, bool unit, float4 (&rb)[4][2]) {
+  const ConvDesc& d = *T.d;
+  unsigned ok = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    rb[i][0] = make_float4(0.f, 0.f, 0.f, 0.f);
+    rb[i][1] = rb[i][0];
+    const int pix = pixa + i;
+    if (unit && ko0 < d.K && pix < T.pend) {
+      ok |= 1u << i;
+      const float4* src = reinterpret_cast<const float4*>(d.dy + (int64_t)pix * d.K + ko0);
+      if (PNN_ALIGNED(src, 16)) { rb[i][0] = __ldg(src); rb[i][1] = __ldg(src + 1); }
+    }
+  }
+  return ok;
+}
+// rows kg*8 + c (c = k_out offset) of the B operand, pixels 4*half .. 4*half+3
+// of pixel group pg: an 8 (k_out) x 4 (pixel) transpose into 8-byte half chunks
+__device__ __forceinline__ void store_dy_half(const float4 (&rb)[4][2], unsigned ok, uint8_t* Bt, int kg, int pg,
+                                              int half) {
+  uint32_t w[4][4];  // w[pixel][pair of k_out]
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const bool in = (ok >> i) & 1;
+    w[i][0] = in ? pack_bf16(rb[i][0].x, rb[i][0].y) : 0u;
+    w[i][1] = in ? pack_bf16(rb[i][0].z, rb[i][0].w) : 0u;
+    w[i][2] = in ? pack_bf16(rb[i][1].x, rb[i][1].y) : 0u;
+    w[i][3] = in ? pack_bf16(rb[i][1].z, rb[i][1].w) : 0u;
+  }
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const uint32_t sel = (c & 1) ? 0x7632 : 0x5410;
+    const uint2 o = make_uint2(__byte_perm(w[0][c / 2], w[1][c / 2], sel), __byte_perm(w[2][c / 2], w[3][c / 2], sel));
+    *reinterpret_cast<uint2*>(Bt + swz(kg * 8 + c, pg) + 8 * half) = o;
+  }
+}
+
+// Weight gradient: A (rows j = (r,s,c), 16 row groups x 8 pixel groups = 128
+// units, one per thread) and B (rows k_out, BN/8 row groups x 8 pixel
+// groups, BN/128 units per thread) in units of 8 rows x 8 pixels, transposed
+// in registers.  The A unit and the first half of the B unit (4 pixels) are
+// loaded together, the second half once A is stored (128 registers a thread
+// do not hold both whole).  XBF: the activation is stored as bf16, else fp32.
+template <bool XBF>
+__device__ __forceinline__ void gather_wgrad(const Tile& T, int kt, uint8_t* A, uint8_t* Bt, int p) {
+  const ConvDesc& d = *T.d;
+  const int pix0 = T.pbeg + kt * kBK;
+  const int jg = p >> 3, pg = p & 7;
+  const int j0 = T.m0 + jg * 8;
+  const bool jin = j0 < T.Mrows;
+  int c0 = 0, r_ = 0, s_ = 0;
+  if (jin) { c0 = j0 % d.C; const int rs = j0 / d.C; s_ = rs % d.S; r_ = rs / d.S; }
+  const bool tr = jin && d.x.scale != nullptr;
+  float sc[8], sf[8];
+  if (tr) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) { sc[i] = __ldg(d.x.scale + c0 + i); sf[i] = __ldg(d.x.shift + c0 + i); }
+  }
+  uint4 ra[8][XBF ? 1 : 2];
+  unsigned have = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    ra[i][0] = make_uint4(0, 0, 0, 0);
+    if (!XBF) ra[i][XBF ? 0 : 1] = make_uint4(0, 0, 0, 0);
+    const int pix = pix0 + pg * 8 + i;
+    const int q = pix % d.Q, tmp = pix / d.Q, pp = tmp % d.P, nb = tmp / d.P;
+    const int h = pp * d.stride + r_ - d.pad, w = q * d.stride + s_ - d.pad;
+    if (jin && pix < T.pend && h >= 0 && h < d.H && w >= 0 && w < d.W) {
+      have |= 1u << i;
+      const int64_t e = ((int64_t)(nb * d.H + h) * d.W + w) * d.C + c0;
+      const uint4* src = XBF ? reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(d.x.ptr) + e)
+                             : reinterpret_cast<const uint4*>(reinterpret_cast<const float*>(d.x.ptr) + e);
+      if (PNN_ALIGNED(src, 16)) {
+        ra[i][0] = __ldg(src);
+        if (!XBF) ra[i][XBF ? 0 : 1] = __ldg(src + 1);
+      }
+    }
+  }
+  const int kg = p >> 3;
+  const bool bunit = p < T.BN;
+  float4 rb0[4][2], rb1[4][2];
+  const unsigned ok0 = load_dy_half(T, pix0 + pg * 8, T.n0 + kg * 8, bunit, rb0);
+  // A: BN scale/shift + ReLU of the producing layer, bf16, 8x8 transpose
+  {
+    uint4 in[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      have[i] = false;
-      const int m = T.m0 + rg + 16 * i;
-      if (!kin || m >= T.Mrows) continue;
-      if (MODE == FWD) {
-        const int q = m % d.Q, tmp = m / d.Q, pp = tmp % d.P, nb = tmp / d.P;
-        const int h = pp * d.stride - d.pad + r_, w = q * d.stride - d.pad + s_;
-        if (h >= 0 && h < d.H && w >= 0 && w < d.W) {
-          load8(d.x.ptr, d.x.dt, ((int64_t)(nb * d.H + h) * d.W + w) * d.C + c0, v[i]);
-          have[i] = true;
+      float v[8];
+      if (XBF) {
+        const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&ra[i][0]);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float2 f = __bfloat1622float2(hh[j]);
+          v[2 * j] = f.x;
+          v[2 * j + 1] = f.y;
         }
       } else {
-        const int w = m % d.W, tmp = m / d.W, h = tmp % d.H, nb = tmp / d.H;
-        const int pn = h + d.pad - r_, qn = w + d.pad - s_;
-        if (pn >= 0 && qn >= 0 && pn % d.stride == 0 && qn % d.stride == 0) {
-          const int pp = pn / d.stride, q = qn / d.stride;
-          if (pp < d.P && q < d.Q) {
-            load8(d.dy, 0, ((int64_t)(nb * d.P + pp) * d.Q + q) * d.K + c0, v[i]);
-            have[i] = true;
-          }
-        }
-      }
-    }
+        const float* f0 = reinterpret_cast<const float*>(&ra[i][0]);
+        const float* f1 = reinterpret_cast<const float*>(&ra[i][XBF ? 0 : 1]);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int row = rg + 16 * i;
-      uint4 out = make_uint4(0, 0, 0, 0);
-      if (have[i]) {
-        if (tr) act8(v[i], sc, sf, d.x.relu);
-        out = pack8(v[i]);
+        for (int j = 0; j < 4; ++j) { v[j] = f0[j]; v[4 + j] = f1[j]; }
       }
-      *reinterpret_cast<uint4*>(A + swz(row, cc)) = out;
+      if (tr) act8(v, sc, sf, d.x.relu);
+      in[i] = (have >> i) & 1 ? pack8(v) : make_uint4(0, 0, 0, 0);
     }
-    // B: weight rows (forward W[n][k], dgrad Wt[c][k]), K-contiguous
-    for (int idx = p; idx < T.BN * 8; idx += kGroup) {
-      const int n = idx >> 3, ch = idx & 7;
-      const int kk = kt * kBK + ch * 8;
-      uint4 val = make_uint4(0, 0, 0, 0);
-      if (T.n0 + n < T.Ncols && kk < T.Kt) {
-        const uint4* q = reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(d.w) +
-                                                        (int64_t)(T.n0 + n) * T.Kt + kk);
-        if (PNN_ALIGNED(q, 16)) val = __ldg(q);
-      }
-      *reinterpret_cast<uint4*>(Bt + swz(n, ch)) = val;
-    }
+    uint4 out[8];
+    transpose8(in, out);
+#pragma unroll
+    for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(A + swz(jg * 8 + c, pg)) = out[c];
+  }
+  // B: bf16, transposed half by half
+  const unsigned ok1 = load_dy_half(T, pix0 + pg * 8 + 4, T.n0 + kg * 8, bunit, rb1);
+  if (bunit) {
+    store_dy_half(rb0, ok0, Bt, kg, pg, 0);
+    store_dy_half(rb1, ok1, Bt, kg, pg, 1);
+  }
+  // BN = 256: a second B unit per thread
+  for (int idx = p + kGroup; idx < T.BN; idx += kGroup) {
+    const int kg2 = idx >> 3;
+    const unsigned m0 = load_dy_half(T, pix0 + pg * 8, T.n0 + kg2 * 8, true, rb0);
+    const unsigned m1 = load_dy_half(T, pix0 + pg * 8 + 4, T.n0 + kg2 * 8, true, rb1);
+    store_dy_half(rb0, m0, Bt, kg2, pg, 0);
+    store_dy_half(rb1, m1, Bt, kg2, pg, 1);
+  }
+}
+
+template <int MODE>
+__device__ __forceinline__ void gather_stage(const Tile& T, int kt, uint8_t* A, uint8_t* Bt, int p) {
+  if (MODE == FWD) {
+    if (T.d->x.dt == DT_BF16) gather_fd<FWD, true>(T, kt, A, Bt, p);
+    else gather_fd<FWD, false>(T, kt, A, Bt, p);
+  } else if (MODE == DGRAD) {
+    gather_fd<DGRAD, false>(T, kt, A, Bt, p);
   } else {
-    // wgrad: units of 8 rows x 8 pixels, transposed in registers.
-    // A (rows j = (r,s,c)): 16 row groups x 8 pixel groups = 128 units, one per thread;
-    // B (rows k_out):       BN/8 row groups x 8 pixel groups, BN/128 per thread.
-    const int pix0 = T.pbeg + kt * kBK;
-    {
-      const int jg = p >> 3, pg = p & 7;
-      const int j0 = T.m0 + jg * 8;
-      const bool jin = j0 < T.Mrows;
-      int c0 = 0, r_ = 0, s_ = 0;
-      if (jin) { c0 = j0 % d.C; const int rs = j0 / d.C; s_ = rs % d.S; r_ = rs / d.S; }
-      float sc[8], sf[8];
-      const bool tr = jin && d.x.scale != nullptr;
-      if (tr) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) { sc[i] = __ldg(d.x.scale + c0 + i); sf[i] = __ldg(d.x.shift + c0 + i); }
-      }
-      uint4 in[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        in[i] = make_uint4(0, 0, 0, 0);
-        const int pix = pix0 + pg * 8 + i;
-        if (jin && pix < T.pend) {
-          const int q = pix % d.Q, tmp = pix / d.Q, pp = tmp % d.P, nb = tmp / d.P;
-          const int h = pp * d.stride + r_ - d.pad, w = q * d.stride + s_ - d.pad;
-          if (h >= 0 && h < d.H && w >= 0 && w < d.W) {
-            float v[8];
-            load8(d.x.ptr, d.x.dt, ((int64_t)(nb * d.H + h) * d.W + w) * d.C + c0, v);
-            if (tr) act8(v, sc, sf, d.x.relu);
-            in[i] = pack8(v);
-          }
-        }
-      }
-      uint4 out[8];
-      transpose8(in, out);
-#pragma unroll
-      for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(A + swz(jg * 8 + c, pg)) = out[c];
-    }
-    {
-      for (int idx = p; idx < T.BN; idx += kGroup) {
-        const int kg = idx >> 3, pg = idx & 7;
-        const int ko0 = T.n0 + kg * 8;
-        uint4 in[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          in[i] = make_uint4(0, 0, 0, 0);
-          const int pix = pix0 + pg * 8 + i;
-          if (ko0 < d.K && pix < T.pend) {
-            float v[8];
-            load8(d.dy, 0, (int64_t)pix * d.K + ko0, v);
-            in[i] = pack8(v);
-          }
-        }
-        uint4 out[8];
-        transpose8(in, out);
-#pragma unroll
-        for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(Bt + swz(kg * 8 + c, pg)) = out[c];
-      }
-    }
+    if (T.d->x.dt == DT_BF16) gather_wgrad<true>(T, kt, A, Bt, p);
+    else gather_wgrad<false>(T, kt, A, Bt, p);
   }
 }
 
 // ---------------------------------------------------------------- epilogue of one tile
+// Column sums over the warp's 32 lanes of x[0..15] (lane = row) by
+// reduce-scatter: each step hands half of the remaining columns to the
+// partner lane (xor 16, 8, 4, 2) and a last exchange (xor 1) completes the
+// sum -- 16 shuffles instead of 80.  Lane l returns the sum of column l >> 1.
+__device__ __forceinline__ float warp_colsum16(const float (&x)[16], int lane) {
+  float y8[8], y4[4], y2[2];
+  const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4, b1 = lane & 2;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    y8[i] = (b4 ? x[i + 8] : x[i]) + __shfl_xor_sync(0xffffffffu, b4 ? x[i] : x[i + 8], 16);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    y4[i] = (b3 ? y8[i + 4] : y8[i]) + __shfl_xor_sync(0xffffffffu, b3 ? y8[i] : y8[i + 4], 8);
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+    y2[i] = (b2 ? y4[i + 2] : y4[i]) + __shfl_xor_sync(0xffffffffu, b2 ? y4[i] : y4[i + 2], 4);
+  const float y = (b1 ? y2[1] : y2[0]) + __shfl_xor_sync(0xffffffffu, b1 ? y2[0] : y2[1], 2);
+  return y + __shfl_xor_sync(0xffffffffu, y, 1);
+}
+
+// 16 residual values of row m from column nb as raw 16-byte words (fp32: 4
+// words, bf16: 2); a chunk that is not entirely inside the row reads the
+// tensor's first elements (that chunk takes the element-wise path instead)
+__device__ __forceinline__ void res_raw(const ConvDesc& d, int m, int nb, int ncols, uint4 (&rr)[4]) {
+  const int64_t o = nb + 16 <= ncols ? (int64_t)m * d.K + nb : 0;
+  if (d.res_dt == DT_BF16) {
+    const uint4* src = reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(d.res) + o);
+    rr[0] = __ldg(src);
+    rr[1] = __ldg(src + 1);
+  } else {
+    const uint4* src = reinterpret_cast<const uint4*>(reinterpret_cast<const float*>(d.res) + o);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) rr[i] = __ldg(src + i);
+  }
+}
+
 template <int MODE>
 __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, int lane, Shared& sh) {
   const ConvDesc& d = *T.d;
@@ -249,7 +401,13 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
   const bool mvalid = m < T.Mrows;
   const uint32_t tbase = tacc + ((uint32_t)(q * 32) << 16);
   const bool stats = MODE == FWD && d.stats != nullptr;
+  // forward residual: 16 columns a chunk, the next chunk's loads issued
+  // before the current chunk is consumed
+  const bool rvec = MODE == FWD && d.res != nullptr && mvalid && (d.K % 8) == 0;
+  uint4 rcur[4], rnext[4];
+  if (rvec) res_raw(d, m, T.n0, T.Ncols, rcur);
   for (int j0 = 0; j0 < T.BN; j0 += 16) {
+    if (rvec && j0 + 16 < T.BN) res_raw(d, m, T.n0 + j0 + 16, T.Ncols, rnext);
     float v[16];
     tmem_ld16(tbase + j0, v);
     const int nb = T.n0 + j0;
@@ -263,13 +421,19 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
         const bool vec = full && (d.K % 8) == 0;
         if (d.res) {
           if (vec) {
-            float r8[8];
-            load8(d.res, d.res_dt == DT_BF16, o, r8);
+            if (d.res_dt == DT_BF16) {
+              const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(rcur);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) v[i] += r8[i];
-            load8(d.res, d.res_dt == DT_BF16, o + 8, r8);
+              for (int i = 0; i < 8; ++i) {
+                const float2 f = __bfloat1622float2(hh[i]);
+                v[2 * i] += f.x;
+                v[2 * i + 1] += f.y;
+              }
+            } else {
+              const float* f = reinterpret_cast<const float*>(rcur);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) v[8 + i] += r8[i];
+              for (int i = 0; i < 16; ++i) v[i] += f[i];
+            }
           } else {
             for (int i = 0; i < 16 && nb + i < d.K; ++i)
               v[i] += d.res_dt == DT_F32 ? reinterpret_cast<const float*>(d.res)[o + i]
@@ -308,17 +472,10 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
         }
       }
       if (stats) {
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-#pragma unroll
-          for (int off = 16; off > 0; off >>= 1) {
-            s1[i] += __shfl_xor_sync(0xffffffffu, s1[i], off);
-            s2[i] += __shfl_xor_sync(0xffffffffu, s2[i], off);
-          }
-        }
-        if (lane == 0) {
-#pragma unroll
-          for (int i = 0; i < 16; ++i) { sh.red[q][j0 + i][0] = s1[i]; sh.red[q][j0 + i][1] = s2[i]; }
+        const float a = warp_colsum16(s1, lane), b = warp_colsum16(s2, lane);
+        if ((lane & 1) == 0) {
+          sh.red[q][j0 + (lane >> 1)][0] = a;
+          sh.red[q][j0 + (lane >> 1)][1] = b;
         }
       }
     } else if (mvalid) {
@@ -341,6 +498,10 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
         for (int i = 0; i < 16 && nb + i < T.Ncols; ++i) out[i] = acc ? out[i] + v[i] : v[i];
       }
     }
+    if (rvec) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) rcur[i] = rnext[i];
+    }
   }
   if (stats) {
     asm volatile("bar.sync 2, 128;" ::: "memory");
@@ -362,6 +523,7 @@ template <int MODE>
 __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, const int* __restrict__ tstart,
                                              int ninst, int total, int bnmax, int32_t* status) {
   extern __shared__ uint8_t smem_raw[];
+  RT(const unsigned long long rt_start = clock64();)
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* const gbase = smem_raw + (base - raw);
@@ -398,19 +560,28 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
     const int gi = threadIdx.x / kGroup, p = threadIdx.x % kGroup;
     uint32_t g = 0;
     bool ok = true;
+    RT(unsigned long long rt_wait = 0, rt_work = 0, rt_n = 0;)
     for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
       const Tile T = decode<MODE>(tab, tstart, ninst, tile);
       for (int kt = 0; kt < T.nkt; ++kt, ++g) {
         if ((int)(g & 1) != gi) continue;
         const int s = g % kStages;
+        RT(const unsigned long long rt0 = clock64();)
         if (!mbar_wait(smem_u32(&sh.empty[s]), ((g / kStages) & 1) ^ 1, abort_flag)) { ok = false; break; }
+        RT(const unsigned long long rt1 = clock64(); rt_wait += rt1 - rt0;)
         uint8_t* A = gbase + s * stage_bytes;
         gather_stage<MODE>(T, kt, A, A + kABytes, p);
         fence_proxy_async();
         mbar_arrive(smem_u32(&sh.full[s]));
+        RT(rt_work += clock64() - rt1; ++rt_n;)
       }
     }
     if (!ok) { sh.abort_flag = 1; atomicExch(status, 3); }
+    RT(if (p == 0) {
+      atomicAdd(&g_role_cycles[MODE][0], rt_wait);
+      atomicAdd(&g_role_cycles[MODE][1], rt_work);
+      atomicAdd(&g_role_cycles[MODE][2], rt_n);
+    })
   } else if (warp == kMmaWarp) {
     // ================================================= MMA issuer
     if (lane == 0) {
@@ -418,16 +589,21 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
       int li = 0;
       bool ok = true;
       bool issued = false;
+      RT(unsigned long long rt_acc = 0, rt_full = 0, rt_issue = 0;)
       for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++li) {
         const Tile T = decode<MODE>(tab, tstart, ninst, tile);
         const int b = li & 1;
+        RT(unsigned long long rt0 = clock64();)
         if (!mbar_wait(smem_u32(&sh.tempty[b]), ((li >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
+        RT(rt_acc += clock64() - rt0;)
         fence_after();
         const uint32_t tacc = tmem + b * colstride;
         const uint32_t idesc = idesc_bf16(kBM, T.BN);
         for (int kt = 0; kt < T.nkt; ++kt, ++g) {
           const int s = g % kStages;
+          RT(rt0 = clock64();)
           if (!mbar_wait(smem_u32(&sh.full[s]), (g / kStages) & 1, abort_flag)) { ok = false; break; }
+          RT(const unsigned long long rt1 = clock64(); rt_full += rt1 - rt0;)
           fence_after();
           const uint32_t a_addr = base + s * stage_bytes;
           const uint32_t b_addr = a_addr + kABytes;
@@ -437,9 +613,12 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
             mma_bf16(tacc, sw128_desc(a_addr + kk * 32), sw128_desc(b_addr + kk * 32), idesc, (kt | kk) ? 1u : 0u);
           issued = true;
           mma_commit(smem_u32(&sh.empty[s]));
+          RT(rt_issue += clock64() - rt1;)
         }
         if (ok) mma_commit(smem_u32(&sh.tfull[b]));
       }
+      RT(atomicAdd(&g_role_cycles[MODE][3], rt_acc); atomicAdd(&g_role_cycles[MODE][4], rt_full);
+         atomicAdd(&g_role_cycles[MODE][5], rt_issue);)
       if (!ok) {
         sh.abort_flag = 1;
         atomicExch(status, 3);
@@ -455,10 +634,13 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     int li = 0;
     bool ok = true;
+    RT(unsigned long long rt_wait = 0, rt_work = 0;)
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++li) {
       const Tile T = decode<MODE>(tab, tstart, ninst, tile);
       const int b = li & 1;
+      RT(const unsigned long long rt0 = clock64();)
       bool got = mbar_wait(smem_u32(&sh.tfull[b]), (li >> 1) & 1, abort_flag);
+      RT(const unsigned long long rt1 = clock64(); rt_wait += rt1 - rt0;)
       got = __all_sync(0xffffffffu, got);  // tcgen05.ld is warp-collective
       // the four epilogue warps decide together (they meet at named barrier 2
       // inside epilogue(); every warp reaches this vote after a bounded wait)
@@ -471,7 +653,13 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
       epilogue<MODE>(T, tmem + b * colstride, q, lane, sh);
       fence_before();
       mbar_arrive(smem_u32(&sh.tempty[b]));
+      RT(rt_work += clock64() - rt1;)
     }
+    RT(if (threadIdx.x == (kMmaWarp + 1) * 32) {
+      atomicAdd(&g_role_cycles[MODE][6], rt_wait);
+      atomicAdd(&g_role_cycles[MODE][7], rt_work);
+      atomicAdd(&g_role_cycles[MODE][8], (unsigned long long)li);
+    })
     if (!ok) {
       sh.abort_flag = 1;
       atomicExch(status, 3);
@@ -483,6 +671,10 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
     fence_after();
     tmem_dealloc(tmem, ncols);
   }
+  RT(if (threadIdx.x == 0) {
+    atomicAdd(&g_role_cycles[MODE][9], clock64() - rt_start);
+    atomicAdd(&g_role_cycles[MODE][10], 1ull);
+  })
 }
 
 // one kernel name per mode (profiler filters and launch lists name the mode)
@@ -551,6 +743,19 @@ cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
 }
 
 }  // namespace pnn
+
+#ifdef PNN_ROLE_TIMING
+// Diagnostic build only: copy (and optionally clear) the role counters
+// (3 modes x 12 counters).
+extern "C" int pnn_role_cycles(unsigned long long* out, int reset) {
+  cudaError_t e = cudaMemcpyFromSymbol(out, pnn::g_role_cycles, sizeof(pnn::g_role_cycles));
+  if (e == cudaSuccess && reset) {
+    static const unsigned long long zero[3][12] = {};
+    e = cudaMemcpyToSymbol(pnn::g_role_cycles, zero, sizeof zero);
+  }
+  return e == cudaSuccess ? 0 : 1;
+}
+#endif
 
 // ============================================================================
 // Allocation-free weight gradient: the same tensor-core kernel, with its

@@ -166,6 +166,13 @@ __device__ __forceinline__ void transpose8(const uint4* in, uint4* out) {
       o[c * 4 + p / 2] = __byte_perm(a, b, (c & 1) ? 0x7632 : 0x5410);
     }
 }
+// 16-byte global -> shared copy that does not block the issuing thread
+// (L2-cached); n_src < 16 fills the rest of the 16 bytes with zeros (0: all
+// zeros, nothing is read).  cp_async_wait_all() waits for this thread's copies.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int n_src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 // byte offset of 16-byte chunk `ch` of row `row` in the 128-byte-swizzled K-major layout
 __device__ __forceinline__ uint32_t swz(int row, int ch) { return (uint32_t)(row * 128 + ((ch ^ (row & 7)) << 4)); }
 
