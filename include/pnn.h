@@ -108,8 +108,11 @@ typedef struct {
   int32_t nesterov;
   int32_t stream_fp32;   /* bf16 mode: keep the residual stream (block outputs,
                             correction tensors) in fp32 storage */
-  int32_t conv_impl;     /* 0 = tensor cores wherever the shape allows, 1 = CUDA-core
-                            kernels only, 2 = CUDA-core forward + tensor-core gradients */
+  int32_t conv_impl;     /* 0 = tensor cores wherever the shape allows (stride-1
+                            forward and data-gradient convs fed by TMA), 1 = CUDA-core
+                            kernels only, 2 = CUDA-core forward + tensor-core gradients,
+                            3 = tensor cores with every operand gathered by threads
+                            (no TMA producer; same results as 0) */
   int32_t grad_fp32;     /* bf16 mode: contract gradients (dgrad, wgrad) with fp32
                             operands instead of bf16 ones */
   void* stream;          /* cudaStream_t; NULL = legacy default stream */
@@ -212,7 +215,9 @@ int pnn_profile(pnn_net* net, int32_t enable);
 int pnn_profile_read(pnn_net* net, int32_t kind, double* ms, int64_t* launches, double* flops, double* bytes);
 
 /* One record per kernel launch bracketed since pnn_profile(net, 1), in launch
- * order: kind (as for pnn_kernel_kind_name), step phase (0 preprocessing
+ * order: kind (as for pnn_kernel_kind_name), variant (tensor-core forward and
+ * data-gradient convs: 1 = operands fed by TMA, 0 = gathered by threads),
+ * step phase (0 preprocessing
  * forward, 1 fine forward, 2 coarse forward, 3 head forward, 4 head backward,
  * 5 coarse backward, 6 correction backward, 7 fine backward, 8
  * preprocessing backward), the number of layer instances grouped in the
@@ -224,7 +229,7 @@ int pnn_profile_read(pnn_net* net, int32_t kind, double* ms, int64_t* launches, 
  * *count; synchronises the library stream.  Records stay until the next
  * pnn_profile call. */
 typedef struct pnn_trace {
-  int32_t kind, phase, instances, tiles;
+  int32_t kind, variant, phase, instances, tiles;
   int32_t shape[6];
   double ms, flops, bytes;
 } pnn_trace;

@@ -553,7 +553,7 @@ __global__ void __launch_bounds__(256) k_bnb_reduce8(const BnBwdDesc* __restrict
                                                      const int* __restrict__ tstart, int n) {
   __shared__ float red[256][16];
   const int inst = find_instance(tstart, n, blockIdx.x);
-  const BnBwdDesc& d = tab[inst];
+  const BnBwdDesc d = tab[inst];
   const int tile = blockIdx.x - tstart[inst];
   const int C = d.C, CG = C / 8;
   const int G = 256 / CG;  // row groups (CG <= 256)
@@ -601,46 +601,44 @@ __global__ void __launch_bounds__(256) k_bnb_reduce8(const BnBwdDesc* __restrict
   }
 }
 
+// Each thread keeps one group of 8 channels (cg = thread % (C/8)) for the
+// whole tile, with that group's per-channel parameters in registers, and
+// walks the tile's rows G = 256 / (C/8) apart.
 __global__ void __launch_bounds__(256) k_bnb_apply8(const BnBwdDesc* __restrict__ tab,
                                                     const int* __restrict__ tstart, int n) {
   const int inst = find_instance(tstart, n, blockIdx.x);
-  const BnBwdDesc& d = tab[inst];
+  const BnBwdDesc d = tab[inst];  // a private copy: the stores below cannot force reloads
   const int tile = blockIdx.x - tstart[inst];
   const int C = d.C, CG = C / 8;
+  const int G = 256 / CG;
+  const int cg = threadIdx.x % CG, g = threadIdx.x / CG;
+  if (g >= G) return;
+  const int c0 = cg * 8;
+  float sc[8], sh[8], mean[8], rstd[8], k0[8], k1[8], k2[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    sc[k] = d.scale[c0 + k]; sh[k] = d.shift[c0 + k]; mean[k] = d.mean[c0 + k]; rstd[k] = d.rstd[c0 + k];
+    k0[k] = d.coef[(c0 + k) * 3]; k1[k] = d.coef[(c0 + k) * 3 + 1]; k2[k] = d.coef[(c0 + k) * 3 + 2];
+  }
   const int64_t r0 = (int64_t)tile * d.rows_per_tile;
   const int64_t r1 = min((int64_t)d.M, r0 + d.rows_per_tile);
-  const int64_t groups = (r1 - r0) * CG;
-  for (int64_t e = threadIdx.x; e < groups; e += blockDim.x) {
-    const int64_t r = r0 + e / CG;
-    const int c0 = (int)(e % CG) * 8;
+  for (int64_t r = r0 + g; r < r1; r += G) {
     const int64_t o = r * C + c0;
     float h[8], dz[8], out[8];
     ld8any(d.h, d.h_dt, o, h);
     ld8f(d.da + o, dz);
+    float a0[8], a1[8], ac[8];
+    if (d.add0) ld8f(d.add0 + o, a0);
+    if (d.add1) ld8f(d.add1 + o, a1);
+    if (d.accumulate) ld8f(d.dh + o, ac);
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
-      const int c = c0 + k;
-      if (d.relu && !(fmaf(d.scale[c], h[k], d.shift[c]) > 0.f)) dz[k] = 0.f;
-      const float xhat = (h[k] - d.mean[c]) * d.rstd[c];
-      out[k] = d.coef[c * 3] * (dz[k] - d.coef[c * 3 + 1] - xhat * d.coef[c * 3 + 2]);
-    }
-    if (d.add0) {
-      float a[8];
-      ld8f(d.add0 + o, a);
-#pragma unroll
-      for (int k = 0; k < 8; ++k) out[k] += a[k];
-    }
-    if (d.add1) {
-      float a[8];
-      ld8f(d.add1 + o, a);
-#pragma unroll
-      for (int k = 0; k < 8; ++k) out[k] += a[k];
-    }
-    if (d.accumulate) {
-      float a[8];
-      ld8f(d.dh + o, a);
-#pragma unroll
-      for (int k = 0; k < 8; ++k) out[k] += a[k];
+      if (d.relu && !(fmaf(sc[k], h[k], sh[k]) > 0.f)) dz[k] = 0.f;
+      const float xhat = (h[k] - mean[k]) * rstd[k];
+      out[k] = k0[k] * (dz[k] - k1[k] - xhat * k2[k]);
+      if (d.add0) out[k] += a0[k];
+      if (d.add1) out[k] += a1[k];
+      if (d.accumulate) out[k] += ac[k];
     }
     st8f(d.dh + o, out);
   }

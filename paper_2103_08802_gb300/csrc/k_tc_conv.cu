@@ -128,7 +128,7 @@ __device__ __forceinline__ void act8(float* v, const float* sc, const float* sf,
 // source rows are bf16, else fp32.
 template <int MODE, bool XBF>
 __device__ __forceinline__ void gather_fd(const Tile& T, int kt, uint8_t* A, uint8_t* Bt, int p) {
-  const ConvDesc& d = *T.d;
+  const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
   const int cc = p & 7, rg = p >> 3;
   const int k = kt * kBK + cc * 8;
   const bool kin = k < T.Kt;
@@ -218,7 +218,7 @@ __device__ __forceinline__ void gather_fd(const Tile& T, int kt, uint8_t* A, uin
 // wgrad B operand: dY[pix][ko0 .. ko0+8) (fp32) for the 4 pixels pixa ..
 // pixa+3, loaded but not consumed; returns the mask of pixels inside the split
 __device__ __forceinline__ unsigned load_dy_half(const Tile& T, int pixa, int ko0, bool unit, float4 (&rb)[4][2]) {
-  const ConvDesc& d = *T.d;
+  const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
   unsigned ok = 0;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
@@ -262,7 +262,7 @@ __device__ __forceinline__ void store_dy_half(const float4 (&rb)[4][2], unsigned
 // do not hold both whole).  XBF: the activation is stored as bf16, else fp32.
 template <bool XBF>
 __device__ __forceinline__ void gather_wgrad(const Tile& T, int kt, uint8_t* A, uint8_t* Bt, int p) {
-  const ConvDesc& d = *T.d;
+  const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
   const int pix0 = T.pbeg + kt * kBK;
   const int jg = p >> 3, pg = p & 7;
   const int j0 = T.m0 + jg * 8;
@@ -393,9 +393,13 @@ __device__ __forceinline__ void res_raw(const ConvDesc& d, int m, int nb, int nc
   }
 }
 
+// One warp drains TMEM lanes 32q .. 32q+31 (its rows) for the 16-column
+// chunks j_first, j_first + j_step, ...; the ethreads epilogue threads
+// (etid = this thread's index among them) meet at named barrier 2.
 template <int MODE>
-__device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, int lane, Shared& sh) {
-  const ConvDesc& d = *T.d;
+__device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, int lane, float (&red)[4][256][2],
+                                         int j_first, int j_step, int etid, int ethreads) {
+  const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
   const int row = q * 32 + lane;
   const int m = T.m0 + row;
   const bool mvalid = m < T.Mrows;
@@ -405,9 +409,9 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
   // before the current chunk is consumed
   const bool rvec = MODE == FWD && d.res != nullptr && mvalid && (d.K % 8) == 0;
   uint4 rcur[4], rnext[4];
-  if (rvec) res_raw(d, m, T.n0, T.Ncols, rcur);
-  for (int j0 = 0; j0 < T.BN; j0 += 16) {
-    if (rvec && j0 + 16 < T.BN) res_raw(d, m, T.n0 + j0 + 16, T.Ncols, rnext);
+  if (rvec && j_first < T.BN) res_raw(d, m, T.n0 + j_first, T.Ncols, rcur);
+  for (int j0 = j_first; j0 < T.BN; j0 += j_step) {
+    if (rvec && j0 + j_step < T.BN) res_raw(d, m, T.n0 + j0 + j_step, T.Ncols, rnext);
     float v[16];
     tmem_ld16(tbase + j0, v);
     const int nb = T.n0 + j0;
@@ -474,8 +478,8 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
       if (stats) {
         const float a = warp_colsum16(s1, lane), b = warp_colsum16(s2, lane);
         if ((lane & 1) == 0) {
-          sh.red[q][j0 + (lane >> 1)][0] = a;
-          sh.red[q][j0 + (lane >> 1)][1] = b;
+          red[q][j0 + (lane >> 1)][0] = a;
+          red[q][j0 + (lane >> 1)][1] = b;
         }
       }
     } else if (mvalid) {
@@ -504,16 +508,16 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
     }
   }
   if (stats) {
-    asm volatile("bar.sync 2, 128;" ::: "memory");
-    for (int j = q * 32 + lane; j < T.BN; j += 128) {
+    asm volatile("bar.sync 2, %0;" ::"r"(ethreads) : "memory");
+    for (int j = etid; j < T.BN; j += ethreads) {
       if (T.n0 + j < d.K) {
-        const float a = sh.red[0][j][0] + sh.red[1][j][0] + sh.red[2][j][0] + sh.red[3][j][0];
-        const float b = sh.red[0][j][1] + sh.red[1][j][1] + sh.red[2][j][1] + sh.red[3][j][1];
+        const float a = red[0][j][0] + red[1][j][0] + red[2][j][0] + red[3][j][0];
+        const float b = red[0][j][1] + red[1][j][1] + red[2][j][1] + red[3][j][1];
         d.stats[((int64_t)T.tm * d.K + T.n0 + j) * 2] = a;
         d.stats[((int64_t)T.tm * d.K + T.n0 + j) * 2 + 1] = b;
       }
     }
-    asm volatile("bar.sync 2, 128;" ::: "memory");  // red[] is reused by the next tile
+    asm volatile("bar.sync 2, %0;" ::"r"(ethreads) : "memory");  // red[] is reused by the next tile
   }
 }
 
@@ -650,7 +654,7 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
       asm volatile("bar.sync 2, 128;" ::: "memory");  // epi_ok is rewritten next tile
       if (!got) { ok = false; break; }
       fence_after();
-      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh);
+      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red, 0, 16, q * 32 + lane, 128);
       fence_before();
       mbar_arrive(smem_u32(&sh.tempty[b]));
       RT(rt_work += clock64() - rt1;)
@@ -675,6 +679,407 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
     atomicAdd(&g_role_cycles[MODE][9], clock64() - rt_start);
     atomicAdd(&g_role_cycles[MODE][10], 1ull);
   })
+}
+
+// ============================================================================
+// TMA-fed variant for stride-1 convolutions (1x1 pad 0, 3x3 pad 1), forward
+// and data gradient.  The A rows of filter tap (r,s) are the source rows
+// shifted by a constant in the flattened pixel index ((r-pad)*W + (s-pad);
+// data gradient: the negated offset), so one 2-D tensor-map box [128 rows x
+// min(channels, 64)] per tap brings a k-step's raw operand; rows that fall in
+// the zero padding are zeroed by the transform, which knows each row's
+// pixel.  Channel counts are 8, 16, 32, 64 or multiples of 64.  Roles (14
+// warps, one CTA per SM, persistent):
+//   warp 13     producer: waits for a free stage, issues the A boxes into the
+//               stage's raw slot and the weight box (128-byte swizzle, the
+//               MMA's layout) into its operand slot, all completing on one
+//               transaction mbarrier;
+//   warps 0-3   transform: thread = A row; converts the row's 8 chunks of 8
+//               K elements -- BN scale/shift + ReLU of the producing layer
+//               (forward; staged in shared memory per instance), bf16,
+//               padding mask -- from the raw slot into the swizzled operand;
+//   warp 12     TMEM owner and MMA issuer;
+//   warps 4-11  epilogue: two warps per TMEM lane quarter, alternate
+//               16-column chunks.
+// Every wait is bounded; the producer drains its copies before the CTA exits.
+constexpr int kTmaThreads = 14 * 32;
+constexpr int kTmaTransform = 128;    // warps 0-3
+constexpr int kTmaEpiWarp0 = 4;       // warps 4-11
+constexpr int kTmaEpilogue = 256;
+constexpr int kTmaMmaWarp = 12;
+constexpr int kTmaProducerWarp = 13;
+constexpr int kTmaMaxStages = 8;
+constexpr int kTmaMaxC = 512;         // channels of a BN-transformed source
+constexpr int kTmaSmemBudget = 227 * 1024;
+
+#ifdef PNN_ROLE_TIMING
+// Diagnostic build only, TMA-fed variant (mode 0 forward, 1 dgrad): [0]
+// producer wait for a free stage, [1] producer issue, [2] stages, [3]
+// transform wait for TMA data, [4] transform work (thread 0), [5] MMA wait
+// for a free accumulator, [6] MMA wait for operands, [7] MMA issue, [8]
+// epilogue wait, [9] epilogue work, [10] CTA lifetime, [11] CTAs.
+__device__ unsigned long long g_tma_cycles[2][16];
+#endif
+
+struct TmaShared {
+  uint64_t tma_full[kTmaMaxStages];
+  uint64_t op_full[kTmaMaxStages];
+  uint64_t op_empty[kTmaMaxStages];
+  uint64_t tfull[2];
+  uint64_t tempty[2];
+  uint64_t drain;
+  uint32_t tmem;
+  int abort_flag;
+  int epi_ok[8];
+  float red[4][256][2];
+  float scale[kTmaMaxC];
+  float shift[kTmaMaxC];
+};
+
+__host__ __device__ constexpr int tma_raw_bytes(int esz) { return kBM * kBK * esz; }
+__host__ __device__ constexpr int tma_op_bytes(int bnmax) { return kABytes + bnmax * 128; }
+__host__ __device__ inline int tma_stages(int bnmax, int esz) {
+  const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared);
+  int s = avail / (tma_raw_bytes(esz) + tma_op_bytes(bnmax));
+  return s < 2 ? 2 : (s > kTmaMaxStages ? kTmaMaxStages : s);
+}
+__host__ __device__ inline size_t tma_smem_bytes(int bnmax, int esz) {
+  return 1024 + (size_t)tma_stages(bnmax, esz) * (tma_raw_bytes(esz) + tma_op_bytes(bnmax)) + sizeof(TmaShared);
+}
+
+// One transform thread's share of a stage: row `row` of the A operand, its
+// 8 chunks of 8 K elements, in groups of 4 (bf16) or 2 (fp32): each group's
+// raw loads are issued before any of its chunks is converted and stored (the restrict-qualified
+// pointers tell the compiler the operand stores cannot alias the raw slot
+// or the scale/shift arrays).
+struct TStage {
+  int row, hrow, kread, lg, cdim, tapb, cb;
+  uint32_t tapok;
+  int taps;
+  bool tr;
+  int relu;
+};
+template <bool XBF, bool BIG>
+__device__ __forceinline__ void transform_stage(const uint8_t* __restrict__ rawp, uint8_t* __restrict__ A,
+                                                const float* __restrict__ scs, const float* __restrict__ sfs,
+                                                const TStage& t) {
+  constexpr int G = XBF ? 4 : 2;  // chunks per group (fp32 raw: two 16-byte words a chunk)
+#pragma unroll
+  for (int h = 0; h < 8; h += G) {
+  uint4 raw[G][XBF ? 1 : 2];
+#pragma unroll
+  for (int jj = 0; jj < G; ++jj) {
+    const int j = h + jj;
+    const int cc = j ^ t.hrow;
+    const int e8 = cc * 8;
+    if (e8 >= t.kread) continue;
+    const int ti = BIG ? 0 : e8 >> t.lg;
+    const int off = BIG ? t.row * 64 + e8 : ((ti * kBM + t.row) << t.lg) + (e8 & (t.cdim - 1));
+    if (XBF) {
+      raw[jj][0] = *reinterpret_cast<const uint4*>(rawp + off * 2);
+    } else {
+      raw[jj][0] = *reinterpret_cast<const uint4*>(rawp + off * 4);
+      raw[jj][XBF ? 0 : 1] = *reinterpret_cast<const uint4*>(rawp + off * 4 + 16);
+    }
+  }
+#pragma unroll
+  for (int jj = 0; jj < G; ++jj) {
+    const int j = h + jj;
+    const int cc = j ^ t.hrow;
+    const int e8 = cc * 8;
+    if (e8 >= t.kread) continue;
+    const int ti = BIG ? 0 : e8 >> t.lg;
+    const int tap = t.tapb + ti;
+    const int c = t.cb + (BIG ? e8 : (e8 & (t.cdim - 1)));
+    const bool valid = tap < t.taps && ((t.tapok >> tap) & 1);
+    float v[8];
+    if (XBF) {
+      const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&raw[jj][0]);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 f = __bfloat1622float2(hh[e]);
+        v[2 * e] = f.x;
+        v[2 * e + 1] = f.y;
+      }
+    } else {
+      const float* f0 = reinterpret_cast<const float*>(&raw[jj][0]);
+      const float* f1 = reinterpret_cast<const float*>(&raw[jj][XBF ? 0 : 1]);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) { v[e] = f0[e]; v[4 + e] = f1[e]; }
+    }
+    if (t.tr) {
+      const float4 s0 = *reinterpret_cast<const float4*>(scs + c);
+      const float4 s1 = *reinterpret_cast<const float4*>(scs + c + 4);
+      const float4 f0 = *reinterpret_cast<const float4*>(sfs + c);
+      const float4 f1 = *reinterpret_cast<const float4*>(sfs + c + 4);
+      const float sc[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+      const float sf[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+      act8(v, sc, sf, t.relu);
+    }
+    *reinterpret_cast<uint4*>(A + swz(t.row, cc)) = valid ? pack8(v) : make_uint4(0, 0, 0, 0);
+  }
+  }
+}
+
+template <int MODE>
+__device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, const int* __restrict__ tstart,
+                                              int ninst, int total, int bnmax, int esz_max, int32_t* status) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw0 = smem_u32(smem_raw);
+  const uint32_t base = (raw0 + 1023u) & ~1023u;
+  uint8_t* const gbase = smem_raw + (base - raw0);
+  const int S = tma_stages(bnmax, esz_max);
+  const int raw_bytes = tma_raw_bytes(esz_max);
+  const int op_bytes = tma_op_bytes(bnmax);
+  const uint32_t op_base = base + S * raw_bytes;
+  RT(const unsigned long long rt_start = clock64();)
+  TmaShared& sh = *reinterpret_cast<TmaShared*>(gbase + S * (raw_bytes + op_bytes));
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  uint32_t colstride = 32;
+  while ((int)colstride < bnmax) colstride <<= 1;
+  const uint32_t ncols = 2 * colstride;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(smem_u32(&sh.tma_full[s]), 1);
+      mbar_init(smem_u32(&sh.op_full[s]), kTmaTransform);
+      mbar_init(smem_u32(&sh.op_empty[s]), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&sh.tfull[b]), 1);
+      mbar_init(smem_u32(&sh.tempty[b]), kTmaEpilogue);
+    }
+    mbar_init(smem_u32(&sh.drain), 1);
+    sh.abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == kTmaMmaWarp) tmem_alloc(smem_u32(&sh.tmem), ncols);
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = sh.tmem;
+  volatile int* abort_flag = &sh.abort_flag;
+
+  if (warp == kTmaProducerWarp) {
+    // ================================================= TMA producer
+    if (lane == 0) {
+      uint32_t g = 0;
+      bool ok = true;
+      RT(unsigned long long rt_a = 0, rt_b = 0;)
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+        const Tile T = decode<MODE>(tab, tstart, ninst, tile);
+        const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
+        const int cdim = MODE == FWD ? d.C : d.K;
+        const int cw = cdim < 64 ? cdim : 64;
+        const int esz = (MODE == FWD && d.x.dt == DT_BF16) ? 2 : 4;
+        const uint32_t box = (uint32_t)(kBM * cw * esz);
+        const int taps = d.R * d.S;
+        for (int kt = 0; kt < T.nkt; ++kt, ++g) {
+          const int s = g % S;
+          RT(const unsigned long long rt0 = clock64();)
+          if (!mbar_wait(smem_u32(&sh.op_empty[s]), ((g / S) & 1) ^ 1, abort_flag)) { ok = false; break; }
+          RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
+          const int k0 = kt * kBK;
+          const int tap0 = k0 / cdim, c0 = k0 % cdim;
+          const int ntap = cdim >= 64 ? 1 : min(64 / cdim, taps - tap0);
+          const uint32_t full = smem_u32(&sh.tma_full[s]);
+          mbar_expect_tx(full, ntap * box + (uint32_t)T.BN * 128u);
+          for (int i = 0; i < ntap; ++i) {
+            const int tap = tap0 + i, r = tap / d.S, sx = tap % d.S;
+            const int shift = MODE == FWD ? (r - d.pad) * d.W + (sx - d.pad) : (d.pad - r) * d.W + (d.pad - sx);
+            tma_load_2d(base + s * raw_bytes + i * box, d.tma_a, c0, T.m0 + shift, full);
+          }
+          tma_load_2d(op_base + s * op_bytes + kABytes, d.tma_b, k0, T.n0, full);
+          RT(rt_b += clock64() - rt1;)
+        }
+      }
+      RT(atomicAdd(&g_tma_cycles[MODE][0], rt_a); atomicAdd(&g_tma_cycles[MODE][1], rt_b);
+         atomicAdd(&g_tma_cycles[MODE][2], (unsigned long long)g);)
+      if (!ok) { sh.abort_flag = 1; atomicExch(status, 3); }
+      // the copies of the last stages issued must land before the CTA exits
+      for (uint32_t i = g > (uint32_t)S ? g - S : 0; i < g; ++i)
+        mbar_wait_drain(smem_u32(&sh.tma_full[i % S]), (i / S) & 1);
+    }
+    __syncwarp();
+  } else if (warp < kTmaEpiWarp0) {
+    // ================================================= transform (thread = A row)
+    // Control flow is the same for every transform thread (they meet at named
+    // barrier 1): a thread whose wait fails raises the abort flag and walks
+    // the remaining stages without waiting or working.
+    const int row = threadIdx.x;
+    uint32_t g = 0;
+    bool ok = true;
+    const ConvDesc* staged = nullptr;  // instance whose scale/shift sit in shared memory
+    RT(unsigned long long rt_a = 0, rt_b = 0, rt_c = 0, rt_d = 0;)
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+      const Tile T = decode<MODE>(tab, tstart, ninst, tile);
+      const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
+      const int cdim = MODE == FWD ? d.C : d.K;
+      const bool big = cdim >= 64;                  // one tap per k-step, 64 channels
+      const int lg = 31 - __clz(big ? 64 : cdim);   // log2 of the box width
+      const bool xbf = MODE == FWD && d.x.dt == DT_BF16;
+      const bool tr = MODE == FWD && d.x.scale != nullptr;
+      if (tr && staged != T.d) {
+        // all transform threads are past the previous tile's stages
+        asm volatile("bar.sync 1, %0;" ::"r"(kTmaTransform) : "memory");
+        for (int c = row; c < cdim; c += kTmaTransform) { sh.scale[c] = __ldg(d.x.scale + c); sh.shift[c] = __ldg(d.x.shift + c); }
+        asm volatile("bar.sync 1, %0;" ::"r"(kTmaTransform) : "memory");
+        staged = T.d;
+      }
+      // this row's pixel and which of the R x S taps stay inside the image
+      const int m = T.m0 + row;
+      const bool mvalid = m < T.Mrows;
+      const int qx = m % d.W, py = (m / d.W) % d.H;
+      uint32_t tapok = 0;
+      for (int r = 0; r < d.R; ++r)
+        for (int sx = 0; sx < d.S; ++sx) {
+          const int dy = MODE == FWD ? r - d.pad : d.pad - r, dx = MODE == FWD ? sx - d.pad : d.pad - sx;
+          const bool in = py + dy >= 0 && py + dy < d.H && qx + dx >= 0 && qx + dx < d.W;
+          tapok |= (mvalid && in ? 1u : 0u) << (r * d.S + sx);
+        }
+      const int taps = d.R * d.S;
+      const int per_tap = big ? cdim / 64 : 1;      // k-steps per tap (big)
+      const int relu = tr ? d.x.relu : 0;
+      // chunk order: cc = j ^ h(row & 7), h = multiplication by x in GF(8);
+      // h(u) and h(u) ^ u are both permutations, so the raw reads (bank
+      // group cc) and the swizzled stores (group cc ^ (row & 7)) of a warp
+      // each spread over all eight bank groups
+      const int hrow = (((row & 7) << 1) & 7) ^ ((row & 4) ? 3 : 0);
+      for (int kt = 0; kt < T.nkt; ++kt, ++g) {
+        const int s = g % S;
+        RT(const unsigned long long rt0 = clock64();)
+        if (ok && !mbar_wait(smem_u32(&sh.tma_full[s]), (g / S) & 1, abort_flag)) {
+          ok = false;
+          sh.abort_flag = 1;
+        }
+        if (!ok) continue;
+        RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
+        const uint8_t* rawp = gbase + s * raw_bytes;
+        uint8_t* A = gbase + S * raw_bytes + s * op_bytes;
+        // big: tap kt / per_tap, channels cb + 8 cc; small: tap kt * (64 / cdim) + (8 cc >> lg)
+        const int tapb = big ? kt / per_tap : kt << (6 - lg);
+        const int cb = big ? (kt - tapb * per_tap) * 64 : 0;
+        // K elements of this stage the MMA reads (16-element steps)
+        const int kread = min(kBK, (T.Kt - kt * kBK + 15) & ~15);
+        TStage st{row, hrow, kread, lg, cdim, tapb, cb, tapok, taps, tr, relu};
+        if (xbf) {
+          if (big) transform_stage<true, true>(rawp, A, sh.scale, sh.shift, st);
+          else transform_stage<true, false>(rawp, A, sh.scale, sh.shift, st);
+        } else {
+          if (big) transform_stage<false, true>(rawp, A, sh.scale, sh.shift, st);
+          else transform_stage<false, false>(rawp, A, sh.scale, sh.shift, st);
+        }
+        RT(const unsigned long long rt2 = clock64(); rt_c += rt2 - rt1;)
+        fence_proxy_async();
+        RT(const unsigned long long rt3 = clock64(); rt_d += rt3 - rt2;)
+        mbar_arrive(smem_u32(&sh.op_full[s]));
+        RT(rt_b += clock64() - rt1;)
+      }
+    }
+    RT(if (threadIdx.x == 0) {
+      atomicAdd(&g_tma_cycles[MODE][3], rt_a); atomicAdd(&g_tma_cycles[MODE][4], rt_b);
+      atomicAdd(&g_tma_cycles[MODE][12], rt_c); atomicAdd(&g_tma_cycles[MODE][13], rt_d);
+    })
+    if (!ok) { sh.abort_flag = 1; atomicExch(status, 3); }
+  } else if (warp == kTmaMmaWarp) {
+    // ================================================= MMA issuer
+    if (lane == 0) {
+      uint32_t g = 0;
+      int li = 0;
+      bool ok = true;
+      bool issued = false;
+      RT(unsigned long long rt_acc = 0, rt_full = 0, rt_issue = 0;)
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++li) {
+        const Tile T = decode<MODE>(tab, tstart, ninst, tile);
+        const int b = li & 1;
+        RT(unsigned long long rt0 = clock64();)
+        if (!mbar_wait(smem_u32(&sh.tempty[b]), ((li >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
+        RT(rt_acc += clock64() - rt0;)
+        fence_after();
+        const uint32_t tacc = tmem + b * colstride;
+        const uint32_t idesc = idesc_bf16(kBM, T.BN);
+        for (int kt = 0; kt < T.nkt; ++kt, ++g) {
+          const int s = g % S;
+          RT(rt0 = clock64();)
+          if (!mbar_wait(smem_u32(&sh.op_full[s]), (g / S) & 1, abort_flag)) { ok = false; break; }
+          RT(const unsigned long long rt1 = clock64(); rt_full += rt1 - rt0;)
+          fence_after();
+          const uint32_t a_addr = op_base + s * op_bytes;
+          const uint32_t b_addr = a_addr + kABytes;
+          const int ksub = min(4, (T.Kt - kt * kBK + 15) / 16);
+          for (int kk = 0; kk < ksub; ++kk)
+            mma_bf16(tacc, sw128_desc(a_addr + kk * 32), sw128_desc(b_addr + kk * 32), idesc, (kt | kk) ? 1u : 0u);
+          issued = true;
+          mma_commit(smem_u32(&sh.op_empty[s]));
+          RT(rt_issue += clock64() - rt1;)
+        }
+        if (ok) mma_commit(smem_u32(&sh.tfull[b]));
+      }
+      RT(atomicAdd(&g_tma_cycles[MODE][5], rt_acc); atomicAdd(&g_tma_cycles[MODE][6], rt_full);
+         atomicAdd(&g_tma_cycles[MODE][7], rt_issue);)
+      if (!ok) {
+        sh.abort_flag = 1;
+        atomicExch(status, 3);
+        if (issued) {
+          mma_commit(smem_u32(&sh.drain));
+          mbar_wait_drain(smem_u32(&sh.drain), 0);
+        }
+      }
+    }
+    __syncwarp();
+  } else {
+    // ================================================= epilogue (warps 4-11)
+    const int ew = warp - kTmaEpiWarp0;   // 0..7
+    const int q = warp & 3;               // TMEM lane quarter this warp may access
+    const int chalf = ew >> 2;            // which 16-column chunks
+    int li = 0;
+    bool ok = true;
+    RT(unsigned long long rt_a = 0, rt_b = 0;)
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++li) {
+      const Tile T = decode<MODE>(tab, tstart, ninst, tile);
+      const int b = li & 1;
+      RT(const unsigned long long rt0 = clock64();)
+      bool got = mbar_wait(smem_u32(&sh.tfull[b]), (li >> 1) & 1, abort_flag);
+      RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
+      got = __all_sync(0xffffffffu, got);
+      if (lane == 0) sh.epi_ok[ew] = got ? 1 : 0;
+      asm volatile("bar.sync 2, %0;" ::"r"(kTmaEpilogue) : "memory");
+      for (int i = 0; i < 8; ++i) got = got && sh.epi_ok[i];
+      asm volatile("bar.sync 2, %0;" ::"r"(kTmaEpilogue) : "memory");
+      if (!got) { ok = false; break; }
+      fence_after();
+      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red, chalf * 16, 32, ew * 32 + lane, kTmaEpilogue);
+      fence_before();
+      mbar_arrive(smem_u32(&sh.tempty[b]));
+      RT(rt_b += clock64() - rt1;)
+    }
+    RT(if (threadIdx.x == kTmaEpiWarp0 * 32) { atomicAdd(&g_tma_cycles[MODE][8], rt_a); atomicAdd(&g_tma_cycles[MODE][9], rt_b); })
+    if (!ok) {
+      sh.abort_flag = 1;
+      atomicExch(status, 3);
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == kTmaMmaWarp) {
+    fence_after();
+    tmem_dealloc(tmem, ncols);
+  }
+  RT(if (threadIdx.x == 0) {
+    atomicAdd(&g_tma_cycles[MODE][10], clock64() - rt_start);
+    atomicAdd(&g_tma_cycles[MODE][11], 1ull);
+  })
+}
+
+__global__ void __launch_bounds__(kTmaThreads, 1) k_conv_fwd_tma(const ConvDesc* __restrict__ tab,
+                                                                 const int* __restrict__ tstart, int ninst, int total,
+                                                                 int bnmax, int esz, int32_t* status) {
+  conv_tma_body<FWD>(tab, tstart, ninst, total, bnmax, esz, status);
+}
+__global__ void __launch_bounds__(kTmaThreads, 1) k_conv_dgrad_tma(const ConvDesc* __restrict__ tab,
+                                                                   const int* __restrict__ tstart, int ninst, int total,
+                                                                   int bnmax, int esz, int32_t* status) {
+  conv_tma_body<DGRAD>(tab, tstart, ninst, total, bnmax, esz, status);
 }
 
 // one kernel name per mode (profiler filters and launch lists name the mode)
@@ -719,6 +1124,30 @@ static cudaError_t launch_mode(ConvKernel kern, const ConvDesc* tab, const int* 
   return cudaGetLastError();
 }
 
+cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax, int esz,
+                            int32_t* status, cudaStream_t st) {
+  if (total <= 0) return cudaSuccess;
+  if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || (esz != 2 && esz != 4) || (mode != 0 && mode != 1))
+    return cudaErrorInvalidValue;
+  static bool attr[2] = {false, false};
+  static int sms = 0;
+  auto kern = mode == 0 ? k_conv_fwd_tma : k_conv_dgrad_tma;
+  if (!attr[mode]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kTmaSmemBudget);
+    if (e != cudaSuccess) return e;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 148;
+    attr[mode] = true;
+  }
+  const size_t smem = tma_smem_bytes(bnmax, esz);
+  if (smem > (size_t)kTmaSmemBudget) return cudaErrorInvalidValue;
+  const int grid = total < sms ? total : sms;
+  kern<<<grid, kTmaThreads, smem, st>>>(tab, tstart, n, total, bnmax, esz, status);
+  return cudaGetLastError();
+}
+
 unsigned long long conv_tc_debug_word() {
 #ifdef PNN_DEBUG_CHECKS
   unsigned long long v = 0;
@@ -746,12 +1175,15 @@ cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
 
 #ifdef PNN_ROLE_TIMING
 // Diagnostic build only: copy (and optionally clear) the role counters
-// (3 modes x 12 counters).
+// (3 modes x 12 counters, then the TMA-fed variant's 2 modes x 16).
 extern "C" int pnn_role_cycles(unsigned long long* out, int reset) {
   cudaError_t e = cudaMemcpyFromSymbol(out, pnn::g_role_cycles, sizeof(pnn::g_role_cycles));
+  if (e == cudaSuccess) e = cudaMemcpyFromSymbol(out + 36, pnn::g_tma_cycles, sizeof(pnn::g_tma_cycles));  // 2 x 16
   if (e == cudaSuccess && reset) {
     static const unsigned long long zero[3][12] = {};
     e = cudaMemcpyToSymbol(pnn::g_role_cycles, zero, sizeof zero);
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(pnn::g_tma_cycles, zero, 2 * 12 * sizeof(unsigned long long));
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(pnn::g_tma_cycles, zero, 8 * sizeof(unsigned long long), 24 * 8);
   }
   return e == cudaSuccess ? 0 : 1;
 }

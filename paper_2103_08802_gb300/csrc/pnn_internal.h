@@ -43,6 +43,13 @@ struct ConvDesc {
   int32_t splits, pix_per_split;
   int32_t mtiles, ntiles;             // tile grid of this instance
   int32_t op_bf16;                    // round both contraction operands to bf16 (bf16 mode)
+  // TMA-fed tensor-core variant (stride 1): device addresses of two 2-D tensor
+  // maps (CUtensorMap, 128-byte aligned) -- tma_a over the A source rows
+  // [pixels][channels] (forward: x, dgrad: dy; box min(channels, 64) x 128,
+  // no swizzle), tma_b over the bf16 weight rows [N][K] (box 64 x BN,
+  // 128-byte swizzle)
+  const void* tma_a;
+  const void* tma_b;
 };
 
 // out = act( sum_i coef_i * in_i ), optional BN partials of out, NHWC [M][C].
@@ -167,6 +174,10 @@ cudaError_t launch_conv_dgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
                                  int32_t* status, cudaStream_t st);
 cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int bnmax,
                                  int32_t* status, cudaStream_t st);
+// TMA-fed stride-1 forward (mode 0) or data-gradient (mode 1) tensor-core conv;
+// esz: largest element size of the A sources of the launch (2 or 4)
+cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax, int esz,
+                            int32_t* status, cudaStream_t st);
 // record a message for pnn_last_error(NULL) and return `code`
 int set_last_error(int code, const char* msg);
 
@@ -192,7 +203,9 @@ cudaError_t launch_weight_cast(const float* in, void* out, int32_t out_dt, int64
 
 // tile geometry helpers shared by runtime and kernels
 constexpr int kEwRowsPerTile = 64;
-constexpr int kBnbRowsPerTile = 256;  // BN backward reduce/apply tiles
+constexpr int kBnbRowsPerTile = 256;  // BN backward reduce/apply tiles: at least this many rows
+// rows of a BN-backward tile for C channels: about 32K elements a CTA
+inline int bnb_rows_per_tile(int C) { return C > 0 && 32768 / C > kBnbRowsPerTile ? 32768 / C : kBnbRowsPerTile; }
 struct ConvTile { int BM, BN; };
 inline ConvTile simt_tile(int variant) {
   return variant == 0 ? ConvTile{64, 64} : (variant == 1 ? ConvTile{128, 32} : ConvTile{256, 16});

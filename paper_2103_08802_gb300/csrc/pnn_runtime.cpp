@@ -26,6 +26,9 @@
 #include "../../include/pnn.h"
 #include "pnn_internal.h"
 
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 using namespace pnn;
 
 namespace {
@@ -95,7 +98,17 @@ struct Launch {
   int aux;  // tcgen05 conv: largest N tile of the group
   double flops, bytes;  // algorithmic work of this launch
   int shape[6];         // first op: conv (C_in, C_out, k, stride, H_out, W_out); else (C, H, W, 0, 0, 0)
+  int esz = 4;          // TMA-fed conv: largest element size of the A sources
 };
+
+// The TMA-fed tensor-core conv (variant 1 of the TC forward / data-gradient
+// kinds) loads each filter tap as one [128 rows x min(channels, 64)] box:
+// stride 1, same padding, and a channel count that divides 64 or is a
+// multiple of it.
+static bool tma_shape_ok(int k, int stride, int pad, int ch) {
+  const bool geom = stride == 1 && ((k == 1 && pad == 0) || (k == 3 && pad == 1));
+  return geom && ch % 8 == 0 && (ch <= 64 ? 64 % ch == 0 : ch % 64 == 0);
+}
 
 const char* kKindName[K_NKINDS] = {"conv_fwd", "conv_dgrad", "conv_wgrad", "wgrad_reduce", "elementwise",
                                    "elementwise_bwd", "bn_finalize", "bn_bwd_reduce", "bn_bwd_finalize",
@@ -256,10 +269,12 @@ struct pnn_net {
     c.in = in; c.out = out; c.res = res; c.w = w; c.k = k; c.stride = stride; c.pad = k / 2;
     c.key[0] = key0; c.key[1] = slot;
     int M = B * P * Q;
-    if (act_dt == DT_BF16 && opt.conv_impl == 0 && iv.C % 8 == 0 && cout % 8 == 0) {
+    if (act_dt == DT_BF16 && (opt.conv_impl == 0 || opt.conv_impl == 3) && iv.C % 8 == 0 && cout % 8 == 0) {
       // tcgen05 path: 128-pixel tiles, all output channels (<= 256) per tile
       c.kind = K_CONV_FWD_TC;
-      c.variant = 0;
+      // the TMA-fed forward (eight epilogue warps) pays off when the epilogue
+      // is wide; narrow outputs keep the thread-gathered kernel
+      c.variant = opt.conv_impl == 0 && cout >= 64 && tma_shape_ok(k, stride, k / 2, iv.C) ? 1 : 0;
       c.mtiles = cdiv(M, kTcBM);
       c.ntiles = cdiv(cout, 256);
     } else {
@@ -459,6 +474,7 @@ struct pnn_net {
           const Value& iv = vals[f.in];
           if (act_dt == DT_BF16 && opt.conv_impl != 1 && iv.C % 8 == 0 && ov.C % 8 == 0 && params[f.w].off % 8 == 0) {
             dg.kind = K_DGRAD_TC;
+            dg.variant = opt.conv_impl == 0 && tma_shape_ok(f.k, f.stride, f.pad, ov.C) ? 1 : 0;
             dg.mtiles = cdiv((int64_t)B * iv.H * iv.W, kTcBM);
             dg.ntiles = cdiv(iv.C, 256);
           } else {
@@ -514,7 +530,7 @@ struct pnn_net {
         POp r;
         r.kind = K_BNB_RED; r.norm = f.norm; r.in = vv;
         r.variant = (n.C % 8 == 0 && n.C <= 2048) ? 1 : 0;  // 1: 8 channels per thread
-        r.tiles = cdiv(n.count, kBnbRowsPerTile);
+        r.tiles = cdiv(n.count, bnb_rows_per_tile(n.C));
         key(r, 0);
         new_op(L, r);
         POp fi = r;
@@ -524,7 +540,7 @@ struct pnn_net {
         new_op(L, fi);
         POp ap = r;
         ap.kind = K_BNB_APPLY;
-        ap.tiles = cdiv(n.count, kBnbRowsPerTile);
+        ap.tiles = cdiv(n.count, bnb_rows_per_tile(n.C));
         if (vals[n.h].need_grad) {
           ap.acc = grad_acc(n.h);
           ap.out = n.h;
@@ -557,6 +573,32 @@ struct pnn_net {
     for (int i = (int)fwd.size() - 1; i >= 0; --i) backward_of(bwd, fwd[i]);
   }
 
+  // 2-D tensor map over rows x inner elements (row pitch inner * element
+  // size) with box [box_rows][box_inner]; sw128: 128-byte swizzle (the MMA's
+  // K-major operand layout), else dense rows.  Out-of-range boxes read zeros.
+  int encode_map(CUtensorMap* m, const void* base, bool bf16, int64_t inner, int64_t rows, int box_inner,
+                 int box_rows, bool sw128) {
+    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    if (!encode) {
+      void* fn = nullptr;
+      cudaDriverEntryPointQueryResult q;
+      cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+      if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
+        return fail(PNN_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
+      encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    const int esz = bf16 ? 2 : 4;
+    const cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)rows};
+    const cuuint64_t pitch[1] = {(cuuint64_t)inner * esz};
+    const cuuint32_t box[2] = {(cuuint32_t)box_inner, (cuuint32_t)box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = encode(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
+                              const_cast<void*>(base), dims, pitch, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                              sw128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(PNN_ECUDA, "cuTensorMapEncodeTiled rejected a conv operand map");
+    return PNN_OK;
+  }
   size_t put_table(const void* p, size_t n) {
     size_t o = align256(host_tables.size());
     host_tables.resize(o + n);
@@ -788,7 +830,7 @@ int pnn_net::plan(const pnn_desc* d) {
   for (auto& n : norms) {
     n.part = alloc((size_t)n.tiles * n.C * 8);
     n.mean = alloc(n.C * 4); n.rstd = alloc(n.C * 4); n.scale = alloc(n.C * 4); n.shift = alloc(n.C * 4);
-    n.btiles = cdiv(n.count, kBnbRowsPerTile);
+    n.btiles = cdiv(n.count, bnb_rows_per_tile(n.C));
     n.bpart = alloc((size_t)n.btiles * n.C * 8);
     n.coef = alloc((size_t)n.C * 12);
   }
@@ -916,6 +958,26 @@ int pnn_net::build_tables() {
             c.mtiles = o.mtiles; c.ntiles = o.ntiles;
             c.op_bf16 = act_dt == DT_BF16 && ((o.kind != K_DGRAD && o.kind != K_WGRAD) || !opt.grad_fp32);
             if (o.kind == K_DGRAD_TC) c.w = (const char*)(ws + off_wt) + params[o.w].off * 2;
+            if ((o.kind == K_CONV_FWD_TC || o.kind == K_DGRAD_TC) && o.variant == 1) {
+              const bool fwd = o.kind == K_CONV_FWD_TC;
+              const int ch = fwd ? iv.C : ov.C;            // channels of the A source
+              const int ncols = fwd ? ov.C : iv.C;          // GEMM N
+              const int kt = o.k * o.k * ch;
+              const void* a_src = fwd ? c.x.ptr : (const void*)P<float>(gptr(o.out));
+              const bool a_bf16 = fwd && c.x.dt == DT_BF16;
+              const int64_t a_rows = fwd ? (int64_t)B * iv.H * iv.W : (int64_t)B * ov.H * ov.W;
+              const int bn = o.ntiles == 1 ? ((ncols + 15) & ~15) : 256;
+              CUtensorMap maps[2];
+              memset(maps, 0, sizeof maps);
+              if (ws) {
+                int r = encode_map(&maps[0], a_src, a_bf16, ch, a_rows, std::min(ch, 64), kTcBM, false);
+                if (!r) r = encode_map(&maps[1], c.w, true, kt, ncols, 64, bn, true);
+                if (r) return r;
+              }
+              const size_t mo = put(maps, sizeof maps);
+              c.tma_a = ws ? ws + tables_off + mo : nullptr;
+              c.tma_b = ws ? ws + tables_off + mo + sizeof(CUtensorMap) : nullptr;
+            }
             if (o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC) {
               c.y = ws + ov.off; c.y_dt = ov.dt;
               if (o.res >= 0) { c.res = ws + vals[o.res].off; c.res_dt = vals[o.res].dt; }
@@ -1007,7 +1069,7 @@ int pnn_net::build_tables() {
             b.dgamma = grad + params[n.gamma].off; b.dbeta = grad + params[n.beta].off;
             b.coef = P<float>(n.coef);
             b.M = n.count; b.C = n.C;
-            b.rows_per_tile = kBnbRowsPerTile; b.tiles = n.btiles;
+            b.rows_per_tile = bnb_rows_per_tile(n.C); b.tiles = n.btiles;
             if (o.kind == K_BNB_FIN) b.accumulate = o.acc_in[0];
             if (o.kind == K_BNB_APPLY) {
               b.dh = P<float>(gptr(n.h));
@@ -1057,10 +1119,16 @@ int pnn_net::build_tables() {
           L.shape[0] = vals[v].C; L.shape[1] = vals[v].H; L.shape[2] = vals[v].W;
         }
       }
+      L.esz = 2;
       for (int id : g.ops)
         if (ops[id].kind == K_CONV_FWD_TC || ops[id].kind == K_DGRAD_TC || ops[id].kind == K_WGRAD_TC) {
           const int K = ops[id].kind == K_DGRAD_TC ? vals[ops[id].in].C : vals[ops[id].out].C;
           L.aux = std::max(L.aux, ops[id].ntiles == 1 ? ((K + 15) & ~15) : 256);
+          if (ops[id].kind == K_DGRAD_TC) L.esz = 4;
+          else if (ops[id].kind == K_CONV_FWD_TC) {
+            const int src = vals[ops[id].in].virt ? vals[ops[id].in].src : ops[id].in;
+            if (vals[src].dt == DT_F32) L.esz = 4;
+          }
         }
       for (int id : g.ops) {
         const POp& o = ops[id];
@@ -1225,10 +1293,17 @@ int pnn_net::run_phase(int p) {
     switch (L.kind) {
       case K_CONV_FWD: e = launch_conv_fwd_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, stream); break;
       case K_CONV_FWD_TC:
-        e = launch_conv_fwd_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
+        e = L.variant == 1
+                ? launch_conv_tma(0, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.esz, P<int32_t>(status_off),
+                                  stream)
+                : launch_conv_fwd_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
         break;
       case K_DGRAD_TC:
-        e = launch_conv_dgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
+        e = L.variant == 1
+                ? launch_conv_tma(1, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.esz, P<int32_t>(status_off),
+                                  stream)
+                : launch_conv_dgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
+                                       stream);
         break;
       case K_WGRAD_TC:
         e = launch_conv_wgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
@@ -1782,7 +1857,7 @@ int pnn_profile_trace(pnn_net* n, int32_t max, pnn_trace* out, int32_t* count) {
     pnn_trace& r = out[i];
     float t = 0.f;
     cudaEventElapsedTime(&t, n->pev[2 * i], n->pev[2 * i + 1]);
-    r.kind = L.kind; r.phase = L.phase; r.instances = L.count; r.tiles = L.total;
+    r.kind = L.kind; r.variant = L.variant; r.phase = L.phase; r.instances = L.count; r.tiles = L.total;
     for (int j = 0; j < 6; ++j) r.shape[j] = L.shape[j];
     r.ms = t; r.flops = L.flops; r.bytes = L.bytes;
   }

@@ -54,7 +54,8 @@ class Options(C.Structure):
 
 
 class Trace(C.Structure):
-    _fields_ = [("kind", C.c_int32), ("phase", C.c_int32), ("instances", C.c_int32), ("tiles", C.c_int32),
+    _fields_ = [("kind", C.c_int32), ("variant", C.c_int32), ("phase", C.c_int32), ("instances", C.c_int32),
+                ("tiles", C.c_int32),
                 ("shape", C.c_int32 * 6), ("ms", C.c_double), ("flops", C.c_double), ("bytes", C.c_double)]
 
 
@@ -306,7 +307,7 @@ class ParaNet:
         self._check(self.lib.pnn_profile_trace(self.h, 0, None, C.byref(n)))
         buf = (Trace * max(1, n.value))()
         self._check(self.lib.pnn_profile_trace(self.h, n.value, buf, C.byref(n)))
-        return [{"kind": self.lib.pnn_kernel_kind_name(r.kind).decode(), "phase": r.phase,
+        return [{"kind": self.lib.pnn_kernel_kind_name(r.kind).decode(), "variant": r.variant, "phase": r.phase,
                  "instances": r.instances, "tiles": r.tiles, "shape": tuple(r.shape),
                  "ms": r.ms, "flops": r.flops, "bytes": r.bytes} for r in buf[:n.value]]
 

@@ -213,6 +213,40 @@ def test_tensor_core_forward_matches_cuda_core(idx):
     assert max(fwd.values()) <= 2e-2, fwd
 
 
+def _conv_variants(desc, theta, x, labels, conv_impl):
+    """Kernel variants of the tensor-core conv launches of one eager step."""
+    import torch
+    from paper_2103_08802_gb300 import pnn
+    net = pnn.ParaNet(desc, conv_impl=conv_impl)
+    net.set_params(theta)
+    net.profile(True)
+    net.forward(torch.from_numpy(x).cuda(), torch.from_numpy(labels).cuda())
+    net.backward()
+    tr = net.profile_trace()
+    net.profile(False)
+    return {(r["kind"], r["variant"]) for r in tr if r["kind"] in ("conv_fwd_tc", "conv_dgrad_tc")}
+
+
+@pytest.mark.parametrize("idx", [1, 2, 4])
+def test_tma_fed_convs_match_thread_gathered(idx):
+    """The TMA-fed stride-1 convolutions (the default) and the thread-gathered
+    tensor-core convolutions (conv_impl=3) build the same bf16 operands and
+    accumulate them in the same K order with the same epilogue: every tensor
+    of the step agrees bit for bit.  (VGG-16's 3x3 convs with 64..512
+    channels, ResNet's 1x1 and 3x3 bottleneck convs; stride-2 convs take the
+    gathered kernel on both sides.)"""
+    desc = reduced(idx)
+    onet, theta, x, labels = inputs(desc)
+    assert ("conv_fwd_tc", 1) in _conv_variants(desc, theta, x, labels, 0)
+    assert ("conv_dgrad_tc", 1) in _conv_variants(desc, theta, x, labels, 0)
+    assert all(v == 0 for _, v in _conv_variants(desc, theta, x, labels, 3))
+    a = run_gpu(desc, theta, x, labels)
+    b = run_gpu(desc, theta, x, labels, conv_impl=3)
+    keys = [k for k in a if k not in ("net", "onet")]
+    for k in keys:
+        np.testing.assert_array_equal(np.asarray(a[k]), np.asarray(b[k]), err_msg=k)
+
+
 def test_step_is_deterministic():
     desc = W.config(2, batch=4)
     onet, theta, x, labels = inputs(desc)
