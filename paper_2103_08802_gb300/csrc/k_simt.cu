@@ -551,7 +551,7 @@ __device__ __forceinline__ void ld8any(const void* base, int dt, int64_t i, floa
 
 __global__ void __launch_bounds__(256) k_bnb_reduce8(const BnBwdDesc* __restrict__ tab,
                                                      const int* __restrict__ tstart, int n) {
-  __shared__ float red[256][16];
+  __shared__ float red[16][256];  // [quantity x channel][thread]: a warp touches 32 consecutive words
   const int inst = find_instance(tstart, n, blockIdx.x);
   const BnBwdDesc d = tab[inst];
   const int tile = blockIdx.x - tstart[inst];
@@ -584,15 +584,27 @@ __global__ void __launch_bounds__(256) k_bnb_reduce8(const BnBwdDesc* __restrict
     }
   }
 #pragma unroll
-  for (int k = 0; k < 8; ++k) { red[threadIdx.x][k] = s1[k]; red[threadIdx.x][8 + k] = s2[k]; }
+  for (int k = 0; k < 8; ++k) { red[k][threadIdx.x] = s1[k]; red[8 + k][threadIdx.x] = s2[k]; }
   __syncthreads();
+  int groups = G;
+  if ((G & (G - 1)) == 0) {
+    // tree over the row groups: red[.][g * CG + cg] += red[.][(g + st) * CG + cg]
+    for (int st = G >> 1; st > 0; st >>= 1) {
+      if (g < st) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) red[k][threadIdx.x] += red[k][threadIdx.x + st * CG];
+      }
+      __syncthreads();
+    }
+    groups = 1;
+  }
   if ((int)threadIdx.x < CG) {
     float a[8], b[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) { a[k] = 0.f; b[k] = 0.f; }
-    for (int gg = 0; gg < G; ++gg)
+    for (int gg = 0; gg < groups; ++gg)
 #pragma unroll
-      for (int k = 0; k < 8; ++k) { a[k] += red[gg * CG + threadIdx.x][k]; b[k] += red[gg * CG + threadIdx.x][8 + k]; }
+      for (int k = 0; k < 8; ++k) { a[k] += red[k][gg * CG + threadIdx.x]; b[k] += red[8 + k][gg * CG + threadIdx.x]; }
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       d.part[((int64_t)tile * C + threadIdx.x * 8 + k) * 2] = a[k];

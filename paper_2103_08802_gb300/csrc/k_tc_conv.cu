@@ -116,6 +116,29 @@ __device__ __forceinline__ void act8(float* v, const float* sc, const float* sf,
   }
 }
 
+// (image, row, column) of a flattened pixel index over a rows x cols grid;
+// step() advances it by a fixed count with carries, so only the first index
+// of a run is divided
+struct Pix {
+  int nb, y, x;
+  __device__ __forceinline__ void init(int m, int rows, int cols) {
+    x = m % cols;
+    const int t = m / cols;
+    y = t % rows;
+    nb = t / rows;
+  }
+  __device__ __forceinline__ void step(int n, int rows, int cols) {
+    x += n;
+    while (x >= cols) {
+      x -= cols;
+      if (++y == rows) { y = 0; ++nb; }
+    }
+  }
+};
+// v / stride and v % stride for v >= 0 (strides 1 and 2 without a division)
+__device__ __forceinline__ int sdiv(int v, int st) { return st == 1 ? v : (st == 2 ? v >> 1 : v / st); }
+__device__ __forceinline__ int smod(int v, int st) { return st == 1 ? 0 : (st == 2 ? v & 1 : v % st); }
+
 // ---------------------------------------------------------------- gather one stage
 // The gatherers form two groups of 128 threads that fill alternating stages.
 // Each stage issues all of its global loads before it consumes any, so that a
@@ -145,22 +168,25 @@ __device__ __forceinline__ void gather_fd(const Tile& T, int kt, uint8_t* A, uin
   // phase 1: addresses and loads
   uint4 raw[8][XBF ? 1 : 2];
   unsigned have = 0;
+  const int grows = MODE == FWD ? d.P : d.H, gcols = MODE == FWD ? d.Q : d.W;
+  Pix px;
+  px.init(T.m0 + rg, grows, gcols);
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const int m = T.m0 + rg + 16 * i;
+    if (i) px.step(16, grows, gcols);
     int64_t e = 0;
     bool ok = false;
     if (MODE == FWD) {
-      const int q = m % d.Q, tmp = m / d.Q, pp = tmp % d.P, nb = tmp / d.P;
-      const int h = pp * d.stride - d.pad + r_, w = q * d.stride - d.pad + s_;
+      const int h = px.y * d.stride - d.pad + r_, w = px.x * d.stride - d.pad + s_;
       ok = h >= 0 && h < d.H && w >= 0 && w < d.W;
-      e = ((int64_t)(nb * d.H + h) * d.W + w) * d.C + c0;
+      e = ((int64_t)(px.nb * d.H + h) * d.W + w) * d.C + c0;
     } else {
-      const int w = m % d.W, tmp = m / d.W, h = tmp % d.H, nb = tmp / d.H;
-      const int pn = h + d.pad - r_, qn = w + d.pad - s_;
-      const int pp = pn / d.stride, q = qn / d.stride;
-      ok = pn >= 0 && qn >= 0 && pn % d.stride == 0 && qn % d.stride == 0 && pp < d.P && q < d.Q;
-      e = ((int64_t)(nb * d.P + pp) * d.Q + q) * d.K + c0;
+      const int pn = px.y + d.pad - r_, qn = px.x + d.pad - s_;
+      ok = pn >= 0 && qn >= 0 && smod(pn, d.stride) == 0 && smod(qn, d.stride) == 0;
+      const int pp = ok ? sdiv(pn, d.stride) : 0, q = ok ? sdiv(qn, d.stride) : 0;
+      ok = ok && pp < d.P && q < d.Q;
+      e = ((int64_t)(px.nb * d.P + pp) * d.Q + q) * d.K + c0;
     }
     ok = ok && kin && m < T.Mrows;
     if (!ok) e = 0;
@@ -277,16 +303,18 @@ __device__ __forceinline__ void gather_wgrad(const Tile& T, int kt, uint8_t* A, 
   }
   uint4 ra[8][XBF ? 1 : 2];
   unsigned have = 0;
+  Pix px;
+  px.init(pix0 + pg * 8, d.P, d.Q);
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     ra[i][0] = make_uint4(0, 0, 0, 0);
     if (!XBF) ra[i][XBF ? 0 : 1] = make_uint4(0, 0, 0, 0);
     const int pix = pix0 + pg * 8 + i;
-    const int q = pix % d.Q, tmp = pix / d.Q, pp = tmp % d.P, nb = tmp / d.P;
-    const int h = pp * d.stride + r_ - d.pad, w = q * d.stride + s_ - d.pad;
+    if (i) px.step(1, d.P, d.Q);
+    const int h = px.y * d.stride + r_ - d.pad, w = px.x * d.stride + s_ - d.pad;
     if (jin && pix < T.pend && h >= 0 && h < d.H && w >= 0 && w < d.W) {
       have |= 1u << i;
-      const int64_t e = ((int64_t)(nb * d.H + h) * d.W + w) * d.C + c0;
+      const int64_t e = ((int64_t)(px.nb * d.H + h) * d.W + w) * d.C + c0;
       const uint4* src = XBF ? reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(d.x.ptr) + e)
                              : reinterpret_cast<const uint4*>(reinterpret_cast<const float*>(d.x.ptr) + e);
       if (PNN_ALIGNED(src, 16)) {
