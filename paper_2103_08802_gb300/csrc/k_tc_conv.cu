@@ -731,9 +731,18 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
 //               16-column chunks.
 // Every wait is bounded; the producer drains its copies before the CTA exits.
 constexpr int kTmaThreads = 14 * 32;
-constexpr int kTmaTransform = 128;    // warps 0-3
-constexpr int kTmaEpiWarp0 = 4;       // warps 4-11
-constexpr int kTmaEpilogue = 256;
+// transform / epilogue split of warps 0-11 per mode: the forward and data
+// gradient have a wide epilogue (4 transform + 8 epilogue warps); the weight
+// gradient builds two transposed operands and drains a small accumulator
+// (8 transform + 4 epilogue warps)
+template <int MODE>
+struct TmaRoles {
+  static constexpr int kTransformWarps = MODE == WGRAD ? 8 : 4;
+  static constexpr int kEpiWarps = 12 - kTransformWarps;
+  static constexpr int kTransform = 32 * kTransformWarps;
+  static constexpr int kEpilogue = 32 * kEpiWarps;
+  static constexpr int kEpiWarp0 = kTransformWarps;
+};
 constexpr int kTmaMmaWarp = 12;
 constexpr int kTmaProducerWarp = 13;
 constexpr int kTmaMaxStages = 8;
@@ -746,7 +755,7 @@ constexpr int kTmaSmemBudget = 227 * 1024;
 // transform wait for TMA data, [4] transform work (thread 0), [5] MMA wait
 // for a free accumulator, [6] MMA wait for operands, [7] MMA issue, [8]
 // epilogue wait, [9] epilogue work, [10] CTA lifetime, [11] CTAs.
-__device__ unsigned long long g_tma_cycles[2][16];
+__device__ unsigned long long g_tma_cycles[3][16];
 #endif
 
 struct TmaShared {
@@ -764,15 +773,15 @@ struct TmaShared {
   float shift[kTmaMaxC];
 };
 
-__host__ __device__ constexpr int tma_raw_bytes(int esz) { return kBM * kBK * esz; }
+// raw_bytes: one stage's raw slot (a multiple of 1024), per launch
 __host__ __device__ constexpr int tma_op_bytes(int bnmax) { return kABytes + bnmax * 128; }
-__host__ __device__ inline int tma_stages(int bnmax, int esz) {
+__host__ __device__ inline int tma_stages(int bnmax, int raw_bytes) {
   const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared);
-  int s = avail / (tma_raw_bytes(esz) + tma_op_bytes(bnmax));
+  int s = avail / (raw_bytes + tma_op_bytes(bnmax));
   return s < 2 ? 2 : (s > kTmaMaxStages ? kTmaMaxStages : s);
 }
-__host__ __device__ inline size_t tma_smem_bytes(int bnmax, int esz) {
-  return 1024 + (size_t)tma_stages(bnmax, esz) * (tma_raw_bytes(esz) + tma_op_bytes(bnmax)) + sizeof(TmaShared);
+__host__ __device__ inline size_t tma_smem_bytes(int bnmax, int raw_bytes) {
+  return 1024 + (size_t)tma_stages(bnmax, raw_bytes) * (raw_bytes + tma_op_bytes(bnmax)) + sizeof(TmaShared);
 }
 
 // One transform thread's share of a stage: row `row` of the A operand, its
@@ -849,15 +858,136 @@ __device__ __forceinline__ void transform_stage(const uint8_t* __restrict__ rawp
   }
 }
 
+// Weight-gradient transform of one tile (256 threads): thread u < 128 builds A unit u (rows
+// jg*8 .. jg*8+7 = (tap, c .. c+7)) from the halo box -- BN scale/shift +
+// ReLU of the producing layer, zero outside the image or the split -- and
+// thread 128 + u, u < BN, B unit u (k_out kg*8 .. +7) from the gradient box, both for the
+// k-step pixels pg, pg+8, .., pg+56, 8x8-transposed into K positions 8*pg ..
+// 8*pg+7 of the K(pixel)-major operands.  The contraction sums over pixels,
+// so a permutation of K shared by A and B leaves it unchanged; this one makes
+// the lanes of a warp read consecutive raw rows.
+template <typename Sh>
+__device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDesc& d, int u, bool tr, uint32_t& g,
+                                                     bool& ok, int S, int raw_bytes, int op_bytes, uint8_t* gbase,
+                                                     Sh& sh RT(, unsigned long long& rt_a, unsigned long long& rt_b)) {
+  const bool xbf = d.x.dt == DT_BF16;
+  const WgBoxes bx = wg_boxes(d.C, d.K, d.W, d.pad, xbf);
+  const int cbase = d.C <= 64 ? 0 : T.m0 % d.C;
+  // threads 0-127 build the A units, threads 128-255 the B units
+  const bool aside = u < 128;
+  if (!aside) u -= 128;
+  const int jg = u >> 3, pg = u & 7;
+  const int j0 = T.m0 + jg * 8;
+  const bool jin = aside && j0 < T.Mrows;
+  const int tap = j0 / d.C, c0 = j0 - tap * d.C;
+  const int r = tap / d.S, sx = tap - r * d.S;
+  const int hoff = r * d.W + sx;                // halo row of pixel 0 for this tap
+  const int dyr = r - d.pad, dxs = sx - d.pad;
+  const int cl = c0 - cbase;                    // channel within the box
+  const bool bunit = !aside && u < T.BN;
+  const int kg = u >> 3;
+  const bool bcols = bunit && T.n0 + kg * 8 < d.K;
+  const int relu = tr ? d.x.relu : 0;
+  // this unit's 8 channels of the producing layer's BN scale/shift (fixed for the tile)
+  float sc[8], sf[8];
+  if (jin && tr) {
+    const float4 s0 = *reinterpret_cast<const float4*>(&sh.scale[c0]);
+    const float4 s1 = *reinterpret_cast<const float4*>(&sh.scale[c0 + 4]);
+    const float4 f0 = *reinterpret_cast<const float4*>(&sh.shift[c0]);
+    const float4 f1 = *reinterpret_cast<const float4*>(&sh.shift[c0 + 4]);
+    sc[0] = s0.x; sc[1] = s0.y; sc[2] = s0.z; sc[3] = s0.w; sc[4] = s1.x; sc[5] = s1.y; sc[6] = s1.z; sc[7] = s1.w;
+    sf[0] = f0.x; sf[1] = f0.y; sf[2] = f0.z; sf[3] = f0.w; sf[4] = f1.x; sf[5] = f1.y; sf[6] = f1.z; sf[7] = f1.w;
+  }
+  for (int kt = 0; kt < T.nkt; ++kt, ++g) {
+    const int s = g % S;
+    RT(const unsigned long long rt0 = clock64();)
+    if (ok && !mbar_wait(smem_u32(&sh.tma_full[s]), (g / S) & 1, &sh.abort_flag)) {
+      ok = false;
+      sh.abort_flag = 1;
+    }
+    if (!ok) continue;
+    RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
+    const uint8_t* __restrict__ rawx = gbase + s * raw_bytes;
+    const uint8_t* __restrict__ rawy = rawx + bx.yoff;
+    uint8_t* __restrict__ A = gbase + S * raw_bytes + s * op_bytes;
+    uint8_t* __restrict__ Bt = A + kABytes;
+    const int pix0 = T.pbeg + kt * kBK;
+    // validity of the unit's 8 pixels (inside the split; tap inside the image)
+    unsigned pin = 0, xin = 0;
+    {
+      Pix px;
+      px.init(pix0 + pg, d.P, d.Q);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        if (i) px.step(8, d.P, d.Q);
+        const bool in = pix0 + pg + 8 * i < T.pend;
+        pin |= (in ? 1u : 0u) << i;
+        const bool ii = in && px.y + dyr >= 0 && px.y + dyr < d.H && px.x + dxs >= 0 && px.x + dxs < d.W;
+        xin |= (ii ? 1u : 0u) << i;
+      }
+    }
+    if (!jin) xin = 0;
+    // A
+    if (aside) {
+      uint4 in[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int row = pg + 8 * i + hoff;
+        float v[8];
+        if (xbf) {
+          const uint4 w = *reinterpret_cast<const uint4*>(rawx + (row * bx.cwx + cl) * 2);
+          const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&w);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(hh[e]);
+            v[2 * e] = f.x;
+            v[2 * e + 1] = f.y;
+          }
+        } else {
+          const float4 a = *reinterpret_cast<const float4*>(rawx + (row * bx.cwx + cl) * 4);
+          const float4 b = *reinterpret_cast<const float4*>(rawx + (row * bx.cwx + cl) * 4 + 16);
+          v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+          v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+        }
+        if (tr) act8(v, sc, sf, relu);
+        in[i] = (xin >> i) & 1 ? pack8(v) : make_uint4(0, 0, 0, 0);
+      }
+      uint4 out[8];
+      transpose8(in, out);
+#pragma unroll
+      for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(A + swz(jg * 8 + c, pg)) = out[c];
+    }
+    // B
+    if (bunit) {
+      uint4 in[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int row = pg + 8 * i;
+        const float* src = reinterpret_cast<const float*>(rawy) + row * d.K + kg * 8;
+        const float4 a = *reinterpret_cast<const float4*>(src);
+        const float4 b = *reinterpret_cast<const float4*>(src + 4);
+        const float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        in[i] = bcols && ((pin >> i) & 1) ? pack8(v) : make_uint4(0, 0, 0, 0);
+      }
+      uint4 out[8];
+      transpose8(in, out);
+#pragma unroll
+      for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(Bt + swz(kg * 8 + c, pg)) = out[c];
+    }
+    fence_proxy_async();
+    mbar_arrive(smem_u32(&sh.op_full[s]));
+    RT(rt_b += clock64() - rt1;)
+  }
+}
+
 template <int MODE>
 __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, const int* __restrict__ tstart,
-                                              int ninst, int total, int bnmax, int esz_max, int32_t* status) {
+                                              int ninst, int total, int bnmax, int raw_bytes, int32_t* status) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw0 = smem_u32(smem_raw);
   const uint32_t base = (raw0 + 1023u) & ~1023u;
   uint8_t* const gbase = smem_raw + (base - raw0);
-  const int S = tma_stages(bnmax, esz_max);
-  const int raw_bytes = tma_raw_bytes(esz_max);
+  const int S = tma_stages(bnmax, raw_bytes);
   const int op_bytes = tma_op_bytes(bnmax);
   const uint32_t op_base = base + S * raw_bytes;
   RT(const unsigned long long rt_start = clock64();)
@@ -870,12 +1000,12 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_u32(&sh.tma_full[s]), 1);
-      mbar_init(smem_u32(&sh.op_full[s]), kTmaTransform);
+      mbar_init(smem_u32(&sh.op_full[s]), TmaRoles<MODE>::kTransform);
       mbar_init(smem_u32(&sh.op_empty[s]), 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(smem_u32(&sh.tfull[b]), 1);
-      mbar_init(smem_u32(&sh.tempty[b]), kTmaEpilogue);
+      mbar_init(smem_u32(&sh.tempty[b]), TmaRoles<MODE>::kEpilogue);
     }
     mbar_init(smem_u32(&sh.drain), 1);
     sh.abort_flag = 0;
@@ -897,6 +1027,25 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
         const Tile T = decode<MODE>(tab, tstart, ninst, tile);
         const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
+        if constexpr (MODE == WGRAD) {
+          // per k-step: the activation rows of all taps (a halo of pad*W+pad
+          // rows each side) and the gradient rows of the k-step's 64 pixels
+          const WgBoxes bx = wg_boxes(d.C, d.K, d.W, d.pad, d.x.dt == DT_BF16);
+          const int cbase = d.C <= 64 ? 0 : T.m0 % d.C;
+          for (int kt = 0; kt < T.nkt; ++kt, ++g) {
+            const int s = g % S;
+            RT(const unsigned long long rt0 = clock64();)
+            if (!mbar_wait(smem_u32(&sh.op_empty[s]), ((g / S) & 1) ^ 1, abort_flag)) { ok = false; break; }
+            RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
+            const int pix0 = T.pbeg + kt * kBK;
+            const uint32_t full = smem_u32(&sh.tma_full[s]);
+            mbar_expect_tx(full, (uint32_t)(bx.xbytes + bx.ybytes));
+            tma_load_2d(base + s * raw_bytes, d.tma_a, cbase, pix0 - bx.halo, full);
+            tma_load_2d(base + s * raw_bytes + bx.yoff, d.tma_b, 0, pix0, full);
+            RT(rt_b += clock64() - rt1;)
+          }
+          continue;
+        }
         const int cdim = MODE == FWD ? d.C : d.K;
         const int cw = cdim < 64 ? cdim : 64;
         const int esz = (MODE == FWD && d.x.dt == DT_BF16) ? 2 : 4;
@@ -929,7 +1078,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
         mbar_wait_drain(smem_u32(&sh.tma_full[i % S]), (i / S) & 1);
     }
     __syncwarp();
-  } else if (warp < kTmaEpiWarp0) {
+  } else if (warp < TmaRoles<MODE>::kEpiWarp0) {
     // ================================================= transform (thread = A row)
     // Control flow is the same for every transform thread (they meet at named
     // barrier 1): a thread whose wait fails raises the abort flag and walks
@@ -946,13 +1095,20 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       const bool big = cdim >= 64;                  // one tap per k-step, 64 channels
       const int lg = 31 - __clz(big ? 64 : cdim);   // log2 of the box width
       const bool xbf = MODE == FWD && d.x.dt == DT_BF16;
-      const bool tr = MODE == FWD && d.x.scale != nullptr;
+      const bool tr = MODE != DGRAD && d.x.scale != nullptr;
       if (tr && staged != T.d) {
         // all transform threads are past the previous tile's stages
-        asm volatile("bar.sync 1, %0;" ::"r"(kTmaTransform) : "memory");
-        for (int c = row; c < cdim; c += kTmaTransform) { sh.scale[c] = __ldg(d.x.scale + c); sh.shift[c] = __ldg(d.x.shift + c); }
-        asm volatile("bar.sync 1, %0;" ::"r"(kTmaTransform) : "memory");
+        asm volatile("bar.sync 1, %0;" ::"r"(TmaRoles<MODE>::kTransform) : "memory");
+        for (int c = row; c < d.C; c += TmaRoles<MODE>::kTransform) {
+          sh.scale[c] = __ldg(d.x.scale + c);
+          sh.shift[c] = __ldg(d.x.shift + c);
+        }
+        asm volatile("bar.sync 1, %0;" ::"r"(TmaRoles<MODE>::kTransform) : "memory");
         staged = T.d;
+      }
+      if constexpr (MODE == WGRAD) {
+        wgrad_transform_tile(T, d, row, tr, g, ok, S, raw_bytes, op_bytes, gbase, sh RT(, rt_a, rt_b));
+        continue;
       }
       // this row's pixel and which of the R x S taps stay inside the image
       const int m = T.m0 + row;
@@ -1034,7 +1190,9 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
           fence_after();
           const uint32_t a_addr = op_base + s * op_bytes;
           const uint32_t b_addr = a_addr + kABytes;
-          const int ksub = min(4, (T.Kt - kt * kBK + 15) / 16);
+          // (weight gradient: pixels sit at permuted K positions, all 64 are read)
+          const int krem = MODE == WGRAD ? kBK : T.Kt - kt * kBK;
+          const int ksub = min(4, (krem + 15) / 16);
           for (int kk = 0; kk < ksub; ++kk)
             mma_bf16(tacc, sw128_desc(a_addr + kk * 32), sw128_desc(b_addr + kk * 32), idesc, (kt | kk) ? 1u : 0u);
           issued = true;
@@ -1057,9 +1215,11 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     __syncwarp();
   } else {
     // ================================================= epilogue (warps 4-11)
-    const int ew = warp - kTmaEpiWarp0;   // 0..7
+    using R = TmaRoles<MODE>;
+    const int ew = warp - R::kEpiWarp0;   // 0 .. kEpiWarps-1
     const int q = warp & 3;               // TMEM lane quarter this warp may access
-    const int chalf = ew >> 2;            // which 16-column chunks
+    const int chalf = ew >> 2;            // which 16-column chunks (two warps a quarter)
+    constexpr int jstep = 16 * (R::kEpiWarps / 4);
     int li = 0;
     bool ok = true;
     RT(unsigned long long rt_a = 0, rt_b = 0;)
@@ -1071,17 +1231,17 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
       got = __all_sync(0xffffffffu, got);
       if (lane == 0) sh.epi_ok[ew] = got ? 1 : 0;
-      asm volatile("bar.sync 2, %0;" ::"r"(kTmaEpilogue) : "memory");
-      for (int i = 0; i < 8; ++i) got = got && sh.epi_ok[i];
-      asm volatile("bar.sync 2, %0;" ::"r"(kTmaEpilogue) : "memory");
+      asm volatile("bar.sync 2, %0;" ::"r"(R::kEpilogue) : "memory");
+      for (int i = 0; i < R::kEpiWarps; ++i) got = got && sh.epi_ok[i];
+      asm volatile("bar.sync 2, %0;" ::"r"(R::kEpilogue) : "memory");
       if (!got) { ok = false; break; }
       fence_after();
-      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red, chalf * 16, 32, ew * 32 + lane, kTmaEpilogue);
+      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red, chalf * 16, jstep, ew * 32 + lane, R::kEpilogue);
       fence_before();
       mbar_arrive(smem_u32(&sh.tempty[b]));
       RT(rt_b += clock64() - rt1;)
     }
-    RT(if (threadIdx.x == kTmaEpiWarp0 * 32) { atomicAdd(&g_tma_cycles[MODE][8], rt_a); atomicAdd(&g_tma_cycles[MODE][9], rt_b); })
+    RT(if (threadIdx.x == R::kEpiWarp0 * 32) { atomicAdd(&g_tma_cycles[MODE][8], rt_a); atomicAdd(&g_tma_cycles[MODE][9], rt_b); })
     if (!ok) {
       sh.abort_flag = 1;
       atomicExch(status, 3);
@@ -1101,13 +1261,18 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
 
 __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_fwd_tma(const ConvDesc* __restrict__ tab,
                                                                  const int* __restrict__ tstart, int ninst, int total,
-                                                                 int bnmax, int esz, int32_t* status) {
-  conv_tma_body<FWD>(tab, tstart, ninst, total, bnmax, esz, status);
+                                                                 int bnmax, int raw_bytes, int32_t* status) {
+  conv_tma_body<FWD>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
 __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_dgrad_tma(const ConvDesc* __restrict__ tab,
                                                                    const int* __restrict__ tstart, int ninst, int total,
-                                                                   int bnmax, int esz, int32_t* status) {
-  conv_tma_body<DGRAD>(tab, tstart, ninst, total, bnmax, esz, status);
+                                                                   int bnmax, int raw_bytes, int32_t* status) {
+  conv_tma_body<DGRAD>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+}
+__global__ void __launch_bounds__(kTmaThreads, 1) k_conv_wgrad_tma(const ConvDesc* __restrict__ tab,
+                                                                   const int* __restrict__ tstart, int ninst, int total,
+                                                                   int bnmax, int raw_bytes, int32_t* status) {
+  conv_tma_body<WGRAD>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
 
 // one kernel name per mode (profiler filters and launch lists name the mode)
@@ -1152,14 +1317,19 @@ static cudaError_t launch_mode(ConvKernel kern, const ConvDesc* tab, const int* 
   return cudaGetLastError();
 }
 
-cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax, int esz,
-                            int32_t* status, cudaStream_t st) {
+bool conv_tma_fits(int bnmax, int raw_bytes) {
+  const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared);
+  return avail / (raw_bytes + tma_op_bytes(bnmax)) >= 2;
+}
+
+cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
+                            int raw_bytes, int32_t* status, cudaStream_t st) {
   if (total <= 0) return cudaSuccess;
-  if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || (esz != 2 && esz != 4) || (mode != 0 && mode != 1))
+  if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || raw_bytes <= 0 || (raw_bytes & 1023) || mode < 0 || mode > 2)
     return cudaErrorInvalidValue;
-  static bool attr[2] = {false, false};
+  static bool attr[3] = {false, false, false};
   static int sms = 0;
-  auto kern = mode == 0 ? k_conv_fwd_tma : k_conv_dgrad_tma;
+  auto kern = mode == 0 ? k_conv_fwd_tma : (mode == 1 ? k_conv_dgrad_tma : k_conv_wgrad_tma);
   if (!attr[mode]) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kTmaSmemBudget);
     if (e != cudaSuccess) return e;
@@ -1169,10 +1339,10 @@ cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, in
     if (sms <= 0) sms = 148;
     attr[mode] = true;
   }
-  const size_t smem = tma_smem_bytes(bnmax, esz);
+  const size_t smem = tma_smem_bytes(bnmax, raw_bytes);
   if (smem > (size_t)kTmaSmemBudget) return cudaErrorInvalidValue;
   const int grid = total < sms ? total : sms;
-  kern<<<grid, kTmaThreads, smem, st>>>(tab, tstart, n, total, bnmax, esz, status);
+  kern<<<grid, kTmaThreads, smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, status);
   return cudaGetLastError();
 }
 
@@ -1203,15 +1373,15 @@ cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
 
 #ifdef PNN_ROLE_TIMING
 // Diagnostic build only: copy (and optionally clear) the role counters
-// (3 modes x 12 counters, then the TMA-fed variant's 2 modes x 16).
+// (3 modes x 12 counters, then the TMA-fed variant's 3 modes x 16).
 extern "C" int pnn_role_cycles(unsigned long long* out, int reset) {
   cudaError_t e = cudaMemcpyFromSymbol(out, pnn::g_role_cycles, sizeof(pnn::g_role_cycles));
-  if (e == cudaSuccess) e = cudaMemcpyFromSymbol(out + 36, pnn::g_tma_cycles, sizeof(pnn::g_tma_cycles));  // 2 x 16
+  if (e == cudaSuccess) e = cudaMemcpyFromSymbol(out + 36, pnn::g_tma_cycles, sizeof(pnn::g_tma_cycles));  // 3 x 16
   if (e == cudaSuccess && reset) {
     static const unsigned long long zero[3][12] = {};
     e = cudaMemcpyToSymbol(pnn::g_role_cycles, zero, sizeof zero);
-    if (e == cudaSuccess) e = cudaMemcpyToSymbol(pnn::g_tma_cycles, zero, 2 * 12 * sizeof(unsigned long long));
-    if (e == cudaSuccess) e = cudaMemcpyToSymbol(pnn::g_tma_cycles, zero, 8 * sizeof(unsigned long long), 24 * 8);
+    for (int part = 0; part < 2 && e == cudaSuccess; ++part)
+      e = cudaMemcpyToSymbol(pnn::g_tma_cycles, zero, 24 * sizeof(unsigned long long), part * 24 * 8);
   }
   return e == cudaSuccess ? 0 : 1;
 }

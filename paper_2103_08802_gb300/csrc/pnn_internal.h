@@ -174,10 +174,13 @@ cudaError_t launch_conv_dgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
                                  int32_t* status, cudaStream_t st);
 cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int bnmax,
                                  int32_t* status, cudaStream_t st);
-// TMA-fed stride-1 forward (mode 0) or data-gradient (mode 1) tensor-core conv;
-// esz: largest element size of the A sources of the launch (2 or 4)
-cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax, int esz,
-                            int32_t* status, cudaStream_t st);
+// TMA-fed stride-1 forward (mode 0), data-gradient (mode 1) or weight-gradient
+// (mode 2) tensor-core conv; raw_bytes: one pipeline stage's raw slot (the
+// largest over the launch's instances, a multiple of 1024)
+cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
+                            int raw_bytes, int32_t* status, cudaStream_t st);
+// whether the TMA-fed kernel holds at least two stages of this size
+bool conv_tma_fits(int bnmax, int raw_bytes);
 // record a message for pnn_last_error(NULL) and return `code`
 int set_last_error(int code, const char* msg);
 
@@ -203,6 +206,30 @@ cudaError_t launch_weight_cast(const float* in, void* out, int32_t out_dt, int64
 
 // tile geometry helpers shared by runtime and kernels
 constexpr int kEwRowsPerTile = 64;
+#ifdef __CUDACC__
+#define PNN_HD __host__ __device__
+#else
+#define PNN_HD
+#endif
+// TMA-fed weight gradient: the two boxes of a k-step (64 pixels) -- the
+// activation rows of every tap (halo of pad*W + pad rows each side) x cwx
+// channels, and the output-gradient rows x K -- and their raw-slot offsets
+struct WgBoxes {
+  int halo, hrows, cwx, escx, xbytes, yoff, ybytes;
+};
+PNN_HD inline WgBoxes wg_boxes(int C, int K, int W, int pad, bool xbf) {
+  WgBoxes b;
+  b.halo = pad * W + pad;
+  b.hrows = 64 + 2 * b.halo;
+  b.cwx = C <= 64 ? C : 128;
+  b.escx = xbf ? 2 : 4;
+  b.xbytes = b.hrows * b.cwx * b.escx;
+  b.yoff = (b.xbytes + 127) & ~127;
+  b.ybytes = 64 * K * 4;
+  return b;
+}
+PNN_HD inline int wg_raw_bytes(const WgBoxes& b) { return (b.yoff + b.ybytes + 1023) & ~1023; }
+
 constexpr int kBnbRowsPerTile = 256;  // BN backward reduce/apply tiles: at least this many rows
 // rows of a BN-backward tile for C channels: about 32K elements a CTA
 inline int bnb_rows_per_tile(int C) { return C > 0 && 32768 / C > kBnbRowsPerTile ? 32768 / C : kBnbRowsPerTile; }

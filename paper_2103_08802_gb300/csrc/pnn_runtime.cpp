@@ -99,6 +99,7 @@ struct Launch {
   double flops, bytes;  // algorithmic work of this launch
   int shape[6];         // first op: conv (C_in, C_out, k, stride, H_out, W_out); else (C, H, W, 0, 0, 0)
   int esz = 4;          // TMA-fed conv: largest element size of the A sources
+  int raw = 0;          // TMA-fed conv: raw slot bytes of one stage
 };
 
 // The TMA-fed tensor-core conv (variant 1 of the TC forward / data-gradient
@@ -108,6 +109,18 @@ struct Launch {
 static bool tma_shape_ok(int k, int stride, int pad, int ch) {
   const bool geom = stride == 1 && ((k == 1 && pad == 0) || (k == 3 && pad == 1));
   return geom && ch % 8 == 0 && (ch <= 64 ? 64 % ch == 0 : ch % 64 == 0);
+}
+
+// The TMA-fed weight gradient loads a k-step's activation rows for all taps
+// as one halo box and the output-gradient rows as another: channels 8..64
+// (dividing 64) or multiples of 128 up to 512, at most 128 output channels
+// (one N tile), a halo of at most 256 rows, and two stages in shared memory.
+static bool tma_wgrad_ok(int k, int stride, int pad, int C, int K, int W, bool xbf) {
+  if (!(stride == 1 && ((k == 1 && pad == 0) || (k == 3 && pad == 1)))) return false;
+  if (!(C % 8 == 0 && ((C <= 64 && 64 % C == 0) || (C % 128 == 0 && C <= 512)))) return false;
+  if (K % 8 != 0 || K > 128) return false;
+  const WgBoxes b = wg_boxes(C, K, W, pad, xbf);
+  return b.hrows <= 256 && conv_tma_fits(128, wg_raw_bytes(b));
 }
 
 const char* kKindName[K_NKINDS] = {"conv_fwd", "conv_dgrad", "conv_wgrad", "wgrad_reduce", "elementwise",
@@ -447,6 +460,13 @@ struct pnn_net {
         if (tc_ok) {
           // tensor cores: rows (r,s,c) in 128-row tiles, all k_out per tile, pixels split across CTAs
           wg.kind = K_WGRAD_TC;
+          {
+            const int src = vals[f.in].virt ? vals[f.in].src : f.in;
+            wg.variant = opt.conv_impl == 0 && tma_wgrad_ok(f.k, f.stride, f.pad, vals[f.in].C, ov.C, vals[f.in].W,
+                                                             vals[src].dt == DT_BF16)
+                             ? 1
+                             : 0;
+          }
           wg.mtiles = cdiv(RSC, kTcBM);
           wg.ntiles = cdiv(ov.C, 256);
           pix_align = 64;
@@ -978,6 +998,22 @@ int pnn_net::build_tables() {
               c.tma_a = ws ? ws + tables_off + mo : nullptr;
               c.tma_b = ws ? ws + tables_off + mo + sizeof(CUtensorMap) : nullptr;
             }
+            if (o.kind == K_WGRAD_TC && o.variant == 1) {
+              // activation halo box [hrows][cwx] (its dtype), gradient box [64][K] fp32
+              const WgBoxes bx = wg_boxes(iv.C, ov.C, iv.W, o.pad, c.x.dt == DT_BF16);
+              CUtensorMap maps[2];
+              memset(maps, 0, sizeof maps);
+              if (ws) {
+                int r = encode_map(&maps[0], c.x.ptr, c.x.dt == DT_BF16, iv.C, (int64_t)B * iv.H * iv.W, bx.cwx,
+                                   bx.hrows, false);
+                if (!r) r = encode_map(&maps[1], P<float>(gptr(o.out)), false, ov.C, (int64_t)B * ov.H * ov.W, ov.C,
+                                       64, false);
+                if (r) return r;
+              }
+              const size_t mo = put(maps, sizeof maps);
+              c.tma_a = ws ? ws + tables_off + mo : nullptr;
+              c.tma_b = ws ? ws + tables_off + mo + sizeof(CUtensorMap) : nullptr;
+            }
             if (o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC) {
               c.y = ws + ov.off; c.y_dt = ov.dt;
               if (o.res >= 0) { c.res = ws + vals[o.res].off; c.res_dt = vals[o.res].dt; }
@@ -1128,8 +1164,14 @@ int pnn_net::build_tables() {
           else if (ops[id].kind == K_CONV_FWD_TC) {
             const int src = vals[ops[id].in].virt ? vals[ops[id].in].src : ops[id].in;
             if (vals[src].dt == DT_F32) L.esz = 4;
+          } else if (ops[id].variant == 1) {
+            const int src = vals[ops[id].in].virt ? vals[ops[id].in].src : ops[id].in;
+            const WgBoxes b = wg_boxes(vals[ops[id].in].C, vals[ops[id].out].C, vals[ops[id].in].W, ops[id].pad,
+                                       vals[src].dt == DT_BF16);
+            L.raw = std::max(L.raw, wg_raw_bytes(b));
           }
         }
+      if (g.kind == K_CONV_FWD_TC || g.kind == K_DGRAD_TC) L.raw = kTcBM * 64 * L.esz;
       for (int id : g.ops) {
         const POp& o = ops[id];
         auto esz = [&](int v) { return vals[v].virt ? (vals[vals[v].src].dt == DT_F32 ? 4.0 : 2.0) : (vals[v].dt == DT_F32 ? 4.0 : 2.0); };
@@ -1294,19 +1336,23 @@ int pnn_net::run_phase(int p) {
       case K_CONV_FWD: e = launch_conv_fwd_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, stream); break;
       case K_CONV_FWD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(0, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.esz, P<int32_t>(status_off),
+                ? launch_conv_tma(0, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
                                   stream)
                 : launch_conv_fwd_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
         break;
       case K_DGRAD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(1, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.esz, P<int32_t>(status_off),
+                ? launch_conv_tma(1, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
                                   stream)
                 : launch_conv_dgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
                                        stream);
         break;
       case K_WGRAD_TC:
-        e = launch_conv_wgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
+        e = L.variant == 1
+                ? launch_conv_tma(2, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
+                                  stream)
+                : launch_conv_wgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
+                                       stream);
         break;
       case K_DGRAD: e = launch_conv_dgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, stream); break;
       case K_WGRAD: e = launch_conv_wgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, stream); break;

@@ -224,27 +224,38 @@ def _conv_variants(desc, theta, x, labels, conv_impl):
     net.backward()
     tr = net.profile_trace()
     net.profile(False)
-    return {(r["kind"], r["variant"]) for r in tr if r["kind"] in ("conv_fwd_tc", "conv_dgrad_tc")}
+    return {(r["kind"], r["variant"]) for r in tr if r["kind"] in ("conv_fwd_tc", "conv_dgrad_tc", "conv_wgrad_tc")}
 
 
 @pytest.mark.parametrize("idx", [1, 2, 4])
 def test_tma_fed_convs_match_thread_gathered(idx):
     """The TMA-fed stride-1 convolutions (the default) and the thread-gathered
-    tensor-core convolutions (conv_impl=3) build the same bf16 operands and
-    accumulate them in the same K order with the same epilogue: every tensor
-    of the step agrees bit for bit.  (VGG-16's 3x3 convs with 64..512
-    channels, ResNet's 1x1 and 3x3 bottleneck convs; stride-2 convs take the
-    gathered kernel on both sides.)"""
+    tensor-core convolutions (conv_impl=3) build the same bf16 operands.  The
+    forward and data-gradient kernels also accumulate them in the same K order
+    with the same epilogue, so every activation, correction tensor, D_j and
+    the loss agree bit for bit.  The TMA-fed weight gradient sums the pixels
+    of each 64-pixel k-step in a permuted order, so weight gradients (and the
+    SGD update built on them) agree to fp32 reordering error: 1e-5 of the
+    largest element.  (VGG-16's 3x3 convs with 64..512 channels, ResNet's 1x1
+    and 3x3 bottleneck convs; stride-2 convs take the gathered kernel on both
+    sides.)"""
     desc = reduced(idx)
     onet, theta, x, labels = inputs(desc)
-    assert ("conv_fwd_tc", 1) in _conv_variants(desc, theta, x, labels, 0)
-    assert ("conv_dgrad_tc", 1) in _conv_variants(desc, theta, x, labels, 0)
+    tma = _conv_variants(desc, theta, x, labels, 0)
+    assert ("conv_fwd_tc", 1) in tma and ("conv_dgrad_tc", 1) in tma and ("conv_wgrad_tc", 1) in tma, tma
     assert all(v == 0 for _, v in _conv_variants(desc, theta, x, labels, 3))
     a = run_gpu(desc, theta, x, labels)
     b = run_gpu(desc, theta, x, labels, conv_impl=3)
-    keys = [k for k in a if k not in ("net", "onet")]
-    for k in keys:
-        np.testing.assert_array_equal(np.asarray(a[k]), np.asarray(b[k]), err_msg=k)
+    reordered = ("grad", "theta_new", "momentum")
+    for k in a:
+        if k in ("net", "onet"):
+            continue
+        ak, bk = np.asarray(a[k]), np.asarray(b[k])
+        if k in reordered:
+            err = np.abs(ak - bk).max() / max(np.abs(bk).max(), 1e-30)
+            assert err <= 1e-5, (k, err)
+        else:
+            np.testing.assert_array_equal(ak, bk, err_msg=k)
 
 
 def test_step_is_deterministic():
