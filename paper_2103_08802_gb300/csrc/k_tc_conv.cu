@@ -50,6 +50,12 @@ constexpr int kThreads = 13 * 32;
 enum { FWD = 0, DGRAD = 1, WGRAD = 2 };
 
 #ifdef PNN_ROLE_TIMING
+// Diagnostic build only: forward epilogue phases (cycles, summed over the
+// first thread of each epilogue warp): TMEM load, residual + store, column
+// sums, statistics barrier + write; [4] chunks.
+__device__ unsigned long long g_epi_cycles[6];
+#endif
+#ifdef PNN_ROLE_TIMING
 // Diagnostic build only: SM cycles each role spends waiting and working,
 // summed over CTAs, per mode: [0] gather wait for a free stage, [1] gather
 // work, [2] stages gathered (both counted for thread 0 of each group), [3]
@@ -424,9 +430,12 @@ __device__ __forceinline__ void res_raw(const ConvDesc& d, int m, int nb, int nc
 // One warp drains TMEM lanes 32q .. 32q+31 (its rows) for the 16-column
 // chunks j_first, j_first + j_step, ...; the ethreads epilogue threads
 // (etid = this thread's index among them) meet at named barrier 2.
+// ystage (forward, may be null): this warp's two 2 KB staging tiles for TMA
+// stores of the output (box 32 rows x 16 columns, swizzled as the output map
+// says); ybuf alternates between them across chunks and tiles.
 template <int MODE>
 __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, int lane, float (&red)[4][256][2],
-                                         int j_first, int j_step, int etid, int ethreads) {
+                                         int j_first, int j_step, int etid, int ethreads, uint8_t* ystage, int& ybuf) {
   const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
   const int row = q * 32 + lane;
   const int m = T.m0 + row;
@@ -438,19 +447,23 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
   const bool rvec = MODE == FWD && d.res != nullptr && mvalid && (d.K % 8) == 0;
   uint4 rcur[4], rnext[4];
   if (rvec && j_first < T.BN) res_raw(d, m, T.n0 + j_first, T.Ncols, rcur);
+  RT(unsigned long long e0 = 0, e1 = 0, e2 = 0, e3 = 0, en = 0, e5 = 0;)
   for (int j0 = j_first; j0 < T.BN; j0 += j_step) {
     if (rvec && j0 + j_step < T.BN) res_raw(d, m, T.n0 + j0 + j_step, T.Ncols, rnext);
     float v[16];
+    RT(unsigned long long c0 = clock64();)
     tmem_ld16(tbase + j0, v);
+    RT(unsigned long long c1 = clock64(); e0 += c1 - c0; ++en;)
     const int nb = T.n0 + j0;
     const bool full = nb + 16 <= T.Ncols;
     if (MODE == FWD) {
       float s1[16], s2[16];
 #pragma unroll
       for (int i = 0; i < 16; ++i) { s1[i] = 0.f; s2[i] = 0.f; }
+      const bool vec = full && (d.K % 8) == 0;
+      const bool tstore = vec && ystage != nullptr && d.tma_y != nullptr;
       if (mvalid) {
         const int64_t o = (int64_t)m * d.K + nb;
-        const bool vec = full && (d.K % 8) == 0;
         if (d.res) {
           if (vec) {
             if (d.res_dt == DT_BF16) {
@@ -472,11 +485,14 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
                                          : __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(d.res)[o + i]);
           }
         }
+        RT(if (true) { const unsigned long long cr = clock64(); e5 += cr - c1; })
         if (d.y_dt == DT_BF16) {
 #pragma unroll
           for (int i = 0; i < 16; ++i) v[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
         }
-        if (vec) {
+        if (tstore) {
+          // staged below by every lane
+        } else if (vec) {
           if (d.y_dt == DT_BF16) {
             uint4* p = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(d.y) + o);
             if (PNN_ALIGNED(p, 16)) {
@@ -503,6 +519,32 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
           if (nb + i < d.K) { s1[i] = v[i]; s2[i] = v[i] * v[i]; }
         }
       }
+      if (tstore) {
+        // the store issued from this buffer two chunks ago must have read it
+        if (lane == 0) bulk_wait_read<1>();
+        __syncwarp();
+        uint8_t* st = ystage + ybuf * 2048;
+        if (d.y_dt == DT_BF16) {
+          // 32-byte rows, 32-byte swizzle: 16-byte chunk c at c ^ ((row >> 2) & 1)
+#pragma unroll
+          for (int c = 0; c < 2; ++c)
+            *reinterpret_cast<uint4*>(st + lane * 32 + ((c ^ ((lane >> 2) & 1)) << 4)) = pack8(v + 8 * c);
+        } else {
+          // 64-byte rows, 64-byte swizzle: 16-byte chunk c at c ^ ((row >> 1) & 3)
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+            *reinterpret_cast<float4*>(st + lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4)) =
+                make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+        }
+        fence_proxy_async();
+        __syncwarp();
+        if (lane == 0 && T.m0 + q * 32 < T.Mrows) {
+          tma_store_2d(d.tma_y, nb, T.m0 + q * 32, smem_u32(st));
+          bulk_commit();
+        }
+        ybuf ^= 1;
+      }
+      RT(const unsigned long long c2 = clock64(); e1 += c2 - c1;)
       if (stats) {
         const float a = warp_colsum16(s1, lane), b = warp_colsum16(s2, lane);
         if ((lane & 1) == 0) {
@@ -510,6 +552,7 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
           red[q][j0 + (lane >> 1)][1] = b;
         }
       }
+      RT(e2 += clock64() - c2;)
     } else if (mvalid) {
       float* out = MODE == DGRAD ? d.dx + (int64_t)m * d.C + nb
                                  : d.dw_part + ((int64_t)T.split * T.Mrows + m) * d.K + nb;
@@ -535,6 +578,7 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
       for (int i = 0; i < 4; ++i) rcur[i] = rnext[i];
     }
   }
+  RT(const unsigned long long c3 = clock64();)
   if (stats) {
     asm volatile("bar.sync 2, %0;" ::"r"(ethreads) : "memory");
     for (int j = etid; j < T.BN; j += ethreads) {
@@ -547,6 +591,11 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
     }
     asm volatile("bar.sync 2, %0;" ::"r"(ethreads) : "memory");  // red[] is reused by the next tile
   }
+  RT(e3 += clock64() - c3;
+     if (MODE == FWD && lane == 0 && ethreads == 256) {
+       atomicAdd(&g_epi_cycles[0], e0); atomicAdd(&g_epi_cycles[1], e1); atomicAdd(&g_epi_cycles[2], e2);
+       atomicAdd(&g_epi_cycles[3], e3); atomicAdd(&g_epi_cycles[4], en); atomicAdd(&g_epi_cycles[5], e5);
+     })
 }
 
 }  // namespace
@@ -682,7 +731,8 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
       asm volatile("bar.sync 2, 128;" ::: "memory");  // epi_ok is rewritten next tile
       if (!got) { ok = false; break; }
       fence_after();
-      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red, 0, 16, q * 32 + lane, 128);
+      int ybuf_unused = 0;
+      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red, 0, 16, q * 32 + lane, 128, nullptr, ybuf_unused);
       fence_before();
       mbar_arrive(smem_u32(&sh.tempty[b]));
       RT(rt_work += clock64() - rt1;)
@@ -775,13 +825,17 @@ struct TmaShared {
 
 // raw_bytes: one stage's raw slot (a multiple of 1024), per launch
 __host__ __device__ constexpr int tma_op_bytes(int bnmax) { return kABytes + bnmax * 128; }
-__host__ __device__ inline int tma_stages(int bnmax, int raw_bytes) {
-  const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared);
+// forward: eight epilogue warps x two 2 KB output staging tiles after the rings
+constexpr int kTmaYStage = 8 * 2 * 2048;
+__host__ __device__ constexpr int tma_extra(int mode) { return mode == 0 ? kTmaYStage : 0; }
+__host__ __device__ inline int tma_stages(int bnmax, int raw_bytes, int extra) {
+  const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - extra;
   int s = avail / (raw_bytes + tma_op_bytes(bnmax));
   return s < 2 ? 2 : (s > kTmaMaxStages ? kTmaMaxStages : s);
 }
-__host__ __device__ inline size_t tma_smem_bytes(int bnmax, int raw_bytes) {
-  return 1024 + (size_t)tma_stages(bnmax, raw_bytes) * (raw_bytes + tma_op_bytes(bnmax)) + sizeof(TmaShared);
+__host__ __device__ inline size_t tma_smem_bytes(int bnmax, int raw_bytes, int extra) {
+  return 1024 + (size_t)tma_stages(bnmax, raw_bytes, extra) * (raw_bytes + tma_op_bytes(bnmax)) + extra +
+         sizeof(TmaShared);
 }
 
 // One transform thread's share of a stage: row `row` of the A operand, its
@@ -987,11 +1041,12 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
   const uint32_t raw0 = smem_u32(smem_raw);
   const uint32_t base = (raw0 + 1023u) & ~1023u;
   uint8_t* const gbase = smem_raw + (base - raw0);
-  const int S = tma_stages(bnmax, raw_bytes);
+  const int S = tma_stages(bnmax, raw_bytes, tma_extra(MODE));
   const int op_bytes = tma_op_bytes(bnmax);
   const uint32_t op_base = base + S * raw_bytes;
   RT(const unsigned long long rt_start = clock64();)
-  TmaShared& sh = *reinterpret_cast<TmaShared*>(gbase + S * (raw_bytes + op_bytes));
+  uint8_t* const ystage0 = gbase + S * (raw_bytes + op_bytes);  // forward output staging (1024-aligned)
+  TmaShared& sh = *reinterpret_cast<TmaShared*>(ystage0 + tma_extra(MODE));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   uint32_t colstride = 32;
   while ((int)colstride < bnmax) colstride <<= 1;
@@ -1220,6 +1275,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     const int q = warp & 3;               // TMEM lane quarter this warp may access
     const int chalf = ew >> 2;            // which 16-column chunks (two warps a quarter)
     constexpr int jstep = 16 * (R::kEpiWarps / 4);
+    int ybuf = 0;
     int li = 0;
     bool ok = true;
     RT(unsigned long long rt_a = 0, rt_b = 0;)
@@ -1236,11 +1292,15 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       asm volatile("bar.sync 2, %0;" ::"r"(R::kEpilogue) : "memory");
       if (!got) { ok = false; break; }
       fence_after();
-      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red, chalf * 16, jstep, ew * 32 + lane, R::kEpilogue);
+      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red, chalf * 16, jstep, ew * 32 + lane, R::kEpilogue,
+                     MODE == FWD ? ystage0 + ew * 4096 : nullptr, ybuf);
       fence_before();
       mbar_arrive(smem_u32(&sh.tempty[b]));
       RT(rt_b += clock64() - rt1;)
     }
+    // the output stores must complete before the CTA exits
+    if (MODE == FWD && lane == 0) bulk_wait_all();
+    __syncwarp();
     RT(if (threadIdx.x == R::kEpiWarp0 * 32) { atomicAdd(&g_tma_cycles[MODE][8], rt_a); atomicAdd(&g_tma_cycles[MODE][9], rt_b); })
     if (!ok) {
       sh.abort_flag = 1;
@@ -1318,7 +1378,7 @@ static cudaError_t launch_mode(ConvKernel kern, const ConvDesc* tab, const int* 
 }
 
 bool conv_tma_fits(int bnmax, int raw_bytes) {
-  const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared);
+  const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - kTmaYStage;
   return avail / (raw_bytes + tma_op_bytes(bnmax)) >= 2;
 }
 
@@ -1339,7 +1399,7 @@ cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, in
     if (sms <= 0) sms = 148;
     attr[mode] = true;
   }
-  const size_t smem = tma_smem_bytes(bnmax, raw_bytes);
+  const size_t smem = tma_smem_bytes(bnmax, raw_bytes, tma_extra(mode));
   if (smem > (size_t)kTmaSmemBudget) return cudaErrorInvalidValue;
   const int grid = total < sms ? total : sms;
   kern<<<grid, kTmaThreads, smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, status);
@@ -1377,11 +1437,13 @@ cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
 extern "C" int pnn_role_cycles(unsigned long long* out, int reset) {
   cudaError_t e = cudaMemcpyFromSymbol(out, pnn::g_role_cycles, sizeof(pnn::g_role_cycles));
   if (e == cudaSuccess) e = cudaMemcpyFromSymbol(out + 36, pnn::g_tma_cycles, sizeof(pnn::g_tma_cycles));  // 3 x 16
+  if (e == cudaSuccess) e = cudaMemcpyFromSymbol(out + 84, pnn::g_epi_cycles, sizeof(pnn::g_epi_cycles));
   if (e == cudaSuccess && reset) {
     static const unsigned long long zero[3][12] = {};
     e = cudaMemcpyToSymbol(pnn::g_role_cycles, zero, sizeof zero);
     for (int part = 0; part < 2 && e == cudaSuccess; ++part)
       e = cudaMemcpyToSymbol(pnn::g_tma_cycles, zero, 24 * sizeof(unsigned long long), part * 24 * 8);
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(pnn::g_epi_cycles, zero, sizeof(pnn::g_epi_cycles));
   }
   return e == cudaSuccess ? 0 : 1;
 }

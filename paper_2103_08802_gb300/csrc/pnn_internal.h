@@ -50,6 +50,9 @@ struct ConvDesc {
   // 128-byte swizzle)
   const void* tma_a;
   const void* tma_b;
+  // TMA-fed forward: tensor map over the output y [pixels][K] (box 16
+  // columns x 32 rows, 64-byte swizzle for fp32, 32-byte for bf16), or null
+  const void* tma_y;
 };
 
 // out = act( sum_i coef_i * in_i ), optional BN partials of out, NHWC [M][C].

@@ -594,10 +594,11 @@ struct pnn_net {
   }
 
   // 2-D tensor map over rows x inner elements (row pitch inner * element
-  // size) with box [box_rows][box_inner]; sw128: 128-byte swizzle (the MMA's
-  // K-major operand layout), else dense rows.  Out-of-range boxes read zeros.
+  // size) with box [box_rows][box_inner]; swz: swizzle span in bytes (128: the
+  // MMA's K-major operand layout; 64 / 32: epilogue staging tiles; 0: dense
+  // rows).  Loads read zeros outside the tensor; stores skip it.
   int encode_map(CUtensorMap* m, const void* base, bool bf16, int64_t inner, int64_t rows, int box_inner,
-                 int box_rows, bool sw128) {
+                 int box_rows, int swz) {
     static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     if (!encode) {
       void* fn = nullptr;
@@ -614,7 +615,10 @@ struct pnn_net {
     const cuuint32_t estr[2] = {1, 1};
     const CUresult r = encode(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
                               const_cast<void*>(base), dims, pitch, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                              sw128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                              swz == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                              : swz == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                              : swz == 32 ? CU_TENSOR_MAP_SWIZZLE_32B
+                                          : CU_TENSOR_MAP_SWIZZLE_NONE,
                               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return fail(PNN_ECUDA, "cuTensorMapEncodeTiled rejected a conv operand map");
     return PNN_OK;
@@ -987,16 +991,21 @@ int pnn_net::build_tables() {
               const bool a_bf16 = fwd && c.x.dt == DT_BF16;
               const int64_t a_rows = fwd ? (int64_t)B * iv.H * iv.W : (int64_t)B * ov.H * ov.W;
               const int bn = o.ntiles == 1 ? ((ncols + 15) & ~15) : 256;
-              CUtensorMap maps[2];
+              // forward: a third map over the output for the epilogue's TMA stores
+              CUtensorMap maps[3];
               memset(maps, 0, sizeof maps);
               if (ws) {
-                int r = encode_map(&maps[0], a_src, a_bf16, ch, a_rows, std::min(ch, 64), kTcBM, false);
-                if (!r) r = encode_map(&maps[1], c.w, true, kt, ncols, 64, bn, true);
+                int r = encode_map(&maps[0], a_src, a_bf16, ch, a_rows, std::min(ch, 64), kTcBM, 0);
+                if (!r) r = encode_map(&maps[1], c.w, true, kt, ncols, 64, bn, 128);
+                if (!r && fwd)
+                  r = encode_map(&maps[2], ws + ov.off, ov.dt == DT_BF16, ov.C, (int64_t)B * ov.H * ov.W, 16, 32,
+                                 ov.dt == DT_BF16 ? 32 : 64);
                 if (r) return r;
               }
               const size_t mo = put(maps, sizeof maps);
               c.tma_a = ws ? ws + tables_off + mo : nullptr;
               c.tma_b = ws ? ws + tables_off + mo + sizeof(CUtensorMap) : nullptr;
+              c.tma_y = ws && fwd ? ws + tables_off + mo + 2 * sizeof(CUtensorMap) : nullptr;
             }
             if (o.kind == K_WGRAD_TC && o.variant == 1) {
               // activation halo box [hrows][cwx] (its dtype), gradient box [64][K] fp32
@@ -1005,9 +1014,9 @@ int pnn_net::build_tables() {
               memset(maps, 0, sizeof maps);
               if (ws) {
                 int r = encode_map(&maps[0], c.x.ptr, c.x.dt == DT_BF16, iv.C, (int64_t)B * iv.H * iv.W, bx.cwx,
-                                   bx.hrows, false);
+                                   bx.hrows, 0);
                 if (!r) r = encode_map(&maps[1], P<float>(gptr(o.out)), false, ov.C, (int64_t)B * ov.H * ov.W, ov.C,
-                                       64, false);
+                                       64, 0);
                 if (r) return r;
               }
               const size_t mo = put(maps, sizeof maps);

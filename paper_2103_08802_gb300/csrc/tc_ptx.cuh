@@ -192,6 +192,23 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, int 
           "r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar)
       : "memory");
 }
+// 2-D tiled TMA store of one box from shared memory to element coordinates
+// (x inner, y outer) of the tensor map; parts of the box outside the tensor
+// are not written.  x * element size must be a multiple of 16 bytes and both
+// coordinates non-negative.  Completion is tracked per thread by bulk groups.
+__device__ __forceinline__ void tma_store_2d(const void* tmap, int x, int y, uint32_t src) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(tmap), "r"(x),
+               "r"(y), "r"(src)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// wait until at most N of this thread's bulk groups still read shared memory
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// wait until all of this thread's bulk groups are complete
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 // byte offset of 16-byte chunk `ch` of row `row` in the 128-byte-swizzled K-major layout
 __device__ __forceinline__ uint32_t swz(int row, int ch) { return (uint32_t)(row * 128 + ((ch ^ (row & 7)) << 4)); }
 
