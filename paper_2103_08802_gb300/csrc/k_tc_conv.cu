@@ -435,7 +435,8 @@ __device__ __forceinline__ void res_raw(const ConvDesc& d, int m, int nb, int nc
 // says); ybuf alternates between them across chunks and tiles.
 template <int MODE>
 __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, int lane, float (&red)[4][256][2],
-                                         int j_first, int j_step, int etid, int ethreads, uint8_t* ystage, int& ybuf) {
+                                         int j_first, int j_step, int etid, int ethreads, uint8_t* ystage, int& ybuf,
+                                         int bar_id = 2) {
   const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
   const int row = q * 32 + lane;
   const int m = T.m0 + row;
@@ -580,7 +581,7 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
   }
   RT(const unsigned long long c3 = clock64();)
   if (stats) {
-    asm volatile("bar.sync 2, %0;" ::"r"(ethreads) : "memory");
+    asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "r"(ethreads) : "memory");
     for (int j = etid; j < T.BN; j += ethreads) {
       if (T.n0 + j < d.K) {
         const float a = red[0][j][0] + red[1][j][0] + red[2][j][0] + red[3][j][0];
@@ -589,7 +590,7 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
         d.stats[((int64_t)T.tm * d.K + T.n0 + j) * 2 + 1] = b;
       }
     }
-    asm volatile("bar.sync 2, %0;" ::"r"(ethreads) : "memory");  // red[] is reused by the next tile
+    asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "r"(ethreads) : "memory");  // red[] is reused by the next tile
   }
   RT(e3 += clock64() - c3;
      if (MODE == FWD && lane == 0 && ethreads == 256) {
@@ -777,8 +778,9 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
 //               (forward; staged in shared memory per instance), bf16,
 //               padding mask -- from the raw slot into the swizzled operand;
 //   warp 12     TMEM owner and MMA issuer;
-//   warps 4-11  epilogue: two warps per TMEM lane quarter, alternate
-//               16-column chunks.
+//   warps 4-11  epilogue: two groups of four warps (one per TMEM lane
+//               quarter); each group owns one of the two accumulators and
+//               drains every other tile, so two tiles drain at once.
 // Every wait is bounded; the producer drains its copies before the CTA exits.
 constexpr int kTmaThreads = 14 * 32;
 // transform / epilogue split of warps 0-11 per mode: the forward and data
@@ -818,7 +820,7 @@ struct TmaShared {
   uint32_t tmem;
   int abort_flag;
   int epi_ok[8];
-  float red[4][256][2];
+  float red[2][4][256][2];  // per epilogue group
   float scale[kTmaMaxC];
   float shift[kTmaMaxC];
 };
@@ -1060,7 +1062,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(smem_u32(&sh.tfull[b]), 1);
-      mbar_init(smem_u32(&sh.tempty[b]), TmaRoles<MODE>::kEpilogue);
+      mbar_init(smem_u32(&sh.tempty[b]), 128);  // one epilogue group drains a buffer
     }
     mbar_init(smem_u32(&sh.drain), 1);
     sh.abort_flag = 0;
@@ -1271,29 +1273,31 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
   } else {
     // ================================================= epilogue (warps 4-11)
     using R = TmaRoles<MODE>;
+    constexpr int kGroups = R::kEpiWarps / 4;
     const int ew = warp - R::kEpiWarp0;   // 0 .. kEpiWarps-1
     const int q = warp & 3;               // TMEM lane quarter this warp may access
-    const int chalf = ew >> 2;            // which 16-column chunks (two warps a quarter)
-    constexpr int jstep = 16 * (R::kEpiWarps / 4);
+    const int eg = ew >> 2;               // epilogue group
+    const int bar = 2 + eg;               // its named barrier
     int ybuf = 0;
-    int li = 0;
+    int li = eg;
     bool ok = true;
     RT(unsigned long long rt_a = 0, rt_b = 0;)
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++li) {
+    for (int tile = blockIdx.x + eg * gridDim.x; tile < total; tile += kGroups * gridDim.x, li += kGroups) {
       const Tile T = decode<MODE>(tab, tstart, ninst, tile);
       const int b = li & 1;
       RT(const unsigned long long rt0 = clock64();)
       bool got = mbar_wait(smem_u32(&sh.tfull[b]), (li >> 1) & 1, abort_flag);
       RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
       got = __all_sync(0xffffffffu, got);
+      // the group's four warps decide together (they meet at its named barrier)
       if (lane == 0) sh.epi_ok[ew] = got ? 1 : 0;
-      asm volatile("bar.sync 2, %0;" ::"r"(R::kEpilogue) : "memory");
-      for (int i = 0; i < R::kEpiWarps; ++i) got = got && sh.epi_ok[i];
-      asm volatile("bar.sync 2, %0;" ::"r"(R::kEpilogue) : "memory");
+      asm volatile("bar.sync %0, 128;" ::"r"(bar) : "memory");
+      for (int i = 0; i < 4; ++i) got = got && sh.epi_ok[eg * 4 + i];
+      asm volatile("bar.sync %0, 128;" ::"r"(bar) : "memory");
       if (!got) { ok = false; break; }
       fence_after();
-      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red, chalf * 16, jstep, ew * 32 + lane, R::kEpilogue,
-                     MODE == FWD ? ystage0 + ew * 4096 : nullptr, ybuf);
+      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red[eg], 0, 16, (ew & 3) * 32 + lane, 128,
+                     MODE == FWD ? ystage0 + ew * 4096 : nullptr, ybuf, bar);
       fence_before();
       mbar_arrive(smem_u32(&sh.tempty[b]));
       RT(rt_b += clock64() - rt1;)
