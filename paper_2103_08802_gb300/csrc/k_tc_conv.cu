@@ -108,8 +108,8 @@ __device__ __forceinline__ Tile decode(const ConvDesc* tab, const int* tstart, i
   t.pbeg = MODE == WGRAD ? t.split * d.pix_per_split : 0;
   t.pend = MODE == WGRAD ? min(d.B * d.P * d.Q, t.pbeg + d.pix_per_split) : 0;
   t.nkt = MODE == WGRAD ? (t.pend - t.pbeg + kBK - 1) / kBK : (t.Kt + kBK - 1) / kBK;
-  t.BN = d.ntiles == 1 ? ((t.Ncols + 15) & ~15) : 256;
-  t.n0 = t.tn * 256;
+  t.BN = d.ntiles == 1 ? ((t.Ncols + 15) & ~15) : d.ntile_w;
+  t.n0 = t.tn * d.ntile_w;
   t.m0 = t.tm * kBM;
   return t;
 }
@@ -554,6 +554,23 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
         }
       }
       RT(e2 += clock64() - c2;)
+    } else if (MODE == DGRAD && ystage != nullptr && d.tma_y != nullptr) {
+      // staged chunk -> TMA store (fresh gradient) or TMA reduce-add (accumulate)
+      if (lane == 0) bulk_wait_read<1>();
+      __syncwarp();
+      uint8_t* st = ystage + ybuf * 2048;
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        *reinterpret_cast<float4*>(st + lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4)) =
+            make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+      fence_proxy_async();
+      __syncwarp();
+      if (lane == 0 && T.m0 + q * 32 < T.Mrows) {
+        if (d.accumulate) tma_reduce_add_2d(d.tma_y, nb, T.m0 + q * 32, smem_u32(st));
+        else tma_store_2d(d.tma_y, nb, T.m0 + q * 32, smem_u32(st));
+        bulk_commit();
+      }
+      ybuf ^= 1;
     } else if (mvalid) {
       float* out = MODE == DGRAD ? d.dx + (int64_t)m * d.C + nb
                                  : d.dw_part + ((int64_t)T.split * T.Mrows + m) * d.K + nb;
@@ -783,13 +800,12 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
 //               drains every other tile, so two tiles drain at once.
 // Every wait is bounded; the producer drains its copies before the CTA exits.
 constexpr int kTmaThreads = 14 * 32;
-// transform / epilogue split of warps 0-11 per mode: the forward and data
-// gradient have a wide epilogue (4 transform + 8 epilogue warps); the weight
-// gradient builds two transposed operands and drains a small accumulator
-// (8 transform + 4 epilogue warps)
+// transform / epilogue split of warps 0-11 per mode: the forward has the
+// heavy epilogue (residual, statistics; 4 transform + 8 epilogue warps); the
+// gradients have the heavy transform (8 transform + 4 epilogue warps)
 template <int MODE>
 struct TmaRoles {
-  static constexpr int kTransformWarps = MODE == WGRAD ? 8 : 4;
+  static constexpr int kTransformWarps = MODE == FWD ? 4 : 8;
   static constexpr int kEpiWarps = 12 - kTransformWarps;
   static constexpr int kTransform = 32 * kTransformWarps;
   static constexpr int kEpilogue = 32 * kEpiWarps;
@@ -827,9 +843,10 @@ struct TmaShared {
 
 // raw_bytes: one stage's raw slot (a multiple of 1024), per launch
 __host__ __device__ constexpr int tma_op_bytes(int bnmax) { return kABytes + bnmax * 128; }
-// forward: eight epilogue warps x two 2 KB output staging tiles after the rings
+// forward / data gradient: two 2 KB output staging tiles per epilogue warp
+// (eight / four warps) after the rings
 constexpr int kTmaYStage = 8 * 2 * 2048;
-__host__ __device__ constexpr int tma_extra(int mode) { return mode == 0 ? kTmaYStage : 0; }
+__host__ __device__ constexpr int tma_extra(int mode) { return mode == 0 ? kTmaYStage : (mode == 1 ? kTmaYStage / 2 : 0); }
 __host__ __device__ inline int tma_stages(int bnmax, int raw_bytes, int extra) {
   const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - extra;
   int s = avail / (raw_bytes + tma_op_bytes(bnmax));
@@ -841,12 +858,13 @@ __host__ __device__ inline size_t tma_smem_bytes(int bnmax, int raw_bytes, int e
 }
 
 // One transform thread's share of a stage: row `row` of the A operand, its
-// 8 chunks of 8 K elements, in groups of 4 (bf16) or 2 (fp32): each group's
+// chunks jbeg .. jend-1 of 8 K elements (all 8, or half when two threads
+// share a row), in groups of 4 (bf16) or 2 (fp32): each group's
 // raw loads are issued before any of its chunks is converted and stored (the restrict-qualified
 // pointers tell the compiler the operand stores cannot alias the raw slot
 // or the scale/shift arrays).
 struct TStage {
-  int row, hrow, kread, lg, cdim, tapb, cb;
+  int row, hrow, kread, lg, cdim, tapb, cb, jbeg, jend;
   uint32_t tapok;
   int taps;
   bool tr;
@@ -859,6 +877,7 @@ __device__ __forceinline__ void transform_stage(const uint8_t* __restrict__ rawp
   constexpr int G = XBF ? 4 : 2;  // chunks per group (fp32 raw: two 16-byte words a chunk)
 #pragma unroll
   for (int h = 0; h < 8; h += G) {
+  if (h < t.jbeg || h >= t.jend) continue;
   uint4 raw[G][XBF ? 1 : 2];
 #pragma unroll
   for (int jj = 0; jj < G; ++jj) {
@@ -1047,7 +1066,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
   const int op_bytes = tma_op_bytes(bnmax);
   const uint32_t op_base = base + S * raw_bytes;
   RT(const unsigned long long rt_start = clock64();)
-  uint8_t* const ystage0 = gbase + S * (raw_bytes + op_bytes);  // forward output staging (1024-aligned)
+  uint8_t* const ystage0 = gbase + S * (raw_bytes + op_bytes);  // output staging (1024-aligned)
   TmaShared& sh = *reinterpret_cast<TmaShared*>(ystage0 + tma_extra(MODE));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   uint32_t colstride = 32;
@@ -1139,8 +1158,11 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     // ================================================= transform (thread = A row)
     // Control flow is the same for every transform thread (they meet at named
     // barrier 1): a thread whose wait fails raises the abort flag and walks
-    // the remaining stages without waiting or working.
-    const int row = threadIdx.x;
+    // the remaining stages without waiting or working.  With 256 transform
+    // threads two share a row (chunks 0-3 and 4-7).
+    const int row = threadIdx.x & 127;
+    constexpr int kRowSplit = TmaRoles<MODE>::kTransform / 128;
+    const int jbeg = (threadIdx.x >> 7) * (8 / kRowSplit), jend = jbeg + 8 / kRowSplit;
     uint32_t g = 0;
     bool ok = true;
     const ConvDesc* staged = nullptr;  // instance whose scale/shift sit in shared memory
@@ -1156,7 +1178,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       if (tr && staged != T.d) {
         // all transform threads are past the previous tile's stages
         asm volatile("bar.sync 1, %0;" ::"r"(TmaRoles<MODE>::kTransform) : "memory");
-        for (int c = row; c < d.C; c += TmaRoles<MODE>::kTransform) {
+        for (int c = threadIdx.x; c < d.C; c += TmaRoles<MODE>::kTransform) {
           sh.scale[c] = __ldg(d.x.scale + c);
           sh.shift[c] = __ldg(d.x.shift + c);
         }
@@ -1164,7 +1186,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
         staged = T.d;
       }
       if constexpr (MODE == WGRAD) {
-        wgrad_transform_tile(T, d, row, tr, g, ok, S, raw_bytes, op_bytes, gbase, sh RT(, rt_a, rt_b));
+        wgrad_transform_tile(T, d, threadIdx.x, tr, g, ok, S, raw_bytes, op_bytes, gbase, sh RT(, rt_a, rt_b));
         continue;
       }
       // this row's pixel and which of the R x S taps stay inside the image
@@ -1202,7 +1224,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
         const int cb = big ? (kt - tapb * per_tap) * 64 : 0;
         // K elements of this stage the MMA reads (16-element steps)
         const int kread = min(kBK, (T.Kt - kt * kBK + 15) & ~15);
-        TStage st{row, hrow, kread, lg, cdim, tapb, cb, tapok, taps, tr, relu};
+        TStage st{row, hrow, kread, lg, cdim, tapb, cb, jbeg, jend, tapok, taps, tr, relu};
         if (xbf) {
           if (big) transform_stage<true, true>(rawp, A, sh.scale, sh.shift, st);
           else transform_stage<true, false>(rawp, A, sh.scale, sh.shift, st);
@@ -1297,13 +1319,13 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       if (!got) { ok = false; break; }
       fence_after();
       epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red[eg], 0, 16, (ew & 3) * 32 + lane, 128,
-                     MODE == FWD ? ystage0 + ew * 4096 : nullptr, ybuf, bar);
+                     MODE != WGRAD ? ystage0 + ew * 4096 : nullptr, ybuf, bar);
       fence_before();
       mbar_arrive(smem_u32(&sh.tempty[b]));
       RT(rt_b += clock64() - rt1;)
     }
     // the output stores must complete before the CTA exits
-    if (MODE == FWD && lane == 0) bulk_wait_all();
+    if (MODE != WGRAD && lane == 0) bulk_wait_all();
     __syncwarp();
     RT(if (threadIdx.x == R::kEpiWarp0 * 32) { atomicAdd(&g_tma_cycles[MODE][8], rt_a); atomicAdd(&g_tma_cycles[MODE][9], rt_b); })
     if (!ok) {
@@ -1534,6 +1556,7 @@ extern "C" int pnn_conv_wgrad_noalloc(const float* x, const float* dy, float* dw
   cd.dw_part = sym->part;
   cd.mtiles = (rsc + kTcBM - 1) / kTcBM;
   cd.ntiles = (k + 255) / 256;
+  cd.ntile_w = 256;
   cd.op_bf16 = 1;
   const int base = cd.mtiles * cd.ntiles;
   int splits = (int)std::min<int64_t>((mp + 255) / 256, (2 * 152 + base - 1) / base);

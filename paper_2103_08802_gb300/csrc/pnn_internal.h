@@ -42,6 +42,7 @@ struct ConvDesc {
   float* dw_part;
   int32_t splits, pix_per_split;
   int32_t mtiles, ntiles;             // tile grid of this instance
+  int32_t ntile_w;                    // N columns of a tile when ntiles > 1 (256, or 128 TMA-fed)
   int32_t op_bf16;                    // round both contraction operands to bf16 (bf16 mode)
   // TMA-fed tensor-core variant (stride 1): device addresses of two 2-D tensor
   // maps (CUtensorMap, 128-byte aligned) -- tma_a over the A source rows

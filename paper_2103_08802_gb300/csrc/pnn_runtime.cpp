@@ -111,6 +111,13 @@ static bool tma_shape_ok(int k, int stride, int pad, int ch) {
   return geom && ch % 8 == 0 && (ch <= 64 ? 64 % ch == 0 : ch % 64 == 0);
 }
 
+// N columns of a tensor-core conv tile when the layer needs several: 128 for
+// the TMA-fed forward and data gradient (a smaller operand slot leaves room for
+// more pipeline stages), 256 otherwise.
+static int tc_ntile_w(int kind, int variant) {
+  return variant == 1 && (kind == K_CONV_FWD_TC || kind == K_DGRAD_TC) ? 128 : 256;
+}
+
 // The TMA-fed weight gradient loads a k-step's activation rows for all taps
 // as one halo box and the output-gradient rows as another: channels 8..64
 // (dividing 64) or multiples of 128 up to 512, at most 128 output channels
@@ -289,7 +296,7 @@ struct pnn_net {
       // is wide; narrow outputs keep the thread-gathered kernel
       c.variant = opt.conv_impl == 0 && cout >= 64 && tma_shape_ok(k, stride, k / 2, iv.C) ? 1 : 0;
       c.mtiles = cdiv(M, kTcBM);
-      c.ntiles = cdiv(cout, 256);
+      c.ntiles = cdiv(cout, tc_ntile_w(c.kind, c.variant));
     } else {
       c.variant = cout <= 16 ? 2 : (cout <= 32 ? 1 : 0);
       ConvTile t = simt_tile(c.variant);
@@ -496,7 +503,7 @@ struct pnn_net {
             dg.kind = K_DGRAD_TC;
             dg.variant = opt.conv_impl == 0 && tma_shape_ok(f.k, f.stride, f.pad, ov.C) ? 1 : 0;
             dg.mtiles = cdiv((int64_t)B * iv.H * iv.W, kTcBM);
-            dg.ntiles = cdiv(iv.C, 256);
+            dg.ntiles = cdiv(iv.C, tc_ntile_w(dg.kind, dg.variant));
           } else {
             dg.variant = iv.C <= 16 ? 2 : (iv.C <= 32 ? 1 : 0);
             ConvTile t = simt_tile(dg.variant);
@@ -980,6 +987,7 @@ int pnn_net::build_tables() {
             c.B = B; c.H = iv.H; c.W = iv.W; c.C = iv.C; c.P = ov.H; c.Q = ov.W; c.K = ov.C;
             c.R = o.k; c.S = o.k; c.stride = o.stride; c.pad = o.pad;
             c.mtiles = o.mtiles; c.ntiles = o.ntiles;
+            c.ntile_w = tc_ntile_w(o.kind, o.variant);
             c.op_bf16 = act_dt == DT_BF16 && ((o.kind != K_DGRAD && o.kind != K_WGRAD) || !opt.grad_fp32);
             if (o.kind == K_DGRAD_TC) c.w = (const char*)(ws + off_wt) + params[o.w].off * 2;
             if ((o.kind == K_CONV_FWD_TC || o.kind == K_DGRAD_TC) && o.variant == 1) {
@@ -990,8 +998,8 @@ int pnn_net::build_tables() {
               const void* a_src = fwd ? c.x.ptr : (const void*)P<float>(gptr(o.out));
               const bool a_bf16 = fwd && c.x.dt == DT_BF16;
               const int64_t a_rows = fwd ? (int64_t)B * iv.H * iv.W : (int64_t)B * ov.H * ov.W;
-              const int bn = o.ntiles == 1 ? ((ncols + 15) & ~15) : 256;
-              // forward: a third map over the output for the epilogue's TMA stores
+              const int bn = o.ntiles == 1 ? ((ncols + 15) & ~15) : tc_ntile_w(o.kind, o.variant);
+              // a third map over the output for the epilogue's TMA stores
               CUtensorMap maps[3];
               memset(maps, 0, sizeof maps);
               if (ws) {
@@ -1000,12 +1008,14 @@ int pnn_net::build_tables() {
                 if (!r && fwd)
                   r = encode_map(&maps[2], ws + ov.off, ov.dt == DT_BF16, ov.C, (int64_t)B * ov.H * ov.W, 16, 32,
                                  ov.dt == DT_BF16 ? 32 : 64);
+                if (!r && !fwd)  // data gradient: dx [pixels][C] fp32, stored or reduce-added
+                  r = encode_map(&maps[2], P<float>(gptr(o.in)), false, iv.C, (int64_t)B * iv.H * iv.W, 16, 32, 64);
                 if (r) return r;
               }
               const size_t mo = put(maps, sizeof maps);
               c.tma_a = ws ? ws + tables_off + mo : nullptr;
               c.tma_b = ws ? ws + tables_off + mo + sizeof(CUtensorMap) : nullptr;
-              c.tma_y = ws && fwd ? ws + tables_off + mo + 2 * sizeof(CUtensorMap) : nullptr;
+              c.tma_y = ws ? ws + tables_off + mo + 2 * sizeof(CUtensorMap) : nullptr;
             }
             if (o.kind == K_WGRAD_TC && o.variant == 1) {
               // activation halo box [hrows][cwx] (its dtype), gradient box [64][K] fp32
@@ -1168,7 +1178,7 @@ int pnn_net::build_tables() {
       for (int id : g.ops)
         if (ops[id].kind == K_CONV_FWD_TC || ops[id].kind == K_DGRAD_TC || ops[id].kind == K_WGRAD_TC) {
           const int K = ops[id].kind == K_DGRAD_TC ? vals[ops[id].in].C : vals[ops[id].out].C;
-          L.aux = std::max(L.aux, ops[id].ntiles == 1 ? ((K + 15) & ~15) : 256);
+          L.aux = std::max(L.aux, ops[id].ntiles == 1 ? ((K + 15) & ~15) : tc_ntile_w(ops[id].kind, ops[id].variant));
           if (ops[id].kind == K_DGRAD_TC) L.esz = 4;
           else if (ops[id].kind == K_CONV_FWD_TC) {
             const int src = vals[ops[id].in].virt ? vals[ops[id].in].src : ops[id].in;

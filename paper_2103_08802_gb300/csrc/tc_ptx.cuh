@@ -201,6 +201,12 @@ __device__ __forceinline__ void tma_store_2d(const void* tmap, int x, int y, uin
                "r"(y), "r"(src)
                : "memory");
 }
+// the same box added element-wise (fp32) into global memory (done in L2)
+__device__ __forceinline__ void tma_reduce_add_2d(const void* tmap, int x, int y, uint32_t src) {
+  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(tmap),
+               "r"(x), "r"(y), "r"(src)
+               : "memory");
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 // wait until at most N of this thread's bulk groups still read shared memory
 template <int N>
