@@ -933,39 +933,50 @@ __device__ __forceinline__ void transform_stage(const uint8_t* __restrict__ rawp
   }
 }
 
-// Weight-gradient transform of one tile (256 threads): thread u < 128 builds A unit u (rows
-// jg*8 .. jg*8+7 = (tap, c .. c+7)) from the halo box -- BN scale/shift +
-// ReLU of the producing layer, zero outside the image or the split -- and
-// thread 128 + u, u < BN, B unit u (k_out kg*8 .. +7) from the gradient box, both for the
-// k-step pixels pg, pg+8, .., pg+56, 8x8-transposed into K positions 8*pg ..
-// 8*pg+7 of the K(pixel)-major operands.  The contraction sums over pixels,
-// so a permutation of K shared by A and B leaves it unchanged; this one makes
-// the lanes of a warp read consecutive raw rows.
+// Weight-gradient transform of one tile (256 threads).  The operands are
+// built in half-units of 8 rows x 4 pixels: A half-unit h (rows jg*8 ..
+// jg*8+7 = (tap, c .. c+7) of the m-tile; BN scale/shift + ReLU of the
+// producing layer; zero outside the image or the split) from the halo box,
+// B half-unit h (k_out kg*8 .. +7) from the gradient box.  Unit (g, pg) holds
+// the k-step pixels pg, pg+8, .., pg+56 at K positions 8*pg .. 8*pg+7, half
+// `hf` the pixels pg + 8*(4*hf + i), i < 4, at K bytes 8*hf of chunk pg.  The
+// contraction sums over pixels, so a K permutation shared by A and B leaves it
+// unchanged; this one makes the lanes of a warp read consecutive raw rows.
+// Thread t takes A half-unit t (if the m-tile has it) and B half-unit t (if
+// BN has it); rows past the layer's M are not written (the MMA rows are
+// independent and the epilogue does not store them).
+__device__ __forceinline__ void store_half8x4(const uint32_t (&w)[4][4], uint8_t* base, int row0, int chunk,
+                                              int hf) {
+  // w[pixel][pair of rows] -> rows row0 + c, 4 pixels each (8 bytes)
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const uint32_t sel = (c & 1) ? 0x7632 : 0x5410;
+    const uint2 o = make_uint2(__byte_perm(w[0][c / 2], w[1][c / 2], sel), __byte_perm(w[2][c / 2], w[3][c / 2], sel));
+    *reinterpret_cast<uint2*>(base + swz(row0 + c, chunk) + 8 * hf) = o;
+  }
+}
 template <typename Sh>
-__device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDesc& d, int u, bool tr, uint32_t& g,
+__device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDesc& d, int t, bool tr, uint32_t& g,
                                                      bool& ok, int S, int raw_bytes, int op_bytes, uint8_t* gbase,
                                                      Sh& sh RT(, unsigned long long& rt_a, unsigned long long& rt_b)) {
   const bool xbf = d.x.dt == DT_BF16;
   const WgBoxes bx = wg_boxes(d.C, d.K, d.W, d.pad, xbf);
   const int cbase = d.C <= 64 ? 0 : T.m0 % d.C;
-  // threads 0-127 build the A units, threads 128-255 the B units
-  const bool aside = u < 128;
-  if (!aside) u -= 128;
-  const int jg = u >> 3, pg = u & 7;
+  const bool one = d.R == 1 && d.S == 1;
+  // A half-unit of this thread
+  const int arows = min(kBM, T.Mrows - T.m0);           // rows of the m-tile in the layer (multiple of 8)
+  const bool aside = t < (arows >> 3) * 16;
+  const int au = t >> 1, ahf = t & 1;
+  const int jg = au >> 3, apg = au & 7;
   const int j0 = T.m0 + jg * 8;
-  const bool jin = aside && j0 < T.Mrows;
   const int tap = j0 / d.C, c0 = j0 - tap * d.C;
   const int r = tap / d.S, sx = tap - r * d.S;
   const int hoff = r * d.W + sx;                // halo row of pixel 0 for this tap
   const int dyr = r - d.pad, dxs = sx - d.pad;
   const int cl = c0 - cbase;                    // channel within the box
-  const bool bunit = !aside && u < T.BN;
-  const int kg = u >> 3;
-  const bool bcols = bunit && T.n0 + kg * 8 < d.K;
   const int relu = tr ? d.x.relu : 0;
-  // this unit's 8 channels of the producing layer's BN scale/shift (fixed for the tile)
   float sc[8], sf[8];
-  if (jin && tr) {
+  if (aside && tr) {
     const float4 s0 = *reinterpret_cast<const float4*>(&sh.scale[c0]);
     const float4 s1 = *reinterpret_cast<const float4*>(&sh.scale[c0 + 4]);
     const float4 f0 = *reinterpret_cast<const float4*>(&sh.shift[c0]);
@@ -973,6 +984,14 @@ __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDe
     sc[0] = s0.x; sc[1] = s0.y; sc[2] = s0.z; sc[3] = s0.w; sc[4] = s1.x; sc[5] = s1.y; sc[6] = s1.z; sc[7] = s1.w;
     sf[0] = f0.x; sf[1] = f0.y; sf[2] = f0.z; sf[3] = f0.w; sf[4] = f1.x; sf[5] = f1.y; sf[6] = f1.z; sf[7] = f1.w;
   }
+  // B half-unit of this thread
+  const bool bside = t < 2 * T.BN;
+  const int bu = t >> 1, bhf = t & 1;
+  const int kg = bu >> 3, bpg = bu & 7;
+  const bool bcols = bside && T.n0 + kg * 8 < d.K;
+  // A pixel coordinates, advanced incrementally (3x3 only): first pixel of the half-unit
+  Pix apx;
+  if (!one) apx.init(T.pbeg + apg + 32 * ahf, d.P, d.Q);
   for (int kt = 0; kt < T.nkt; ++kt, ++g) {
     const int s = g % S;
     RT(const unsigned long long rt0 = clock64();)
@@ -987,31 +1006,31 @@ __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDe
     uint8_t* __restrict__ A = gbase + S * raw_bytes + s * op_bytes;
     uint8_t* __restrict__ Bt = A + kABytes;
     const int pix0 = T.pbeg + kt * kBK;
-    // validity of the unit's 8 pixels (inside the split; tap inside the image)
-    unsigned pin = 0, xin = 0;
-    {
-      Pix px;
-      px.init(pix0 + pg, d.P, d.Q);
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        if (i) px.step(8, d.P, d.Q);
-        const bool in = pix0 + pg + 8 * i < T.pend;
-        pin |= (in ? 1u : 0u) << i;
-        const bool ii = in && px.y + dyr >= 0 && px.y + dyr < d.H && px.x + dxs >= 0 && px.x + dxs < d.W;
-        xin |= (ii ? 1u : 0u) << i;
-      }
-    }
-    if (!jin) xin = 0;
-    // A
     if (aside) {
-      uint4 in[8];
+      // validity of the 4 pixels pix0 + apg + 8 * (4 * ahf + i)
+      unsigned xin = 0;
+      if (one) {
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int row = pg + 8 * i + hoff;
+        for (int i = 0; i < 4; ++i) xin |= (pix0 + apg + 8 * (4 * ahf + i) < T.pend ? 1u : 0u) << i;
+      } else {
+        Pix px = apx;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          if (i) px.step(8, d.P, d.Q);
+          const bool in = pix0 + apg + 8 * (4 * ahf + i) < T.pend && px.y + dyr >= 0 && px.y + dyr < d.H &&
+                          px.x + dxs >= 0 && px.x + dxs < d.W;
+          xin |= (in ? 1u : 0u) << i;
+        }
+        apx.step(kBK, d.P, d.Q);
+      }
+      uint32_t w[4][4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int row = apg + 8 * (4 * ahf + i) + hoff;
         float v[8];
         if (xbf) {
-          const uint4 w = *reinterpret_cast<const uint4*>(rawx + (row * bx.cwx + cl) * 2);
-          const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&w);
+          const uint4 q = *reinterpret_cast<const uint4*>(rawx + (row * bx.cwx + cl) * 2);
+          const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&q);
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
             const float2 f = __bfloat1622float2(hh[e]);
@@ -1025,29 +1044,27 @@ __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDe
           v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
         }
         if (tr) act8(v, sc, sf, relu);
-        in[i] = (xin >> i) & 1 ? pack8(v) : make_uint4(0, 0, 0, 0);
+        const bool in = (xin >> i) & 1;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) w[i][e] = in ? pack_bf16(v[2 * e], v[2 * e + 1]) : 0u;
       }
-      uint4 out[8];
-      transpose8(in, out);
-#pragma unroll
-      for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(A + swz(jg * 8 + c, pg)) = out[c];
+      store_half8x4(w, A, jg * 8, apg, ahf);
     }
-    // B
-    if (bunit) {
-      uint4 in[8];
+    if (bside) {
+      uint32_t w[4][4];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int row = pg + 8 * i;
+      for (int i = 0; i < 4; ++i) {
+        const int row = bpg + 8 * (4 * bhf + i);
         const float* src = reinterpret_cast<const float*>(rawy) + row * d.K + kg * 8;
         const float4 a = *reinterpret_cast<const float4*>(src);
         const float4 b = *reinterpret_cast<const float4*>(src + 4);
-        const float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-        in[i] = bcols && ((pin >> i) & 1) ? pack8(v) : make_uint4(0, 0, 0, 0);
+        const bool in = bcols && pix0 + row < T.pend;
+        w[i][0] = in ? pack_bf16(a.x, a.y) : 0u;
+        w[i][1] = in ? pack_bf16(a.z, a.w) : 0u;
+        w[i][2] = in ? pack_bf16(b.x, b.y) : 0u;
+        w[i][3] = in ? pack_bf16(b.z, b.w) : 0u;
       }
-      uint4 out[8];
-      transpose8(in, out);
-#pragma unroll
-      for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(Bt + swz(kg * 8 + c, pg)) = out[c];
+      store_half8x4(w, Bt, kg * 8, bpg, bhf);
     }
     fence_proxy_async();
     mbar_arrive(smem_u32(&sh.op_full[s]));
