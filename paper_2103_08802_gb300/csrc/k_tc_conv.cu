@@ -800,12 +800,12 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
 //               drains every other tile, so two tiles drain at once.
 // Every wait is bounded; the producer drains its copies before the CTA exits.
 constexpr int kTmaThreads = 14 * 32;
-// transform / epilogue split of warps 0-11 per mode: the forward has the
-// heavy epilogue (residual, statistics; 4 transform + 8 epilogue warps); the
-// gradients have the heavy transform (8 transform + 4 epilogue warps)
-template <int MODE>
+// transform / epilogue split of warps 0-11 (XW transform warps): the forward
+// (wide outputs) has the heavy epilogue (residual, statistics; 4 + 8 warps);
+// the gradients have the heavy transform (8 + 4 warps)
+template <int MODE, int XW>
 struct TmaRoles {
-  static constexpr int kTransformWarps = MODE == FWD ? 4 : 8;
+  static constexpr int kTransformWarps = XW;
   static constexpr int kEpiWarps = 12 - kTransformWarps;
   static constexpr int kTransform = 32 * kTransformWarps;
   static constexpr int kEpilogue = 32 * kEpiWarps;
@@ -844,9 +844,9 @@ struct TmaShared {
 // raw_bytes: one stage's raw slot (a multiple of 1024), per launch
 __host__ __device__ constexpr int tma_op_bytes(int bnmax) { return kABytes + bnmax * 128; }
 // forward / data gradient: two 2 KB output staging tiles per epilogue warp
-// (eight / four warps) after the rings
+// (12 - XW warps) after the rings
 constexpr int kTmaYStage = 8 * 2 * 2048;
-__host__ __device__ constexpr int tma_extra(int mode) { return mode == 0 ? kTmaYStage : (mode == 1 ? kTmaYStage / 2 : 0); }
+__host__ __device__ constexpr int tma_extra(int mode, int xw) { return mode == 2 ? 0 : (12 - xw) * 2 * 2048; }
 __host__ __device__ inline int tma_stages(int bnmax, int raw_bytes, int extra) {
   const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - extra;
   int s = avail / (raw_bytes + tma_op_bytes(bnmax));
@@ -1072,19 +1072,19 @@ __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDe
   }
 }
 
-template <int MODE>
+template <int MODE, int XW>
 __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, const int* __restrict__ tstart,
                                               int ninst, int total, int bnmax, int raw_bytes, int32_t* status) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw0 = smem_u32(smem_raw);
   const uint32_t base = (raw0 + 1023u) & ~1023u;
   uint8_t* const gbase = smem_raw + (base - raw0);
-  const int S = tma_stages(bnmax, raw_bytes, tma_extra(MODE));
+  const int S = tma_stages(bnmax, raw_bytes, tma_extra(MODE, XW));
   const int op_bytes = tma_op_bytes(bnmax);
   const uint32_t op_base = base + S * raw_bytes;
   RT(const unsigned long long rt_start = clock64();)
   uint8_t* const ystage0 = gbase + S * (raw_bytes + op_bytes);  // output staging (1024-aligned)
-  TmaShared& sh = *reinterpret_cast<TmaShared*>(ystage0 + tma_extra(MODE));
+  TmaShared& sh = *reinterpret_cast<TmaShared*>(ystage0 + tma_extra(MODE, XW));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   uint32_t colstride = 32;
   while ((int)colstride < bnmax) colstride <<= 1;
@@ -1093,7 +1093,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_u32(&sh.tma_full[s]), 1);
-      mbar_init(smem_u32(&sh.op_full[s]), TmaRoles<MODE>::kTransform);
+      mbar_init(smem_u32(&sh.op_full[s]), TmaRoles<MODE, XW>::kTransform);
       mbar_init(smem_u32(&sh.op_empty[s]), 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -1171,14 +1171,14 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
         mbar_wait_drain(smem_u32(&sh.tma_full[i % S]), (i / S) & 1);
     }
     __syncwarp();
-  } else if (warp < TmaRoles<MODE>::kEpiWarp0) {
+  } else if (warp < TmaRoles<MODE, XW>::kEpiWarp0) {
     // ================================================= transform (thread = A row)
     // Control flow is the same for every transform thread (they meet at named
     // barrier 1): a thread whose wait fails raises the abort flag and walks
     // the remaining stages without waiting or working.  With 256 transform
     // threads two share a row (chunks 0-3 and 4-7).
     const int row = threadIdx.x & 127;
-    constexpr int kRowSplit = TmaRoles<MODE>::kTransform / 128;
+    constexpr int kRowSplit = TmaRoles<MODE, XW>::kTransform / 128;
     const int jbeg = (threadIdx.x >> 7) * (8 / kRowSplit), jend = jbeg + 8 / kRowSplit;
     uint32_t g = 0;
     bool ok = true;
@@ -1194,12 +1194,12 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       const bool tr = MODE != DGRAD && d.x.scale != nullptr;
       if (tr && staged != T.d) {
         // all transform threads are past the previous tile's stages
-        asm volatile("bar.sync 1, %0;" ::"r"(TmaRoles<MODE>::kTransform) : "memory");
-        for (int c = threadIdx.x; c < d.C; c += TmaRoles<MODE>::kTransform) {
+        asm volatile("bar.sync 1, %0;" ::"r"(TmaRoles<MODE, XW>::kTransform) : "memory");
+        for (int c = threadIdx.x; c < d.C; c += TmaRoles<MODE, XW>::kTransform) {
           sh.scale[c] = __ldg(d.x.scale + c);
           sh.shift[c] = __ldg(d.x.shift + c);
         }
-        asm volatile("bar.sync 1, %0;" ::"r"(TmaRoles<MODE>::kTransform) : "memory");
+        asm volatile("bar.sync 1, %0;" ::"r"(TmaRoles<MODE, XW>::kTransform) : "memory");
         staged = T.d;
       }
       if constexpr (MODE == WGRAD) {
@@ -1311,7 +1311,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     __syncwarp();
   } else {
     // ================================================= epilogue (warps 4-11)
-    using R = TmaRoles<MODE>;
+    using R = TmaRoles<MODE, XW>;
     constexpr int kGroups = R::kEpiWarps / 4;
     const int ew = warp - R::kEpiWarp0;   // 0 .. kEpiWarps-1
     const int q = warp & 3;               // TMEM lane quarter this warp may access
@@ -1365,17 +1365,18 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
 __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_fwd_tma(const ConvDesc* __restrict__ tab,
                                                                  const int* __restrict__ tstart, int ninst, int total,
                                                                  int bnmax, int raw_bytes, int32_t* status) {
-  conv_tma_body<FWD>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+  conv_tma_body<FWD, 4>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
+
 __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_dgrad_tma(const ConvDesc* __restrict__ tab,
                                                                    const int* __restrict__ tstart, int ninst, int total,
                                                                    int bnmax, int raw_bytes, int32_t* status) {
-  conv_tma_body<DGRAD>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+  conv_tma_body<DGRAD, 8>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
 __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_wgrad_tma(const ConvDesc* __restrict__ tab,
                                                                    const int* __restrict__ tstart, int ninst, int total,
                                                                    int bnmax, int raw_bytes, int32_t* status) {
-  conv_tma_body<WGRAD>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+  conv_tma_body<WGRAD, 8>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
 
 // one kernel name per mode (profiler filters and launch lists name the mode)
@@ -1430,6 +1431,7 @@ cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, in
   if (total <= 0) return cudaSuccess;
   if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || raw_bytes <= 0 || (raw_bytes & 1023) || mode < 0 || mode > 2)
     return cudaErrorInvalidValue;
+  const int xw = mode == 0 ? 4 : 8;  // transform warps of the mode's kernel
   static bool attr[3] = {false, false, false};
   static int sms = 0;
   auto kern = mode == 0 ? k_conv_fwd_tma : (mode == 1 ? k_conv_dgrad_tma : k_conv_wgrad_tma);
@@ -1442,7 +1444,7 @@ cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, in
     if (sms <= 0) sms = 148;
     attr[mode] = true;
   }
-  const size_t smem = tma_smem_bytes(bnmax, raw_bytes, tma_extra(mode));
+  const size_t smem = tma_smem_bytes(bnmax, raw_bytes, tma_extra(mode, xw));
   if (smem > (size_t)kTmaSmemBudget) return cudaErrorInvalidValue;
   const int grid = total < sms ? total : sms;
   kern<<<grid, kTmaThreads, smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, status);

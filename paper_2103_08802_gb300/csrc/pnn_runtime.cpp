@@ -293,7 +293,8 @@ struct pnn_net {
       // tcgen05 path: 128-pixel tiles, all output channels (<= 256) per tile
       c.kind = K_CONV_FWD_TC;
       // the TMA-fed forward (eight epilogue warps) pays off when the epilogue
-      // is wide; narrow outputs keep the thread-gathered kernel
+      // is wide (measured: 2x on 16->64 with the residual); narrow outputs keep
+      // the thread-gathered kernel, which is faster there
       c.variant = opt.conv_impl == 0 && cout >= 64 && tma_shape_ok(k, stride, k / 2, iv.C) ? 1 : 0;
       c.mtiles = cdiv(M, kTcBM);
       c.ntiles = cdiv(cout, tc_ntile_w(c.kind, c.variant));
