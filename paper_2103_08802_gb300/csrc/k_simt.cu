@@ -284,23 +284,29 @@ __global__ void __launch_bounds__(256) k_conv_wgrad(const ConvDesc* __restrict__
 
 // 32 elements per CTA, 8 lanes per element: lane l sums splits l, l+8, ...
 // in order, then a fixed xor-shuffle tree combines the 8 lanes.
+// 32 consecutive partial positions e per CTA; warp w sums splits w, w+8, ..
+// (coalesced 128-byte rows of one split), then the eight warp sums are added
+// in warp order: a fixed order, so the result is deterministic.  Transposed
+// partials ([split][j][k_out], the tensor-core layout) land in dw[k_out][j].
 __global__ void __launch_bounds__(256) k_wreduce(const WReduceDesc* __restrict__ tab, const int* __restrict__ tstart,
                                                  int n) {
+  __shared__ float red[8][32];
   const int inst = find_instance(tstart, n, blockIdx.x);
-  const WReduceDesc& d = tab[inst];
-  const int64_t i = (int64_t)(blockIdx.x - tstart[inst]) * 32 + threadIdx.x / 8;
-  const int l = threadIdx.x % 8;
+  const WReduceDesc d = tab[inst];
+  const int64_t e = (int64_t)(blockIdx.x - tstart[inst]) * 32 + (threadIdx.x & 31);
+  const int w = threadIdx.x >> 5;
   float s = 0.f;
-  int64_t src = 0;
-  if (i < d.n) {
-    // i indexes dw[k_out][j]; transposed partials are stored [s][j][k_out]
-    src = d.transposed ? (int64_t)(i % d.rsc) * d.kout + i / d.rsc : i;
-    for (int k = l; k < d.splits; k += 8) s += d.part[(int64_t)k * d.n + src];
+  if (e < d.n)
+    for (int k = w; k < d.splits; k += 8) s += d.part[(int64_t)k * d.n + e];
+  red[w][threadIdx.x & 31] = s;
+  __syncthreads();
+  if (w == 0 && e < d.n) {
+    float t = red[0][threadIdx.x];
+#pragma unroll
+    for (int i = 1; i < 8; ++i) t += red[i][threadIdx.x];
+    const int64_t i = d.transposed ? (e % d.kout) * d.rsc + e / d.kout : e;
+    d.dw[i] = d.accumulate ? d.dw[i] + t : t;
   }
-  s += __shfl_xor_sync(0xffffffffu, s, 4);
-  s += __shfl_xor_sync(0xffffffffu, s, 2);
-  s += __shfl_xor_sync(0xffffffffu, s, 1);
-  if (i < d.n && l == 0) d.dw[i] = d.accumulate ? d.dw[i] + s : s;
 }
 
 __global__ void k_wtrans(const WtDesc* __restrict__ tab, const int* __restrict__ tstart, int n) {

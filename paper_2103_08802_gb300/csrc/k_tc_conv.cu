@@ -442,15 +442,30 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
   const int m = T.m0 + row;
   const bool mvalid = m < T.Mrows;
   const uint32_t tbase = tacc + ((uint32_t)(q * 32) << 16);
-  const bool stats = MODE == FWD && d.stats != nullptr;
+  // forward: BN statistics of the output; fused data gradient: BN-backward
+  // partial sums of the input's BN (same per-tile layout [m-tile][cols][2])
+  const bool stats = (MODE == FWD && d.stats != nullptr) || (MODE == DGRAD && d.bnb_part != nullptr);
+  float* const spart = MODE == FWD ? d.stats : d.bnb_part;
   // forward residual: 16 columns a chunk, the next chunk's loads issued
   // before the current chunk is consumed
   const bool rvec = MODE == FWD && d.res != nullptr && mvalid && (d.K % 8) == 0;
   uint4 rcur[4], rnext[4];
   if (rvec && j_first < T.BN) res_raw(d, m, T.n0 + j_first, T.Ncols, rcur);
   RT(unsigned long long e0 = 0, e1 = 0, e2 = 0, e3 = 0, en = 0, e5 = 0;)
+  // fused data gradient: the chunk's BN input h (16 values of this row)
+  const bool hload = MODE == DGRAD && stats && mvalid;
   for (int j0 = j_first; j0 < T.BN; j0 += j_step) {
     if (rvec && j0 + j_step < T.BN) res_raw(d, m, T.n0 + j0 + j_step, T.Ncols, rnext);
+    uint4 hraw[4];
+    if (hload) {
+      const bool hb = d.x.dt == DT_BF16;
+      const int64_t o = (int64_t)m * d.C + T.n0 + j0;
+      const uint4* src = hb ? reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(d.x.ptr) + o)
+                            : reinterpret_cast<const uint4*>(reinterpret_cast<const float*>(d.x.ptr) + o);
+      hraw[0] = __ldg(src);
+      hraw[1] = __ldg(src + 1);
+      if (!hb) { hraw[2] = __ldg(src + 2); hraw[3] = __ldg(src + 3); }
+    }
     float v[16];
     RT(unsigned long long c0 = clock64();)
     tmem_ld16(tbase + j0, v);
@@ -555,6 +570,51 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
       }
       RT(e2 += clock64() - c2;)
     } else if (MODE == DGRAD && ystage != nullptr && d.tma_y != nullptr) {
+      if (stats) {
+        // BN-backward partial sums of the input's BN: g = dA masked by the
+        // ReLU of the forward BN output, xhat = (h - mean) * rstd
+        float s1[16], s2[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) { s1[i] = 0.f; s2[i] = 0.f; }
+        if (mvalid) {
+          float h[16];
+          if (d.x.dt == DT_BF16) {
+            const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(hraw);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const float2 f = __bfloat1622float2(hh[i]);
+              h[2 * i] = f.x;
+              h[2 * i + 1] = f.y;
+            }
+          } else {
+            const float* f = reinterpret_cast<const float*>(hraw);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) h[i] = f[i];
+          }
+#pragma unroll
+          for (int i4 = 0; i4 < 16; i4 += 4) {
+            const float4 sc = __ldg(reinterpret_cast<const float4*>(d.x.scale + nb + i4));
+            const float4 sh = __ldg(reinterpret_cast<const float4*>(d.x.shift + nb + i4));
+            const float4 mu = __ldg(reinterpret_cast<const float4*>(d.bn_mean + nb + i4));
+            const float4 rs = __ldg(reinterpret_cast<const float4*>(d.bn_rstd + nb + i4));
+            const float scv[4] = {sc.x, sc.y, sc.z, sc.w}, shv[4] = {sh.x, sh.y, sh.z, sh.w};
+            const float muv[4] = {mu.x, mu.y, mu.z, mu.w}, rsv[4] = {rs.x, rs.y, rs.z, rs.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const int i = i4 + k;
+              float gv = v[i];
+              if (d.x.relu && !(fmaf(scv[k], h[i], shv[k]) > 0.f)) gv = 0.f;
+              s1[i] = gv;
+              s2[i] = gv * ((h[i] - muv[k]) * rsv[k]);
+            }
+          }
+        }
+        const float a = warp_colsum16(s1, lane), b = warp_colsum16(s2, lane);
+        if ((lane & 1) == 0) {
+          red[q][j0 + (lane >> 1)][0] = a;
+          red[q][j0 + (lane >> 1)][1] = b;
+        }
+      }
       // staged chunk -> TMA store (fresh gradient) or TMA reduce-add (accumulate)
       if (lane == 0) bulk_wait_read<1>();
       __syncwarp();
@@ -600,11 +660,12 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
   if (stats) {
     asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "r"(ethreads) : "memory");
     for (int j = etid; j < T.BN; j += ethreads) {
-      if (T.n0 + j < d.K) {
+      if (T.n0 + j < T.Ncols) {
         const float a = red[0][j][0] + red[1][j][0] + red[2][j][0] + red[3][j][0];
         const float b = red[0][j][1] + red[1][j][1] + red[2][j][1] + red[3][j][1];
-        d.stats[((int64_t)T.tm * d.K + T.n0 + j) * 2] = a;
-        d.stats[((int64_t)T.tm * d.K + T.n0 + j) * 2 + 1] = b;
+        const int scols = T.Ncols;
+        spart[((int64_t)T.tm * scols + T.n0 + j) * 2] = a;
+        spart[((int64_t)T.tm * scols + T.n0 + j) * 2 + 1] = b;
       }
     }
     asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "r"(ethreads) : "memory");  // red[] is reused by the next tile
@@ -1371,7 +1432,7 @@ __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_fwd_tma(const ConvDesc*
 __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_dgrad_tma(const ConvDesc* __restrict__ tab,
                                                                    const int* __restrict__ tstart, int ninst, int total,
                                                                    int bnmax, int raw_bytes, int32_t* status) {
-  conv_tma_body<DGRAD, 8>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+  conv_tma_body<DGRAD, 4>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
 __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_wgrad_tma(const ConvDesc* __restrict__ tab,
                                                                    const int* __restrict__ tstart, int ninst, int total,
@@ -1431,7 +1492,7 @@ cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, in
   if (total <= 0) return cudaSuccess;
   if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || raw_bytes <= 0 || (raw_bytes & 1023) || mode < 0 || mode > 2)
     return cudaErrorInvalidValue;
-  const int xw = mode == 0 ? 4 : 8;  // transform warps of the mode's kernel
+  const int xw = mode == 2 ? 8 : 4;  // transform warps of the mode's kernel
   static bool attr[3] = {false, false, false};
   static int sms = 0;
   auto kern = mode == 0 ? k_conv_fwd_tma : (mode == 1 ? k_conv_dgrad_tma : k_conv_wgrad_tma);

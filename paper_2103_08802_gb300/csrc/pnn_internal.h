@@ -54,6 +54,13 @@ struct ConvDesc {
   // TMA-fed forward: tensor map over the output y [pixels][K] (box 16
   // columns x 32 rows, 64-byte swizzle for fp32, 32-byte for bf16), or null
   const void* tma_y;
+  // TMA-fed data gradient of a BN(+ReLU) value (x = that virtual value): when
+  // bnb_part is set, the epilogue also writes the BN-backward partial sums of
+  // its tile, [m-tile][C][2] = (sum g, sum g * xhat) with g = dA masked by the
+  // ReLU and xhat = (h - mean) * rstd
+  const float* bn_mean;
+  const float* bn_rstd;
+  float* bnb_part;
 };
 
 // out = act( sum_i coef_i * in_i ), optional BN partials of out, NHWC [M][C].

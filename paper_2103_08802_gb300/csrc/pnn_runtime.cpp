@@ -56,10 +56,13 @@ struct Value {
   size_t off = 0, goff = 0;
   int galias = -1;  // gradient lives in another value's gradient buffer
   bool grad_written = false;
+  int gwrites = 0;           // ops that wrote (stored or accumulated) this gradient
+  int gwriter_dgrad = -1;    // the last data-gradient op among them
   std::vector<int> pending;  // values whose gradient is to be added into this one's
 };
 
 struct Norm {
+  int fused_tiles = 0;                       // BN-backward partials written by a data-gradient epilogue: its m-tiles
   int C = 0, h = -1, gamma = -1, beta = -1;  // gamma/beta: param ids
   int virt = -1;                             // the virtual BN(+ReLU) value
   int tiles = 0;
@@ -85,6 +88,7 @@ struct POp {
   int acc_in[3] = {0, 0, 0};
   int addv[2] = {-1, -1};                    // BNB_APPLY: extra gradients added into dh
   int splits = 1, pix_per_split = 0;
+  int bn_fuse = -1;                          // TMA dgrad: norm whose BN-backward partials the epilogue writes
   size_t scratch = 0;                        // wgrad partial buffer offset
   int tiles = 0, mtiles = 0, ntiles = 0;
   int head = 0;
@@ -411,6 +415,7 @@ struct pnn_net {
   int grad_acc(int v) {
     int a = vals[v].grad_written ? 1 : 0;
     vals[v].grad_written = true;
+    vals[v].gwrites++;
     return a;
   }
   void flush_pending(std::vector<int>& L, int v, const int* key) {
@@ -514,7 +519,7 @@ struct pnn_net {
           dg.tiles = dg.mtiles * dg.ntiles;
           dg.acc = grad_acc(f.in);
           key(dg, 2);
-          new_op(L, dg);
+          vals[f.in].gwriter_dgrad = new_op(L, dg);
         }
         break;
       }
@@ -560,7 +565,19 @@ struct pnn_net {
         r.variant = (n.C % 8 == 0 && n.C <= 2048) ? 1 : 0;  // 1: 8 channels per thread
         r.tiles = cdiv(n.count, bnb_rows_per_tile(n.C));
         key(r, 0);
-        new_op(L, r);
+        // The reduction is fused into the data gradient that wrote the whole
+        // gradient of the BN(+ReLU) value (TMA-fed, stored, sole writer): its
+        // epilogue writes the partial sums of each 128-row tile.
+        const int wr = vals[vv].gwriter_dgrad;
+        const bool fuse = vals[vv].gwrites == 1 && wr >= 0 && ops[wr].kind == K_DGRAD_TC && ops[wr].variant == 1 &&
+                          ops[wr].acc == 0 &&
+                          ops[wr].in == vv && vals[vv].galias < 0 && vals[vv].pending.empty() && n.C % 16 == 0;
+        if (fuse) {
+          ops[wr].bn_fuse = f.norm;
+          norms[f.norm].fused_tiles = ops[wr].mtiles;
+        } else {
+          new_op(L, r);
+        }
         POp fi = r;
         fi.kind = K_BNB_FIN;
         fi.tiles = n.C;  // one CTA per channel
@@ -863,7 +880,8 @@ int pnn_net::plan(const pnn_desc* d) {
     n.part = alloc((size_t)n.tiles * n.C * 8);
     n.mean = alloc(n.C * 4); n.rstd = alloc(n.C * 4); n.scale = alloc(n.C * 4); n.shift = alloc(n.C * 4);
     n.btiles = cdiv(n.count, bnb_rows_per_tile(n.C));
-    n.bpart = alloc((size_t)n.btiles * n.C * 8);
+    // room for the reduce kernel's tiles or a fused data gradient's 128-row tiles
+    n.bpart = alloc((size_t)std::max(n.btiles, cdiv(n.count, kTcBM)) * n.C * 8);
     n.coef = alloc((size_t)n.C * 12);
   }
   // wgrad scratch: one region per op (sized per op)
@@ -1042,6 +1060,10 @@ int pnn_net::build_tables() {
             } else if (o.kind == K_DGRAD || o.kind == K_DGRAD_TC) {
               c.dy = P<float>(gptr(o.out));
               c.dx = P<float>(gptr(o.in)); c.accumulate = o.acc;
+              if (o.bn_fuse >= 0) {
+                const Norm& nf = norms[o.bn_fuse];
+                c.bn_mean = P<float>(nf.mean); c.bn_rstd = P<float>(nf.rstd); c.bnb_part = P<float>(nf.bpart);
+              }
               add(&c, sizeof c, o.tiles);
             } else {
               c.dy = P<float>(gptr(o.out));
@@ -1125,7 +1147,7 @@ int pnn_net::build_tables() {
             b.dgamma = grad + params[n.gamma].off; b.dbeta = grad + params[n.beta].off;
             b.coef = P<float>(n.coef);
             b.M = n.count; b.C = n.C;
-            b.rows_per_tile = bnb_rows_per_tile(n.C); b.tiles = n.btiles;
+            b.rows_per_tile = bnb_rows_per_tile(n.C); b.tiles = n.fused_tiles ? n.fused_tiles : n.btiles;
             if (o.kind == K_BNB_FIN) b.accumulate = o.acc_in[0];
             if (o.kind == K_BNB_APPLY) {
               b.dh = P<float>(gptr(n.h));

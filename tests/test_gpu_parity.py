@@ -230,15 +230,21 @@ def _conv_variants(desc, theta, x, labels, conv_impl):
 @pytest.mark.parametrize("idx", [1, 2, 4])
 def test_tma_fed_convs_match_thread_gathered(idx):
     """The TMA-fed stride-1 convolutions (the default) and the thread-gathered
-    tensor-core convolutions (conv_impl=3) build the same bf16 operands.  The
-    forward and data-gradient kernels also accumulate them in the same K order
-    with the same epilogue, so every activation, correction tensor, D_j and
-    the loss agree bit for bit.  The TMA-fed weight gradient sums the pixels
-    of each 64-pixel k-step in a permuted order, so weight gradients (and the
-    SGD update built on them) agree to fp32 reordering error: 1e-5 of the
-    largest element.  (VGG-16's 3x3 convs with 64..512 channels, ResNet's 1x1
-    and 3x3 bottleneck convs; stride-2 convs take the gathered kernel on both
-    sides.)"""
+    tensor-core convolutions (conv_impl=3) build the same bf16 operands, and the
+    forward kernels accumulate them in the same K order with the same
+    epilogue: every activation, correction tensor, logit and the loss agree bit
+    for bit.  The backward differs only in fp32 summation order -- the TMA-fed
+    weight gradient sums each 64-pixel k-step in a permuted order, and the
+    TMA-fed data gradient of a BN(+ReLU) value also forms that BN's backward
+    sums over its 128-row tiles (the thread-gathered path runs the separate
+    reduction kernel).  A last-bit change of a BN-backward sum can flip the
+    bf16 rounding of gradient operands further down (one bf16 ulp is 4e-3
+    relative), so D_j, the gradients and the SGD update agree to the level of
+    such flips: norm-relative 2e-2, the bound the tensor-core / CUDA-core
+    backward comparison uses; correctness of each path against the oracle is
+    what the parity tests above check.  (VGG-16's 3x3 convs with 64..512
+    channels, ResNet's 1x1 and 3x3 bottleneck convs; stride-2 convs take the
+    gathered kernel on both sides.)"""
     desc = reduced(idx)
     onet, theta, x, labels = inputs(desc)
     tma = _conv_variants(desc, theta, x, labels, 0)
@@ -246,14 +252,14 @@ def test_tma_fed_convs_match_thread_gathered(idx):
     assert all(v == 0 for _, v in _conv_variants(desc, theta, x, labels, 3))
     a = run_gpu(desc, theta, x, labels)
     b = run_gpu(desc, theta, x, labels, conv_impl=3)
-    reordered = ("grad", "theta_new", "momentum")
+    backward = ("grad", "theta_new", "momentum")
     for k in a:
         if k in ("net", "onet"):
             continue
         ak, bk = np.asarray(a[k]), np.asarray(b[k])
-        if k in reordered:
-            err = np.abs(ak - bk).max() / max(np.abs(bk).max(), 1e-30)
-            assert err <= 1e-5, (k, err)
+        if k in backward or k.startswith("D"):
+            err = np.linalg.norm(ak - bk) / max(np.linalg.norm(bk), 1e-30)
+            assert err <= 2e-2, (k, err)
         else:
             np.testing.assert_array_equal(ak, bk, err_msg=k)
 
