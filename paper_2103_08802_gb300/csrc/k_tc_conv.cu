@@ -110,7 +110,7 @@ __device__ __forceinline__ Tile decode(const ConvDesc* tab, const int* tstart, i
   t.nkt = MODE == WGRAD ? (t.pend - t.pbeg + kBK - 1) / kBK : (t.Kt + kBK - 1) / kBK;
   t.BN = d.ntiles == 1 ? ((t.Ncols + 15) & ~15) : d.ntile_w;
   t.n0 = t.tn * d.ntile_w;
-  t.m0 = t.tm * kBM;
+  t.m0 = t.tm * (d.mtile_rows > 0 ? d.mtile_rows : kBM);
   return t;
 }
 
@@ -902,19 +902,22 @@ struct TmaShared {
   float shift[kTmaMaxC];
 };
 
-// raw_bytes: one stage's raw slot (a multiple of 1024), per launch
-__host__ __device__ constexpr int tma_op_bytes(int bnmax) { return kABytes + bnmax * 128; }
+// raw_bytes: one stage's raw slot (a multiple of 1024), per launch.  Operand
+// slot: A (one 128-row half, or two for the weight gradient's 256-row tiles)
+// then B (bnmax rows).
+__host__ __device__ constexpr int tma_amult(int mode) { return mode == 2 ? 2 : 1; }
+__host__ __device__ constexpr int tma_op_bytes(int mode, int bnmax) { return tma_amult(mode) * kABytes + bnmax * 128; }
 // forward / data gradient: two 2 KB output staging tiles per epilogue warp
 // (12 - XW warps) after the rings
 constexpr int kTmaYStage = 8 * 2 * 2048;
 __host__ __device__ constexpr int tma_extra(int mode, int xw) { return mode == 2 ? 0 : (12 - xw) * 2 * 2048; }
-__host__ __device__ inline int tma_stages(int bnmax, int raw_bytes, int extra) {
+__host__ __device__ inline int tma_stages(int mode, int bnmax, int raw_bytes, int extra) {
   const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - extra;
-  int s = avail / (raw_bytes + tma_op_bytes(bnmax));
+  int s = avail / (raw_bytes + tma_op_bytes(mode, bnmax));
   return s < 2 ? 2 : (s > kTmaMaxStages ? kTmaMaxStages : s);
 }
-__host__ __device__ inline size_t tma_smem_bytes(int bnmax, int raw_bytes, int extra) {
-  return 1024 + (size_t)tma_stages(bnmax, raw_bytes, extra) * (raw_bytes + tma_op_bytes(bnmax)) + extra +
+__host__ __device__ inline size_t tma_smem_bytes(int mode, int bnmax, int raw_bytes, int extra) {
+  return 1024 + (size_t)tma_stages(mode, bnmax, raw_bytes, extra) * (raw_bytes + tma_op_bytes(mode, bnmax)) + extra +
          sizeof(TmaShared);
 }
 
@@ -994,18 +997,45 @@ __device__ __forceinline__ void transform_stage(const uint8_t* __restrict__ rawp
   }
 }
 
-// Weight-gradient transform of one tile (256 threads).  The operands are
-// built in half-units of 8 rows x 4 pixels: A half-unit h (rows jg*8 ..
-// jg*8+7 = (tap, c .. c+7) of the m-tile; BN scale/shift + ReLU of the
+// one A half-unit of the weight-gradient transform (constants for a tile)
+struct WgA {
+  bool on;
+  int jg, pg, hf;         // row group (of the up to 256 tile rows), pixel group, half
+  int c0, cl, hoff, dyr, dxs;
+  Pix px;                 // pixel of K position 8*pg + 4*hf (3x3 only)
+};
+__device__ __forceinline__ WgA wg_aunit(const Tile& T, const ConvDesc& d, int a, int nA, int cbase) {
+  WgA u;
+  u.on = a < nA;
+  const int au = a >> 1;
+  u.hf = a & 1;
+  u.jg = au >> 3;
+  u.pg = au & 7;
+  const int j0 = T.m0 + u.jg * 8;
+  const int tap = j0 / d.C;
+  u.c0 = j0 - tap * d.C;
+  const int r = tap / d.S, sx = tap - r * d.S;
+  u.hoff = r * d.W + sx;
+  u.dyr = r - d.pad;
+  u.dxs = sx - d.pad;
+  u.cl = u.c0 - cbase;
+  if (u.on && !(d.R == 1 && d.S == 1)) u.px.init(T.pbeg + u.pg + 32 * u.hf, d.P, d.Q);
+  return u;
+}
+
+// Weight-gradient transform of one tile (256 threads, up to 256 rows).  The
+// operands are built in half-units of 8 rows x 4 pixels: A half-unit (rows
+// jg*8 .. jg*8+7 = (tap, c .. c+7) of the tile; BN scale/shift + ReLU of the
 // producing layer; zero outside the image or the split) from the halo box,
-// B half-unit h (k_out kg*8 .. +7) from the gradient box.  Unit (g, pg) holds
+// B half-unit (k_out kg*8 .. +7) from the gradient box.  Unit (g, pg) holds
 // the k-step pixels pg, pg+8, .., pg+56 at K positions 8*pg .. 8*pg+7, half
 // `hf` the pixels pg + 8*(4*hf + i), i < 4, at K bytes 8*hf of chunk pg.  The
 // contraction sums over pixels, so a K permutation shared by A and B leaves it
 // unchanged; this one makes the lanes of a warp read consecutive raw rows.
-// Thread t takes A half-unit t (if the m-tile has it) and B half-unit t (if
-// BN has it); rows past the layer's M are not written (the MMA rows are
-// independent and the epilogue does not store them).
+// Thread t takes A half-units t and t + 256 and B half-unit 255 - t (those
+// that exist); rows 128-255 go to the second 16 KB half of A; rows past the
+// layer's M are not written (the MMA rows are independent and the epilogue
+// does not store them).
 __device__ __forceinline__ void store_half8x4(const uint32_t (&w)[4][4], uint8_t* base, int row0, int chunk,
                                               int hf) {
   // w[pixel][pair of rows] -> rows row0 + c, 4 pixels each (8 bytes)
@@ -1017,42 +1047,81 @@ __device__ __forceinline__ void store_half8x4(const uint32_t (&w)[4][4], uint8_t
   }
 }
 template <typename Sh>
+__device__ __forceinline__ void wg_a_stage(const ConvDesc& d, const Tile& T, WgA& u, bool one, bool xbf, bool tr,
+                                           int relu, int pix0, const WgBoxes& bx, const uint8_t* __restrict__ rawx,
+                                           uint8_t* __restrict__ A, const Sh& sh) {
+  // validity of the 4 pixels pix0 + pg + 8 * (4 * hf + i)
+  unsigned xin = 0;
+  if (one) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) xin |= (pix0 + u.pg + 8 * (4 * u.hf + i) < T.pend ? 1u : 0u) << i;
+  } else {
+    Pix px = u.px;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (i) px.step(8, d.P, d.Q);
+      const bool in = pix0 + u.pg + 8 * (4 * u.hf + i) < T.pend && px.y + u.dyr >= 0 && px.y + u.dyr < d.H &&
+                      px.x + u.dxs >= 0 && px.x + u.dxs < d.W;
+      xin |= (in ? 1u : 0u) << i;
+    }
+    u.px.step(kBK, d.P, d.Q);
+  }
+  float sc[8], sf[8];
+  if (tr) {
+    const float4 s0 = *reinterpret_cast<const float4*>(&sh.scale[u.c0]);
+    const float4 s1 = *reinterpret_cast<const float4*>(&sh.scale[u.c0 + 4]);
+    const float4 f0 = *reinterpret_cast<const float4*>(&sh.shift[u.c0]);
+    const float4 f1 = *reinterpret_cast<const float4*>(&sh.shift[u.c0 + 4]);
+    sc[0] = s0.x; sc[1] = s0.y; sc[2] = s0.z; sc[3] = s0.w; sc[4] = s1.x; sc[5] = s1.y; sc[6] = s1.z; sc[7] = s1.w;
+    sf[0] = f0.x; sf[1] = f0.y; sf[2] = f0.z; sf[3] = f0.w; sf[4] = f1.x; sf[5] = f1.y; sf[6] = f1.z; sf[7] = f1.w;
+  }
+  uint32_t w[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int row = u.pg + 8 * (4 * u.hf + i) + u.hoff;
+    float v[8];
+    if (xbf) {
+      const uint4 q = *reinterpret_cast<const uint4*>(rawx + (row * bx.cwx + u.cl) * 2);
+      const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&q);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 f = __bfloat1622float2(hh[e]);
+        v[2 * e] = f.x;
+        v[2 * e + 1] = f.y;
+      }
+    } else {
+      const float4 a = *reinterpret_cast<const float4*>(rawx + (row * bx.cwx + u.cl) * 4);
+      const float4 b = *reinterpret_cast<const float4*>(rawx + (row * bx.cwx + u.cl) * 4 + 16);
+      v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+      v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+    if (tr) act8(v, sc, sf, relu);
+    const bool in = (xin >> i) & 1;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) w[i][e] = in ? pack_bf16(v[2 * e], v[2 * e + 1]) : 0u;
+  }
+  store_half8x4(w, A + (u.jg >> 4) * kABytes, (u.jg & 15) * 8, u.pg, u.hf);
+}
+template <typename Sh>
 __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDesc& d, int t, bool tr, uint32_t& g,
                                                      bool& ok, int S, int raw_bytes, int op_bytes, uint8_t* gbase,
                                                      Sh& sh RT(, unsigned long long& rt_a, unsigned long long& rt_b)) {
   const bool xbf = d.x.dt == DT_BF16;
   const WgBoxes bx = wg_boxes(d.C, d.K, d.W, d.pad, xbf);
+  const int tile_rows = d.mtile_rows > 0 ? d.mtile_rows : kBM;
   const int cbase = d.C <= 64 ? 0 : T.m0 % d.C;
   const bool one = d.R == 1 && d.S == 1;
-  // A half-unit of this thread
-  const int arows = min(kBM, T.Mrows - T.m0);           // rows of the m-tile in the layer (multiple of 8)
-  const bool aside = t < (arows >> 3) * 16;
-  const int au = t >> 1, ahf = t & 1;
-  const int jg = au >> 3, apg = au & 7;
-  const int j0 = T.m0 + jg * 8;
-  const int tap = j0 / d.C, c0 = j0 - tap * d.C;
-  const int r = tap / d.S, sx = tap - r * d.S;
-  const int hoff = r * d.W + sx;                // halo row of pixel 0 for this tap
-  const int dyr = r - d.pad, dxs = sx - d.pad;
-  const int cl = c0 - cbase;                    // channel within the box
   const int relu = tr ? d.x.relu : 0;
-  float sc[8], sf[8];
-  if (aside && tr) {
-    const float4 s0 = *reinterpret_cast<const float4*>(&sh.scale[c0]);
-    const float4 s1 = *reinterpret_cast<const float4*>(&sh.scale[c0 + 4]);
-    const float4 f0 = *reinterpret_cast<const float4*>(&sh.shift[c0]);
-    const float4 f1 = *reinterpret_cast<const float4*>(&sh.shift[c0 + 4]);
-    sc[0] = s0.x; sc[1] = s0.y; sc[2] = s0.z; sc[3] = s0.w; sc[4] = s1.x; sc[5] = s1.y; sc[6] = s1.z; sc[7] = s1.w;
-    sf[0] = f0.x; sf[1] = f0.y; sf[2] = f0.z; sf[3] = f0.w; sf[4] = f1.x; sf[5] = f1.y; sf[6] = f1.z; sf[7] = f1.w;
-  }
+  const int arows = min(tile_rows, T.Mrows - T.m0);       // rows of the tile in the layer (multiple of 8)
+  const int nA = (arows >> 3) * 16;
+  WgA u0 = wg_aunit(T, d, t, nA, cbase);
+  WgA u1 = wg_aunit(T, d, t + 256, nA, cbase);
   // B half-unit of this thread
-  const bool bside = t < 2 * T.BN;
-  const int bu = t >> 1, bhf = t & 1;
+  const int bh = 255 - t;
+  const bool bside = bh < 2 * T.BN;
+  const int bu = bh >> 1, bhf = bh & 1;
   const int kg = bu >> 3, bpg = bu & 7;
   const bool bcols = bside && T.n0 + kg * 8 < d.K;
-  // A pixel coordinates, advanced incrementally (3x3 only): first pixel of the half-unit
-  Pix apx;
-  if (!one) apx.init(T.pbeg + apg + 32 * ahf, d.P, d.Q);
   for (int kt = 0; kt < T.nkt; ++kt, ++g) {
     const int s = g % S;
     RT(const unsigned long long rt0 = clock64();)
@@ -1065,52 +1134,10 @@ __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDe
     const uint8_t* __restrict__ rawx = gbase + s * raw_bytes;
     const uint8_t* __restrict__ rawy = rawx + bx.yoff;
     uint8_t* __restrict__ A = gbase + S * raw_bytes + s * op_bytes;
-    uint8_t* __restrict__ Bt = A + kABytes;
+    uint8_t* __restrict__ Bt = A + 2 * kABytes;
     const int pix0 = T.pbeg + kt * kBK;
-    if (aside) {
-      // validity of the 4 pixels pix0 + apg + 8 * (4 * ahf + i)
-      unsigned xin = 0;
-      if (one) {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) xin |= (pix0 + apg + 8 * (4 * ahf + i) < T.pend ? 1u : 0u) << i;
-      } else {
-        Pix px = apx;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          if (i) px.step(8, d.P, d.Q);
-          const bool in = pix0 + apg + 8 * (4 * ahf + i) < T.pend && px.y + dyr >= 0 && px.y + dyr < d.H &&
-                          px.x + dxs >= 0 && px.x + dxs < d.W;
-          xin |= (in ? 1u : 0u) << i;
-        }
-        apx.step(kBK, d.P, d.Q);
-      }
-      uint32_t w[4][4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int row = apg + 8 * (4 * ahf + i) + hoff;
-        float v[8];
-        if (xbf) {
-          const uint4 q = *reinterpret_cast<const uint4*>(rawx + (row * bx.cwx + cl) * 2);
-          const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&q);
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 f = __bfloat1622float2(hh[e]);
-            v[2 * e] = f.x;
-            v[2 * e + 1] = f.y;
-          }
-        } else {
-          const float4 a = *reinterpret_cast<const float4*>(rawx + (row * bx.cwx + cl) * 4);
-          const float4 b = *reinterpret_cast<const float4*>(rawx + (row * bx.cwx + cl) * 4 + 16);
-          v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-          v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-        }
-        if (tr) act8(v, sc, sf, relu);
-        const bool in = (xin >> i) & 1;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) w[i][e] = in ? pack_bf16(v[2 * e], v[2 * e + 1]) : 0u;
-      }
-      store_half8x4(w, A, jg * 8, apg, ahf);
-    }
+    if (u0.on) wg_a_stage(d, T, u0, one, xbf, tr, relu, pix0, bx, rawx, A, sh);
+    if (u1.on) wg_a_stage(d, T, u1, one, xbf, tr, relu, pix0, bx, rawx, A, sh);
     if (bside) {
       uint32_t w[4][4];
 #pragma unroll
@@ -1140,8 +1167,9 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
   const uint32_t raw0 = smem_u32(smem_raw);
   const uint32_t base = (raw0 + 1023u) & ~1023u;
   uint8_t* const gbase = smem_raw + (base - raw0);
-  const int S = tma_stages(bnmax, raw_bytes, tma_extra(MODE, XW));
-  const int op_bytes = tma_op_bytes(bnmax);
+  const int S = tma_stages(MODE, bnmax, raw_bytes, tma_extra(MODE, XW));
+  const int op_bytes = tma_op_bytes(MODE, bnmax);
+  constexpr int kAMult = tma_amult(MODE);
   const uint32_t op_base = base + S * raw_bytes;
   RT(const unsigned long long rt_start = clock64();)
   uint8_t* const ystage0 = gbase + S * (raw_bytes + op_bytes);  // output staging (1024-aligned)
@@ -1149,7 +1177,8 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   uint32_t colstride = 32;
   while ((int)colstride < bnmax) colstride <<= 1;
-  const uint32_t ncols = 2 * colstride;
+  const uint32_t bufcols = kAMult * colstride;  // one accumulator buffer (two halves for 256-row tiles)
+  const uint32_t ncols = 2 * bufcols;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -1337,8 +1366,10 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
         if (!mbar_wait(smem_u32(&sh.tempty[b]), ((li >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
         RT(rt_acc += clock64() - rt0;)
         fence_after();
-        const uint32_t tacc = tmem + b * colstride;
+        const uint32_t tacc = tmem + b * bufcols;
         const uint32_t idesc = idesc_bf16(kBM, T.BN);
+        // a second 128-row half: only in a 256-row tile that has more than 128 rows
+        const bool two = kAMult == 2 && min(T.d->mtile_rows, T.Mrows - T.m0) > kBM;
         for (int kt = 0; kt < T.nkt; ++kt, ++g) {
           const int s = g % S;
           RT(rt0 = clock64();)
@@ -1346,12 +1377,16 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
           RT(const unsigned long long rt1 = clock64(); rt_full += rt1 - rt0;)
           fence_after();
           const uint32_t a_addr = op_base + s * op_bytes;
-          const uint32_t b_addr = a_addr + kABytes;
+          const uint32_t b_addr = a_addr + kAMult * kABytes;
           // (weight gradient: pixels sit at permuted K positions, all 64 are read)
           const int krem = MODE == WGRAD ? kBK : T.Kt - kt * kBK;
           const int ksub = min(4, (krem + 15) / 16);
-          for (int kk = 0; kk < ksub; ++kk)
+          for (int kk = 0; kk < ksub; ++kk) {
             mma_bf16(tacc, sw128_desc(a_addr + kk * 32), sw128_desc(b_addr + kk * 32), idesc, (kt | kk) ? 1u : 0u);
+            if (two)
+              mma_bf16(tacc + colstride, sw128_desc(a_addr + kABytes + kk * 32), sw128_desc(b_addr + kk * 32), idesc,
+                       (kt | kk) ? 1u : 0u);
+          }
           issued = true;
           mma_commit(smem_u32(&sh.op_empty[s]));
           RT(rt_issue += clock64() - rt1;)
@@ -1396,8 +1431,15 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       asm volatile("bar.sync %0, 128;" ::"r"(bar) : "memory");
       if (!got) { ok = false; break; }
       fence_after();
-      epilogue<MODE>(T, tmem + b * colstride, q, lane, sh.red[eg], 0, 16, (ew & 3) * 32 + lane, 128,
+      epilogue<MODE>(T, tmem + b * bufcols, q, lane, sh.red[eg], 0, 16, (ew & 3) * 32 + lane, 128,
                      MODE != WGRAD ? ystage0 + ew * 4096 : nullptr, ybuf, bar);
+      if (kAMult == 2 && min(T.d->mtile_rows, T.Mrows - T.m0) > kBM) {
+        // rows 128-255 of the tile, from the second accumulator half
+        Tile T2 = T;
+        T2.m0 += kBM;
+        epilogue<MODE>(T2, tmem + b * bufcols + colstride, q, lane, sh.red[eg], 0, 16, (ew & 3) * 32 + lane, 128,
+                       nullptr, ybuf, bar);
+      }
       fence_before();
       mbar_arrive(smem_u32(&sh.tempty[b]));
       RT(rt_b += clock64() - rt1;)
@@ -1482,9 +1524,9 @@ static cudaError_t launch_mode(ConvKernel kern, const ConvDesc* tab, const int* 
   return cudaGetLastError();
 }
 
-bool conv_tma_fits(int bnmax, int raw_bytes) {
+bool conv_tma_fits(int mode, int bnmax, int raw_bytes) {
   const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - kTmaYStage;
-  return avail / (raw_bytes + tma_op_bytes(bnmax)) >= 2;
+  return avail / (raw_bytes + tma_op_bytes(mode, bnmax)) >= 2;
 }
 
 cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
@@ -1505,7 +1547,7 @@ cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, in
     if (sms <= 0) sms = 148;
     attr[mode] = true;
   }
-  const size_t smem = tma_smem_bytes(bnmax, raw_bytes, tma_extra(mode, xw));
+  const size_t smem = tma_smem_bytes(mode, bnmax, raw_bytes, tma_extra(mode, xw));
   if (smem > (size_t)kTmaSmemBudget) return cudaErrorInvalidValue;
   const int grid = total < sms ? total : sms;
   kern<<<grid, kTmaThreads, smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, status);
@@ -1637,6 +1679,7 @@ extern "C" int pnn_conv_wgrad_noalloc(const float* x, const float* dy, float* dw
   cd.mtiles = (rsc + kTcBM - 1) / kTcBM;
   cd.ntiles = (k + 255) / 256;
   cd.ntile_w = 256;
+  cd.mtile_rows = kBM;
   cd.op_bf16 = 1;
   const int base = cd.mtiles * cd.ntiles;
   int splits = (int)std::min<int64_t>((mp + 255) / 256, (2 * 152 + base - 1) / base);

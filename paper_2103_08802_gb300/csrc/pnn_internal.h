@@ -43,6 +43,7 @@ struct ConvDesc {
   int32_t splits, pix_per_split;
   int32_t mtiles, ntiles;             // tile grid of this instance
   int32_t ntile_w;                    // N columns of a tile when ntiles > 1 (256, or 128 TMA-fed)
+  int32_t mtile_rows;                 // M rows of a tile: 128, or 256 (TMA-fed weight gradient: two MMA halves)
   int32_t op_bf16;                    // round both contraction operands to bf16 (bf16 mode)
   // TMA-fed tensor-core variant (stride 1): device addresses of two 2-D tensor
   // maps (CUtensorMap, 128-byte aligned) -- tma_a over the A source rows
@@ -190,8 +191,8 @@ cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
 // largest over the launch's instances, a multiple of 1024)
 cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
                             int raw_bytes, int32_t* status, cudaStream_t st);
-// whether the TMA-fed kernel holds at least two stages of this size
-bool conv_tma_fits(int bnmax, int raw_bytes);
+// whether the TMA-fed kernel of `mode` holds at least two stages of this size
+bool conv_tma_fits(int mode, int bnmax, int raw_bytes);
 // record a message for pnn_last_error(NULL) and return `code`
 int set_last_error(int code, const char* msg);
 

@@ -122,6 +122,14 @@ static int tc_ntile_w(int kind, int variant) {
   return variant == 1 && (kind == K_CONV_FWD_TC || kind == K_DGRAD_TC) ? 128 : 256;
 }
 
+// M rows of a tensor-core conv tile: 256 for the TMA-fed weight gradient of a
+// layer with at most 128 input channels (two MMA halves share each B operand, so
+// a layer with up to 256 (r,s,c) rows makes one pass over the pixels; a tile
+// then holds whole taps, all inside the activation box), 128 otherwise.
+static int tc_mtile_rows(int kind, int variant, int C) {
+  return kind == K_WGRAD_TC && variant == 1 && C <= 128 ? 256 : kTcBM;
+}
+
 // The TMA-fed weight gradient loads a k-step's activation rows for all taps
 // as one halo box and the output-gradient rows as another: channels 8..64
 // (dividing 64) or multiples of 128 up to 512, at most 128 output channels
@@ -131,7 +139,7 @@ static bool tma_wgrad_ok(int k, int stride, int pad, int C, int K, int W, bool x
   if (!(C % 8 == 0 && ((C <= 64 && 64 % C == 0) || (C % 128 == 0 && C <= 512)))) return false;
   if (K % 8 != 0 || K > 128) return false;
   const WgBoxes b = wg_boxes(C, K, W, pad, xbf);
-  return b.hrows <= 256 && conv_tma_fits(128, wg_raw_bytes(b));
+  return b.hrows <= 256 && conv_tma_fits(2, 128, wg_raw_bytes(b));
 }
 
 const char* kKindName[K_NKINDS] = {"conv_fwd", "conv_dgrad", "conv_wgrad", "wgrad_reduce", "elementwise",
@@ -480,7 +488,7 @@ struct pnn_net {
                              ? 1
                              : 0;
           }
-          wg.mtiles = cdiv(RSC, kTcBM);
+          wg.mtiles = cdiv(RSC, tc_mtile_rows(wg.kind, wg.variant, vals[f.in].C));
           wg.ntiles = cdiv(ov.C, 256);
           pix_align = 64;
         } else {
@@ -1007,6 +1015,7 @@ int pnn_net::build_tables() {
             c.R = o.k; c.S = o.k; c.stride = o.stride; c.pad = o.pad;
             c.mtiles = o.mtiles; c.ntiles = o.ntiles;
             c.ntile_w = tc_ntile_w(o.kind, o.variant);
+            c.mtile_rows = tc_mtile_rows(o.kind, o.variant, iv.C);
             c.op_bf16 = act_dt == DT_BF16 && ((o.kind != K_DGRAD && o.kind != K_WGRAD) || !opt.grad_fp32);
             if (o.kind == K_DGRAD_TC) c.w = (const char*)(ws + off_wt) + params[o.w].off * 2;
             if ((o.kind == K_CONV_FWD_TC || o.kind == K_DGRAD_TC) && o.variant == 1) {
