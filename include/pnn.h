@@ -269,6 +269,17 @@ uint64_t pnn_debug_word(void);
 int pnn_conv_wgrad_noalloc(const float* x, const float* dy, float* dw, int32_t batch, int32_t h, int32_t w,
                            int32_t c, int32_t k, int32_t ksize, int32_t stride, void* stream);
 
+/* Failure-detection self-test (no counterpart in the paper).  Every device
+ * wait of the library's kernels is bounded: on expiry a kernel records status
+ * 3, releases what it holds and returns, and the host reports PNN_ETIMEOUT.
+ * This call exercises that path on purpose: it launches one thread that
+ * arrives once on an mbarrier expecting two arrivals and waits on it with the
+ * kernels' bounded wait, limited to limit_ns (0 < limit_ns <= 1e10).  The
+ * phase never completes, so the call returns PNN_ETIMEOUT after about
+ * limit_ns, and the CUDA context stays usable.  stream: cudaStream_t (NULL =
+ * legacy default stream); synchronises it.  Allocates nothing. */
+int pnn_selftest_wait_timeout(int64_t limit_ns, void* stream);
+
 const char* pnn_last_error(const pnn_net* net);
 const char* pnn_status_string(int status);
 

@@ -1598,6 +1598,47 @@ extern "C" int pnn_role_cycles(unsigned long long* out, int reset) {
 #endif
 
 // ============================================================================
+// Bounded-wait self-test: one thread arrives once on an mbarrier that expects
+// two arrivals and then waits on it through the conv kernels' bounded wait;
+// the phase can never complete, so the wait gives up after limit_ns and the
+// kernel records status 3 (the code the conv kernels use for an expired wait)
+// and returns normally.
+namespace pnn {
+namespace {
+static __device__ int32_t g_wait_probe_status;
+__global__ void k_wait_probe(unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  abort_flag = 0;
+  mbar_init(smem_u32(&bar), 2);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  mbar_arrive(smem_u32(&bar));
+  const bool ok = mbar_wait_for(smem_u32(&bar), 0, &abort_flag, limit_ns);
+  g_wait_probe_status = ok ? 0 : 3;
+}
+}  // namespace
+}  // namespace pnn
+
+extern "C" int pnn_selftest_wait_timeout(int64_t limit_ns, void* stream) {
+  if (limit_ns <= 0 || limit_ns > 10000000000ll)
+    return pnn::set_last_error(PNN_EINVAL, "pnn_selftest_wait_timeout: limit_ns must be in (0, 1e10]");
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int32_t host = -1;
+  cudaError_t e = cudaMemcpyToSymbolAsync(pnn::g_wait_probe_status, &host, sizeof host, 0, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) {
+    pnn::k_wait_probe<<<1, 32, 0, st>>>((unsigned long long)limit_ns);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess)
+    e = cudaMemcpyFromSymbolAsync(&host, pnn::g_wait_probe_status, sizeof host, 0, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return pnn::set_last_error(PNN_ECUDA, cudaGetErrorString(e));
+  if (host == 3) return pnn::set_last_error(PNN_ETIMEOUT, "device wait gave up after its limit (self-test)");
+  return host == 0 ? PNN_OK : pnn::set_last_error(PNN_ECUDA, "wait self-test did not report");
+}
+
+// ============================================================================
 // Allocation-free weight gradient: the same tensor-core kernel, with its
 // split-K partial sums, launch descriptors and status word in fixed-size
 // file-scope device arrays instead of memory from the caller or the library.

@@ -58,15 +58,19 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// bounded wait: false on timeout or when another thread of the CTA aborted
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+// bounded wait: false after limit_ns or when another thread of the CTA aborted
+__device__ __forceinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                              unsigned long long limit_ns) {
   if (mbar_try(bar, parity)) return true;
   const unsigned long long t0 = gtimer();
   while (true) {
     if (mbar_try(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (gtimer() - t0 > kWaitNs) return false;
+    if (gtimer() - t0 > limit_ns) return false;
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  return mbar_wait_for(bar, parity, abort_flag, kWaitNs);
 }
 // time-bounded wait that ignores the abort flag (drains committed MMAs)
 __device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity) {

@@ -103,6 +103,7 @@ def load():
         "pnn_debug_word": (C.c_uint64, []),
         "pnn_kernel_kind_name": (C.c_char_p, [I32]),
         "pnn_conv_wgrad_noalloc": (C.c_int, [P, P, P, I32, I32, I32, I32, I32, I32, I32, P]),
+        "pnn_selftest_wait_timeout": (C.c_int, [C.c_int64, P]),
         "pnn_last_error": (C.c_char_p, [P]),
         "pnn_status_string": (C.c_char_p, [C.c_int]),
     }

@@ -88,3 +88,10 @@ def test_calls_without_workspace_fail_cleanly(pnn):
     assert lib.pnn_sgd_step(net.h, 0.1) == 7
     assert lib.pnn_backward(None) == 1            # null handle
     assert lib.pnn_status_string(5) == b"device wait timed out"
+
+
+def test_wait_selftest_rejects_bad_limits(pnn):
+    lib = pnn.load()
+    assert lib.pnn_selftest_wait_timeout(0, None) == 1          # PNN_EINVAL, before any CUDA call
+    assert lib.pnn_selftest_wait_timeout(-5, None) == 1
+    assert b"limit_ns" in lib.pnn_last_error(None)
