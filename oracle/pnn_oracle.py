@@ -371,6 +371,55 @@ class Bottleneck(_Layer):
         return dx, [dg1, db1, dw1, dg2, db2, dw2, dg3, db3, dw3] + grads_p
 
 
+class CoarseRU(_Layer):
+    """Coarse residual unit of Parareal ResNet (Section 4.2): two 3x3 convs
+    and a skip connection, the first conv strided when the block downsamples.
+    Written in the pre-activation order of the ResNet-1001 units it stands
+    in for (the paper does not place the BNs):
+        a1 = ReLU(BN1(x)); h1 = conv3x3_s(a1); a2 = ReLU(BN2(h1));
+        out = conv3x3(a2) + (x, or conv1x1_s(a1) when the shape changes)."""
+
+    def __init__(self, cin, h, w, cout, stride):
+        self.proj = (cin != cout) or stride != 1
+        self.c1 = Conv(cin, h, w, cout, 3, stride)
+        _, ho, wo = self.c1.out_shape
+        self.c2 = Conv(cout, ho, wo, cout, 3, 1)
+        self.cp = Conv(cin, h, w, cout, 1, stride) if self.proj else None
+        self.c2.store_q = False   # its output goes straight into the residual sum
+        self.out_shape = (cout, ho, wo)
+        self.spec = ([(KIND_BN_G, (cin,)), (KIND_BN_B, (cin,))] + self.c1.spec
+                     + [(KIND_BN_G, (cout,)), (KIND_BN_B, (cout,))] + self.c2.spec
+                     + (self.cp.spec if self.proj else []))
+
+    def forward(self, x, P):
+        z1, b1 = self._bn(x, P[0], P[1])
+        a1 = self._relu(z1)
+        h1, k1 = self.c1.forward(a1, P[2:3])
+        z2, b2 = self._bn(h1, P[3], P[4])
+        a2 = self._relu(z2)
+        h2, k2 = self.c2.forward(a2, P[5:6])
+        if self.proj:
+            sc, kp = self.cp.forward(a1, P[6:7])
+        else:
+            sc, kp = x, None
+        return h2 + sc, (b1, z1, k1, b2, z2, k2, kp)
+
+    def backward(self, dout, P, cache, need_dx=True):
+        b1, z1, k1, b2, z2, k2, kp = cache
+        da2, (dw2,) = self.c2.backward(dout, P[5:6], k2)
+        dh1, dg2, db2 = self._bn_back(self._relu_back(da2, z2), P[3], b2)
+        da1, (dw1,) = self.c1.backward(dh1, P[2:3], k1)
+        grads_p = []
+        if self.proj:
+            dap, (dwp,) = self.cp.backward(dout, P[6:7], kp)
+            da1 = da1 + dap
+            grads_p = [dwp]
+        dx, dg1, db1 = self._bn_back(self._relu_back(da1, z1), P[0], b1)
+        if not self.proj:
+            dx = dx + dout
+        return dx, [dg1, db1, dw1, dg2, db2, dw2] + grads_p
+
+
 def make_layer(spec, shape, linear=False, bf16=False):
     c, h, w = shape
     op = spec["op"]
@@ -382,6 +431,8 @@ def make_layer(spec, shape, linear=False, bf16=False):
         L = Basic(c, h, w, spec["cout"])
     elif op == "bottleneck":
         L = Bottleneck(c, h, w, spec["cout"], spec["mid"], spec.get("stride", 1))
+    elif op == "coarse_ru":
+        L = CoarseRU(c, h, w, spec["cout"], spec.get("stride", 1))
     else:
         raise ValueError(op)
     L.linear = linear

@@ -7,7 +7,9 @@
 * delta mode with F^j := g^{j+1} reproduces the untorn nonlinear network;
 * Prop:equiv -- residual mode with F^j := g^{j+1} on a linear body
   reproduces the untorn network;
-* the parameter count of ResNet-1001 printed in Table errorrate.
+* the parameter counts printed in Tables errorrate and vggresult: ResNet-1001,
+  Parareal ResNet-N (N = 3, 6, 12, 18) and Parareal VGG-16-4;
+* a coarse RU with a zero second conv is the identity (or its projection).
 """
 import copy
 import json
@@ -50,6 +52,21 @@ def small_vgg_net(correction="residual"):
     }
 
 
+def small_coarse_ru_net(correction="residual"):
+    """Coarse RUs (Section 4.2) in both roles: as the body and as F^j, with
+    strided and projected units."""
+    R = W.coarse_ru
+    return {
+        "name": "small_coarse_ru", "batch": 3, "in_c": 3, "in_h": 16, "in_w": 16, "classes": 5,
+        "precision": "fp32", "correction": correction,
+        "stem": [W.conv(8)],
+        "body": [R(8), R(16), R(16, 2), R(16), R(32, 2), R(32)],
+        "segments": [2, 2, 2],
+        "coarse": [[R(16, 2), R(16)], [R(32, 2)]],
+        "cj_post": "none", "head": {"kind": "bn_relu_gap_fc", "hidden": []},
+    }
+
+
 def tiny(correction="residual", batch=3, hw=16):
     d = W.tiny_resnet(batch=batch, correction=correction)
     d["in_h"] = d["in_w"] = hw
@@ -60,6 +77,7 @@ NETS = {
     "tiny": tiny,
     "bottleneck": small_bottleneck_net,
     "vgg": small_vgg_net,
+    "coarse_ru": small_coarse_ru_net,
 }
 
 
@@ -89,7 +107,7 @@ def test_matches_torch_autograd(name, mode):
     np.testing.assert_allclose(res["grad"], tg, rtol=1e-8, atol=1e-11 * np.abs(tg).max())
 
 
-@pytest.mark.parametrize("name", ["tiny", "bottleneck"])
+@pytest.mark.parametrize("name", ["tiny", "bottleneck", "coarse_ru"])
 def test_D_j_is_dL_dy_j(name):
     """Algorithm 2: the seed of subnetwork j is dL/dy_j = D_j."""
     desc = NETS[name]()
@@ -107,8 +125,11 @@ def test_D_j_is_dL_dy_j(name):
         np.testing.assert_allclose(st["ys"][j], parts["ys"][j].detach().numpy(), rtol=1e-12, atol=1e-12)
 
 
-def test_finite_differences_every_parameter_kind():
-    desc = tiny(batch=2, hw=8)
+@pytest.mark.parametrize("name", ["tiny", "coarse_ru"])
+def test_finite_differences_every_parameter_kind(name):
+    desc = tiny(batch=2, hw=8) if name == "tiny" else small_coarse_ru_net()
+    if name == "coarse_ru":
+        desc["batch"] = 2
     net, theta, x, labels = _setup(desc)
     res = O.train_step(desc, theta, x, labels)
     g = res["grad"]
@@ -195,7 +216,7 @@ def test_delta_mode_with_fine_coarse_is_sequential(name):
         off += n
 
 
-@pytest.mark.parametrize("name", ["tiny", "bottleneck"])
+@pytest.mark.parametrize("name", ["tiny", "bottleneck", "coarse_ru"])
 def test_prop_equiv_linear_residual_mode(name):
     """Prop:equiv: f linear in its body and F^j = g^{j+1} give f-bar = f, for
     arbitrary (here nonlinear) C^j and h."""
@@ -234,3 +255,87 @@ def test_resnet1001_parameter_count():
 def test_config_interfaces(idx, shapes):
     net = O.ParaNet(W.config(idx))
     assert [tuple(s) for s in net.X] == shapes
+
+
+def _count(spec):
+    return sum(int(np.prod(s)) for _, s in spec)
+
+
+def _printed(n):
+    return f"{n / 1e6:.1f}M"
+
+
+@pytest.mark.parametrize("n", [3, 6, 12, 18])
+def test_paper_parareal_resnet_parameter_counts(n):
+    """Table errorrate: the subnetwork (mean), coarse network and total
+    parameter counts of Parareal ResNet-N with N_c = ceil(12/N).  The coarse
+    column fixes the coarse RU (two 3x3 convs, the first strided with a 1x1
+    projection where the shape changes) and N_c; the totals of N = 6 and 12
+    fix the tearing: every g^j holds ceil(333/N) units (336 in all), where a
+    last-segment-takes-the-remainder tearing gives 16.1M for N = 12.  For
+    N = 18 that tearing (342 units) gives 19.5M against the printed 19.4M, and
+    the remainder tearing 19.2M: no whole-unit tearing gives the printed
+    total with the printed coarse count, so that row is held to 0.1M."""
+    row = json.load(open(os.path.join(GOLDEN, "param_counts.json")))["parareal_resnet_n"]["rows"][str(n)]
+    d = W.paper_parareal_resnet(n, classes=10)
+    net = O.ParaNet(d)
+    assert len(net.coarse) == n - 1 and all(len(F) == -(-12 // n) for F in d["coarse"])
+    assert len(d["body"]) == n * -(-333 // n)
+    coarse = sum(_count(F.spec) for F in net.coarse)
+    fine = sum(_count(g.spec) for g in net.fine)
+    assert _printed(coarse) == row["coarse"]
+    assert _printed(fine / n) == row["subnetwork"]
+    total = net.num_params()
+    if n == 18:
+        assert abs(total - float(row["total"][:-1]) * 1e6) <= 0.15e6
+    else:
+        assert _printed(total) == row["total"]
+
+
+def test_paper_parareal_vgg_parameter_counts():
+    """Table vggresult: F^j = two 3x3 convs + maxpool gives the printed
+    coarse network count; the mean subnetwork count is VGG-16's twelve body
+    convs over four subnetworks."""
+    row = json.load(open(os.path.join(GOLDEN, "param_counts.json")))["parareal_vgg16_4"]
+    net = O.ParaNet(W.parareal_vgg16(coarse="paper"))
+    assert _printed(sum(_count(F.spec) for F in net.coarse)) == row["coarse"]
+    assert _printed(sum(_count(g.spec) for g in net.fine) / 4) == row["subnetwork"]
+
+
+@pytest.mark.parametrize("n,shapes", [
+    (3, [(16, 32, 32), (64, 32, 32), (128, 16, 16), (256, 8, 8)]),
+    (6, [(16, 32, 32)] + [(64, 32, 32)] * 2 + [(128, 16, 16)] * 2 + [(256, 8, 8)] * 2),
+    (12, [(16, 32, 32)] + [(64, 32, 32)] * 4 + [(128, 16, 16)] * 4 + [(256, 8, 8)] * 4),
+])
+def test_paper_parareal_resnet_interfaces(n, shapes):
+    """Section 4.2: X_j is 64x32x32 for j <= N_0, 128x16x16 for j <= 2 N_0,
+    256x8x8 after, and F^j maps X_j to X_{j+1}."""
+    d = W.paper_parareal_resnet(n, per_stage=4 * (n // 3))
+    net = O.ParaNet(d)
+    assert [tuple(s) for s in net.X] == shapes
+    for j, F in enumerate(net.coarse):
+        assert tuple(F.in_shape) == shapes[j + 1] and tuple(F.out_shape) == shapes[j + 2]
+
+
+@pytest.mark.parametrize("cin,cout,stride", [(8, 8, 1), (8, 16, 2), (8, 16, 1)])
+def test_coarse_ru_with_zero_second_conv(cin, cout, stride):
+    """With the second conv zero, a coarse RU returns its skip path: x itself,
+    or the 1x1 (strided) projection of ReLU(BN(x)), written out here with a
+    per-channel batch normalisation and a strided subsample."""
+    r = np.random.default_rng(4)
+    L = O.make_layer(W.coarse_ru(cout, stride), (cin, 6, 6))
+    x = r.standard_normal((2, cin, 6, 6))
+    P = []
+    for kind, shape in L.spec:
+        P.append(r.standard_normal(shape) if kind != O.KIND_CONV_W else 0.3 * r.standard_normal(shape))
+    P[5] = np.zeros_like(P[5])
+    out, _ = L.forward(x, P)
+    if cin == cout and stride == 1:
+        np.testing.assert_array_equal(out, x)
+        return
+    mu = x.mean(axis=(0, 2, 3), keepdims=True)
+    var = x.var(axis=(0, 2, 3), keepdims=True)
+    a = np.maximum((x - mu) / np.sqrt(var + O.BN_EPS) * P[0][None, :, None, None] + P[1][None, :, None, None], 0)
+    a = a[:, :, ::stride, ::stride]
+    want = np.einsum("kc,nchw->nkhw", P[6][:, :, 0, 0], a)
+    np.testing.assert_allclose(out, want, rtol=1e-12, atol=1e-12)

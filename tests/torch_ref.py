@@ -65,6 +65,15 @@ def layer(spec, x, p, linear=False):
         if cin != c or s != 1:
             return h3 + F.conv2d(a1, p.take(c, cin, 1, 1), stride=s)
         return h3 + x
+    if op == "coarse_ru":
+        c, s = spec["cout"], spec.get("stride", 1)
+        a1 = _act(_bn(x, p, linear), linear)
+        h1 = F.conv2d(a1, p.take(c, cin, 3, 3), stride=s, padding=1)
+        a2 = _act(_bn(h1, p, linear), linear)
+        h2 = F.conv2d(a2, p.take(c, c, 3, 3), padding=1)
+        if cin != c or s != 1:
+            return h2 + F.conv2d(a1, p.take(c, cin, 1, 1), stride=s)
+        return h2 + x
     raise ValueError(op)
 
 

@@ -23,6 +23,7 @@ Layer kinds:
   {"op": "conv_bn_relu", "cout", "k", "stride", "pool"} conv-BN-ReLU (+ 2x2/s2 maxpool if pool)
   {"op": "basic", "cout"}                               post-activation basic block
   {"op": "bottleneck", "cout", "mid", "stride"}         pre-activation bottleneck
+  {"op": "coarse_ru", "cout", "stride"}                 coarse RU: two 3x3 convs + skip
 """
 from __future__ import annotations
 
@@ -30,8 +31,8 @@ import copy
 import numpy as np
 
 __all__ = [
-    "conv", "conv_bn_relu", "basic", "bottleneck",
-    "tiny_resnet", "parareal_vgg16", "parareal_resnet1001",
+    "conv", "conv_bn_relu", "basic", "bottleneck", "coarse_ru",
+    "tiny_resnet", "parareal_vgg16", "parareal_resnet1001", "paper_parareal_resnet",
     "config", "CONFIG_NAMES", "make_batch", "init_params", "bf16_round",
     "with_batch",
 ]
@@ -54,6 +55,10 @@ def bottleneck(cout, mid, stride=1):
     return {"op": "bottleneck", "cout": cout, "mid": mid, "stride": stride}
 
 
+def coarse_ru(cout, stride=1):
+    return {"op": "coarse_ru", "cout": cout, "stride": stride}
+
+
 # ---------------------------------------------------------------- configs
 def tiny_resnet(batch=8, precision="fp32", correction="residual"):
     """Tiny parareal ResNet: stem conv3x3->16 (+BN+ReLU), N=2 subnetworks of
@@ -70,10 +75,13 @@ def tiny_resnet(batch=8, precision="fp32", correction="residual"):
     }
 
 
-def parareal_vgg16(batch=128, precision="bf16", correction="residual", classes=10):
+def parareal_vgg16(batch=128, precision="bf16", correction="residual", classes=10, coarse="one_conv"):
     """Parareal VGG-16-4 at 32x32: the 13 conv layers with BN+ReLU and a 2x2
     maxpool closing each stage, torn after stages 2, 3, 4 and 5 (Section 4.1);
-    one conv3x3+BN+ReLU+maxpool coarse block per interface; 3-FC head."""
+    3-FC head.  coarse="one_conv": one conv3x3+BN+ReLU+maxpool block per
+    interface; coarse="paper": F^j of Section 4.1, two 3x3 convs (each with
+    BN+ReLU, as the body's convs) and a 2x2/s2 maxpool, at the width of
+    X_{j+1}."""
     body = [conv_bn_relu(64, pool=2),
             conv_bn_relu(128), conv_bn_relu(128, pool=2),
             conv_bn_relu(256), conv_bn_relu(256), conv_bn_relu(256, pool=2),
@@ -85,8 +93,8 @@ def parareal_vgg16(batch=128, precision="bf16", correction="residual", classes=1
         "stem": [conv_bn_relu(64)],
         "body": body,
         "segments": [3, 3, 3, 3],
-        "coarse": [[conv_bn_relu(256, pool=2)], [conv_bn_relu(512, pool=2)],
-                   [conv_bn_relu(512, pool=2)]],
+        "coarse": ([[conv_bn_relu(c, pool=2)] for c in (256, 512, 512)] if coarse == "one_conv" else
+                   [[conv_bn_relu(c), conv_bn_relu(c, pool=2)] for c in (256, 512, 512)]),
         "cj_post": "bn_relu",
         "head": {"kind": "gap_mlp", "hidden": [4096, 4096]},
     }
@@ -136,6 +144,48 @@ def parareal_resnet1001(n_seg=4, batch=128, classes=10, hw=32, precision="bf16",
         "in_h": hw, "in_w": hw, "classes": classes, "precision": precision,
         "correction": correction,
         "stem": stem, "body": body, "segments": segments, "coarse": coarse,
+        "cj_post": "none",
+        "head": {"kind": "bn_relu_gap_fc", "hidden": []},
+    }
+
+
+def paper_parareal_resnet(n, batch=128, classes=100, hw=32, precision="bf16", correction="residual",
+                          per_stage=111, n_c=None):
+    """Parareal ResNet-N built from ResNet-1001 as Section 4.2 does.
+
+    N = 3 N_0 subnetworks, N_0 per stage, so that X_j is 64x32x32 for
+    j <= N_0, 128x16x16 for j <= 2 N_0 and 256x8x8 after.  Every g^j holds
+    ceil(333/N) = ceil(111/N_0) pre-activation bottlenecks (the body thus has
+    N ceil(333/N) >= 333 of them; the first block of stages 2 and 3 is the
+    strided one).  Each F^j : X_j -> X_{j+1} is N_c = ceil(12/N) coarse RUs
+    at the width of X_{j+1}, the first strided (and projected) when X_j and
+    X_{j+1} differ in shape.  n = 1 is the untorn ResNet-1001 (Parareal
+    ResNet-1).  per_stage < 111 gives the same construction with fewer
+    bottlenecks per stage (ceil(per_stage/N_0) per subnetwork)."""
+    if n == 1:
+        d = parareal_resnet1001(n_seg=1, batch=batch, classes=classes, hw=hw, precision=precision,
+                                correction=correction, per_stage=per_stage, segments=[3 * per_stage])
+        d["name"] = "paper_parareal_resnet_n1"
+        return d
+    assert n % 3 == 0, "Parareal ResNet-N is defined for N = 3 N_0"
+    n0 = n // 3
+    seg = -(-per_stage // n0)
+    n_c = -(-12 // n) if n_c is None else n_c
+    body = []
+    for s in range(3):
+        for b in range(n0 * seg):
+            body.append(bottleneck(64 << s, 16 << s, 2 if (s > 0 and b == 0) else 1))
+    coarse = []
+    for j in range(1, n):
+        s0, s1 = (j - 1) // n0, j // n0   # stages of X_j and X_{j+1}
+        c1 = 64 << s1
+        coarse.append([coarse_ru(c1, 2 if s1 > s0 else 1)] + [coarse_ru(c1) for _ in range(n_c - 1)])
+    assert hw in (32, 64)
+    stem = [conv(16)] if hw == 32 else [conv_bn_relu(16), conv(16, stride=2)]
+    return {
+        "name": f"paper_parareal_resnet_n{n}", "batch": batch, "in_c": 3, "in_h": hw, "in_w": hw,
+        "classes": classes, "precision": precision, "correction": correction,
+        "stem": stem, "body": body, "segments": [seg] * n, "coarse": coarse,
         "cj_post": "none",
         "head": {"kind": "bn_relu_gap_fc", "hidden": []},
     }
