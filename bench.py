@@ -7,6 +7,7 @@ subnetworks, batch 256, 3x64x64 synthetic N(0,1) images (stride-2 stem),
 training iteration (Algorithm 1 forward, Algorithm 2 backward, SGD update).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config I]
+                  [--paper-net resnet_nN|vgg16_4]
 
 Prints one JSON line (rank 0).  For N > 1 (launched by torchrun) every rank
 trains an independent replica on its own batch (the path is single-GPU by
@@ -37,6 +38,10 @@ FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 CONV_KINDS = ("conv_fwd", "conv_dgrad", "conv_wgrad", "conv_fwd_tc", "conv_dgrad_tc", "conv_wgrad_tc")
 
 
+PAPER_NETS = {f"resnet_n{n}": (lambda n=n: W.paper_parareal_resnet(n)) for n in (1, 3, 6, 12, 18, 24)}
+PAPER_NETS["vgg16_4"] = lambda: W.parareal_vgg16(coarse="paper")
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -48,6 +53,12 @@ def parse():
     ap.add_argument("--cpu-sample-batch", type=int, default=1)
     ap.add_argument("--stream-fp32", type=int, default=1, choices=[0, 1],
                     help="keep the residual stream and correction tensors in fp32 (1) or bf16 (0)")
+    ap.add_argument("--paper-net", default=None, choices=sorted(PAPER_NETS),
+                    help="time one of the paper's own constructions instead of --config: Parareal "
+                         "ResNet-N of Section 4.2 (batch 128, 3x32x32, 100 classes, the workload of "
+                         "Table grad) or Parareal VGG-16-4 with the two-conv coarse blocks of Section 4.1")
+    ap.add_argument("--lr", type=float, default=0.1,
+                    help="SGD learning rate (Section 4 uses 0.1; the step's work does not depend on it)")
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch (profiling a small case of the same network)")
     return ap.parse_args()
@@ -181,12 +192,16 @@ def our_arm(args, desc, rank, local, world, dist):
     build.build()
     torch.cuda.set_device(local)
     stream = torch.cuda.Stream()
-    net = pnn.ParaNet(desc, seed=0, stream=stream, stream_fp32=bool(args.stream_fp32))
+    net = pnn.ParaNet(desc, seed=0, stream=stream, stream_fp32=bool(args.stream_fp32), lr=args.lr)
     B = desc["batch"]
     x, labels = W.make_batch(desc, seed=1000 + desc.get("config_index", 0) + rank)
     xd = torch.from_numpy(x).cuda()
     ld = torch.from_numpy(labels).cuda()
     loss = torch.zeros(1, device="cuda")
+    # every measured section below starts again from the initial weights: a
+    # fixed synthetic batch trained for dozens of steps at Section 4's lr can
+    # diverge, and the step's work does not depend on the weights' values
+    theta0 = net.get_params()
     torch.cuda.synchronize()
 
     for _ in range(max(3, args.warmup)):
@@ -212,6 +227,7 @@ def our_arm(args, desc, rank, local, world, dist):
     value = B * args.steps * world / (ms / 1e3)
 
     # ------------------------------------------------ per-kernel profile (eager steps)
+    net.set_params(theta0)
     net.profile(True)
     for _ in range(args.steps):
         net.forward(xd, ld, loss)
@@ -221,9 +237,12 @@ def our_arm(args, desc, rank, local, world, dist):
     net.profile(False)
     fw, bw, up = net.launch_counts()
     launches_per_step = fw + bw + up
-    phases = net.timings()
+    phases_eager = net.timings()
+    net.set_params(theta0)
+    phases = net.time_phases(xd, ld, args.steps)
 
     # ------------------------------------------------ end to end through the host API
+    net.set_params(theta0)
     xh = torch.from_numpy(x).pin_memory()
     lh = torch.from_numpy(labels).pin_memory()
     net.train_step_host(xh, lh)  # captures the host-staged step graph
@@ -273,7 +292,7 @@ def our_arm(args, desc, rank, local, world, dist):
         "config": {"workload": desc["name"] + "_b%d_%dpx_c%d" % (B, desc["in_h"], desc["classes"]),
                    "batch": B, "input": "3x%dx%d" % (desc["in_h"], desc["in_w"]), "classes": desc["classes"],
                    "subnetworks": len(desc["segments"]), "correction": desc.get("correction", "residual"),
-                   "residual_stream": "fp32" if args.stream_fp32 else "bf16",
+                   "residual_stream": "fp32" if args.stream_fp32 else "bf16", "lr": args.lr,
                    "l2": "inputs larger than L2 (%.1f GB workspace per step)" % (net.workspace_bytes / 1e9),
                    "parallelism": "replicas" if world > 1 else "single-gpu"},
         "conv_tflops": conv_flops / (conv_ms / 1e3) / 1e12 if conv_ms else None,
@@ -289,6 +308,7 @@ def our_arm(args, desc, rank, local, world, dist):
                         "gflop_per_step": v[2] / args.steps / 1e9, "gb_per_step": v[3] / args.steps / 1e9}
                     for k, v in sorted(prof.items(), key=lambda kv: -kv[1][0])},
         "phases_ms": phases,
+        "phases_ms_eager": phases_eager,
         "cpu_baseline": cpu,
         "e2e": e2e,
         "gpu_launches": launches_per_step * args.steps,
@@ -301,7 +321,12 @@ def our_arm(args, desc, rank, local, world, dist):
 def main():
     args = parse()
     rank, local, world, dist = dist_setup(args.gpus)
-    desc = W.config(args.config, batch=args.batch)
+    if args.paper_net:
+        desc = PAPER_NETS[args.paper_net]()
+        if args.batch:
+            desc["batch"] = args.batch
+    else:
+        desc = W.config(args.config, batch=args.batch)
     if args.impl == "reference":
         reference_arm(args, desc, rank)
     else:

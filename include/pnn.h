@@ -58,8 +58,15 @@ typedef enum { PNN_CORR_RESIDUAL = 0, PNN_CORR_DELTA = 1 } pnn_correction;
  *   PNN_CONV_BN_RELU    conv -> BN -> ReLU, then a 2x2/s2 maxpool if pool != 0
  *   PNN_BASIC           post-activation basic block: ReLU(BN(conv(ReLU(BN(conv x)))) + x)
  *   PNN_BOTTLENECK      pre-activation bottleneck (cout, mid, stride on the 3x3
- *                       conv, 1x1 projection shortcut when the shape changes) */
-typedef enum { PNN_CONV = 0, PNN_CONV_BN_RELU = 1, PNN_BASIC = 2, PNN_BOTTLENECK = 3 } pnn_layer_op;
+ *                       conv, 1x1 projection shortcut when the shape changes)
+ *   PNN_COARSE_RU       coarse RU of Parareal ResNet (Section 4.2): two 3x3 convs
+ *                       and a skip, in pre-activation order
+ *                       conv3x3(ReLU(BN(conv3x3_s(ReLU(BN x))))) + skip, the
+ *                       stride on the first conv, the skip a 1x1 (strided)
+ *                       projection of ReLU(BN x) when the shape changes */
+typedef enum {
+  PNN_CONV = 0, PNN_CONV_BN_RELU = 1, PNN_BASIC = 2, PNN_BOTTLENECK = 3, PNN_COARSE_RU = 4
+} pnn_layer_op;
 
 /* Postprocessing h (eq:barf's epsilon part) */
 typedef enum { PNN_HEAD_GAP_FC = 0, PNN_HEAD_BN_RELU_GAP_FC = 1, PNN_HEAD_GAP_MLP = 2 } pnn_head_kind;
@@ -200,6 +207,17 @@ int pnn_get_tensor(pnn_net* net, int32_t which, int32_t j, float* host, size_t n
  * post for forward, the same four for backward, then the SGD update and the
  * total: ms[10]. */
 int pnn_get_timings(pnn_net* net, float ms[10]);
+/* Per-phase device time of whole training steps replayed from CUDA graphs,
+ * in the order of pnn_get_timings (ms[10]): each phase (pre, fine, coarse,
+ * post forward; post, coarse, fine, pre backward; update) is captured as its
+ * own graph and bracketed by events on the library stream, and the times are
+ * the mean over `steps` steps.  The phases of Tables gradvgg and grad, without
+ * the launch gaps of an eager step.  x and labels are device pointers as for
+ * pnn_train_step; each step updates the parameters.  A network that has not
+ * stepped yet first takes one untimed eager step (it initialises the momentum
+ * buffers), so it then takes steps + 1 steps in all.  Synchronises the library
+ * stream.  PNN_ESTATE while profiling is enabled; PNN_EINVAL for steps <= 0. */
+int pnn_time_phases(pnn_net* net, const float* x, const int32_t* labels, int32_t steps, float ms[10]);
 /* Counts of the step's kernel launches: forward, backward, update. */
 int pnn_launch_counts(const pnn_net* net, int32_t counts[3]);
 

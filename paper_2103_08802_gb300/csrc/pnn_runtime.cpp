@@ -212,6 +212,11 @@ struct pnn_net {
   const float* g_x = nullptr;
   const int32_t* g_labels = nullptr;
   float* g_loss = nullptr;
+  // one graph per phase for pnn_time_phases (pre, fine, coarse, post forward;
+  // post, coarse, fine, pre backward; update), captured for (px, plabels)
+  cudaGraphExec_t pgexec[9] = {};
+  const float* px = nullptr;
+  const int32_t* plabels = nullptr;
   std::string err;
   int counts[3] = {0, 0, 0};
   // profiling: events around every launch, accumulated per kind
@@ -410,6 +415,20 @@ struct pnn_net {
         int sc = proj ? conv(L, a1, wp, ly.cout, 1, ly.stride, -1, act_dt, key0, 5) : x;
         if (vals[sc].virt) sc = ew(L, {sc}, {1.f}, false, sdt, key0, 5);
         return conv(L, a3, w3, ly.cout, 1, 1, sc, sdt, key0, 6);
+      }
+      case PNN_COARSE_RU: {
+        const bool proj = cin != ly.cout || ly.stride != 1;
+        int g1 = take(pc, 1, cin), b1 = take(pc, 2, cin);
+        int w1 = take(pc, 0, ly.cout, cin, 3, 3);
+        int g2 = take(pc, 1, ly.cout), b2 = take(pc, 2, ly.cout);
+        int w2 = take(pc, 0, ly.cout, ly.cout, 3, 3);
+        int wp = proj ? take(pc, 0, ly.cout, cin, 1, 1) : -1;
+        int a1 = bn_virtual(L, x, g1, b1, true, key0, 0);
+        int h1 = conv(L, a1, w1, ly.cout, 3, ly.stride, -1, act_dt, key0, 1);
+        int a2 = bn_virtual(L, h1, g2, b2, true, key0, 2);
+        int sc = proj ? conv(L, a1, wp, ly.cout, 1, ly.stride, -1, act_dt, key0, 3) : x;
+        if (vals[sc].virt) sc = ew(L, {sc}, {1.f}, false, sdt, key0, 3);
+        return conv(L, a2, w2, ly.cout, 3, 1, sc, sdt, key0, 4);
       }
     }
     return -1;
@@ -706,7 +725,7 @@ int pnn_net::plan(const pnn_desc* d) {
   auto check_layers = [&](const pnn_layer* ls, int n) -> bool {
     for (int i = 0; i < n; ++i) {
       const pnn_layer& l = ls[i];
-      if (l.op < 0 || l.op > 3 || l.cout <= 0 || (l.stride != 1 && l.stride != 2)) return false;
+      if (l.op < 0 || l.op > 4 || l.cout <= 0 || (l.stride != 1 && l.stride != 2)) return false;
       if ((l.op == PNN_CONV || l.op == PNN_CONV_BN_RELU) && l.k != 1 && l.k != 3) return false;
       if (l.op == PNN_BOTTLENECK && l.mid <= 0) return false;
       if (l.op == PNN_BASIC && l.stride != 1) return false;
@@ -1718,6 +1737,99 @@ int pnn_train_step(pnn_net* n, const float* x, const int32_t* labels, float* los
   return n->cuda_check(cudaGraphLaunch(n->gexec, n->stream), "graph launch");
 }
 
+static void drop_phase_graphs(pnn_net* n) {
+  for (auto& g : n->pgexec)
+    if (g) {
+      cudaGraphExecDestroy(g);
+      g = nullptr;
+    }
+}
+
+int pnn_time_phases(pnn_net* n, const float* x, const int32_t* labels, int32_t steps, float ms[10]) {
+  BOUND_OR_FAIL(n);
+  if (!x || !labels || !ms) return n->fail(PNN_EINVAL, "null argument");
+  if (steps <= 0) return n->fail(PNN_EINVAL, "steps must be positive");
+  if (n->prof) return n->fail(PNN_ESTATE, "phase timing needs profiling off");
+  if (n->first_step) {
+    int r = pnn_train_step(n, x, labels, nullptr);
+    if (r) return r;
+  }
+  if (n->pgexec[0] && (x != n->px || labels != n->plabels)) drop_phase_graphs(n);
+  n->x_dev = x;
+  n->labels_dev = labels;
+  if (!n->pgexec[0]) {
+    for (int k = 0; k < 9; ++k) {
+      cudaError_t e = cudaStreamBeginCapture(n->stream, cudaStreamCaptureModeThreadLocal);
+      if (e != cudaSuccess) return n->cuda_check(e, "begin capture");
+      int r = PNN_OK;
+      if (k == 0) {
+        e = launch_pack_input(x, n->ws + n->vals[n->x_in].off, n->vals[n->x_in].dt, n->B, n->in_c, n->in_h, n->in_w,
+                              n->stream);
+        r = e == cudaSuccess ? n->run_phase(0) : n->cuda_check(e, "pack input");
+      } else if (k < 4) {
+        r = n->run_phase(k);
+      } else if (k == 6) {
+        r = n->run_phase(6);
+        if (!r) r = n->run_phase(7);
+      } else if (k < 8) {
+        r = n->run_phase(k == 7 ? 8 : k);
+      } else {
+        r = n->do_sgd(0.f, false);
+        n->first_step = false;
+      }
+      cudaGraph_t g = nullptr;
+      e = cudaStreamEndCapture(n->stream, &g);
+      if (r || e != cudaSuccess) {
+        if (g) cudaGraphDestroy(g);
+        drop_phase_graphs(n);
+        return r ? r : n->cuda_check(e, "end capture");
+      }
+      e = cudaGraphInstantiate(&n->pgexec[k], g, 0);
+      cudaGraphDestroy(g);
+      if (e != cudaSuccess) {
+        drop_phase_graphs(n);
+        return n->cuda_check(e, "instantiate graph");
+      }
+    }
+    n->px = x;
+    n->plabels = labels;
+  }
+  // events: ev[k] before phase graph k, ev[9] after the update
+  cudaEvent_t ev[10];
+  for (auto& e : ev)
+    if (cudaEventCreate(&e) != cudaSuccess) return n->cuda_check(cudaGetLastError(), "event");
+  double acc[9] = {};
+  cudaError_t e = cudaSuccess;
+  for (int s = 0; s < steps && e == cudaSuccess; ++s) {
+    for (int k = 0; k < 9 && e == cudaSuccess; ++k) {
+      e = cudaEventRecord(ev[k], n->stream);
+      if (e == cudaSuccess) e = cudaGraphLaunch(n->pgexec[k], n->stream);
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(ev[9], n->stream);
+    if (e == cudaSuccess) e = cudaEventSynchronize(ev[9]);
+    for (int k = 0; k < 9 && e == cudaSuccess; ++k) {
+      float t = 0.f;
+      e = cudaEventElapsedTime(&t, ev[k], ev[k + 1]);
+      acc[k] += t;
+    }
+  }
+  for (auto& v : ev) cudaEventDestroy(v);
+  if (e != cudaSuccess) return n->cuda_check(e, "phase timing");
+  n->state = 0;
+  // graph order pre_f fine_f coarse_f post_f post_b coarse_b fine_b pre_b update
+  // -> the order of pnn_get_timings: four forward, four backward (pre, fine,
+  // coarse, post), update, total
+  const int map[8] = {0, 1, 2, 3, 7, 6, 5, 4};
+  float tot = 0.f;
+  for (int i = 0; i < 8; ++i) {
+    ms[i] = (float)(acc[map[i]] / steps);
+    tot += ms[i];
+  }
+  ms[8] = (float)(acc[8] / steps);
+  ms[9] = tot + ms[8];
+  return pnn_sync(n);
+}
+
 int pnn_train_step_host(pnn_net* n, const float* x_host, const int32_t* labels_host, float* loss_host) {
   BOUND_OR_FAIL(n);
   if (!x_host || !labels_host) return n->fail(PNN_EINVAL, "null x or labels");
@@ -1752,6 +1864,7 @@ void pnn_destroy(pnn_net* n) {
   if (!n) return;
   if (n->gexec) cudaGraphExecDestroy(n->gexec);
   if (n->graph) cudaGraphDestroy(n->graph);
+  drop_phase_graphs(n);
   for (auto& v : n->ev)
     if (v) cudaEventDestroy(v);
   for (auto& v : n->pev)
@@ -1913,6 +2026,7 @@ int pnn_profile(pnn_net* n, int32_t enable) {
     n->gexec = nullptr;
     n->graph = nullptr;
   }
+  drop_phase_graphs(n);
   n->prof = enable != 0;
   n->pnext = 0;
   n->pfold = 0;

@@ -17,7 +17,7 @@ LIB_PATH = os.path.join(HERE, "libpnn.so")
 PNN_OK = 0
 PRECISION = {"bf16": 0, "fp32": 1}
 CORRECTION = {"residual": 0, "delta": 1}
-LAYER_OP = {"conv": 0, "conv_bn_relu": 1, "basic": 2, "bottleneck": 3}
+LAYER_OP = {"conv": 0, "conv_bn_relu": 1, "basic": 2, "bottleneck": 3, "coarse_ru": 4}
 HEAD = {"gap_fc": 0, "bn_relu_gap_fc": 1, "gap_mlp": 2}
 CJ_POST = {"none": 0, "bn_relu": 1}
 TENSOR = {"x": 0, "y": 1, "r": 2, "rtilde": 3, "ytilde": 4, "D": 5, "logits": 6}
@@ -94,6 +94,7 @@ def load():
         "pnn_tensor_size": (C.c_int, [P, I32, I32, C.POINTER(SZ)]),
         "pnn_get_tensor": (C.c_int, [P, I32, I32, P, SZ]),
         "pnn_get_timings": (C.c_int, [P, C.POINTER(C.c_float)]),
+        "pnn_time_phases": (C.c_int, [P, C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_float)]),
         "pnn_launch_counts": (C.c_int, [P, C.POINTER(I32)]),
         "pnn_profile": (C.c_int, [P, I32]),
         "pnn_profile_read": (C.c_int, [P, I32, C.POINTER(C.c_double), C.POINTER(C.c_int64),
@@ -286,6 +287,15 @@ class ParaNet:
     def timings(self):
         ms = (C.c_float * 10)()
         self._check(self.lib.pnn_get_timings(self.h, ms))
+        keys = ["pre_f", "fine_f", "coarse_f", "post_f", "pre_b", "fine_b", "coarse_b", "post_b", "update", "total"]
+        return dict(zip(keys, list(ms)))
+
+    def time_phases(self, x, labels, steps=5):
+        """Per-phase ms of `steps` graph-replayed training steps (device x, labels)."""
+        self._args(x, labels, None)
+        ms = (C.c_float * 10)()
+        self._check(self.lib.pnn_time_phases(self.h, C.c_void_p(x.data_ptr()), C.c_void_p(labels.data_ptr()),
+                                             int(steps), ms))
         keys = ["pre_f", "fine_f", "coarse_f", "post_f", "pre_b", "fine_b", "coarse_b", "post_b", "update", "total"]
         return dict(zip(keys, list(ms)))
 

@@ -38,9 +38,17 @@ def test_library_exports_every_declared_symbol(pnn):
         assert hasattr(lib, n), n
 
 
-@pytest.mark.parametrize("idx", range(5))
+PAPER_NETS = {
+    "paper_resnet_n3": lambda: W.paper_parareal_resnet(3),
+    "paper_resnet_n18": lambda: W.paper_parareal_resnet(18),
+    "paper_resnet_n24_delta": lambda: W.paper_parareal_resnet(24, correction="delta"),
+    "paper_vgg16_4": lambda: W.parareal_vgg16(coarse="paper"),
+}
+
+
+@pytest.mark.parametrize("idx", list(range(5)) + list(PAPER_NETS))
 def test_plan_matches_oracle_parameter_table(pnn, idx):
-    d = W.config(idx)
+    d = W.config(idx) if isinstance(idx, int) else PAPER_NETS[idx]()
     net = pnn.ParaNet(d, bind=False)
     spec = net.param_spec()
     ospec = O.ParaNet(d).spec
