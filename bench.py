@@ -57,6 +57,11 @@ def parse():
                     help="time one of the paper's own constructions instead of --config: Parareal "
                          "ResNet-N of Section 4.2 (batch 128, 3x32x32, 100 classes, the workload of "
                          "Table grad) or Parareal VGG-16-4 with the two-conv coarse blocks of Section 4.1")
+    ap.add_argument("--tearing", default="none", choices=["none", "uniform", "flops", "bytes", "time"],
+                    help="ResNet-1001 workloads: cut the body into subnetworks of equal RU count (uniform, "
+                         "Section 4.2) or of equal cost (the remark after Table grad): algorithmic FLOPs, "
+                         "HBM bytes, or the device time of each layer measured on the untorn network; "
+                         "every choice but none also reports each subnetwork's measured time")
     ap.add_argument("--lr", type=float, default=0.1,
                     help="SGD learning rate (Section 4 uses 0.1; the step's work does not depend on it)")
     ap.add_argument("--batch", type=int, default=None,
@@ -185,6 +190,59 @@ def reference_arm(args, desc, rank):
 
 
 # ---------------------------------------------------------------- our arm
+def layer_times(desc, stream, steps=2):
+    """Device ms of each body layer's forward and backward launches in the
+    untorn network (the body as one segment), from an eager profiled step."""
+    import copy
+    import torch
+    from paper_2103_08802_gb300 import pnn
+    d1 = copy.deepcopy(desc)
+    d1["segments"] = [len(desc["body"])]
+    d1["coarse"] = []
+    net = pnn.ParaNet(d1, seed=0, stream=stream)
+    x, labels = W.make_batch(d1, seed=7)
+    xd, ld = torch.from_numpy(x).cuda(), torch.from_numpy(labels).cuda()
+    theta0 = net.get_params()
+    for _ in range(2):
+        net.train_step(xd, ld)
+    t = [0.0] * len(desc["body"])
+    for _ in range(steps):
+        net.set_params(theta0)
+        net.profile(True)
+        net.forward(xd, ld)
+        net.backward()
+        for r in net.profile_trace():
+            if r["phase"] in (1, 7) and r["block"] >= 0:
+                t[r["block"]] += r["ms"] / steps
+        net.profile(False)
+    net.close()
+    del net
+    torch.cuda.empty_cache()
+    return t
+
+
+def retear(args, desc, stream):
+    """The workload torn as --tearing asks, and a record of the cut: layers per
+    segment, each segment's summed layer time measured on the untorn network,
+    and the largest of them (the parallel phase's virtual wall-clock of
+    Table grad if every subnetwork had a GPU of its own)."""
+    from paper_2103_08802_gb300 import pnn
+    t = layer_times(desc, stream)
+    n = len(desc["segments"])
+    if args.tearing == "uniform":
+        seg = list(desc["segments"])
+    else:
+        cost = t if args.tearing == "time" else pnn.block_costs(desc, args.tearing)
+        seg = pnn.partition(cost, n)
+        desc = W.config(args.config, batch=args.batch, segments=seg)
+    b = np.cumsum([0] + seg)
+    seg_ms = [float(sum(t[b[j]:b[j + 1]])) for j in range(n)]
+    rec = {"kind": args.tearing, "segments": seg, "segment_fine_ms": seg_ms,
+           "virtual_fine_ms": max(seg_ms), "mean_segment_ms": float(np.mean(seg_ms)),
+           "layer_ms_total": float(sum(t))}
+    return desc, rec
+
+
 def our_arm(args, desc, rank, local, world, dist):
     import torch
     from paper_2103_08802_gb300 import build, pnn
@@ -192,6 +250,11 @@ def our_arm(args, desc, rank, local, world, dist):
     build.build()
     torch.cuda.set_device(local)
     stream = torch.cuda.Stream()
+    tearing = None
+    if args.tearing != "none":
+        if args.paper_net or args.config not in (2, 3, 4):
+            raise SystemExit("--tearing applies to the ResNet-1001 configurations 2, 3 and 4")
+        desc, tearing = retear(args, desc, stream)
     net = pnn.ParaNet(desc, seed=0, stream=stream, stream_fp32=bool(args.stream_fp32), lr=args.lr)
     B = desc["batch"]
     x, labels = W.make_batch(desc, seed=1000 + desc.get("config_index", 0) + rank)
@@ -293,6 +356,7 @@ def our_arm(args, desc, rank, local, world, dist):
                    "batch": B, "input": "3x%dx%d" % (desc["in_h"], desc["in_w"]), "classes": desc["classes"],
                    "subnetworks": len(desc["segments"]), "correction": desc.get("correction", "residual"),
                    "residual_stream": "fp32" if args.stream_fp32 else "bf16", "lr": args.lr,
+                   "tearing": "uniform" if args.tearing == "none" else args.tearing,
                    "l2": "inputs larger than L2 (%.1f GB workspace per step)" % (net.workspace_bytes / 1e9),
                    "parallelism": "replicas" if world > 1 else "single-gpu"},
         "conv_tflops": conv_flops / (conv_ms / 1e3) / 1e12 if conv_ms else None,
@@ -307,6 +371,7 @@ def our_arm(args, desc, rank, local, world, dist):
         "kernels": {k: {"ms_per_step": v[0] / args.steps, "launches_per_step": v[1] / args.steps,
                         "gflop_per_step": v[2] / args.steps / 1e9, "gb_per_step": v[3] / args.steps / 1e9}
                     for k, v in sorted(prof.items(), key=lambda kv: -kv[1][0])},
+        "tearing": tearing,
         "phases_ms": phases,
         "phases_ms_eager": phases_eager,
         "cpu_baseline": cpu,

@@ -207,6 +207,26 @@ int pnn_get_tensor(pnn_net* net, int32_t which, int32_t j, float* host, size_t n
  * post for forward, the same four for backward, then the SGD update and the
  * total: ms[10]. */
 int pnn_get_timings(pnn_net* net, float ms[10]);
+/* ---- tearing (Section 4.2, the remark after Table grad: a decomposition of the
+ * body into subnetworks of equal computational cost rather than equal numbers
+ * of RUs).  Both calls are host-only and need no GPU. */
+typedef enum { PNN_COST_FLOPS = 0, PNN_COST_BYTES = 1 } pnn_cost_kind;
+/* Cost of each of the n = desc->n_body layers of the block-repetitive part g
+ * in the untorn network (desc's body as one segment, no coarse network): the
+ * algorithmic FLOPs (conv FLOPs = 2 * B*P*Q*K*C*R*S over the layer's forward,
+ * data-gradient and weight-gradient convolutions) or HBM bytes (each operand
+ * read once, each result written once, as pnn_profile_read counts them) of the
+ * layer's forward and backward ops under opts (NULL: defaults).  desc->segments
+ * and the coarse fields are ignored.  out: caller-owned, n doubles. */
+int pnn_block_costs(const pnn_desc* desc, const pnn_options* opts, int32_t kind, double* out, int32_t n);
+/* Cut n layers with costs cost[0..n-1] (finite, >= 0) into n_seg consecutive
+ * non-empty segments whose largest cost sum is as small as possible (exact).
+ * Among the optimal cuts it returns the one whose segments, from the first on,
+ * each take as many layers as the optimum allows.  segments: caller-owned,
+ * n_seg ints (layers per segment, summing to n).  PNN_EINVAL unless
+ * 1 <= n_seg <= n. */
+int pnn_partition(const double* cost, int32_t n, int32_t n_seg, int32_t* segments);
+
 /* Per-phase device time of whole training steps replayed from CUDA graphs,
  * in the order of pnn_get_timings (ms[10]): each phase (pre, fine, coarse,
  * post forward; post, coarse, fine, pre backward; update) is captured as its
@@ -249,6 +269,9 @@ int pnn_profile_read(pnn_net* net, int32_t kind, double* ms, int64_t* launches, 
 typedef struct pnn_trace {
   int32_t kind, variant, phase, instances, tiles;
   int32_t shape[6];
+  int32_t block; /* fine-wave launches (phases 1 and 7): the layer's position
+                    in its segment, its index in g for an untorn network
+                    (n_seg = 1); -1 for every other launch */
   double ms, flops, bytes;
 } pnn_trace;
 int pnn_profile_trace(pnn_net* net, int32_t max, pnn_trace* out, int32_t* count);

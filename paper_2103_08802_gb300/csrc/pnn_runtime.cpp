@@ -18,6 +18,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <limits>
 #include <map>
 #include <string>
 #include <tuple>
@@ -104,6 +105,7 @@ struct Launch {
   int shape[6];         // first op: conv (C_in, C_out, k, stride, H_out, W_out); else (C, H, W, 0, 0, 0)
   int esz = 4;          // TMA-fed conv: largest element size of the A sources
   int raw = 0;          // TMA-fed conv: raw slot bytes of one stage
+  int block = -1;       // fine forward / backward: position of the layer in its segment
 };
 
 // The TMA-fed tensor-core conv (variant 1 of the TC forward / data-gradient
@@ -690,6 +692,46 @@ struct pnn_net {
   int plan(const pnn_desc* d);
   int bind(void* dev, size_t bytes);
   int build_tables();
+  // Algorithmic work of one op, added to flops / bytes: conv FLOPs =
+  // 2 * B*P*Q*K*C*R*S; bytes = each operand read once, each result written once
+  // (a read-modify-write for accumulating results).
+  void op_cost(const POp& o, double& flops, double& bytes) const {
+    auto esz = [&](int v) {
+      return vals[v].virt ? (vals[vals[v].src].dt == DT_F32 ? 4.0 : 2.0) : (vals[v].dt == DT_F32 ? 4.0 : 2.0);
+    };
+    auto elems = [&](int v) { return (double)B * vals[v].H * vals[v].W * vals[v].C; };
+    const double wsz = act_dt == DT_BF16 ? 2.0 : 4.0;
+    switch (o.kind) {
+      case K_CONV_FWD: case K_CONV_FWD_TC: case K_DGRAD: case K_DGRAD_TC: case K_WGRAD: case K_WGRAD_TC: {
+        const Value& iv = vals[o.in]; const Value& ov = vals[o.out];
+        const double macs = (double)B * ov.H * ov.W * ov.C * iv.C * o.k * o.k;
+        flops += 2 * macs;
+        const double wbytes = (double)ov.C * iv.C * o.k * o.k * wsz;
+        if (o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC)
+          bytes += elems(o.in) * esz(o.in) + wbytes + elems(o.out) * esz(o.out) + (o.res >= 0 ? elems(o.res) * esz(o.res) : 0);
+        else if (o.kind == K_DGRAD || o.kind == K_DGRAD_TC)
+          bytes += elems(o.out) * 4 + wbytes + elems(o.in) * 4 * (o.acc ? 2 : 1);
+        else
+          bytes += elems(o.in) * esz(o.in) + elems(o.out) * 4 + (double)o.splits * ov.C * iv.C * o.k * o.k * 4;
+        break;
+      }
+      case K_EW: {
+        const int ref = o.out >= 0 ? o.out : o.ins[0];
+        for (int i = 0; i < o.nin; ++i) bytes += elems(o.ins[i]) * esz(o.ins[i]);
+        if (o.out >= 0) bytes += elems(ref) * esz(ref);
+        break;
+      }
+      case K_EW_BWD: bytes += elems(o.in) * 4 * (1 + o.nin) + (o.relu ? elems(o.in) * esz(o.in) : 0); break;
+      case K_BNB_RED: bytes += elems(o.in) * 4 + elems(norms[o.norm].h) * esz(norms[o.norm].h); break;
+      case K_BNB_APPLY:
+        bytes += elems(o.in) * 4 + elems(norms[o.norm].h) * esz(norms[o.norm].h) + elems(norms[o.norm].h) * 4 * (o.acc ? 2 : 1);
+        break;
+      case K_POOL_FWD: bytes += elems(o.in) * esz(o.in) + elems(o.out) * esz(o.out); break;
+      case K_POOL_BWD: bytes += elems(o.out) * 4 + elems(o.in) * (esz(o.in) + 4); break;
+      case K_WREDUCE: bytes += (double)o.splits * params[o.w].n * 4 + params[o.w].n * 4; break;
+      default: break;
+    }
+  }
   int run_phase(int p);
   int do_forward(bool timed);
   int do_backward(bool timed);
@@ -1214,6 +1256,8 @@ int pnn_net::build_tables() {
       L.flops = 0; L.bytes = 0; L.aux = 16;
       {
         const POp& o = ops[g.ops[0]];
+        if (p == 1) L.block = o.key[0];
+        if (p == 7) L.block = -o.key[0];
         const bool conv = o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC || o.kind == K_DGRAD ||
                           o.kind == K_DGRAD_TC || o.kind == K_WGRAD || o.kind == K_WGRAD_TC;
         const int v = o.in >= 0 ? o.in : (o.out >= 0 ? o.out : o.ins[0]);
@@ -1242,40 +1286,7 @@ int pnn_net::build_tables() {
           }
         }
       if (g.kind == K_CONV_FWD_TC || g.kind == K_DGRAD_TC) L.raw = kTcBM * 64 * L.esz;
-      for (int id : g.ops) {
-        const POp& o = ops[id];
-        auto esz = [&](int v) { return vals[v].virt ? (vals[vals[v].src].dt == DT_F32 ? 4.0 : 2.0) : (vals[v].dt == DT_F32 ? 4.0 : 2.0); };
-        auto elems = [&](int v) { return (double)B * vals[v].H * vals[v].W * vals[v].C; };
-        const double wsz = act_dt == DT_BF16 ? 2.0 : 4.0;
-        switch (o.kind) {
-          case K_CONV_FWD: case K_CONV_FWD_TC: case K_DGRAD: case K_DGRAD_TC: case K_WGRAD: case K_WGRAD_TC: {
-            const Value& iv = vals[o.in]; const Value& ov = vals[o.out];
-            const double macs = (double)B * ov.H * ov.W * ov.C * iv.C * o.k * o.k;
-            L.flops += 2 * macs;
-            const double wbytes = (double)ov.C * iv.C * o.k * o.k * wsz;
-            if (o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC)
-              L.bytes += elems(o.in) * esz(o.in) + wbytes + elems(o.out) * esz(o.out) + (o.res >= 0 ? elems(o.res) * esz(o.res) : 0);
-            else if (o.kind == K_DGRAD || o.kind == K_DGRAD_TC)
-              L.bytes += elems(o.out) * 4 + wbytes + elems(o.in) * 4 * (o.acc ? 2 : 1);
-            else
-              L.bytes += elems(o.in) * esz(o.in) + elems(o.out) * 4 + (double)o.splits * ov.C * iv.C * o.k * o.k * 4;
-            break;
-          }
-          case K_EW: {
-            const int ref = o.out >= 0 ? o.out : o.ins[0];
-            for (int i = 0; i < o.nin; ++i) L.bytes += elems(o.ins[i]) * esz(o.ins[i]);
-            if (o.out >= 0) L.bytes += elems(ref) * esz(ref);
-            break;
-          }
-          case K_EW_BWD: L.bytes += elems(o.in) * 4 * (1 + o.nin) + (o.relu ? elems(o.in) * esz(o.in) : 0); break;
-          case K_BNB_RED: L.bytes += elems(o.in) * 4 + elems(norms[o.norm].h) * esz(norms[o.norm].h); break;
-          case K_BNB_APPLY: L.bytes += elems(o.in) * 4 + elems(norms[o.norm].h) * esz(norms[o.norm].h) + elems(norms[o.norm].h) * 4 * (o.acc ? 2 : 1); break;
-          case K_POOL_FWD: L.bytes += elems(o.in) * esz(o.in) + elems(o.out) * esz(o.out); break;
-          case K_POOL_BWD: L.bytes += elems(o.out) * 4 + elems(o.in) * (esz(o.in) + 4); break;
-          case K_WREDUCE: L.bytes += (double)o.splits * params[o.w].n * 4 + params[o.w].n * 4; break;
-          default: break;
-        }
-      }
+      for (int id : g.ops) op_cost(ops[id], L.flops, L.bytes);
       tstart.push_back(total);
       L.table_off = put(tab.data(), tab.size());
       L.tstart_off = put(tstart.data(), tstart.size() * sizeof(int));
@@ -1646,6 +1657,73 @@ int pnn_create(const pnn_desc* desc, const pnn_options* opts, pnn_net** out) {
   n->ws_bytes = n->cursor;
   n->host_tables.clear();
   *out = n;
+  return PNN_OK;
+}
+
+int pnn_block_costs(const pnn_desc* desc, const pnn_options* opts, int32_t kind, double* out, int32_t n) {
+  if (!desc || !out) return set_global(PNN_EINVAL, "null argument");
+  if (kind != PNN_COST_FLOPS && kind != PNN_COST_BYTES) return set_global(PNN_EINVAL, "bad cost kind");
+  if (n <= 0 || n != desc->n_body) return set_global(PNN_EINVAL, "n must equal the body length");
+  // the untorn network: the whole body as one segment, no coarse network
+  pnn_desc d = *desc;
+  const int32_t whole = desc->n_body;
+  d.segments = &whole;
+  d.n_seg = 1;
+  d.coarse = nullptr;
+  d.coarse_len = nullptr;
+  pnn_net* net = nullptr;
+  int r = pnn_create(&d, opts, &net);
+  if (r) return r;
+  std::fill(out, out + n, 0.0);
+  // forward ops of body layer i carry key[0] = i, their backward ops -i
+  auto add = [&](const std::vector<int>& L, int sign) {
+    for (int id : L) {
+      const POp& o = net->ops[id];
+      const int i = sign * o.key[0];
+      if (i < 0 || i >= n) continue;
+      double f = 0.0, b = 0.0;
+      net->op_cost(o, f, b);
+      out[i] += kind == PNN_COST_FLOPS ? f : b;
+    }
+  };
+  add(net->fine_f[0], 1);
+  add(net->fine_b[0], -1);
+  pnn_destroy(net);
+  return PNN_OK;
+}
+
+int pnn_partition(const double* cost, int32_t n, int32_t n_seg, int32_t* segments) {
+  if (!cost || !segments) return set_global(PNN_EINVAL, "null argument");
+  if (n_seg <= 0 || n < n_seg) return set_global(PNN_EINVAL, "need 1 <= n_seg <= n");
+  std::vector<double> S(n + 1, 0.0);
+  for (int i = 0; i < n; ++i) {
+    if (!(cost[i] >= 0.0) || !std::isfinite(cost[i])) return set_global(PNN_EINVAL, "costs must be finite and >= 0");
+    S[i + 1] = S[i] + cost[i];
+  }
+  // best[i]: the smallest possible largest segment sum over partitions of the
+  // first i layers into j segments (j = 1 .. n_seg, one row at a time)
+  const double inf = std::numeric_limits<double>::infinity();
+  std::vector<double> best(n + 1, inf), next(n + 1, inf);
+  for (int i = 1; i <= n; ++i) best[i] = S[i];
+  for (int j = 2; j <= n_seg; ++j) {
+    std::fill(next.begin(), next.end(), inf);
+    for (int i = j; i <= n; ++i)
+      for (int k = j - 1; k < i; ++k) next[i] = std::min(next[i], std::max(best[k], S[i] - S[k]));
+    best.swap(next);
+  }
+  const double T = best[n];
+  // one optimal partition: every segment from the left takes as many layers as
+  // the bound T allows while leaving one layer for each later segment
+  int start = 0;
+  for (int j = 0; j < n_seg; ++j) {
+    const int later = n_seg - 1 - j;
+    int end = start + 1;
+    if (later == 0) end = n;
+    else
+      while (end < n - later && S[end + 1] - S[start] <= T) ++end;
+    segments[j] = end - start;
+    start = end;
+  }
   return PNN_OK;
 }
 
@@ -2070,6 +2148,7 @@ int pnn_profile_trace(pnn_net* n, int32_t max, pnn_trace* out, int32_t* count) {
     cudaEventElapsedTime(&t, n->pev[2 * i], n->pev[2 * i + 1]);
     r.kind = L.kind; r.variant = L.variant; r.phase = L.phase; r.instances = L.count; r.tiles = L.total;
     for (int j = 0; j < 6; ++j) r.shape[j] = L.shape[j];
+    r.block = L.block;
     r.ms = t; r.flops = L.flops; r.bytes = L.bytes;
   }
   *count = have;

@@ -56,7 +56,8 @@ class Options(C.Structure):
 class Trace(C.Structure):
     _fields_ = [("kind", C.c_int32), ("variant", C.c_int32), ("phase", C.c_int32), ("instances", C.c_int32),
                 ("tiles", C.c_int32),
-                ("shape", C.c_int32 * 6), ("ms", C.c_double), ("flops", C.c_double), ("bytes", C.c_double)]
+                ("shape", C.c_int32 * 6), ("block", C.c_int32), ("ms", C.c_double), ("flops", C.c_double),
+                ("bytes", C.c_double)]
 
 
 _lib = None
@@ -95,6 +96,8 @@ def load():
         "pnn_get_tensor": (C.c_int, [P, I32, I32, P, SZ]),
         "pnn_get_timings": (C.c_int, [P, C.POINTER(C.c_float)]),
         "pnn_time_phases": (C.c_int, [P, C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_float)]),
+        "pnn_block_costs": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_double), C.c_int32]),
+        "pnn_partition": (C.c_int, [C.POINTER(C.c_double), C.c_int32, C.c_int32, C.POINTER(C.c_int32)]),
         "pnn_launch_counts": (C.c_int, [P, C.POINTER(I32)]),
         "pnn_profile": (C.c_int, [P, I32]),
         "pnn_profile_read": (C.c_int, [P, I32, C.POINTER(C.c_double), C.POINTER(C.c_int64),
@@ -124,6 +127,66 @@ def _layers(specs):
     return arr
 
 
+def _make_desc(desc):
+    """The C description of a description dict, and the arrays it points to."""
+    d = Desc()
+    d.batch, d.in_c, d.in_h, d.in_w = desc["batch"], desc["in_c"], desc["in_h"], desc["in_w"]
+    d.classes = desc["classes"]
+    stem, body = _layers(desc["stem"]), _layers(desc["body"])
+    segs = (C.c_int32 * len(desc["segments"]))(*desc["segments"])
+    flat = [l for F in desc["coarse"] for l in F]
+    coarse = _layers(flat)
+    clen = (C.c_int32 * max(1, len(desc["coarse"])))(*[len(F) for F in desc["coarse"]])
+    hidden = list(desc["head"].get("hidden", []))
+    hid = (C.c_int32 * max(1, len(hidden)))(*hidden)
+    d.stem, d.n_stem = stem, len(desc["stem"])
+    d.body, d.n_body = body, len(desc["body"])
+    d.segments, d.n_seg = segs, len(desc["segments"])
+    d.coarse, d.coarse_len = coarse, clen
+    d.cj_post = CJ_POST[desc["cj_post"]]
+    d.head_kind = HEAD[desc["head"]["kind"]]
+    d.head_hidden, d.n_hidden = hid, len(hidden)
+    return d, [stem, body, segs, coarse, clen, hid]
+
+
+def _global_check(lib, status):
+    if status != PNN_OK:
+        msg = lib.pnn_last_error(None)
+        raise PnnError(status, msg.decode() if msg else "")
+
+
+COST = {"flops": 0, "bytes": 1}
+
+
+def block_costs(desc, kind="flops"):
+    """Per-layer cost of the body (forward + backward of the untorn network):
+    a list of len(desc["body"]) floats.  Host only."""
+    lib = load()
+    d, keep = _make_desc(desc)
+    o = Options()
+    lib.pnn_default_options(C.byref(o))
+    o.precision = PRECISION[desc["precision"]]
+    n = len(desc["body"])
+    out = (C.c_double * n)()
+    _global_check(lib, lib.pnn_block_costs(C.byref(d), C.byref(o), COST[kind], out, n))
+    return list(out)
+
+
+def partition(costs, n_seg):
+    """Layers per segment of the min-max contiguous cut of `costs`.  Host only."""
+    lib = load()
+    n = len(costs)
+    c = (C.c_double * max(1, n))(*costs)
+    seg = (C.c_int32 * max(1, n_seg))()
+    _global_check(lib, lib.pnn_partition(c, n, n_seg, seg))
+    return list(seg)[:n_seg]
+
+
+def balanced_segments(desc, n_seg, kind="flops"):
+    """Segments of `desc`'s body of equal cost (Section 4.2's remark)."""
+    return partition(block_costs(desc, kind), n_seg)
+
+
 class ParaNet:
     """A parareal network planned and trained by libpnn.
 
@@ -135,25 +198,7 @@ class ParaNet:
                  device="cuda", bind=True):
         self.lib = load()
         self.desc = desc
-        self._keep = []
-        d = Desc()
-        d.batch, d.in_c, d.in_h, d.in_w = desc["batch"], desc["in_c"], desc["in_h"], desc["in_w"]
-        d.classes = desc["classes"]
-        stem, body = _layers(desc["stem"]), _layers(desc["body"])
-        segs = (C.c_int32 * len(desc["segments"]))(*desc["segments"])
-        flat = [l for F in desc["coarse"] for l in F]
-        coarse = _layers(flat)
-        clen = (C.c_int32 * max(1, len(desc["coarse"])))(*[len(F) for F in desc["coarse"]])
-        hidden = list(desc["head"].get("hidden", []))
-        hid = (C.c_int32 * max(1, len(hidden)))(*hidden)
-        self._keep += [stem, body, segs, coarse, clen, hid]
-        d.stem, d.n_stem = stem, len(desc["stem"])
-        d.body, d.n_body = body, len(desc["body"])
-        d.segments, d.n_seg = segs, len(desc["segments"])
-        d.coarse, d.coarse_len = coarse, clen
-        d.cj_post = CJ_POST[desc["cj_post"]]
-        d.head_kind = HEAD[desc["head"]["kind"]]
-        d.head_hidden, d.n_hidden = hid, len(hidden)
+        d, self._keep = _make_desc(desc)
         o = Options()
         self.lib.pnn_default_options(C.byref(o))
         o.precision = PRECISION[precision or desc["precision"]]
@@ -319,7 +364,7 @@ class ParaNet:
         buf = (Trace * max(1, n.value))()
         self._check(self.lib.pnn_profile_trace(self.h, n.value, buf, C.byref(n)))
         return [{"kind": self.lib.pnn_kernel_kind_name(r.kind).decode(), "variant": r.variant, "phase": r.phase,
-                 "instances": r.instances, "tiles": r.tiles, "shape": tuple(r.shape),
+                 "instances": r.instances, "tiles": r.tiles, "shape": tuple(r.shape), "block": r.block,
                  "ms": r.ms, "flops": r.flops, "bytes": r.bytes} for r in buf[:n.value]]
 
     def launch_counts(self):

@@ -200,18 +200,21 @@ CONFIG_NAMES = [
 ]
 
 
-def config(index, batch=None):
-    """The five measured workloads, by index 0..4."""
+def config(index, batch=None, segments=None):
+    """The five measured workloads, by index 0..4.  `segments` re-tears the
+    ResNet-1001 workloads (2..4) with the same number of subnetworks."""
+    if segments is not None and index not in (2, 3, 4):
+        raise ValueError("only the ResNet-1001 workloads take another tearing")
     if index == 0:
         d = tiny_resnet()
     elif index == 1:
         d = parareal_vgg16()
     elif index == 2:
-        d = parareal_resnet1001(n_seg=4, batch=128, classes=10)
+        d = parareal_resnet1001(n_seg=4, batch=128, classes=10, segments=segments)
     elif index == 3:
-        d = parareal_resnet1001(n_seg=16, batch=128, classes=100)
+        d = parareal_resnet1001(n_seg=16, batch=128, classes=100, segments=segments)
     elif index == 4:
-        d = parareal_resnet1001(n_seg=8, batch=256, classes=200, hw=64)
+        d = parareal_resnet1001(n_seg=8, batch=256, classes=200, hw=64, segments=segments)
     else:
         raise ValueError(index)
     d["config_index"] = index
