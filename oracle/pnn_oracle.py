@@ -99,11 +99,72 @@ def conv2d_backward(x, w, stride, pad, dy, need_dx=True):
     return dx, dw
 
 
+BN_MOMENTUM = 0.1
+
+
+class RunningStats:
+    """Running statistics of every BN layer.  The paper trains with BN and
+    states no rule for them; the reading is PyTorch's BatchNorm2d: per layer a
+    running mean (initially 0) and variance (initially 1); every training-mode
+    evaluation moves them the fraction `momentum` towards the batch mean and
+    the unbiased batch variance (n / (n - 1) times the biased one, n values
+    per channel); an evaluation in eval mode normalises with them instead of
+    the batch's statistics.  A layer is identified by the offset of its gamma
+    in the parameter vector, so the delta form's two evaluations of F^j move
+    the same statistics, in the order they run.
+
+    Flat layout (`flat`, `from_flat`): for every BN layer in parameter order,
+    its C running means, then its C running variances."""
+
+    def __init__(self, spec, momentum=BN_MOMENTUM, eval_mode=False):
+        self.momentum, self.eval = momentum, eval_mode
+        self.layers, off = [], 0
+        for kind, shape in spec:
+            if kind == KIND_BN_G:
+                self.layers.append((off, int(shape[0])))
+            off += int(np.prod(shape))
+        self.mean = {o: np.zeros(c) for o, c in self.layers}
+        self.var = {o: np.ones(c) for o, c in self.layers}
+        self.base = None
+
+    def flat(self):
+        return np.concatenate([np.concatenate([self.mean[o], self.var[o]]) for o, _ in self.layers]) \
+            if self.layers else np.zeros(0)
+
+    def from_flat(self, a):
+        a = np.asarray(a, np.float64)
+        i = 0
+        for o, c in self.layers:
+            self.mean[o] = a[i:i + c].copy()
+            self.var[o] = a[i + c:i + 2 * c].copy()
+            i += 2 * c
+        return self
+
+    def key(self, gamma):
+        return (gamma.__array_interface__["data"][0] - self.base) // 8
+
+
+_RUNNING = None   # the RunningStats batchnorm() consults during a forward, if any
+
+
 def batchnorm(h, gamma, beta):
-    """Training-mode batch normalisation: statistics over (batch, H, W),
-    biased variance, eps = 1e-5.  Returns (z, cache)."""
+    """Batch normalisation over (batch, H, W), eps = 1e-5.  Training mode
+    (the default) normalises with the batch mean and biased variance and, when
+    running statistics are attached, moves them; eval mode normalises with the
+    running statistics.  Returns (z, cache)."""
+    if _RUNNING is not None and _RUNNING.eval:
+        k = _RUNNING.key(gamma)
+        rstd = 1.0 / np.sqrt(_RUNNING.var[k] + BN_EPS)
+        xhat = (h - _RUNNING.mean[k].reshape(1, -1, 1, 1)) * rstd.reshape(1, -1, 1, 1)
+        return gamma.reshape(1, -1, 1, 1) * xhat + beta.reshape(1, -1, 1, 1), None
     mean = h.mean(axis=(0, 2, 3), keepdims=True)
     var = ((h - mean) ** 2).mean(axis=(0, 2, 3), keepdims=True)
+    if _RUNNING is not None:
+        k = _RUNNING.key(gamma)
+        n = h.shape[0] * h.shape[2] * h.shape[3]
+        m = _RUNNING.momentum
+        _RUNNING.mean[k] = (1 - m) * _RUNNING.mean[k] + m * mean.ravel()
+        _RUNNING.var[k] = (1 - m) * _RUNNING.var[k] + m * var.ravel() * (n / max(n - 1, 1))
     rstd = 1.0 / np.sqrt(var + BN_EPS)
     xhat = (h - mean) * rstd
     z = gamma.reshape(1, -1, 1, 1) * xhat + beta.reshape(1, -1, 1, 1)
@@ -639,9 +700,32 @@ class ParaNet:
                                for name, j, _ in self.blocks for g in grads[(name, j)]])
 
     # ------------------------------------------------------------ forward
-    def forward(self, theta, x, labels):
+    def forward(self, theta, x, labels, running=None):
         """Algorithm 1.  Returns the loss and a state holding every interface
-        tensor (x_j, y_j, r_j, rt_j, ytilde), the logits and the caches."""
+        tensor (x_j, y_j, r_j, rt_j, ytilde), the logits and the caches.  With
+        `running` (a RunningStats) every BN moves its running statistics, or
+        normalises with them if `running` is in eval mode."""
+        global _RUNNING
+        theta = np.ascontiguousarray(theta, dtype=np.float64)
+        if running is None:
+            return self._forward(theta, x, labels)
+        running.base = theta.__array_interface__["data"][0]
+        _RUNNING = running
+        try:
+            return self._forward(theta, x, labels)
+        finally:
+            _RUNNING = None
+
+    def infer(self, theta, x, running):
+        """The eval-mode forward: every BN normalises with `running` (a
+        RunningStats or its flat layout).  Returns the logits."""
+        if not isinstance(running, RunningStats):
+            running = RunningStats(self.spec).from_flat(running)
+        running.eval = True
+        _, st = self.forward(theta, x, np.zeros(np.asarray(x).shape[0], np.int64), running)
+        return st["logits"]
+
+    def _forward(self, theta, x, labels):
         P = self.unflatten(theta)
         x = np.asarray(x, dtype=np.float64)
         N = self.N
@@ -668,8 +752,10 @@ class ParaNet:
                 cc.append(c)
                 rt.append(r[j + 1] + f)
             else:
-                f1, c1 = self.coarse[j].forward(xs[j + 1] + rt[j], P[("coarse", j)])
+                # F^j(x_{j+1}) first: with running statistics the order of the
+                # two evaluations matters, and this one does not depend on rt_j
                 f0, c0 = self.coarse[j].forward(xs[j + 1], P[("coarse", j)])
+                f1, c1 = self.coarse[j].forward(xs[j + 1] + rt[j], P[("coarse", j)])
                 cc.append(c1)
                 ccx.append(c0)
                 rt.append(r[j + 1] + f1 - f0)
@@ -719,12 +805,19 @@ class ParaNet:
 
 
 def train_step(desc, theta, x, labels, lr=0.1, momentum=0.9, weight_decay=5e-4,
-               nesterov=True, momentum_buf=None, linear_body=False, precision="fp64"):
+               nesterov=True, momentum_buf=None, linear_body=False, precision="fp64", running=None,
+               bn_momentum=BN_MOMENTUM):
     """Forward, backward and one SGD step.  Returns a dict with loss, grad,
-    theta_new, buf_new and the forward state."""
+    theta_new, buf_new, the forward state and running_new, the BN running
+    statistics after the step (flat layout of RunningStats; `running` gives
+    them before it, default zeros / ones)."""
     net = ParaNet(desc, linear_body, precision)
-    loss, st = net.forward(theta, x, labels)
+    rs = RunningStats(net.spec, bn_momentum)
+    if running is not None:
+        rs.from_flat(running)
+    loss, st = net.forward(theta, x, labels, rs)
     grad = net.backward(st)
     theta_new, buf = sgd_step(np.asarray(theta, np.float64), grad, momentum_buf, lr, momentum,
                               weight_decay, nesterov)
-    return {"net": net, "loss": loss, "grad": grad, "theta_new": theta_new, "buf_new": buf, "state": st}
+    return {"net": net, "loss": loss, "grad": grad, "theta_new": theta_new, "buf_new": buf, "state": st,
+            "running_new": rs.flat()}

@@ -9,7 +9,9 @@
   reproduces the untorn network;
 * the parameter counts printed in Tables errorrate and vggresult: ResNet-1001,
   Parareal ResNet-N (N = 3, 6, 12, 18) and Parareal VGG-16-4;
-* a coarse RU with a zero second conv is the identity (or its projection).
+* a coarse RU with a zero second conv is the identity (or its projection);
+* BN running statistics after a training step and the eval-mode forward that
+  uses them, against torch's own batch_norm buffers.
 """
 import copy
 import json
@@ -339,3 +341,63 @@ def test_coarse_ru_with_zero_second_conv(cin, cout, stride):
     a = a[:, :, ::stride, ::stride]
     want = np.einsum("kc,nchw->nkhw", P[6][:, :, 0, 0], a)
     np.testing.assert_allclose(out, want, rtol=1e-12, atol=1e-12)
+
+
+def _random_running(net, seed):
+    """Running statistics away from their defaults: means N(0, 0.3^2),
+    variances in [0.5, 2]."""
+    rs = O.RunningStats(net.spec)
+    r = np.random.default_rng(seed)
+    for o, c in rs.layers:
+        rs.mean[o] = 0.3 * r.standard_normal(c)
+        rs.var[o] = r.uniform(0.5, 2.0, c)
+    return rs
+
+
+def _torch_running(rs, train):
+    return {"train": train, "stats": {o: (torch.tensor(rs.mean[o]), torch.tensor(rs.var[o])) for o, _ in rs.layers}}
+
+
+@pytest.mark.parametrize("name", list(NETS))
+@pytest.mark.parametrize("mode", ["residual", "delta"])
+def test_running_statistics_match_torch(name, mode):
+    """After a training step every BN's running mean and variance equal what
+    torch's batch_norm leaves in its buffers (momentum 0.1, unbiased batch
+    variance), the delta form's F^j moving its statistics twice."""
+    desc = NETS[name](mode)
+    net, theta, x, labels = _setup(desc)
+    rs = _random_running(net, 9)
+    res = O.train_step(desc, theta, x, labels, running=rs.flat())
+    T.RUNNING = _torch_running(rs, True)
+    try:
+        with torch.no_grad():
+            T.parareal_loss(desc, torch.tensor(theta), x, labels)
+        st = T.RUNNING["stats"]
+    finally:
+        T.RUNNING = None
+    want = np.concatenate([np.concatenate([st[o][0].numpy(), st[o][1].numpy()]) for o, _ in rs.layers])
+    np.testing.assert_allclose(res["running_new"], want, rtol=1e-12, atol=1e-13)
+    # and they moved: every layer's statistics differ from where they started
+    assert not np.allclose(res["running_new"], rs.flat())
+
+
+@pytest.mark.parametrize("name", list(NETS))
+@pytest.mark.parametrize("mode", ["residual", "delta"])
+def test_eval_forward_matches_torch(name, mode):
+    """The eval-mode forward normalises every BN with its running statistics:
+    logits against torch's batch_norm(training=False)."""
+    desc = NETS[name](mode)
+    net, theta, x, labels = _setup(desc)
+    rs = _random_running(net, 10)
+    got = net.infer(theta, x, rs.flat())
+    T.RUNNING = _torch_running(rs, False)
+    try:
+        with torch.no_grad():
+            _, parts = T.parareal_loss(desc, torch.tensor(theta), x, labels, return_parts=True)
+    finally:
+        T.RUNNING = None
+    want = parts["logits"].numpy()
+    np.testing.assert_allclose(got, want, rtol=1e-10, atol=1e-12 * np.abs(want).max())
+    # eval mode differs from training mode (batch statistics)
+    _, st = net.forward(theta, x, labels)
+    assert not np.allclose(st["logits"], got)

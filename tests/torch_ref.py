@@ -23,12 +23,23 @@ class _Params:
         return v
 
 
+# Running statistics: None, or {"train": bool, "stats": {gamma offset: (mean, var)}}.
+# torch.nn.functional.batch_norm moves the buffers itself in training mode
+# (momentum 0.1, unbiased variance) and normalises with them in eval mode.
+RUNNING = None
+
+
 def _bn(h, p, linear=False):
+    off = p.i
     g = p.take(h.shape[1])
     b = p.take(h.shape[1])
     if linear:
         return h
-    return F.batch_norm(h, None, None, g, b, training=True, momentum=0.0, eps=1e-5)
+    if RUNNING is None:
+        return F.batch_norm(h, None, None, g, b, training=True, momentum=0.0, eps=1e-5)
+    rm, rv = RUNNING["stats"].setdefault(
+        off, (torch.zeros(h.shape[1], dtype=F64), torch.ones(h.shape[1], dtype=F64)))
+    return F.batch_norm(h, rm, rv, g, b, training=RUNNING["train"], momentum=0.1, eps=1e-5)
 
 
 def _act(z, linear=False):
@@ -110,7 +121,17 @@ def head(desc, y, p):
 
 
 def _shapes(desc, x):
-    """Output shapes X_0..X_N found by a dry run with zero parameters."""
+    """Output shapes X_0..X_N found by a dry run with zero parameters (which
+    leaves running statistics alone)."""
+    global RUNNING
+    saved, RUNNING = RUNNING, None
+    try:
+        return _dry_shapes(desc, x)
+    finally:
+        RUNNING = saved
+
+
+def _dry_shapes(desc, x):
     with torch.no_grad():
         p = _Params(torch.zeros(10 ** 8, dtype=F64))
         h = stack(desc["stem"], x[:2], p)
@@ -145,9 +166,9 @@ def parareal_loss(desc, theta, x, labels, linear_body=False, return_parts=False)
         if mode == "residual":
             rt = r[j + 1] + stack(desc["coarse"][j], rt, p, linear_body)
         else:
-            f1 = stack(desc["coarse"][j], xs[j + 1] + rt, p, linear_body)
-            p.i = start
             f0 = stack(desc["coarse"][j], xs[j + 1], p, linear_body)
+            p.i = start
+            f1 = stack(desc["coarse"][j], xs[j + 1] + rt, p, linear_body)
             rt = r[j + 1] + f1 - f0
     ytilde = ys[-1] + rt
     z = head(desc, ytilde, p)
