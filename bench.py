@@ -62,6 +62,8 @@ def parse():
                          "Section 4.2) or of equal cost (the remark after Table grad): algorithmic FLOPs, "
                          "HBM bytes, or the device time of each layer measured on the untorn network; "
                          "every choice but none also reports each subnetwork's measured time")
+    ap.add_argument("--inference", action="store_true",
+                    help="time the eval-mode forward (pnn_infer) of the workload instead of training")
     ap.add_argument("--lr", type=float, default=0.1,
                     help="SGD learning rate (Section 4 uses 0.1; the step's work does not depend on it)")
     ap.add_argument("--batch", type=int, default=None,
@@ -243,6 +245,122 @@ def retear(args, desc, stream):
     return desc, rec
 
 
+def roofline_of(prof, steps):
+    """Roofline record of the dominant kernel kind of a profiled window of
+    `steps` steps ({kind: (ms, launches, flops, bytes)})."""
+    pk, src = peaks()
+    name, (kms, kn, kfl, kby) = max(prof.items(), key=lambda kv: kv[1][0])
+    per_launch_ms = kms / kn
+    # the bound follows the kernel's algorithmic intensity: below the ridge point
+    # (peak FLOP/s / peak B/s) the roof is HBM bandwidth
+    ridge = pk["bf16_tflops_sustained"] * 1e12 / (pk["hbm_gbs"] * 1e9)
+    intensity = kfl / kby if kby else float("inf")
+    if name.startswith("conv") and not name.endswith("_tc") and intensity >= FP32_ALU_TFLOPS * 1e3 / pk["hbm_gbs"]:
+        bound, peak, unit = "alu", FP32_ALU_TFLOPS, "TFLOP/s"
+        achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
+    elif name.endswith("_tc") and intensity >= ridge:
+        bound, peak, unit = "tensor", pk["bf16_tflops_sustained"], "TFLOP/s"
+        achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
+    else:
+        bound, peak, unit = "hbm", pk["hbm_gbs"], "GB/s"
+        achieved = kby / kn / (per_launch_ms / 1e3) / 1e9
+    return {"kernel": name, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+            "frac": achieved / peak, "traffic": None, "intensity_flop_per_byte": intensity,
+            "peak_source": (src + (" (hbm_gbs)" if bound == "hbm" else " (bf16_tflops_sustained)"))
+            if bound != "alu" else "derived: 152 SM x 128 FP32 lanes x 2 x 2.07 GHz",
+            "launches_per_step": kn / steps}
+
+
+def infer_arm(args, desc, rank, local, world, dist):
+    """Eval-mode forward throughput (pnn_infer, one CUDA graph per pass) of the
+    same network: parameters and running statistics of a fresh net (the work
+    does not depend on their values)."""
+    import torch
+    from paper_2103_08802_gb300 import build, pnn
+    build.build()
+    torch.cuda.set_device(local)
+    stream = torch.cuda.Stream()
+    net = pnn.ParaNet(desc, seed=0, stream=stream, inference=True)
+    B = desc["batch"]
+    x, labels = W.make_batch(desc, seed=2000 + rank)
+    xd = torch.from_numpy(x).cuda()
+    logits = torch.empty(B * desc["classes"], dtype=torch.float32, device="cuda")
+    for _ in range(max(3, args.warmup)):
+        net.infer(xd, logits)
+    net.sync()
+    with Clocks(local) as clk:
+        barrier(dist)
+        torch.cuda.synchronize()
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for _ in range(args.steps):
+            net.infer(xd, logits)
+        end.record(stream)
+        torch.cuda.synchronize()
+        ms = start.elapsed_time(end)
+        barrier(dist)
+    ms = max_over_ranks(dist, ms)
+    clocks = clk.summary()
+    net.sync()
+    value = B * args.steps * world / (ms / 1e3)
+    net.profile(True)
+    for _ in range(args.steps):
+        net.infer(xd, logits)
+    prof = net.profile_read()
+    net.profile(False)
+    # end to end: pinned host images in, host logits out, every pass
+    xh = torch.from_numpy(x).pin_memory()
+    lh = torch.empty(B * desc["classes"], dtype=torch.float32).pin_memory()
+    net.infer(xd, logits)
+    net.sync()
+    barrier(dist)
+    t0 = time.perf_counter()
+    with torch.cuda.stream(stream):
+        for _ in range(args.steps):
+            xd.copy_(xh, non_blocking=True)
+            net.infer(xd, logits)
+            lh.copy_(logits, non_blocking=True)
+            stream.synchronize()
+    e2e_s = max_over_ranks(dist, time.perf_counter() - t0)
+    if rank != 0:
+        return
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        from oracle import pnn_oracle as O
+        d1 = W.with_batch(desc, args.cpu_sample_batch)
+        onet = O.ParaNet(d1, precision="bf16" if d1["precision"] == "bf16" else "fp64")
+        theta = W.init_params(onet.spec, seed=0, bf16=d1["precision"] == "bf16")
+        x1, _ = W.make_batch(d1)
+        t = time.perf_counter()
+        onet.infer(theta, x1, O.RunningStats(onet.spec))
+        t = time.perf_counter() - t
+        cpu = {"value": d1["batch"] / t, "unit": "images/s", "cores": cores(), "kind": "oracle",
+               "sample": f"{d1['batch']} image(s) of the same network, one eval-mode forward of the CPU fp64 "
+                         f"oracle ({t:.1f} s)"}
+    out = {
+        "metric": "parareal-net eval-mode forward images/sec on 1 GB300", "value": value, "unit": "images/s",
+        "n_gpus": world, "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if desc["precision"] == "bf16" else "fp32", "data": "synthetic",
+        "config": {"workload": desc["name"] + "_b%d_%dpx_c%d_inference" % (B, desc["in_h"], desc["classes"]),
+                   "batch": B, "input": "3x%dx%d" % (desc["in_h"], desc["in_w"]), "classes": desc["classes"],
+                   "subnetworks": len(desc["segments"]), "correction": desc.get("correction", "residual"),
+                   "workspace_gb": net.workspace_bytes / 1e9,
+                   "l2": "inputs larger than L2" if net.workspace_bytes > 129e6 else "workspace within L2",
+                   "parallelism": "replicas" if world > 1 else "single-gpu"},
+        "roofline": roofline_of(prof, args.steps),
+        "kernels": {k: {"ms_per_step": v[0] / args.steps, "launches_per_step": v[1] / args.steps,
+                        "gflop_per_step": v[2] / args.steps / 1e9, "gb_per_step": v[3] / args.steps / 1e9}
+                    for k, v in sorted(prof.items(), key=lambda kv: -kv[1][0])},
+        "cpu_baseline": cpu,
+        "e2e": {"value": B * args.steps * world / e2e_s, "unit": "images/s",
+                "h2d_bytes_per_step": int(x.nbytes), "d2h_bytes_per_step": int(B * desc["classes"] * 4)},
+        "gpu_launches": sum(v[1] for v in prof.values()),
+        "clocks": clocks,
+    }
+    print(json.dumps(out), flush=True)
+
+
 def our_arm(args, desc, rank, local, world, dist):
     import torch
     from paper_2103_08802_gb300 import build, pnn
@@ -323,23 +441,7 @@ def our_arm(args, desc, rank, local, world, dist):
     conv_ms = sum(prof[k][0] for k in CONV_KINDS if k in prof)
     conv_flops = sum(prof[k][2] for k in CONV_KINDS if k in prof)
     total_prof_ms = sum(v[0] for v in prof.values())
-    # dominant kernel kind by device time
-    dom = max(prof.items(), key=lambda kv: kv[1][0])
-    name, (kms, kn, kfl, kby) = dom
-    per_launch_ms = kms / kn
-    # the bound follows the kernel's algorithmic intensity: below the ridge point
-    # (peak FLOP/s / peak B/s) the roof is HBM bandwidth
-    ridge = pk["bf16_tflops_sustained"] * 1e12 / (pk["hbm_gbs"] * 1e9)
-    intensity = kfl / kby if kby else float("inf")
-    if name.startswith("conv") and not name.endswith("_tc") and intensity >= FP32_ALU_TFLOPS * 1e3 / pk["hbm_gbs"]:
-        bound, peak, unit = "alu", FP32_ALU_TFLOPS, "TFLOP/s"
-        achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
-    elif name.endswith("_tc") and intensity >= ridge:
-        bound, peak, unit = "tensor", pk["bf16_tflops_sustained"], "TFLOP/s"
-        achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
-    else:
-        bound, peak, unit = "hbm", pk["hbm_gbs"], "GB/s"
-        achieved = kby / kn / (per_launch_ms / 1e3) / 1e9
+    roofline = roofline_of(prof, args.steps)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         b = args.cpu_sample_batch
@@ -362,12 +464,7 @@ def our_arm(args, desc, rank, local, world, dist):
         "conv_tflops": conv_flops / (conv_ms / 1e3) / 1e12 if conv_ms else None,
         "conv_frac_of_bf16_peak": (conv_flops / (conv_ms / 1e3) / 1e12) / pk["bf16_tflops_sustained"] if conv_ms else None,
         "conv_share_of_device_time": conv_ms / total_prof_ms if total_prof_ms else None,
-        "roofline": {"kernel": name, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                     "frac": achieved / peak, "traffic": None,
-                     "intensity_flop_per_byte": intensity,
-                     "peak_source": (src + (" (hbm_gbs)" if bound == "hbm" else " (bf16_tflops_sustained)"))
-                     if bound != "alu" else "derived: 152 SM x 128 FP32 lanes x 2 x 2.07 GHz",
-                     "launches_per_step": kn / args.steps},
+        "roofline": roofline,
         "kernels": {k: {"ms_per_step": v[0] / args.steps, "launches_per_step": v[1] / args.steps,
                         "gflop_per_step": v[2] / args.steps / 1e9, "gb_per_step": v[3] / args.steps / 1e9}
                     for k, v in sorted(prof.items(), key=lambda kv: -kv[1][0])},
@@ -394,6 +491,8 @@ def main():
         desc = W.config(args.config, batch=args.batch)
     if args.impl == "reference":
         reference_arm(args, desc, rank)
+    elif args.inference:
+        infer_arm(args, desc, rank, local, world, dist)
     else:
         our_arm(args, desc, rank, local, world, dist)
     if dist is not None:

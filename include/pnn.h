@@ -123,10 +123,17 @@ typedef struct {
   int32_t grad_fp32;     /* bf16 mode: contract gradients (dgrad, wgrad) with fp32
                             operands instead of bf16 ones */
   void* stream;          /* cudaStream_t; NULL = legacy default stream */
+  float bn_momentum;     /* rate at which every BN's running statistics follow
+                            the batch's in a training forward (the paper states
+                            no rule; PyTorch's BatchNorm2d default is 0.1) */
+  int32_t inference;     /* 1: plan the forward pass alone for pnn_infer (every BN
+                            normalises with its running statistics; activations
+                            share buffers, no gradients or optimiser state) */
 } pnn_options;
 
 /* Fill o with the defaults: bf16, residual correction, seed 0, lr 0.1,
- * momentum 0.9, weight decay 5e-4, Nesterov (Section 4), stream_fp32 1. */
+ * momentum 0.9, weight decay 5e-4, Nesterov (Section 4), stream_fp32 1,
+ * bn_momentum 0.1, inference 0. */
 void pnn_default_options(pnn_options* o);
 
 /* Plan the network from a description.  Host only: no GPU work, no device
@@ -207,6 +214,34 @@ int pnn_get_tensor(pnn_net* net, int32_t which, int32_t j, float* host, size_t n
  * post for forward, the same four for backward, then the SGD update and the
  * total: ms[10]. */
 int pnn_get_timings(pnn_net* net, float ms[10]);
+/* ---- BN running statistics.  The paper trains with BN and states no rule for
+ * them; this library follows PyTorch's BatchNorm2d: every BN layer keeps a
+ * running mean (0 at pnn_bind_workspace) and variance (1), and each training
+ * forward moves them the fraction opts.bn_momentum towards the batch mean and
+ * the unbiased batch variance (n/(n-1) times the biased one, n values per
+ * channel).  The delta form's two evaluations of F^j move the same statistics,
+ * F^j(x_{j+1}) first.  Layout (host, float): for every BN layer in parameter
+ * order (the order of its gamma in the parameter vector), its C running means,
+ * then its C running variances.  Get and set synchronise the library stream;
+ * n must equal pnn_running_stats_size. */
+int pnn_running_stats_size(const pnn_net* net, size_t* n);
+int pnn_get_running_stats(pnn_net* net, float* host, size_t n);
+int pnn_set_running_stats(pnn_net* net, const float* host, size_t n);
+
+/* ---- inference (Section 3.1's forward, Algorithm 1, in eval mode).  On a net
+ * created with opts.inference = 1: x (device, NCHW float32, batch x in_c x
+ * in_h x in_w) -> logits (device, batch x classes float32, row-major), every
+ * BN normalising with its running statistics (pnn_set_running_stats; a fresh
+ * net holds 0 / 1).  Parameters as pnn_set_params.  The pass is captured as a
+ * CUDA graph on the first call for a given (x, logits) pair and replayed after
+ * that (with profiling enabled, pnn_profile, it runs eagerly so that every
+ * launch is timed); it runs asynchronously on the library stream (pnn_sync
+ * waits).
+ * PNN_ESTATE on a training net; pnn_forward, pnn_backward, pnn_sgd_step,
+ * pnn_train_step, pnn_time_phases and the gradient accessors return PNN_ESTATE
+ * on an inference net, and pnn_get_tensor gives only PNN_T_LOGITS there. */
+int pnn_infer(pnn_net* net, const float* x, float* logits);
+
 /* ---- tearing (Section 4.2, the remark after Table grad: a decomposition of the
  * body into subnetworks of equal computational cost rather than equal numbers
  * of RUs).  Both calls are host-only and need no GPU. */

@@ -425,6 +425,19 @@ __global__ void __launch_bounds__(256) k_bn_fin(const BnFinDesc* __restrict__ ta
   const int inst = find_instance(tstart, n, blockIdx.x);
   const BnFinDesc& d = tab[inst];
   const int c = blockIdx.x - tstart[inst];
+  if (d.eval) {
+    // eval mode: the running statistics stand in for the batch's
+    if (threadIdx.x == 0) {
+      const double mean = d.run_mean[c];
+      const double rstd = 1.0 / sqrt((double)d.run_var[c] + 1e-5);
+      const double sc = (double)d.gamma[c] * rstd;
+      d.mean[c] = (float)mean;
+      d.rstd[c] = (float)rstd;
+      d.scale[c] = (float)sc;
+      d.shift[c] = (float)((double)d.beta[c] - mean * sc);
+    }
+    return;
+  }
   double s1 = 0.0, s2 = 0.0;
   for (int t = threadIdx.x; t < d.tiles; t += 256) {
     s1 += (double)d.part[((int64_t)t * d.C + c) * 2];
@@ -435,6 +448,13 @@ __global__ void __launch_bounds__(256) k_bn_fin(const BnFinDesc* __restrict__ ta
     const double mean = s1 / (double)d.count;
     double var = s2 / (double)d.count - mean * mean;
     if (var < 0.0) var = 0.0;
+    if (d.run_mean) {
+      // running statistics follow the batch mean and the unbiased variance
+      const double m = d.momentum;
+      const double unbiased = d.count > 1 ? var * (double)d.count / (double)(d.count - 1) : var;
+      d.run_mean[c] = (float)((1.0 - m) * (double)d.run_mean[c] + m * mean);
+      d.run_var[c] = (float)((1.0 - m) * (double)d.run_var[c] + m * unbiased);
+    }
     const double rstd = 1.0 / sqrt(var + 1e-5);
     const double sc = (double)d.gamma[c] * rstd;
     d.mean[c] = (float)mean;

@@ -95,6 +95,9 @@ struct BnFinDesc {
   int64_t count;         // number of rows M
   const float* gamma; const float* beta;
   float* mean; float* rstd; float* scale; float* shift;
+  float* run_mean; float* run_var;  // running statistics of this BN layer
+  float momentum;                   // training: rate at which they follow the batch
+  int32_t eval;                     // 1: normalise with the running statistics
 };
 
 // BN backward: dz = da * [z > 0 if relu], z = scale*h + shift, xhat = (h-mean)*rstd

@@ -70,6 +70,7 @@ struct Norm {
   int64_t count = 0;
   size_t part = 0, mean = 0, rstd = 0, scale = 0, shift = 0, bpart = 0, coef = 0;
   int btiles = 0;
+  size_t run = 0;  // running mean (C floats) followed by running variance (C floats)
 };
 
 // One planned op (forward or backward).  Fields are interpreted per kind.
@@ -154,6 +155,11 @@ struct Phase { std::vector<Launch> launches; };
 int cdiv(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+struct Group {
+  int kind, variant;
+  std::vector<int> ops;
+};
+
 }  // namespace
 
 struct pnn_net {
@@ -198,6 +204,12 @@ struct pnn_net {
   // 0 pre_f 1 fine_f(+delta_f) 2 coarse_f 3 head_f 4 head_b 5 coarse_b 6 delta_b 7 fine_b 8 pre_b
   Phase ph[9];
   std::vector<uint8_t> host_tables;
+  std::vector<size_t> run_at;   // param id of a BN gamma -> float offset of its running statistics
+  size_t running_floats = 0, off_running = 0;
+  // pnn_infer's graph, captured for (ix, ilogits)
+  cudaGraphExec_t igexec = nullptr;
+  const float* ix = nullptr;
+  float* ilogits = nullptr;
   // runtime state
   cudaStream_t stream = nullptr;
   bool own_stream = false;
@@ -286,7 +298,7 @@ struct pnn_net {
     n.count = rows(h);
     norms.push_back(n);
     int nid = (int)norms.size() - 1;
-    request_stats(list, nid, h, key0);
+    if (!opt.inference) request_stats(list, nid, h, key0);  // inference normalises with running statistics
     POp f;
     f.kind = K_BN_FIN; f.norm = nid;
     f.key[0] = key0; f.key[1] = slot;
@@ -692,6 +704,53 @@ struct pnn_net {
   int plan(const pnn_desc* d);
   int bind(void* dev, size_t bytes);
   int build_tables();
+  std::vector<Group> phase_groups(int p) const;
+  // Inference plan: a value's buffer is handed to a later value of the same
+  // size once the last launch that reads it has been issued.
+  void share_activation_buffers() {
+    std::vector<int> def(vals.size(), -1), last(vals.size(), -1);
+    auto reads = [&](int v, int at) {
+      if (v < 0) return;
+      if (vals[v].virt) v = vals[v].src;
+      last[v] = std::max(last[v], at);
+    };
+    int li = 0;
+    for (int p = 0; p < 4; ++p)
+      for (const Group& g : phase_groups(p)) {
+        for (int id : g.ops) {
+          const POp& o = ops[id];
+          reads(o.in, li);
+          reads(o.res, li);
+          for (int i = 0; i < o.nin; ++i) reads(o.ins[i], li);
+          if (o.out >= 0 && !vals[o.out].virt && def[o.out] < 0) def[o.out] = li;
+        }
+        ++li;
+      }
+    std::vector<std::vector<int>> born(li + 1), dies(li + 1);
+    for (size_t v = 0; v < vals.size(); ++v) {
+      if (vals[v].virt) continue;
+      const int d = std::max(def[v], 0);  // the packed input is written before launch 0
+      born[d].push_back((int)v);
+      dies[std::max(last[v], d)].push_back((int)v);
+    }
+    auto bytes = [&](int v) {
+      const Value& x = vals[v];
+      return align256((size_t)B * x.H * x.W * x.C * (x.dt == DT_F32 ? 4 : 2));
+    };
+    std::map<size_t, std::vector<size_t>> free_at;  // size -> free offsets
+    for (int t = 0; t <= li; ++t) {
+      for (int v : born[t]) {
+        std::vector<size_t>& f = free_at[bytes(v)];
+        if (f.empty()) {
+          vals[v].off = alloc(bytes(v));
+        } else {
+          vals[v].off = f.back();
+          f.pop_back();
+        }
+      }
+      for (int v : dies[t]) free_at[bytes(v)].push_back(vals[v].off);
+    }
+  }
   // Algorithmic work of one op, added to flops / bytes: conv FLOPs =
   // 2 * B*P*Q*K*C*R*S; bytes = each operand read once, each result written once
   // (a read-modify-write for accumulating results).
@@ -904,6 +963,22 @@ int pnn_net::plan(const pnn_desc* d) {
     c.tiles = c.mtiles;
     if (c.stats_norm >= 0) norms[c.stats_norm].tiles = c.tiles;
   }
+  // BN running statistics: one slot of 2C floats per BN layer, in the order of
+  // its gamma in the parameter vector (the delta form's two evaluations of F^j
+  // share their layers' slots)
+  {
+    std::vector<int> gam;
+    for (size_t i = 0; i < params.size(); ++i)
+      if (params[i].kind == 1) gam.push_back((int)i);
+    std::sort(gam.begin(), gam.end(), [&](int a, int b) { return params[a].off < params[b].off; });
+    run_at.assign(params.size(), 0);
+    running_floats = 0;
+    for (int g : gam) {
+      run_at[g] = running_floats;
+      running_floats += 2 * params[g].n;
+    }
+  }
+  if (!opt.inference) {
   // backward lists (Algorithm 2): head, coarse chain, fine wave, pre wave
   backward_list(head_f, head_b);
   backward_list(coarse_f, coarse_b);
@@ -934,20 +1009,28 @@ int pnn_net::plan(const pnn_desc* d) {
     for (auto& L : fine_b) visit(L);
     for (auto& L : pre_b) visit(L);
   }
+  }  // !opt.inference
   // ---------------------------------------------------------- memory plan
   cursor = 0;
   off_master = alloc(nparams * 4);
-  off_grad = alloc(nparams * 4);
-  off_mom = alloc(nparams * 4);
+  off_grad = opt.inference ? 0 : alloc(nparams * 4);
+  off_mom = opt.inference ? 0 : alloc(nparams * 4);
   off_shadow = act_dt == DT_BF16 ? alloc(nparams * 2) : 0;
   off_wt = act_dt == DT_BF16 ? alloc(nparams * 2) : 0;
-  for (auto& v : vals) {
-    if (!v.virt) v.off = alloc((size_t)B * v.H * v.W * v.C * (v.dt == DT_F32 ? 4 : 2));
-    if (v.need_grad) v.goff = alloc((size_t)B * v.H * v.W * v.C * 4);
+  off_running = alloc(running_floats * 4);
+  if (opt.inference) {
+    share_activation_buffers();
+  } else {
+    for (auto& v : vals) {
+      if (!v.virt) v.off = alloc((size_t)B * v.H * v.W * v.C * (v.dt == DT_F32 ? 4 : 2));
+      if (v.need_grad) v.goff = alloc((size_t)B * v.H * v.W * v.C * 4);
+    }
   }
   for (auto& n : norms) {
     n.part = alloc((size_t)n.tiles * n.C * 8);
     n.mean = alloc(n.C * 4); n.rstd = alloc(n.C * 4); n.scale = alloc(n.C * 4); n.shift = alloc(n.C * 4);
+    n.run = off_running + run_at[n.gamma] * 4;
+    if (opt.inference) continue;
     n.btiles = cdiv(n.count, bnb_rows_per_tile(n.C));
     // room for the reduce kernel's tiles or a fused data gradient's 128-row tiles
     n.bpart = alloc((size_t)std::max(n.btiles, cdiv(n.count, kTcBM)) * n.C * 8);
@@ -972,12 +1055,6 @@ int pnn_net::plan(const pnn_desc* d) {
 }
 
 // ====================================================================== tables
-namespace {
-struct Group {
-  int kind, variant;
-  std::vector<int> ops;
-};
-}
 
 static Src make_src(const pnn_net& n, int v) {
   Src s{};
@@ -995,7 +1072,7 @@ static Src make_src(const pnn_net& n, int v) {
   return s;
 }
 
-int pnn_net::build_tables() {
+std::vector<Group> pnn_net::phase_groups(int p) const {
   // merge per-subnetwork lists by key into launch groups
   auto keyless = [&](int a, int b) {
     const POp &x = ops[a], &y = ops[b];
@@ -1031,11 +1108,26 @@ int pnn_net::build_tables() {
     for (int id : L) g.push_back(Group{ops[id].kind, ops[id].variant, {id}});
     return g;
   };
-  std::vector<std::vector<int>> fwd_lists = fine_f;
-  fwd_lists.insert(fwd_lists.end(), delta_f.begin(), delta_f.end());
-  std::vector<Group> phases[9] = {merge(pre_f),    merge(fwd_lists), single(coarse_f),
-                                  single(head_f),  single(head_b),   single(coarse_b),
-                                  merge(delta_b),  merge(fine_b),    merge(pre_b)};
+  switch (p) {
+    case 0: return merge(pre_f);
+    case 1: {
+      std::vector<std::vector<int>> fwd_lists = fine_f;
+      fwd_lists.insert(fwd_lists.end(), delta_f.begin(), delta_f.end());
+      return merge(fwd_lists);
+    }
+    case 2: return single(coarse_f);
+    case 3: return single(head_f);
+    case 4: return single(head_b);
+    case 5: return single(coarse_b);
+    case 6: return merge(delta_b);
+    case 7: return merge(fine_b);
+    default: return merge(pre_b);
+  }
+}
+
+int pnn_net::build_tables() {
+  std::vector<Group> phases[9];
+  for (int p = 0; p < 9; ++p) phases[p] = phase_groups(p);
   host_tables.clear();
   auto put = [&](const void* p, size_t n) { return put_table(p, n); };
   float* master = P<float>(off_master);
@@ -1199,6 +1291,9 @@ int pnn_net::build_tables() {
             f.part = P<float>(n.part); f.tiles = n.tiles; f.C = n.C; f.count = n.count;
             f.gamma = master + params[n.gamma].off; f.beta = master + params[n.beta].off;
             f.mean = P<float>(n.mean); f.rstd = P<float>(n.rstd); f.scale = P<float>(n.scale); f.shift = P<float>(n.shift);
+            f.run_mean = P<float>(n.run); f.run_var = P<float>(n.run) + n.C;
+            f.momentum = opt.bn_momentum;
+            f.eval = opt.inference ? 1 : 0;
             add(&f, sizeof f, n.C);  // one CTA per channel
             break;
           }
@@ -1370,7 +1465,7 @@ int pnn_net::run_head_fwd() {
     const int wo = fc_width[l + 1];
     e = launch_gemm(reinterpret_cast<const GemmDesc*>(tb + head_fwd_tab[l]), tst, 1, cdiv(B, 64) * cdiv(wo, 64), stream);
   }
-  if (e == cudaSuccess)
+  if (e == cudaSuccess && !opt.inference)
     e = launch_softmax_ce(P<float>(feat[nfc]), labels_dev, B, classes, P<float>(loss_off), P<float>(dfeat[nfc]),
                           P<int32_t>(status_off), stream);
   return cuda_check(e, "head forward");
@@ -1575,8 +1670,15 @@ int pnn_net::bind(void* dev, size_t bytes) {
   }
   for (const ParamT& p : params) to_internal(p, theta.data() + p.off, internal.data() + p.off);
   e = cudaMemcpy(ws + off_master, internal.data(), nparams * 4, cudaMemcpyHostToDevice);
-  if (e == cudaSuccess) e = cudaMemset(ws + off_grad, 0, nparams * 4);
-  if (e == cudaSuccess) e = cudaMemset(ws + off_mom, 0, nparams * 4);
+  if (e == cudaSuccess && !opt.inference) e = cudaMemset(ws + off_grad, 0, nparams * 4);
+  if (e == cudaSuccess && !opt.inference) e = cudaMemset(ws + off_mom, 0, nparams * 4);
+  if (e == cudaSuccess && running_floats) {
+    // running means 0, running variances 1
+    std::vector<float> run(running_floats, 0.f);
+    for (size_t i = 0; i < params.size(); ++i)
+      if (params[i].kind == 1) std::fill(run.begin() + run_at[i] + params[i].n, run.begin() + run_at[i] + 2 * params[i].n, 1.f);
+    e = cudaMemcpy(ws + off_running, run.data(), running_floats * 4, cudaMemcpyHostToDevice);
+  }
   if (e == cudaSuccess) e = cudaMemset(ws + status_off, 0, 64);
   if (e == cudaSuccess && act_dt == DT_BF16)
     e = launch_copy_cast(P<float>(off_master), ws + off_shadow, DT_BF16, (int64_t)nparams, stream);
@@ -1608,6 +1710,8 @@ namespace {
 #define BOUND_OR_FAIL(n)  \
   NET_OR_FAIL(n);         \
   if (!(n)->ws) return (n)->fail(PNN_ENOTBOUND, "no workspace bound");
+#define TRAINING_OR_FAIL(n) \
+  if ((n)->opt.inference) return (n)->fail(PNN_ESTATE, "an inference net runs pnn_infer only");
 }  // namespace
 
 extern "C" {
@@ -1625,6 +1729,8 @@ void pnn_default_options(pnn_options* o) {
   o->stream_fp32 = 1;
   o->conv_impl = 0;
   o->stream = nullptr;
+  o->bn_momentum = 0.1f;
+  o->inference = 0;
 }
 
 int pnn_create(const pnn_desc* desc, const pnn_options* opts, pnn_net** out) {
@@ -1741,6 +1847,7 @@ int pnn_bind_workspace(pnn_net* n, void* dev, size_t bytes) {
 
 int pnn_forward(pnn_net* n, const float* x, const int32_t* labels, float* loss) {
   BOUND_OR_FAIL(n);
+  TRAINING_OR_FAIL(n);
   if (!x || !labels) return n->fail(PNN_EINVAL, "null x or labels");
   n->x_dev = x;
   n->labels_dev = labels;
@@ -1756,6 +1863,7 @@ int pnn_forward(pnn_net* n, const float* x, const int32_t* labels, float* loss) 
 
 int pnn_backward(pnn_net* n) {
   BOUND_OR_FAIL(n);
+  TRAINING_OR_FAIL(n);
   if (n->state != 1) return n->fail(PNN_ESTATE, "pnn_backward needs a preceding pnn_forward");
   int r = n->do_backward(true);
   if (r) return r;
@@ -1765,6 +1873,7 @@ int pnn_backward(pnn_net* n) {
 
 int pnn_sgd_step(pnn_net* n, float lr) {
   BOUND_OR_FAIL(n);
+  TRAINING_OR_FAIL(n);
   if (n->state != 2) return n->fail(PNN_ESTATE, "pnn_sgd_step needs a preceding pnn_backward");
   int r = n->do_sgd(lr, true);
   if (r) return r;
@@ -1774,6 +1883,7 @@ int pnn_sgd_step(pnn_net* n, float lr) {
 
 int pnn_train_step(pnn_net* n, const float* x, const int32_t* labels, float* loss) {
   BOUND_OR_FAIL(n);
+  TRAINING_OR_FAIL(n);
   if (!x || !labels) return n->fail(PNN_EINVAL, "null x or labels");
   if (n->first_step) {
     // the first step initialises the momentum buffers; run it eagerly
@@ -1825,6 +1935,7 @@ static void drop_phase_graphs(pnn_net* n) {
 
 int pnn_time_phases(pnn_net* n, const float* x, const int32_t* labels, int32_t steps, float ms[10]) {
   BOUND_OR_FAIL(n);
+  TRAINING_OR_FAIL(n);
   if (!x || !labels || !ms) return n->fail(PNN_EINVAL, "null argument");
   if (steps <= 0) return n->fail(PNN_EINVAL, "steps must be positive");
   if (n->prof) return n->fail(PNN_ESTATE, "phase timing needs profiling off");
@@ -1910,6 +2021,7 @@ int pnn_time_phases(pnn_net* n, const float* x, const int32_t* labels, int32_t s
 
 int pnn_train_step_host(pnn_net* n, const float* x_host, const int32_t* labels_host, float* loss_host) {
   BOUND_OR_FAIL(n);
+  TRAINING_OR_FAIL(n);
   if (!x_host || !labels_host) return n->fail(PNN_EINVAL, "null x or labels");
   const size_t xb = (size_t)n->B * n->in_c * n->in_h * n->in_w * 4;
   cudaError_t e = cudaMemcpyAsync(n->ws + n->x_stage, x_host, xb, cudaMemcpyHostToDevice, n->stream);
@@ -1938,8 +2050,78 @@ int pnn_sync(pnn_net* n) {
   return PNN_OK;
 }
 
+int pnn_running_stats_size(const pnn_net* n, size_t* out) {
+  NET_OR_FAIL(n);
+  if (!out) return set_global(PNN_EINVAL, "null argument");
+  *out = n->running_floats;
+  return PNN_OK;
+}
+
+int pnn_get_running_stats(pnn_net* n, float* host, size_t count) {
+  BOUND_OR_FAIL(n);
+  if ((!host && count) || count != n->running_floats) return n->fail(PNN_EINVAL, "length must equal pnn_running_stats_size");
+  cudaError_t e = cudaStreamSynchronize(n->stream);
+  if (e == cudaSuccess && count) e = cudaMemcpy(host, n->ws + n->off_running, count * 4, cudaMemcpyDeviceToHost);
+  return n->cuda_check(e, "read running statistics");
+}
+
+int pnn_set_running_stats(pnn_net* n, const float* host, size_t count) {
+  BOUND_OR_FAIL(n);
+  if ((!host && count) || count != n->running_floats) return n->fail(PNN_EINVAL, "length must equal pnn_running_stats_size");
+  cudaError_t e = cudaStreamSynchronize(n->stream);
+  if (e == cudaSuccess && count) e = cudaMemcpy(n->ws + n->off_running, host, count * 4, cudaMemcpyHostToDevice);
+  return n->cuda_check(e, "write running statistics");
+}
+
+int pnn_infer(pnn_net* n, const float* x, float* logits) {
+  BOUND_OR_FAIL(n);
+  if (!n->opt.inference) return n->fail(PNN_ESTATE, "pnn_infer needs a net created with opts.inference = 1");
+  if (!x || !logits) return n->fail(PNN_EINVAL, "null x or logits");
+  if (n->prof) {
+    // profiling: eager launches, each bracketed by events
+    n->x_dev = x;
+    n->labels_dev = nullptr;
+    int r = n->do_forward(true);
+    const int nfc = (int)n->fc_width.size() - 1;
+    if (!r)
+      r = n->cuda_check(cudaMemcpyAsync(logits, n->ws + n->feat[nfc], (size_t)n->B * n->classes * 4,
+                                        cudaMemcpyDeviceToDevice, n->stream),
+                        "copy logits");
+    return r;
+  }
+  if (n->igexec && (x != n->ix || logits != n->ilogits)) {
+    cudaGraphExecDestroy(n->igexec);
+    n->igexec = nullptr;
+  }
+  if (!n->igexec) {
+    n->x_dev = x;
+    n->labels_dev = nullptr;
+    cudaError_t e = cudaStreamBeginCapture(n->stream, cudaStreamCaptureModeThreadLocal);
+    if (e != cudaSuccess) return n->cuda_check(e, "begin capture");
+    int r = n->do_forward(false);
+    const int nfc = (int)n->fc_width.size() - 1;
+    if (!r)
+      r = n->cuda_check(cudaMemcpyAsync(logits, n->ws + n->feat[nfc], (size_t)n->B * n->classes * 4,
+                                        cudaMemcpyDeviceToDevice, n->stream),
+                        "copy logits");
+    cudaGraph_t g = nullptr;
+    e = cudaStreamEndCapture(n->stream, &g);
+    if (r || e != cudaSuccess) {
+      if (g) cudaGraphDestroy(g);
+      return r ? r : n->cuda_check(e, "end capture");
+    }
+    e = cudaGraphInstantiate(&n->igexec, g, 0);
+    cudaGraphDestroy(g);
+    if (e != cudaSuccess) return n->cuda_check(e, "instantiate graph");
+    n->ix = x;
+    n->ilogits = logits;
+  }
+  return n->cuda_check(cudaGraphLaunch(n->igexec, n->stream), "graph launch");
+}
+
 void pnn_destroy(pnn_net* n) {
   if (!n) return;
+  if (n->igexec) cudaGraphExecDestroy(n->igexec);
   if (n->gexec) cudaGraphExecDestroy(n->gexec);
   if (n->graph) cudaGraphDestroy(n->graph);
   drop_phase_graphs(n);
@@ -1992,8 +2174,16 @@ static int copy_params_out(pnn_net* n, size_t off, float* host, size_t count) {
 }
 
 int pnn_get_params(pnn_net* n, float* host, size_t count) { NET_OR_FAIL(n); return copy_params_out(n, n->off_master, host, count); }
-int pnn_get_grads(pnn_net* n, float* host, size_t count) { NET_OR_FAIL(n); return copy_params_out(n, n->off_grad, host, count); }
-int pnn_get_momentum(pnn_net* n, float* host, size_t count) { NET_OR_FAIL(n); return copy_params_out(n, n->off_mom, host, count); }
+int pnn_get_grads(pnn_net* n, float* host, size_t count) {
+  NET_OR_FAIL(n);
+  TRAINING_OR_FAIL(n);
+  return copy_params_out(n, n->off_grad, host, count);
+}
+int pnn_get_momentum(pnn_net* n, float* host, size_t count) {
+  NET_OR_FAIL(n);
+  TRAINING_OR_FAIL(n);
+  return copy_params_out(n, n->off_mom, host, count);
+}
 
 int pnn_set_params(pnn_net* n, const float* host, size_t count) {
   BOUND_OR_FAIL(n);
@@ -2038,6 +2228,8 @@ int pnn_tensor_size(const pnn_net* n, int32_t which, int32_t j, size_t* out) {
 
 int pnn_get_tensor(pnn_net* n, int32_t which, int32_t j, float* host, size_t count) {
   BOUND_OR_FAIL(n);
+  if (n->opt.inference && which != PNN_T_LOGITS)
+    return n->fail(PNN_ESTATE, "an inference net keeps only the logits (its activations share buffers)");
   int v; bool g;
   if (tensor_value(n, which, j, &v, &g)) return n->fail(PNN_EINVAL, "no such tensor");
   size_t want;

@@ -50,7 +50,7 @@ class Options(C.Structure):
                 ("lr", C.c_float), ("momentum", C.c_float), ("weight_decay", C.c_float),
                 ("nesterov", C.c_int32), ("stream_fp32", C.c_int32), ("conv_impl", C.c_int32),
                 ("grad_fp32", C.c_int32),
-                ("stream", C.c_void_p)]
+                ("stream", C.c_void_p), ("bn_momentum", C.c_float), ("inference", C.c_int32)]
 
 
 class Trace(C.Structure):
@@ -97,6 +97,10 @@ def load():
         "pnn_get_timings": (C.c_int, [P, C.POINTER(C.c_float)]),
         "pnn_time_phases": (C.c_int, [P, C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_float)]),
         "pnn_block_costs": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.POINTER(C.c_double), C.c_int32]),
+        "pnn_running_stats_size": (C.c_int, [P, C.POINTER(C.c_size_t)]),
+        "pnn_get_running_stats": (C.c_int, [P, C.c_void_p, C.c_size_t]),
+        "pnn_set_running_stats": (C.c_int, [P, C.c_void_p, C.c_size_t]),
+        "pnn_infer": (C.c_int, [P, C.c_void_p, C.c_void_p]),
         "pnn_partition": (C.c_int, [C.POINTER(C.c_double), C.c_int32, C.c_int32, C.POINTER(C.c_int32)]),
         "pnn_launch_counts": (C.c_int, [P, C.POINTER(I32)]),
         "pnn_profile": (C.c_int, [P, I32]),
@@ -195,7 +199,7 @@ class ParaNet:
 
     def __init__(self, desc, precision=None, correction=None, seed=0, lr=0.1, momentum=0.9,
                  weight_decay=5e-4, nesterov=True, stream_fp32=True, conv_impl=0, grad_fp32=False, stream=None,
-                 device="cuda", bind=True):
+                 device="cuda", bind=True, inference=False, bn_momentum=0.1):
         self.lib = load()
         self.desc = desc
         d, self._keep = _make_desc(desc)
@@ -206,6 +210,7 @@ class ParaNet:
         o.seed, o.lr, o.momentum, o.weight_decay = seed, lr, momentum, weight_decay
         o.nesterov, o.stream_fp32, o.conv_impl = int(nesterov), int(stream_fp32), int(conv_impl)
         o.grad_fp32 = int(grad_fp32)
+        o.inference, o.bn_momentum = int(inference), bn_momentum
         self.stream = stream
         o.stream = None if stream is None else C.c_void_p(stream.cuda_stream)
         self.h = C.c_void_p()
@@ -334,6 +339,31 @@ class ParaNet:
         self._check(self.lib.pnn_get_timings(self.h, ms))
         keys = ["pre_f", "fine_f", "coarse_f", "post_f", "pre_b", "fine_b", "coarse_b", "post_b", "update", "total"]
         return dict(zip(keys, list(ms)))
+
+    def running_stats(self):
+        """BN running statistics (per BN layer in parameter order: C means, C variances)."""
+        n = C.c_size_t()
+        self._check(self.lib.pnn_running_stats_size(self.h, C.byref(n)))
+        a = np.empty(n.value, dtype=np.float32)
+        self._check(self.lib.pnn_get_running_stats(self.h, C.c_void_p(a.ctypes.data), n.value))
+        return a
+
+    def set_running_stats(self, a):
+        a = np.ascontiguousarray(a, dtype=np.float32)
+        self._check(self.lib.pnn_set_running_stats(self.h, C.c_void_p(a.ctypes.data), a.size))
+
+    def infer(self, x, logits):
+        """Eval-mode forward of an inference net: x (device NCHW float32) ->
+        logits (device float32 batch x classes), asynchronous on the stream."""
+        import torch
+        d = self.desc
+        if x.dtype != torch.float32 or not x.is_cuda or not x.is_contiguous() \
+                or tuple(x.shape) != (d["batch"], d["in_c"], d["in_h"], d["in_w"]):
+            raise TypeError("x must be a contiguous float32 CUDA tensor of shape (batch, C, H, W)")
+        if logits.dtype != torch.float32 or not logits.is_cuda or not logits.is_contiguous() \
+                or logits.numel() != d["batch"] * d["classes"]:
+            raise TypeError("logits must be a contiguous float32 CUDA tensor of batch x classes")
+        self._check(self.lib.pnn_infer(self.h, C.c_void_p(x.data_ptr()), C.c_void_p(logits.data_ptr())))
 
     def time_phases(self, x, labels, steps=5):
         """Per-phase ms of `steps` graph-replayed training steps (device x, labels)."""
