@@ -62,6 +62,9 @@ def parse():
                          "Section 4.2) or of equal cost (the remark after Table grad): algorithmic FLOPs, "
                          "HBM bytes, or the device time of each layer measured on the untorn network; "
                          "every choice but none also reports each subnetwork's measured time")
+    ap.add_argument("--overlap", type=int, default=0,
+                    help="run the last subnetwork's backward beside the coarse chain's (Algorithm 2 needs only "
+                         "D_N for it), leaving this many SMs to the chain; 0 = phases in sequence")
     ap.add_argument("--inference", action="store_true",
                     help="time the eval-mode forward (pnn_infer) of the workload instead of training")
     ap.add_argument("--lr", type=float, default=0.1,
@@ -373,7 +376,8 @@ def our_arm(args, desc, rank, local, world, dist):
         if args.paper_net or args.config not in (2, 3, 4):
             raise SystemExit("--tearing applies to the ResNet-1001 configurations 2, 3 and 4")
         desc, tearing = retear(args, desc, stream)
-    net = pnn.ParaNet(desc, seed=0, stream=stream, stream_fp32=bool(args.stream_fp32), lr=args.lr)
+    net = pnn.ParaNet(desc, seed=0, stream=stream, stream_fp32=bool(args.stream_fp32), lr=args.lr,
+                      overlap=args.overlap)
     B = desc["batch"]
     x, labels = W.make_batch(desc, seed=1000 + desc.get("config_index", 0) + rank)
     xd = torch.from_numpy(x).cuda()
@@ -420,7 +424,8 @@ def our_arm(args, desc, rank, local, world, dist):
     launches_per_step = fw + bw + up
     phases_eager = net.timings()
     net.set_params(theta0)
-    phases = net.time_phases(xd, ld, args.steps)
+    # the overlapped backward runs two phases at once: no per-phase split
+    phases = net.time_phases(xd, ld, args.steps) if not args.overlap else None
 
     # ------------------------------------------------ end to end through the host API
     net.set_params(theta0)
@@ -459,6 +464,7 @@ def our_arm(args, desc, rank, local, world, dist):
                    "subnetworks": len(desc["segments"]), "correction": desc.get("correction", "residual"),
                    "residual_stream": "fp32" if args.stream_fp32 else "bf16", "lr": args.lr,
                    "tearing": "uniform" if args.tearing == "none" else args.tearing,
+                   "overlap_sms": args.overlap,
                    "l2": "inputs larger than L2 (%.1f GB workspace per step)" % (net.workspace_bytes / 1e9),
                    "parallelism": "replicas" if world > 1 else "single-gpu"},
         "conv_tflops": conv_flops / (conv_ms / 1e3) / 1e12 if conv_ms else None,

@@ -129,11 +129,17 @@ typedef struct {
   int32_t inference;     /* 1: plan the forward pass alone for pnn_infer (every BN
                             normalises with its running statistics; activations
                             share buffers, no gradients or optimiser state) */
+  int32_t overlap;       /* > 0 (residual correction, N > 1): run the last
+                            subnetwork's backward, which needs only D_N (Algorithm
+                            2), beside the coarse chain's backward on a second
+                            stream, its persistent kernels capped to leave
+                            `overlap` SMs to the chain; the chain's term of
+                            dL/dx_N is added after both.  0 = phases in sequence */
 } pnn_options;
 
 /* Fill o with the defaults: bf16, residual correction, seed 0, lr 0.1,
  * momentum 0.9, weight decay 5e-4, Nesterov (Section 4), stream_fp32 1,
- * bn_momentum 0.1, inference 0. */
+ * bn_momentum 0.1, inference 0, overlap 0. */
 void pnn_default_options(pnn_options* o);
 
 /* Plan the network from a description.  Host only: no GPU work, no device

@@ -1505,7 +1505,7 @@ typedef void (*ConvKernel)(const ConvDesc*, const int*, int, int, int, int32_t*)
 
 template <int MODE>
 static cudaError_t launch_mode(ConvKernel kern, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
-                               int32_t* status, cudaStream_t st) {
+                               int32_t* status, cudaStream_t st, int max_ctas) {
   if (total <= 0) return cudaSuccess;
   if (bnmax < 16 || bnmax > 256 || (bnmax & 15)) return cudaErrorInvalidValue;
   static bool attr = false;
@@ -1519,7 +1519,8 @@ static cudaError_t launch_mode(ConvKernel kern, const ConvDesc* tab, const int* 
     if (sms <= 0) sms = 148;
     attr = true;
   }
-  const int grid = total < sms ? total : sms;
+  int grid = total < sms ? total : sms;
+  if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
   kern<<<grid, kThreads, smem_bytes(bnmax), st>>>(tab, tstart, n, total, bnmax, status);
   return cudaGetLastError();
 }
@@ -1530,7 +1531,7 @@ bool conv_tma_fits(int mode, int bnmax, int raw_bytes) {
 }
 
 cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
-                            int raw_bytes, int32_t* status, cudaStream_t st) {
+                            int raw_bytes, int32_t* status, cudaStream_t st, int max_ctas) {
   if (total <= 0) return cudaSuccess;
   if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || raw_bytes <= 0 || (raw_bytes & 1023) || mode < 0 || mode > 2)
     return cudaErrorInvalidValue;
@@ -1549,7 +1550,8 @@ cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, in
   }
   const size_t smem = tma_smem_bytes(mode, bnmax, raw_bytes, tma_extra(mode, xw));
   if (smem > (size_t)kTmaSmemBudget) return cudaErrorInvalidValue;
-  const int grid = total < sms ? total : sms;
+  int grid = total < sms ? total : sms;
+  if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
   kern<<<grid, kTmaThreads, smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, status);
   return cudaGetLastError();
 }
@@ -1565,16 +1567,16 @@ unsigned long long conv_tc_debug_word() {
 }
 
 cudaError_t launch_conv_fwd_tc(const ConvDesc* tab, const int* tstart, int n, int total, int bnmax, int32_t* status,
-                               cudaStream_t st) {
-  return launch_mode<FWD>(k_conv_fwd_tc, tab, tstart, n, total, bnmax, status, st);
+                               cudaStream_t st, int max_ctas) {
+  return launch_mode<FWD>(k_conv_fwd_tc, tab, tstart, n, total, bnmax, status, st, max_ctas);
 }
 cudaError_t launch_conv_dgrad_tc(const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
-                                 int32_t* status, cudaStream_t st) {
-  return launch_mode<DGRAD>(k_conv_dgrad_tc, tab, tstart, n, total, bnmax, status, st);
+                                 int32_t* status, cudaStream_t st, int max_ctas) {
+  return launch_mode<DGRAD>(k_conv_dgrad_tc, tab, tstart, n, total, bnmax, status, st, max_ctas);
 }
 cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
-                                 int32_t* status, cudaStream_t st) {
-  return launch_mode<WGRAD>(k_conv_wgrad_tc, tab, tstart, n, total, bnmax, status, st);
+                                 int32_t* status, cudaStream_t st, int max_ctas) {
+  return launch_mode<WGRAD>(k_conv_wgrad_tc, tab, tstart, n, total, bnmax, status, st, max_ctas);
 }
 
 }  // namespace pnn

@@ -183,17 +183,19 @@ cudaError_t launch_pool_bwd(const PoolDesc* tab, const int* tstart, int n, int t
 cudaError_t launch_gemm(const GemmDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
 // tcgen05 implicit-GEMM convolution (bf16 operands, fp32 accumulate in TMEM);
 // instances need C % 8 == 0; bnmax = largest N tile (multiple of 16, <= 256)
+// (max_ctas > 0 caps the persistent grid below the SM count, leaving SMs to
+// launches of other streams)
 cudaError_t launch_conv_fwd_tc(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int bnmax,
-                               int32_t* status, cudaStream_t st);
+                               int32_t* status, cudaStream_t st, int max_ctas = 0);
 cudaError_t launch_conv_dgrad_tc(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int bnmax,
-                                 int32_t* status, cudaStream_t st);
+                                 int32_t* status, cudaStream_t st, int max_ctas = 0);
 cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int bnmax,
-                                 int32_t* status, cudaStream_t st);
+                                 int32_t* status, cudaStream_t st, int max_ctas = 0);
 // TMA-fed stride-1 forward (mode 0), data-gradient (mode 1) or weight-gradient
 // (mode 2) tensor-core conv; raw_bytes: one pipeline stage's raw slot (the
 // largest over the launch's instances, a multiple of 1024)
 cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
-                            int raw_bytes, int32_t* status, cudaStream_t st);
+                            int raw_bytes, int32_t* status, cudaStream_t st, int max_ctas = 0);
 // whether the TMA-fed kernel of `mode` holds at least two stages of this size
 bool conv_tma_fits(int mode, int bnmax, int raw_bytes);
 // record a message for pnn_last_error(NULL) and return `code`

@@ -202,9 +202,19 @@ struct pnn_net {
   char* ws = nullptr;
   // launch lists
   // 0 pre_f 1 fine_f(+delta_f) 2 coarse_f 3 head_f 4 head_b 5 coarse_b 6 delta_b 7 fine_b 8 pre_b
-  Phase ph[9];
+  Phase ph[11];  // 0-8 the step's phases; 9 the last subnetwork's backward and 10 the
+                 // deferred x_N gradient term when the coarse chain overlaps it
   std::vector<uint8_t> host_tables;
   std::vector<size_t> run_at;   // param id of a BN gamma -> float offset of its running statistics
+  // coarse/fine overlap: the last subnetwork's backward (it needs only D_N) runs
+  // on s_lo beside the coarse chain's backward on s_hi; the chain's term
+  // -dL/dr_{N-1} of dL/dx_N is deferred to fix_b, after both
+  bool overlap_on = false;
+  int defer_x = -1, defer_r = -1;
+  std::vector<int> fix_b;
+  cudaStream_t s_hi = nullptr, s_lo = nullptr;
+  cudaEvent_t fork_ev = nullptr, hi_done = nullptr, lo_done = nullptr;
+  int lo_cap = 0;  // grid cap of s_lo's persistent kernels
   size_t running_floats = 0, off_running = 0;
   // pnn_infer's graph, captured for (ix, ilogits)
   cudaGraphExec_t igexec = nullptr;
@@ -571,6 +581,7 @@ struct pnn_net {
         e.in = f.out; e.out = f.out; e.relu = f.relu;
         for (int i = 0; i < f.nin; ++i) {
           if (!vals[f.ins[i]].need_grad) continue;
+          if (overlap_on && f.out == defer_r && f.ins[i] == defer_x) continue;  // planned into fix_b
           const int key_[2] = {k0, k1};
           flush_pending(L, f.ins[i], key_);
           e.ins[e.nin] = f.ins[i];
@@ -791,7 +802,8 @@ struct pnn_net {
       default: break;
     }
   }
-  int run_phase(int p);
+  int run_phase(int p) { return run_phase(p, stream, 0); }
+  int run_phase(int p, cudaStream_t st, int cap);
   int do_forward(bool timed);
   int do_backward(bool timed);
   int do_sgd(float lr, bool timed);
@@ -910,7 +922,9 @@ int pnn_net::plan(const pnn_desc* d) {
         rts[j + 1] = ew(coarse_f, {out, f0[j]}, {1.f, -1.f}, false, stream_dt, 2000 + 100 * j, 98);
     }
   }
-  ytilde = N > 1 ? ew(coarse_f, {ys[N - 1], rts[N - 1]}, {1.f, 1.f}, false, stream_dt, 9000, 0) : ys[0];
+  // ytilde joins the post phase, so that its backward (which writes dL/dy_N =
+  // D_N) is complete when the head's backward is
+  ytilde = N > 1 ? ew(head_f, {ys[N - 1], rts[N - 1]}, {1.f, 1.f}, false, stream_dt, 9000, 0) : ys[0];
   if (N == 1) rts[0] = ytilde;
   // head h
   std::vector<int> head_ids;
@@ -980,12 +994,31 @@ int pnn_net::plan(const pnn_desc* d) {
   }
   if (!opt.inference) {
   // backward lists (Algorithm 2): head, coarse chain, fine wave, pre wave
+  overlap_on = opt.overlap > 0 && opt.correction == PNN_CORR_RESIDUAL && N > 1;
+  if (overlap_on) {
+    defer_x = xs[N - 1];
+    defer_r = rs[N - 2];
+  }
   backward_list(head_f, head_b);
   backward_list(coarse_f, coarse_b);
   delta_b.resize(delta_f.size());
   for (size_t j = 0; j < delta_f.size(); ++j) backward_list(delta_f[j], delta_b[j]);
   fine_b.resize(fine_f.size());
-  for (size_t j = 0; j < fine_f.size(); ++j) backward_list(fine_f[j], fine_b[j]);
+  if (overlap_on) {
+    // the last subnetwork first (it writes dL/dx_N first), then the deferred
+    // term dL/dx_N -= dL/dr_{N-1}, then the other subnetworks
+    backward_list(fine_f[N - 1], fine_b[N - 1]);
+    POp e;
+    e.kind = K_EW_BWD;
+    e.in = defer_r; e.out = defer_r; e.relu = false;
+    e.nin = 1; e.ins[0] = defer_x; e.coef[0] = -1.f; e.acc_in[0] = grad_acc(defer_x);
+    e.tiles = cdiv(rows(defer_x), kEwRowsPerTile);
+    e.key[0] = -1000; e.key[1] = -(N - 2); e.key[2] = 1;
+    new_op(fix_b, e);
+    for (int j = 0; j + 1 < N; ++j) backward_list(fine_f[j], fine_b[j]);
+  } else {
+    for (size_t j = 0; j < fine_f.size(); ++j) backward_list(fine_f[j], fine_b[j]);
+  }
   pre_b.resize(N);
   for (int j = 0; j < N; ++j) backward_list(pre_f[j], pre_b[j]);
   // gradient-accumulating parameters (delta mode: F^j used twice)
@@ -1120,14 +1153,20 @@ std::vector<Group> pnn_net::phase_groups(int p) const {
     case 4: return single(head_b);
     case 5: return single(coarse_b);
     case 6: return merge(delta_b);
-    case 7: return merge(fine_b);
-    default: return merge(pre_b);
+    case 7:
+      if (overlap_on) return merge(std::vector<std::vector<int>>(fine_b.begin(), fine_b.end() - 1));
+      return merge(fine_b);
+    case 8: return merge(pre_b);
+    case 9:
+      if (overlap_on) return merge(std::vector<std::vector<int>>(fine_b.end() - 1, fine_b.end()));
+      return {};
+    default: return single(fix_b);
   }
 }
 
 int pnn_net::build_tables() {
-  std::vector<Group> phases[9];
-  for (int p = 0; p < 9; ++p) phases[p] = phase_groups(p);
+  std::vector<Group> phases[11];
+  for (int p = 0; p < 11; ++p) phases[p] = phase_groups(p);
   host_tables.clear();
   auto put = [&](const void* p, size_t n) { return put_table(p, n); };
   float* master = P<float>(off_master);
@@ -1137,7 +1176,7 @@ int pnn_net::build_tables() {
   auto wptr = [&](int pid) -> const void* {
     return (const char*)wts + params[pid].off * (wdt == DT_BF16 ? 2 : 4);
   };
-  for (int p = 0; p < 9; ++p) {
+  for (int p = 0; p < 11; ++p) {
     ph[p].launches.clear();
     for (auto& g : phases[p]) {
       std::vector<uint8_t> tab;
@@ -1414,7 +1453,7 @@ int pnn_net::build_tables() {
   }
   counts[0] = counts[1] = 0;
   for (int p = 0; p < 4; ++p) counts[0] += (int)ph[p].launches.size();
-  for (int p = 4; p < 9; ++p) counts[1] += (int)ph[p].launches.size();
+  for (int p = 4; p < 11; ++p) counts[1] += (int)ph[p].launches.size();
   counts[2] = act_dt == DT_BF16 && wt_count ? 2 : 1;
   return PNN_OK;
 }
@@ -1492,7 +1531,7 @@ int pnn_net::run_head_bwd(int opid) {
 }
 
 // ====================================================================== execution
-int pnn_net::run_phase(int p) {
+int pnn_net::run_phase(int p, cudaStream_t st, int cap) {
   const char* tb = ws + tables_off;
   for (const Launch& L : ph[p].launches) {
     const void* tab = tb + L.table_off;
@@ -1506,54 +1545,54 @@ int pnn_net::run_phase(int p) {
         plaunch.resize(pev.size() / 2);
       }
       plaunch[pnext / 2] = &L;
-      cudaEventRecord(pev[pnext], stream);
+      cudaEventRecord(pev[pnext], st);
     }
     switch (L.kind) {
-      case K_CONV_FWD: e = launch_conv_fwd_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, stream); break;
+      case K_CONV_FWD: e = launch_conv_fwd_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, st); break;
       case K_CONV_FWD_TC:
         e = L.variant == 1
                 ? launch_conv_tma(0, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
-                                  stream)
-                : launch_conv_fwd_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), stream);
+                                  st, cap)
+                : launch_conv_fwd_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), st, cap);
         break;
       case K_DGRAD_TC:
         e = L.variant == 1
                 ? launch_conv_tma(1, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
-                                  stream)
+                                  st, cap)
                 : launch_conv_dgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
-                                       stream);
+                                       st, cap);
         break;
       case K_WGRAD_TC:
         e = L.variant == 1
                 ? launch_conv_tma(2, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
-                                  stream)
+                                  st, cap)
                 : launch_conv_wgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
-                                       stream);
+                                       st, cap);
         break;
-      case K_DGRAD: e = launch_conv_dgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, stream); break;
-      case K_WGRAD: e = launch_conv_wgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, stream); break;
-      case K_WREDUCE: e = launch_wreduce((const WReduceDesc*)tab, ts, L.count, L.total, stream); break;
-      case K_EW: e = launch_ew((const EwDesc*)tab, ts, L.count, L.total, stream); break;
-      case K_EW_BWD: e = launch_ew_bwd((const EwBwdDesc*)tab, ts, L.count, L.total, stream); break;
-      case K_BN_FIN: e = launch_bn_fin((const BnFinDesc*)tab, ts, L.count, L.total, stream); break;
+      case K_DGRAD: e = launch_conv_dgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, st); break;
+      case K_WGRAD: e = launch_conv_wgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, st); break;
+      case K_WREDUCE: e = launch_wreduce((const WReduceDesc*)tab, ts, L.count, L.total, st); break;
+      case K_EW: e = launch_ew((const EwDesc*)tab, ts, L.count, L.total, st); break;
+      case K_EW_BWD: e = launch_ew_bwd((const EwBwdDesc*)tab, ts, L.count, L.total, st); break;
+      case K_BN_FIN: e = launch_bn_fin((const BnFinDesc*)tab, ts, L.count, L.total, st); break;
       case K_BNB_RED:
-        e = L.variant ? launch_bnb_reduce8((const BnBwdDesc*)tab, ts, L.count, L.total, stream)
-                      : launch_bnb_reduce((const BnBwdDesc*)tab, ts, L.count, L.total, stream);
+        e = L.variant ? launch_bnb_reduce8((const BnBwdDesc*)tab, ts, L.count, L.total, st)
+                      : launch_bnb_reduce((const BnBwdDesc*)tab, ts, L.count, L.total, st);
         break;
-      case K_BNB_FIN: e = launch_bnb_fin((const BnBwdDesc*)tab, ts, L.count, L.total, stream); break;
+      case K_BNB_FIN: e = launch_bnb_fin((const BnBwdDesc*)tab, ts, L.count, L.total, st); break;
       case K_BNB_APPLY:
-        e = L.variant ? launch_bnb_apply8((const BnBwdDesc*)tab, ts, L.count, L.total, stream)
-                      : launch_bnb_apply((const BnBwdDesc*)tab, ts, L.count, L.total, stream);
+        e = L.variant ? launch_bnb_apply8((const BnBwdDesc*)tab, ts, L.count, L.total, st)
+                      : launch_bnb_apply((const BnBwdDesc*)tab, ts, L.count, L.total, st);
         break;
-      case K_POOL_FWD: e = launch_pool_fwd((const PoolDesc*)tab, ts, L.count, L.total, stream); break;
-      case K_POOL_BWD: e = launch_pool_bwd((const PoolDesc*)tab, ts, L.count, L.total, stream); break;
+      case K_POOL_FWD: e = launch_pool_fwd((const PoolDesc*)tab, ts, L.count, L.total, st); break;
+      case K_POOL_BWD: e = launch_pool_bwd((const PoolDesc*)tab, ts, L.count, L.total, st); break;
       case K_HEAD_FWD: { int r = run_head_fwd(); if (r) return r; break; }
       case K_HEAD_BWD: { int r = run_head_bwd(L.variant); if (r) return r; break; }
       default: return fail(PNN_EINVAL, "internal: unknown launch kind");
     }
     if (e != cudaSuccess) return cuda_check(e, "kernel launch");
     if (prof) {
-      cudaEventRecord(pev[pnext + 1], stream);
+      cudaEventRecord(pev[pnext + 1], st);
       pnext += 2;
     }
   }
@@ -1574,6 +1613,35 @@ int pnn_net::do_forward(bool timed) {
 
 int pnn_net::do_backward(bool timed) {
   if (timed) cudaEventRecord(ev[5], stream);
+  if (overlap_on) {
+    int r = run_phase(4);
+    if (r) return r;
+    if (timed) cudaEventRecord(ev[6], stream);
+    // fork: the coarse chain on the high-priority stream, the last subnetwork's
+    // backward (it needs only D_N) beside it with a capped grid; then join
+    cudaError_t e = cudaEventRecord(fork_ev, stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s_hi, fork_ev, 0);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s_lo, fork_ev, 0);
+    if (e != cudaSuccess) return cuda_check(e, "fork");
+    r = run_phase(9, s_lo, lo_cap);
+    if (!r) r = run_phase(5, s_hi, 0);
+    if (r) return r;
+    e = cudaEventRecord(hi_done, s_hi);
+    if (e == cudaSuccess) e = cudaEventRecord(lo_done, s_lo);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(stream, hi_done, 0);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(stream, lo_done, 0);
+    if (e != cudaSuccess) return cuda_check(e, "join");
+    if (timed) cudaEventRecord(ev[7], stream);
+    for (int p : {6, 10, 7}) {
+      r = run_phase(p);
+      if (r) return r;
+    }
+    if (timed) cudaEventRecord(ev[8], stream);
+    r = run_phase(8);
+    if (r) return r;
+    if (timed) cudaEventRecord(ev[9], stream);
+    return PNN_OK;
+  }
   for (int p = 4; p < 9; ++p) {
     int r = run_phase(p);
     if (r) return r;
@@ -1646,6 +1714,18 @@ int pnn_net::bind(void* dev, size_t bytes) {
     cudaError_t se = cudaStreamCreate(&stream);
     if (se != cudaSuccess) return cuda_check(se, "create stream");
     own_stream = true;
+  }
+  if (overlap_on && !s_hi) {
+    int lo = 0, hi = 0, dev = 0, sms = 0;
+    cudaError_t se = cudaDeviceGetStreamPriorityRange(&lo, &hi);
+    if (se == cudaSuccess) se = cudaStreamCreateWithPriority(&s_hi, cudaStreamNonBlocking, hi);
+    if (se == cudaSuccess) se = cudaStreamCreateWithPriority(&s_lo, cudaStreamNonBlocking, lo);
+    for (cudaEvent_t* ev_ : {&fork_ev, &hi_done, &lo_done})
+      if (se == cudaSuccess) se = cudaEventCreateWithFlags(ev_, cudaEventDisableTiming);
+    if (se == cudaSuccess) se = cudaGetDevice(&dev);
+    if (se == cudaSuccess) se = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (se != cudaSuccess) return cuda_check(se, "create overlap streams");
+    lo_cap = std::max(1, sms - opt.overlap);
   }
   int r = build_tables();
   if (r) return r;
@@ -1731,6 +1811,7 @@ void pnn_default_options(pnn_options* o) {
   o->stream = nullptr;
   o->bn_momentum = 0.1f;
   o->inference = 0;
+  o->overlap = 0;
 }
 
 int pnn_create(const pnn_desc* desc, const pnn_options* opts, pnn_net** out) {
@@ -1939,6 +2020,7 @@ int pnn_time_phases(pnn_net* n, const float* x, const int32_t* labels, int32_t s
   if (!x || !labels || !ms) return n->fail(PNN_EINVAL, "null argument");
   if (steps <= 0) return n->fail(PNN_EINVAL, "steps must be positive");
   if (n->prof) return n->fail(PNN_ESTATE, "phase timing needs profiling off");
+  if (n->overlap_on) return n->fail(PNN_ESTATE, "phase timing needs the phases in sequence (opts.overlap = 0)");
   if (n->first_step) {
     int r = pnn_train_step(n, x, labels, nullptr);
     if (r) return r;
@@ -2130,6 +2212,10 @@ void pnn_destroy(pnn_net* n) {
   for (auto& v : n->pev)
     if (v) cudaEventDestroy(v);
   if (n->own_stream && n->stream) cudaStreamDestroy(n->stream);
+  for (cudaEvent_t v : {n->fork_ev, n->hi_done, n->lo_done})
+    if (v) cudaEventDestroy(v);
+  if (n->s_hi) cudaStreamDestroy(n->s_hi);
+  if (n->s_lo) cudaStreamDestroy(n->s_lo);
   delete n;
 }
 
