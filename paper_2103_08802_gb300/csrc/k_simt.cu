@@ -404,49 +404,103 @@ __global__ void __launch_bounds__(256) k_ew_bwd(const EwBwdDesc* __restrict__ ta
 // ---------------------------------------------------------------- BN
 // one CTA per channel: thread t sums tiles t, t+256, ... in double, then a
 // fixed shared-memory tree combines the 256 partial sums
-__device__ __forceinline__ void block_sum2(double& a, double& b) {
-  __shared__ double ra[256], rb[256];
-  ra[threadIdx.x] = a;
-  rb[threadIdx.x] = b;
-  __syncthreads();
-  for (int w = 128; w > 0; w >>= 1) {
-    if ((int)threadIdx.x < w) {
-      ra[threadIdx.x] += ra[threadIdx.x + w];
-      rb[threadIdx.x] += rb[threadIdx.x + w];
+
+// Sums over one chunk of partial tiles ([tiles][C][2] floats) for the 32
+// channels of a channel group: lane = channel, warp w adds tiles t0+w, t0+w+8,
+// ... (eight independent 256-byte row loads per warp), then warp 0 adds the
+// eight warps' sums in warp order.  When a launch spans several chunks, each
+// CTA leaves its chunk sums in scratch and the last CTA of the channel group
+// (an atomic count) adds them: warp w takes chunks w, w+8, ..., warp 0 adds the
+// warps' sums in order, so the result does not depend on the order the CTAs
+// run in.  Returns true on the threads (warp 0, c < C) that hold the totals in
+// s1 / s2.
+__device__ __forceinline__ bool chunked_sums(const float* __restrict__ part, int C, int tiles, int cg, int chunk,
+                                             int nchunk, double* scratch, int32_t* counter, double& s1, double& s2) {
+  __shared__ double red[8][2][32];
+  __shared__ int is_last;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int c = cg * 32 + lane;
+  const int t0 = chunk * kFinTilesPerCta, t1 = min(tiles, t0 + kFinTilesPerCta);
+  double a = 0.0, b = 0.0;
+  if (c < C) {
+    float2 v[kFinTilesPerCta / 8];
+#pragma unroll
+    for (int k = 0; k < kFinTilesPerCta / 8; ++k) {
+      const int t = t0 + w + 8 * k;
+      v[k] = t < t1 ? *reinterpret_cast<const float2*>(part + ((int64_t)t * C + c) * 2) : make_float2(0.f, 0.f);
     }
-    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < kFinTilesPerCta / 8; ++k) {
+      a += (double)v[k].x;
+      b += (double)v[k].y;
+    }
   }
-  a = ra[0];
-  b = rb[0];
+  red[w][0][lane] = a;
+  red[w][1][lane] = b;
+  __syncthreads();
+  a = 0.0;
+  b = 0.0;
+  if (w == 0)
+    for (int k = 0; k < 8; ++k) {
+      a += red[k][0][lane];
+      b += red[k][1][lane];
+    }
+  if (nchunk == 1) {
+    s1 = a;
+    s2 = b;
+    return w == 0 && c < C;
+  }
+  if (w == 0 && c < C) {
+    scratch[((int64_t)chunk * C + c) * 2] = a;
+    scratch[((int64_t)chunk * C + c) * 2 + 1] = b;
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) is_last = atomicAdd(counter + cg, 1) == nchunk - 1;
+  __syncthreads();
+  if (!is_last) return false;
+  __threadfence();
+  a = 0.0;
+  b = 0.0;
+  if (c < C)
+    for (int k = w; k < nchunk; k += 8) {
+      a += __ldcg(scratch + ((int64_t)k * C + c) * 2);
+      b += __ldcg(scratch + ((int64_t)k * C + c) * 2 + 1);
+    }
+  red[w][0][lane] = a;
+  red[w][1][lane] = b;
+  __syncthreads();
+  a = 0.0;
+  b = 0.0;
+  if (w == 0)
+    for (int k = 0; k < 8; ++k) {
+      a += red[k][0][lane];
+      b += red[k][1][lane];
+    }
+  if (threadIdx.x == 0) counter[cg] = 0;  // ready for the next launch
+  s1 = a;
+  s2 = b;
+  return w == 0 && c < C;
 }
 
 __global__ void __launch_bounds__(256) k_bn_fin(const BnFinDesc* __restrict__ tab, const int* __restrict__ tstart,
                                                 int n) {
   const int inst = find_instance(tstart, n, blockIdx.x);
   const BnFinDesc& d = tab[inst];
-  const int c = blockIdx.x - tstart[inst];
+  const int local = blockIdx.x - tstart[inst];
+  const int cg = local % d.cgroups, chunk = local / d.cgroups;
+  const int c = cg * 32 + (threadIdx.x & 31);
+  double mean, var;
   if (d.eval) {
     // eval mode: the running statistics stand in for the batch's
-    if (threadIdx.x == 0) {
-      const double mean = d.run_mean[c];
-      const double rstd = 1.0 / sqrt((double)d.run_var[c] + 1e-5);
-      const double sc = (double)d.gamma[c] * rstd;
-      d.mean[c] = (float)mean;
-      d.rstd[c] = (float)rstd;
-      d.scale[c] = (float)sc;
-      d.shift[c] = (float)((double)d.beta[c] - mean * sc);
-    }
-    return;
-  }
-  double s1 = 0.0, s2 = 0.0;
-  for (int t = threadIdx.x; t < d.tiles; t += 256) {
-    s1 += (double)d.part[((int64_t)t * d.C + c) * 2];
-    s2 += (double)d.part[((int64_t)t * d.C + c) * 2 + 1];
-  }
-  block_sum2(s1, s2);
-  if (threadIdx.x == 0) {
-    const double mean = s1 / (double)d.count;
-    double var = s2 / (double)d.count - mean * mean;
+    if (threadIdx.x >= 32 || c >= d.C) return;
+    mean = d.run_mean[c];
+    var = d.run_var[c];
+  } else {
+    double s1, s2;
+    if (!chunked_sums(d.part, d.C, d.tiles, cg, chunk, d.nchunk, d.scratch, d.counter, s1, s2)) return;
+    mean = s1 / (double)d.count;
+    var = s2 / (double)d.count - mean * mean;
     if (var < 0.0) var = 0.0;
     if (d.run_mean) {
       // running statistics follow the batch mean and the unbiased variance
@@ -455,13 +509,13 @@ __global__ void __launch_bounds__(256) k_bn_fin(const BnFinDesc* __restrict__ ta
       d.run_mean[c] = (float)((1.0 - m) * (double)d.run_mean[c] + m * mean);
       d.run_var[c] = (float)((1.0 - m) * (double)d.run_var[c] + m * unbiased);
     }
-    const double rstd = 1.0 / sqrt(var + 1e-5);
-    const double sc = (double)d.gamma[c] * rstd;
-    d.mean[c] = (float)mean;
-    d.rstd[c] = (float)rstd;
-    d.scale[c] = (float)sc;
-    d.shift[c] = (float)((double)d.beta[c] - mean * sc);
   }
+  const double rstd = 1.0 / sqrt(var + 1e-5);
+  const double sc = (double)d.gamma[c] * rstd;
+  d.mean[c] = (float)mean;
+  d.rstd[c] = (float)rstd;
+  d.scale[c] = (float)sc;
+  d.shift[c] = (float)((double)d.beta[c] - mean * sc);
 }
 
 __global__ void __launch_bounds__(256) k_bnb_reduce(const BnBwdDesc* __restrict__ tab,
@@ -512,20 +566,16 @@ __global__ void __launch_bounds__(256) k_bnb_fin(const BnBwdDesc* __restrict__ t
                                                  int n) {
   const int inst = find_instance(tstart, n, blockIdx.x);
   const BnBwdDesc& d = tab[inst];
-  const int c = blockIdx.x - tstart[inst];
-  double s1 = 0.0, s2 = 0.0;
-  for (int t = threadIdx.x; t < d.tiles; t += 256) {
-    s1 += (double)d.part[((int64_t)t * d.C + c) * 2];
-    s2 += (double)d.part[((int64_t)t * d.C + c) * 2 + 1];
-  }
-  block_sum2(s1, s2);
-  if (threadIdx.x == 0) {
-    d.dbeta[c] = d.accumulate ? d.dbeta[c] + (float)s1 : (float)s1;
-    d.dgamma[c] = d.accumulate ? d.dgamma[c] + (float)s2 : (float)s2;
-    d.coef[c * 3 + 0] = d.gamma[c] * d.rstd[c];
-    d.coef[c * 3 + 1] = (float)(s1 / (double)d.M);
-    d.coef[c * 3 + 2] = (float)(s2 / (double)d.M);
-  }
+  const int local = blockIdx.x - tstart[inst];
+  const int cg = local % d.cgroups, chunk = local / d.cgroups;
+  const int c = cg * 32 + (threadIdx.x & 31);
+  double s1, s2;
+  if (!chunked_sums(d.part, d.C, d.tiles, cg, chunk, d.nchunk, d.scratch, d.counter, s1, s2)) return;
+  d.dbeta[c] = d.accumulate ? d.dbeta[c] + (float)s1 : (float)s1;
+  d.dgamma[c] = d.accumulate ? d.dgamma[c] + (float)s2 : (float)s2;
+  d.coef[c * 3 + 0] = d.gamma[c] * d.rstd[c];
+  d.coef[c * 3 + 1] = (float)(s1 / (double)d.M);
+  d.coef[c * 3 + 2] = (float)(s2 / (double)d.M);
 }
 
 __global__ void __launch_bounds__(256) k_bnb_apply(const BnBwdDesc* __restrict__ tab,

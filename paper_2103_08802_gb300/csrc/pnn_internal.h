@@ -86,9 +86,11 @@ struct EwBwdDesc {
   int32_t nin;
   int64_t M; int32_t C;
   int32_t rows_per_tile, tiles;
+  double* scratch; int32_t* counter; int32_t cgroups, nchunk;  // fin: as for BnFinDesc
 };
 
 // BN statistics finalisation: partials[tiles][C][2] -> mean, rstd, scale, shift
+constexpr int kFinTilesPerCta = 64;  // BN finalize: partial tiles one CTA adds up (8 per warp)
 struct BnFinDesc {
   const float* part;
   int32_t tiles, C;
@@ -98,6 +100,10 @@ struct BnFinDesc {
   float* run_mean; float* run_var;  // running statistics of this BN layer
   float momentum;                   // training: rate at which they follow the batch
   int32_t eval;                     // 1: normalise with the running statistics
+  // the reduction over tiles: CTAs = cgroups (32 channels each) x nchunk (64
+  // tiles each); chunk sums meet in scratch ([nchunk][C][2] doubles) and the
+  // last CTA of a channel group (counter[cg], zero between launches) adds them
+  double* scratch; int32_t* counter; int32_t cgroups, nchunk;
 };
 
 // BN backward: dz = da * [z > 0 if relu], z = scale*h + shift, xhat = (h-mean)*rstd
@@ -117,6 +123,7 @@ struct BnBwdDesc {
   const float* add0; const float* add1;  // apply: extra gradients added into dh (residual paths)
   int64_t M; int32_t C;
   int32_t rows_per_tile, tiles;
+  double* scratch; int32_t* counter; int32_t cgroups, nchunk;  // fin: as for BnFinDesc
 };
 
 struct PoolDesc {

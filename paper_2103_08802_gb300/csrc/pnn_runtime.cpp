@@ -71,6 +71,9 @@ struct Norm {
   size_t part = 0, mean = 0, rstd = 0, scale = 0, shift = 0, bpart = 0, coef = 0;
   int btiles = 0;
   size_t run = 0;  // running mean (C floats) followed by running variance (C floats)
+  // finalize reductions (forward statistics, backward sums): chunk scratch and
+  // per-channel-group counters
+  size_t fscr = 0, fcnt = 0, bscr = 0, bcnt = 0;
 };
 
 // One planned op (forward or backward).  Fields are interpreted per kind.
@@ -216,6 +219,7 @@ struct pnn_net {
   cudaEvent_t fork_ev = nullptr, hi_done = nullptr, lo_done = nullptr;
   int lo_cap = 0;  // grid cap of s_lo's persistent kernels
   size_t running_floats = 0, off_running = 0;
+  size_t off_fin_cnt = 0, fin_cnt_bytes = 0;
   // pnn_infer's graph, captured for (ix, ilogits)
   cudaGraphExec_t igexec = nullptr;
   const float* ix = nullptr;
@@ -1059,14 +1063,29 @@ int pnn_net::plan(const pnn_desc* d) {
       if (v.need_grad) v.goff = alloc((size_t)B * v.H * v.W * v.C * 4);
     }
   }
+  // finalize counters: one region, zeroed at bind (each launch leaves them zero)
+  {
+    size_t ncnt = 0;
+    for (auto& n : norms) ncnt += 2 * (size_t)cdiv(n.C, 32);
+    off_fin_cnt = alloc(ncnt * 4);
+    fin_cnt_bytes = ncnt * 4;
+    size_t at = off_fin_cnt;
+    for (auto& n : norms) {
+      n.fcnt = at; at += (size_t)cdiv(n.C, 32) * 4;
+      n.bcnt = at; at += (size_t)cdiv(n.C, 32) * 4;
+    }
+  }
   for (auto& n : norms) {
     n.part = alloc((size_t)n.tiles * n.C * 8);
     n.mean = alloc(n.C * 4); n.rstd = alloc(n.C * 4); n.scale = alloc(n.C * 4); n.shift = alloc(n.C * 4);
     n.run = off_running + run_at[n.gamma] * 4;
+    n.fscr = alloc((size_t)cdiv(std::max(n.tiles, 1), kFinTilesPerCta) * n.C * 16);
     if (opt.inference) continue;
     n.btiles = cdiv(n.count, bnb_rows_per_tile(n.C));
     // room for the reduce kernel's tiles or a fused data gradient's 128-row tiles
-    n.bpart = alloc((size_t)std::max(n.btiles, cdiv(n.count, kTcBM)) * n.C * 8);
+    const int bt = std::max(n.btiles, cdiv(n.count, kTcBM));
+    n.bpart = alloc((size_t)bt * n.C * 8);
+    n.bscr = alloc((size_t)cdiv(bt, kFinTilesPerCta) * n.C * 16);
     n.coef = alloc((size_t)n.C * 12);
   }
   // wgrad scratch: one region per op (sized per op)
@@ -1333,7 +1352,10 @@ int pnn_net::build_tables() {
             f.run_mean = P<float>(n.run); f.run_var = P<float>(n.run) + n.C;
             f.momentum = opt.bn_momentum;
             f.eval = opt.inference ? 1 : 0;
-            add(&f, sizeof f, n.C);  // one CTA per channel
+            f.scratch = P<double>(n.fscr); f.counter = P<int32_t>(n.fcnt);
+            f.cgroups = cdiv(n.C, 32);
+            f.nchunk = f.eval ? 1 : cdiv(std::max(n.tiles, 1), kFinTilesPerCta);
+            add(&f, sizeof f, f.cgroups * f.nchunk);
             break;
           }
           case K_BNB_RED:
@@ -1352,6 +1374,9 @@ int pnn_net::build_tables() {
             b.coef = P<float>(n.coef);
             b.M = n.count; b.C = n.C;
             b.rows_per_tile = bnb_rows_per_tile(n.C); b.tiles = n.fused_tiles ? n.fused_tiles : n.btiles;
+            b.scratch = P<double>(n.bscr); b.counter = P<int32_t>(n.bcnt);
+            b.cgroups = cdiv(n.C, 32);
+            b.nchunk = cdiv(std::max(b.tiles, 1), kFinTilesPerCta);
             if (o.kind == K_BNB_FIN) b.accumulate = o.acc_in[0];
             if (o.kind == K_BNB_APPLY) {
               b.dh = P<float>(gptr(n.h));
@@ -1359,7 +1384,7 @@ int pnn_net::build_tables() {
               b.add0 = o.addv[0] >= 0 ? P<float>(gptr(o.addv[0])) : nullptr;
               b.add1 = o.addv[1] >= 0 ? P<float>(gptr(o.addv[1])) : nullptr;
             }
-            add(&b, sizeof b, o.tiles);
+            add(&b, sizeof b, o.kind == K_BNB_FIN ? b.cgroups * b.nchunk : o.tiles);
             break;
           }
           case K_POOL_FWD:
@@ -1760,6 +1785,7 @@ int pnn_net::bind(void* dev, size_t bytes) {
     e = cudaMemcpy(ws + off_running, run.data(), running_floats * 4, cudaMemcpyHostToDevice);
   }
   if (e == cudaSuccess) e = cudaMemset(ws + status_off, 0, 64);
+  if (e == cudaSuccess && fin_cnt_bytes) e = cudaMemset(ws + off_fin_cnt, 0, fin_cnt_bytes);
   if (e == cudaSuccess && act_dt == DT_BF16)
     e = launch_copy_cast(P<float>(off_master), ws + off_shadow, DT_BF16, (int64_t)nparams, stream);
   if (e == cudaSuccess) e = refresh_wt();
