@@ -790,37 +790,68 @@ __global__ void __launch_bounds__(256) k_pool_bwd(const PoolDesc* __restrict__ t
 }
 
 // ---------------------------------------------------------------- GEMM (head)
+// C[m][n] = sum_k A[m][k] B[k][n] (+ bias[n]) (+ beta C[m][n]) (ReLU), fp32.
+// 64 x 64 tiles, 256 threads with 4 x 4 outputs each; the K loop runs in 32-wide
+// steps with the next step's operands loaded into registers while the current
+// one is multiplied from shared memory (double buffered).  Each operand is read
+// along whichever of its two indices is contiguous in memory, so every warp load
+// is coalesced for any of the head's layouts.  Every output sums its k terms in
+// ascending order with one fused multiply-add each.
 __global__ void __launch_bounds__(256) k_gemm(const GemmDesc* __restrict__ tab, const int* __restrict__ tstart,
                                               int n) {
-  constexpr int BM = 64, BN = 64, BK = 16;
-  __shared__ float As[BK][BM + 4];
-  __shared__ float Bs[BK][BN + 4];
+  constexpr int BM = 64, BN = 64, BK = 32, PER = BM * BK / 256;
+  __shared__ float As[2][BK][BM + 4];
+  __shared__ float Bs[2][BK][BN + 4];
   const int inst = find_instance(tstart, n, blockIdx.x);
   const GemmDesc& d = tab[inst];
   const int t = blockIdx.x - tstart[inst];
   const int tm = t % d.mtiles, tn = t / d.mtiles;
   const int m0 = tm * BM, n0 = tn * BN;
   const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+  const bool a_k = d.sak == 1, b_k = d.sbk == 1;  // k contiguous in A / in B
+  float ra[PER], rb[PER];
+  auto slot = [&](int e, bool k_fast, int W, int& kk, int& x) {
+    if (k_fast) { kk = e % BK; x = e / BK; } else { x = e % W; kk = e / W; }
+  };
+  auto load = [&](int k0) {
+#pragma unroll
+    for (int q = 0; q < PER; ++q) {
+      int kk, x;
+      slot(tid + 256 * q, a_k, BM, kk, x);
+      const int m = m0 + x, k = k0 + kk;
+      ra[q] = (m < d.M && k < d.K) ? d.A[(int64_t)m * d.sam + (int64_t)k * d.sak] : 0.f;
+      slot(tid + 256 * q, b_k, BN, kk, x);
+      const int nc = n0 + x, kb = k0 + kk;
+      rb[q] = (nc < d.N && kb < d.K) ? d.Bm[(int64_t)kb * d.sbk + (int64_t)nc * d.sbn] : 0.f;
+    }
+  };
+  auto store = [&](int buf) {
+#pragma unroll
+    for (int q = 0; q < PER; ++q) {
+      int kk, x;
+      slot(tid + 256 * q, a_k, BM, kk, x);
+      As[buf][kk][x] = ra[q];
+      slot(tid + 256 * q, b_k, BN, kk, x);
+      Bs[buf][kk][x] = rb[q];
+    }
+  };
   float acc[4][4] = {};
+  load(0);
+  store(0);
+  __syncthreads();
+  int buf = 0;
   for (int k0 = 0; k0 < d.K; k0 += BK) {
-    for (int e = tid; e < BM * BK; e += 256) {
-      const int kk = e % BK, mm = e / BK;
-      const int m = m0 + mm, k = k0 + kk;
-      As[kk][mm] = (m < d.M && k < d.K) ? d.A[m * d.sam + k * d.sak] : 0.f;
-    }
-    for (int e = tid; e < BN * BK; e += 256) {
-      const int nn = e % BN, kk = e / BN;
-      const int nc = n0 + nn, k = k0 + kk;
-      Bs[kk][nn] = (nc < d.N && k < d.K) ? d.Bm[k * d.sbk + nc * d.sbn] : 0.f;
-    }
-    __syncthreads();
+    const bool more = k0 + BK < d.K;
+    if (more) load(k0 + BK);
 #pragma unroll
     for (int kk = 0; kk < BK; ++kk)
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(As[kk][ty + 16 * i], Bs[kk][tx + 16 * j], acc[i][j]);
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(As[buf][kk][ty + 16 * i], Bs[buf][kk][tx + 16 * j], acc[i][j]);
+    if (more) store(buf ^ 1);
     __syncthreads();
+    buf ^= 1;
   }
 #pragma unroll
   for (int i = 0; i < 4; ++i)
@@ -830,9 +861,9 @@ __global__ void __launch_bounds__(256) k_gemm(const GemmDesc* __restrict__ tab, 
       if (m < d.M && nc < d.N) {
         float v = acc[i][j];
         if (d.bias) v += d.bias[nc];
-        if (d.beta != 0.f) v += d.beta * d.Cm[m * d.scm + nc];
+        if (d.beta != 0.f) v += d.beta * d.Cm[(int64_t)m * d.scm + nc];
         if (d.relu) v = fmaxf(v, 0.f);
-        d.Cm[m * d.scm + nc] = v;
+        d.Cm[(int64_t)m * d.scm + nc] = v;
       }
     }
 }
