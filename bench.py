@@ -176,6 +176,20 @@ def cores():
         return os.cpu_count()
 
 
+def config_of(args, desc, world=1, extra=None):
+    """The `config` object of both arms' JSON lines."""
+    B = desc["batch"]
+    c = {"workload": desc["name"] + "_b%d_%dpx_c%d" % (B, desc["in_h"], desc["classes"]),
+         "batch": B, "input": "3x%dx%d" % (desc["in_h"], desc["in_w"]), "classes": desc["classes"],
+         "subnetworks": len(desc["segments"]), "correction": desc.get("correction", "residual"),
+         "residual_stream": "fp32" if args.stream_fp32 else "bf16", "lr": args.lr,
+         "tearing": "uniform" if args.tearing == "none" else args.tearing,
+         "overlap_sms": args.overlap,
+         "parallelism": "replicas" if world > 1 else "single-gpu"}
+    c.update(extra or {})
+    return c
+
+
 def reference_arm(args, desc, rank):
     if rank != 0:
         return
@@ -190,7 +204,7 @@ def reference_arm(args, desc, rank):
         "impl": "reference", "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": desc["name"] + "_b%d" % desc["batch"], "batch": desc["batch"]},
+        "data": "synthetic", "config": config_of(args, desc, args.gpus),
         "cpu_baseline": {"value": value, "unit": "images/s", "cores": cores(), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
@@ -461,14 +475,8 @@ def our_arm(args, desc, rank, local, world, dist):
         "warmup": max(3, args.warmup), "ms_per_step": ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if desc["precision"] == "bf16" else "fp32",
         "data": "synthetic",
-        "config": {"workload": desc["name"] + "_b%d_%dpx_c%d" % (B, desc["in_h"], desc["classes"]),
-                   "batch": B, "input": "3x%dx%d" % (desc["in_h"], desc["in_w"]), "classes": desc["classes"],
-                   "subnetworks": len(desc["segments"]), "correction": desc.get("correction", "residual"),
-                   "residual_stream": "fp32" if args.stream_fp32 else "bf16", "lr": args.lr,
-                   "tearing": "uniform" if args.tearing == "none" else args.tearing,
-                   "overlap_sms": args.overlap,
-                   "l2": "inputs larger than L2 (%.1f GB workspace per step)" % (net.workspace_bytes / 1e9),
-                   "parallelism": "replicas" if world > 1 else "single-gpu"},
+        "config": config_of(args, desc, world, {
+            "l2": "inputs larger than L2 (%.1f GB workspace per step)" % (net.workspace_bytes / 1e9)}),
         "conv_tflops": conv_flops / (conv_ms / 1e3) / 1e12 if conv_ms else None,
         "conv_frac_of_bf16_peak": (conv_flops / (conv_ms / 1e3) / 1e12) / pk["bf16_tflops_sustained"] if conv_ms else None,
         "conv_share_of_device_time": conv_ms / total_prof_ms if total_prof_ms else None,
