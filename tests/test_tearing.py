@@ -90,3 +90,29 @@ def test_balanced_segments_of_resnet1001(pnn):
     assert sum(fl) == sum(by) == 333
     assert max(fl) - min(fl) <= 1
     assert by[0] < by[-1] / 2
+
+
+# ------------------------------------------------------------ pins of the oracle's own tearing helpers
+def test_oracle_best_cut_textbook_cases():
+    """The classic "split an array into m parts minimising the largest sum"
+    examples, worked by hand."""
+    assert T.best_cut([7, 2, 5, 10, 8], 2) == 18      # 7+2+5 | 10+8
+    assert T.best_cut([1, 2, 3, 4, 5], 2) == 9        # 1+2+3 | 4+5
+    assert T.best_cut([1, 4, 4], 3) == 4
+    assert T.best_cut([5, 5, 5, 5], 1) == 20
+    assert T.best_cut([3, 1, 4, 1, 5, 9, 2, 6], 8) == 9
+
+
+def test_oracle_layer_flops_closed_form():
+    """A non-strided ResNet-1001 bottleneck on a 32x32 map with 64 channels and
+    width 16 takes 1024 * (64*16 + 9*16*16 + 16*64) multiply-adds per image in
+    the forward pass (the same at every stage: 4x the pixels, 1/4 the channels
+    squared), and three times that in training; the whole body of 333 units
+    with its stem comes to about 8.95 GFLOP of training convolutions per 32x32
+    image."""
+    per_unit = 1024 * (64 * 16 + 9 * 16 * 16 + 16 * 64)
+    d = W.parareal_resnet1001(n_seg=1, batch=2, segments=[333])
+    f = T.body_training_flops(d, (16, 32, 32))
+    assert f[5] == f[150] == f[300] == 6 * per_unit * 2
+    stem = 3 * 2 * T.layer_forward_macs(d["stem"][0], (3, 32, 32))[0]
+    assert abs((sum(f) / 2 + stem) / 8.95e9 - 1) < 1e-3
