@@ -103,3 +103,46 @@ def test_wait_selftest_rejects_bad_limits(pnn):
     assert lib.pnn_selftest_wait_timeout(0, None) == 1          # PNN_EINVAL, before any CUDA call
     assert lib.pnn_selftest_wait_timeout(-5, None) == 1
     assert b"limit_ns" in lib.pnn_last_error(None)
+
+
+@pytest.mark.parametrize("idx", range(5))
+def test_running_stats_layout_and_inference_plan(pnn, idx):
+    """The library's running-statistics block has the oracle's layout size
+    (2 C floats per BN layer), and an inference plan of the same network --
+    forward only, activation buffers handed on by liveness -- needs a fraction
+    of the training workspace."""
+    import ctypes as C
+    d = W.config(idx)
+    train = pnn.ParaNet(d, bind=False)
+    infer = pnn.ParaNet(d, bind=False, inference=True)
+    n = C.c_size_t()
+    assert train.lib.pnn_running_stats_size(train.h, C.byref(n)) == 0
+    assert n.value == O.RunningStats(O.ParaNet(d).spec).flat().size
+    assert infer.lib.pnn_running_stats_size(infer.h, C.byref(n)) == 0
+    assert n.value == O.RunningStats(O.ParaNet(d).spec).flat().size
+    assert infer.num_params == train.num_params
+    assert infer.workspace_bytes < train.workspace_bytes / 2
+
+
+def test_overlap_option_plans_the_last_subnetwork_apart(pnn):
+    """opts.overlap moves the last subnetwork's backward out of the grouped
+    launches (more backward launches, the same forward) in the residual form
+    with N > 1, and leaves the delta form and N = 1 as they are."""
+    import ctypes as C
+
+    def counts(d, **kw):
+        net = pnn.ParaNet(d, bind=False, **kw)
+        c = (C.c_int32 * 3)()
+        assert net.lib.pnn_launch_counts(net.h, c) == 0
+        return list(c)
+
+    d = W.config(2)
+    seq, ov = counts(d), counts(d, overlap=32)
+    assert ov[0] == seq[0] and ov[1] > seq[1] and ov[2] == seq[2]
+    dd = W.config(2)
+    dd["correction"] = "delta"
+    assert counts(dd, overlap=32) == counts(dd)
+    d1 = W.config(0)
+    d1["segments"] = [4]
+    d1["coarse"] = []
+    assert counts(d1, overlap=32) == counts(d1)
