@@ -21,6 +21,10 @@ Parallel-in-time Algorithm"):
     the coarse chain backwards for D_j and the eta_j gradients, then every
     subnetwork with seed dL/dy_j = D_j and dL/dx_j -= D_{j-1}.
   * Section 4: SGD with Nesterov momentum and weight decay.
+  * BN running statistics and the eval-mode forward (the paper states no rule;
+    the reading is PyTorch's BatchNorm2d, see RunningStats): ParaNet.forward
+    with a RunningStats moves them, ParaNet.infer normalises with them.
+  * Section 4.2's coarse RU (two 3x3 convs and a skip, CoarseRU).
 
 Layout is NCHW, every value float64.  Each primitive is the textbook
 definition written out; numpy's tensordot (a library matmul) serves as the
