@@ -1,7 +1,7 @@
 """Shared helpers of the GPU parity tests: run one training step through the
 C ABI and through the oracle on the same seeded inputs and compare.
 
-Metrics (the benchmark spec gives the numbers, not the formulas):
+Metrics (the target tolerances; the formulas are these):
   forward tensors  max|a - r| / max|r|            <= 2e-2 (bf16), 1e-4 (fp32 check)
   gradients        ||g - r||_2 / ||r||_2 per tensor <= 5e-2 (bf16), 1e-4 (fp32 check)
 """

@@ -3,7 +3,7 @@ oracle, through the C ABI.
 
 * After a training-mode forward every BN's running mean and variance (momentum 0.1,
   unbiased batch variance) match the oracle's: fp32 check mode within 1e-4
-  (north_star's fp32 bound), bf16 within 2e-2 max-relative (the forward bound;
+  (the fp32 target bound), bf16 within 2e-2 max-relative (the forward bound;
   the statistics are forward quantities).
 * An inference net (opts.inference = 1: forward only, activations sharing
   buffers) given the same parameters and running statistics returns the

@@ -2,7 +2,7 @@
 update) against the CPU oracle on identical seeded inputs and weights,
 through the C ABI.
 
-Tolerances.  the benchmark spec's bounds are 2e-2 (bf16 forward, max-relative),
+Tolerances.  The target bounds are 2e-2 (bf16 forward, max-relative),
 5e-2 (bf16 gradients, norm-relative) and 1e-4 (fp32 check mode).  They are
 applied as they stand wherever they are attainable: every forward tensor in
 bf16 and every quantity in fp32 check mode at small sizes.  Two effects make
@@ -18,7 +18,7 @@ cases, and there the bound is measured instead of assumed:
 * in fp32 beyond the tiny config the same flips occur at the fp32
   accumulation-order level (and amplify with depth); the bound is 3x the
   oracle's own response to a 1e-5 relative perturbation of its parameters,
-  and never below the benchmark spec value.  The same measured bound covers
+  and never below the target bound.  The same measured bound covers
   forward tensors where depth amplifies rounding past 2e-2 / 1e-4.
 """
 import numpy as np
@@ -56,7 +56,7 @@ def _grad_keys(report):
 
 
 def _measured(desc, noise_fn, factor, floor):
-    """Every key is bounded by max(the benchmark spec bound, factor * measured noise):
+    """Every key is bounded by max(target bound, factor * measured noise):
     the forward bound for forward tensors, `floor` for D_j and gradients."""
     onet, theta, x, labels = inputs(desc)
     g = run_gpu(desc, theta, x, labels)
@@ -153,7 +153,7 @@ def paper_reduced(n, precision="bf16", correction="residual", batch=128):
                                    correction=correction)
 
 
-# ------------------------------------------------------------------ strict (the benchmark spec bounds)
+# ------------------------------------------------------------------ strict (target bounds)
 @pytest.mark.parametrize("mode", ["residual", "delta"])
 def test_tiny_fp32_check_mode_step(mode):
     desc = W.config(0)

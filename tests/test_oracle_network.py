@@ -194,7 +194,7 @@ def _sequential_theta(net, theta):
 
 @pytest.mark.parametrize("name", list(NETS))
 def test_delta_mode_with_fine_coarse_is_sequential(name):
-    """The benchmark spec's consistency check, exact for the nonlinear network in the
+    """The consistency check of the delta form, exact for the nonlinear network in the
     delta form: state_{j} = x_{j+1} + rt_j equals g^j(...g^1(C x)) when
     F^j = g^{j+1}."""
     desc = _coarse_is_fine(NETS[name]("delta"))
