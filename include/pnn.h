@@ -264,8 +264,8 @@ int pnn_block_costs(const pnn_desc* desc, const pnn_options* opts, int32_t kind,
  * non-empty segments whose largest cost sum is as small as possible (exact).
  * Among the optimal cuts it returns the one whose segments, from the first on,
  * each take as many layers as the optimum allows.  segments: caller-owned,
- * n_seg ints (layers per segment, summing to n).  PNN_EINVAL unless
- * 1 <= n_seg <= n. */
+ * n_seg ints (layers per segment, summing to n).  Time O(n_seg * n^2);
+ * PNN_EINVAL unless 1 <= n_seg <= n and n_seg * n^2 <= 4e9. */
 int pnn_partition(const double* cost, int32_t n, int32_t n_seg, int32_t* segments);
 
 /* Per-phase device time of whole training steps replayed from CUDA graphs,

@@ -1908,6 +1908,7 @@ int pnn_block_costs(const pnn_desc* desc, const pnn_options* opts, int32_t kind,
 int pnn_partition(const double* cost, int32_t n, int32_t n_seg, int32_t* segments) {
   if (!cost || !segments) return set_global(PNN_EINVAL, "null argument");
   if (n_seg <= 0 || n < n_seg) return set_global(PNN_EINVAL, "need 1 <= n_seg <= n");
+  if ((double)n_seg * n * n > 4e9) return set_global(PNN_EINVAL, "n_seg * n^2 above 4e9 (the exact cut's cost)");
   std::vector<double> S(n + 1, 0.0);
   for (int i = 0; i < n; ++i) {
     if (!(cost[i] >= 0.0) || !std::isfinite(cost[i])) return set_global(PNN_EINVAL, "costs must be finite and >= 0");

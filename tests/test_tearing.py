@@ -116,3 +116,8 @@ def test_oracle_layer_flops_closed_form():
     assert f[5] == f[150] == f[300] == 6 * per_unit * 2
     stem = 3 * 2 * T.layer_forward_macs(d["stem"][0], (3, 32, 32))[0]
     assert abs((sum(f) / 2 + stem) / 8.95e9 - 1) < 1e-3
+
+
+def test_partition_rejects_oversized_problems(pnn):
+    with pytest.raises(pnn.PnnError):
+        pnn.partition([1.0] * 40000, 3)
