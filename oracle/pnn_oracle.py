@@ -33,13 +33,13 @@ open (BN eps, pooling padding, block layout, loss) are the module constants
 and the layer classes below.
 
 Precision model.  The paper fixes no precision.  By default everything is
-float64.  With precision="bf16" the forward pass rounds to bfloat16 exactly
-the values a bf16 tensor-core implementation holds in bf16: every
-convolution operand (input activation and weight) and every stored
-convolution / pooling output that is not followed by a residual add.  This
-makes the floating-point decisions of the forward pass (ReLU masks, maxpool
-argmax) use the kernel's precision; all arithmetic stays float64 and no
-gradient is rounded.
+float64.  With precision="bf16" the pass rounds to bfloat16 exactly the
+values a bf16 tensor-core implementation holds in bf16: every convolution
+operand (input activation, weight, and in the backward pass the output
+gradient), and every stored convolution / pooling output that is not
+followed by a residual add.  This makes the floating-point decisions of the
+forward pass (ReLU masks, maxpool argmax) use the kernel's precision; all
+arithmetic stays float64.
 """
 from __future__ import annotations
 
@@ -267,6 +267,31 @@ def sgd_step(theta, grad, buf, lr, momentum, weight_decay, nesterov):
 
 
 # =================================================================== layers
+# Test hook (never set by the oracle itself): while a `perturbed` context is
+# active every convolution output is multiplied by (1 + rel * N(0, 1)) before
+# any rounding.  Tests use it to measure how far the oracle's own result moves
+# under differences of the size an fp32 accumulation order leaves in a
+# convolution, which bounds how far any correct implementation can be from it.
+_PERTURB = None
+
+
+class perturbed:
+    """Context manager: conv outputs perturbed by a relative `rel`, normal
+    draws from numpy Generator `rng` (see _PERTURB)."""
+
+    def __init__(self, rng, rel):
+        self.rng, self.rel = rng, rel
+
+    def __enter__(self):
+        global _PERTURB
+        _PERTURB = (self.rng, self.rel)
+        return self
+
+    def __exit__(self, *a):
+        global _PERTURB
+        _PERTURB = None
+
+
 class _Layer:
     """A layer maps (C,H,W) -> (C',H',W'); it lists its parameters as
     (kind, shape) and implements forward / backward on numpy arrays."""
@@ -305,10 +330,15 @@ class Conv(_Layer):
     def forward(self, x, P):
         xq = self._q(x)
         y = conv2d(xq, self._q(P[0]), self.stride, self.pad)
+        if _PERTURB is not None:
+            y = y * (1.0 + _PERTURB[1] * _PERTURB[0].standard_normal(y.shape))
         return (self._q(y) if self.store_q else y), xq
 
     def backward(self, dy, P, cache, need_dx=True):
-        dx, dw = conv2d_backward(cache, self._q(P[0]), self.stride, self.pad, dy, need_dx)
+        # the bf16 model: the output gradient is a contraction operand too
+        dx, dw = conv2d_backward(cache, self._q(P[0]), self.stride, self.pad, self._q(dy), need_dx)
+        if _PERTURB is not None and dx is not None:
+            dx = dx * (1.0 + _PERTURB[1] * _PERTURB[0].standard_normal(dx.shape))
         return dx, [dw]
 
 
