@@ -324,6 +324,68 @@ const char* pnn_kernel_kind_name(int32_t kind); /* NULL for a bad kind */
  * address low 40 bits); 0 if none or in release builds. */
 uint64_t pnn_debug_word(void);
 
+/* ---- one grouped convolution on caller buffers ----
+ * The three contractions of a training step's convolution layers (Section 3.2:
+ * Algorithm 1's forward g^j, Algorithm 2's data and weight gradients), run
+ * alone through the same tensor-core kernels pnn_forward / pnn_backward
+ * launch, so that each kernel can be checked element by element.  n instances
+ * (each its own geometry and buffers) form one grouped launch, as the N
+ * subnetworks' layers do in a step.  Zero padding ksize/2; p = (h + 2*pad -
+ * ksize)/stride + 1, q likewise.  Contraction operands are rounded to bf16
+ * (round to nearest even), products accumulate in fp32.
+ *   mode PNN_CONV_FORWARD  y[n][p][q][kk] = res + sum_{r,s,cc} v(x)[n][p*stride+r-pad][q*stride+s-pad][cc] * w[kk][r][s][cc]
+ *                          with v(x) = bn_scale[cc]*x + bn_shift[cc], then max(0, .) when
+ *                          relu != 0, when bn_scale is given (the BN(+ReLU) of the layer
+ *                          before, applied on load), else v(x) = x; y rounded to y_dtype.
+ *                          y_mean / y_rstd (optional, device, k floats): the batch
+ *                          statistics of y that a following BN layer uses (mean, 1/sqrt(var + 1e-5),
+ *                          biased variance over batch*p*q rows, Section 4's BN)
+ *   mode PNN_CONV_DGRAD    dx[n][i][j][cc] (+)= sum_{r,s,kk} dy[n][p][q][kk] * w[kk][r][s][cc]
+ *                          over the (p, q) with p*stride+r-pad = i, q*stride+s-pad = j.
+ *                          With bn_mean / bn_rstd given (x = the BN input h, bn_scale /
+ *                          bn_shift / relu its forward BN): dbeta[cc] = sum g and dgamma[cc] =
+ *                          sum g * (h - mean) * rstd over all rows, g = dx masked by the ReLU of
+ *                          bn_scale*h + bn_shift (the BN-backward sums of that layer)
+ *   mode PNN_CONV_WGRAD    dw[kk][r][s][cc] = sum_{n,p,q} dy[n][p][q][kk] * v(x)[n][p*stride+r-pad][q*stride+s-pad][cc]
+ * impl: 0 = the kernel a training step would choose, 1 = the TMA-fed kernel
+ * (stride 1 only; PNN_EINVAL where the shape does not allow it), 2 = the
+ * thread-gathered kernel.  c and k multiples of 8.  All pointers are device
+ * memory of the current device, NHWC with the batch folded into the rows;
+ * w is bf16 [k][ksize][ksize][c].  The caller owns every buffer and a
+ * workspace of pnn_conv_workspace_bytes bytes (256-byte aligned); the call
+ * allocates nothing, enqueues on `stream` (NULL = legacy default) and
+ * synchronises it.  Errors: PNN_EINVAL, PNN_ENOMEM (workspace too small),
+ * PNN_ECUDA, PNN_ETIMEOUT; message in pnn_last_error(NULL). */
+typedef enum { PNN_CONV_FORWARD = 0, PNN_CONV_DGRAD = 1, PNN_CONV_WGRAD = 2 } pnn_conv_mode;
+typedef enum { PNN_DT_F32 = 0, PNN_DT_BF16 = 1 } pnn_dtype;
+typedef struct pnn_conv_args {
+  int32_t batch, h, w, c;        /* input geometry */
+  int32_t k, ksize, stride;      /* output channels, 1 or 3, 1 or 2 */
+  const void* x;                 /* forward / weight gradient input; data gradient: BN input (optional) */
+  int32_t x_dtype;               /* pnn_dtype */
+  const float* bn_scale;         /* optional, c floats: read v(x) instead of x */
+  const float* bn_shift;
+  int32_t relu;
+  const void* wt;                /* bf16 weights [k][ksize][ksize][c] */
+  void* y;                       /* forward output, batch*p*q x k */
+  int32_t y_dtype;
+  const void* res;               /* forward: optional residual added before rounding, batch*p*q x k */
+  int32_t res_dtype;
+  float* y_mean;                 /* forward: optional batch statistics of y, k floats each */
+  float* y_rstd;
+  const float* dy;               /* gradients: float32, batch*p*q x k */
+  float* dx;                     /* data gradient output, batch*h*w x c float32 */
+  int32_t accumulate;            /* data gradient: add into dx instead of overwriting it */
+  const float* bn_mean;          /* data gradient: optional BN-backward sums (see above) */
+  const float* bn_rstd;
+  float* dgamma;
+  float* dbeta;
+  float* dw;                     /* weight gradient output, k x ksize x ksize x c float32 */
+} pnn_conv_args;
+int pnn_conv_workspace_bytes(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* args, size_t* bytes);
+int pnn_conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* args, void* workspace,
+                 size_t workspace_bytes, void* stream);
+
 /* ---- allocation-free weight gradient of one convolution ----
  * The paper has no counterpart to this call.  It exists for callers that
  * cannot allocate device memory at the point they need the result, e.g.

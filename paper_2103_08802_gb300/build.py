@@ -20,7 +20,7 @@ NVCC = os.path.join(CUDA, "bin", "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 CU_SOURCES = ["k_simt.cu", "k_tc_conv.cu"]
-CPP_SOURCES = ["pnn_runtime.cpp"]
+CPP_SOURCES = ["pnn_runtime.cpp", "pnn_conv_api.cpp"]
 
 
 def _sources():

@@ -11,6 +11,9 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+#include <mutex>
+
 #include "pnn_internal.h"
 
 namespace pnn {
@@ -101,11 +104,16 @@ __global__ void __launch_bounds__(256) k_conv_fwd(const ConvDesc* __restrict__ t
     }
     __syncthreads();
   }
-  // epilogue: residual, store, BN partials of the stored value
+  // epilogue: residual, store, BN partials (mean, M2) of the stored value:
+  // two passes over each thread's TM rows, then chan_merge over the 16 row
+  // groups in order
+  int cnt = 0;  // rows of this thread inside the layer
+#pragma unroll
+  for (int i = 0; i < TM; ++i) cnt += m0 + ty + 16 * i < M ? 1 : 0;
 #pragma unroll
   for (int j = 0; j < TN; ++j) {
     const int co = n0 + tx + 16 * j;
-    float s1 = 0.f, s2 = 0.f;
+    float s1 = 0.f;
 #pragma unroll
     for (int i = 0; i < TM; ++i) {
       const int m = m0 + ty + 16 * i;
@@ -115,22 +123,31 @@ __global__ void __launch_bounds__(256) k_conv_fwd(const ConvDesc* __restrict__ t
         if (d.res) v += ldv(d.res, d.res_dt, o);
         v = rnd(d.y_dt, v);
         stv(d.y, d.y_dt, o, v);
+        acc[i][j] = v;
         s1 += v;
-        s2 += v * v;
       }
     }
-    red[ty][tx + 16 * j][0] = s1;
-    red[ty][tx + 16 * j][1] = s2;
+    const float mean = cnt > 0 ? s1 / (float)cnt : 0.f;
+    float m2 = 0.f;
+#pragma unroll
+    for (int i = 0; i < TM; ++i)
+      if (m0 + ty + 16 * i < M) m2 = fmaf(acc[i][j] - mean, acc[i][j] - mean, m2);
+    red[ty][tx + 16 * j][0] = mean;
+    red[ty][tx + 16 * j][1] = m2;
   }
   if (d.stats) {
     __syncthreads();
     for (int nn = tid; nn < BN; nn += 256) {
       const int co = n0 + nn;
       if (co < d.K) {
-        float s1 = 0.f, s2 = 0.f;
-        for (int r = 0; r < 16; ++r) { s1 += red[r][nn][0]; s2 += red[r][nn][1]; }
-        d.stats[((int64_t)tm * d.K + co) * 2 + 0] = s1;
-        d.stats[((int64_t)tm * d.K + co) * 2 + 1] = s2;
+        float n = 0.f, mean = 0.f, m2 = 0.f;
+        for (int r = 0; r < 16; ++r) {
+          int cr = 0;
+          for (int i = 0; i < TM; ++i) cr += m0 + r + 16 * i < M ? 1 : 0;
+          chan_merge(n, mean, m2, (float)cr, red[r][nn][0], red[r][nn][1]);
+        }
+        d.stats[((int64_t)tm * d.K + co) * 2 + 0] = mean;
+        d.stats[((int64_t)tm * d.K + co) * 2 + 1] = m2;
       }
     }
   }
@@ -345,9 +362,11 @@ __global__ void __launch_bounds__(256) k_ew(const EwDesc* __restrict__ tab, cons
   const RowTile rt(C, threadIdx.x);
   const int64_t r0 = (int64_t)tile * d.rows_per_tile;
   const int64_t r1 = min((int64_t)d.M, r0 + d.rows_per_tile);
+  // BN partials of the output: Welford's update over this thread's rows
+  // (count, mean, M2), then chan_merge over the row groups in order
   for (int ci = 0; ci < rt.cpt; ++ci) {
     const int c = rt.c0 + 256 * ci;
-    float s1 = 0.f, s2 = 0.f;
+    float n = 0.f, mean = 0.f, m2 = 0.f;
     if (c < C) {
       for (int64_t r = r0 + rt.g; r < r1; r += rt.G) {
         const int64_t o = r * C + c;
@@ -358,25 +377,33 @@ __global__ void __launch_bounds__(256) k_ew(const EwDesc* __restrict__ tab, cons
           v = rnd(d.out_dt, v);
           stv(d.out, d.out_dt, o, v);
         }
-        s1 += v;
-        s2 += v * v;
+        if (d.stats) {
+          n += 1.f;
+          const float delta = v - mean;
+          mean += delta / n;
+          m2 = fmaf(delta, v - mean, m2);
+        }
       }
     }
     if (d.stats) {
       if (rt.G == 1) {
         if (c < C) {
-          d.stats[((int64_t)tile * C + c) * 2] = s1;
-          d.stats[((int64_t)tile * C + c) * 2 + 1] = s2;
+          d.stats[((int64_t)tile * C + c) * 2] = mean;
+          d.stats[((int64_t)tile * C + c) * 2 + 1] = m2;
         }
       } else {
-        red[threadIdx.x][0] = s1;
-        red[threadIdx.x][1] = s2;
+        red[threadIdx.x][0] = mean;
+        red[threadIdx.x][1] = m2;
         __syncthreads();
         if ((int)threadIdx.x < C) {
-          float a = 0.f, b = 0.f;
-          for (int g = 0; g < rt.G; ++g) { a += red[g * C + threadIdx.x][0]; b += red[g * C + threadIdx.x][1]; }
-          d.stats[((int64_t)tile * C + threadIdx.x) * 2] = a;
-          d.stats[((int64_t)tile * C + threadIdx.x) * 2 + 1] = b;
+          float a = 0.f, am = 0.f, a2 = 0.f;
+          for (int g = 0; g < rt.G; ++g) {
+            // rows r0 + g, r0 + g + G, ... below r1
+            const float cg = r1 > r0 + g ? (float)((r1 - r0 - g + rt.G - 1) / rt.G) : 0.f;
+            chan_merge(a, am, a2, cg, red[g * C + threadIdx.x][0], red[g * C + threadIdx.x][1]);
+          }
+          d.stats[((int64_t)tile * C + threadIdx.x) * 2] = am;
+          d.stats[((int64_t)tile * C + threadIdx.x) * 2 + 1] = a2;
         }
         __syncthreads();
       }
@@ -483,6 +510,79 @@ __device__ __forceinline__ bool chunked_sums(const float* __restrict__ part, int
   return w == 0 && c < C;
 }
 
+// The same two-level reduction for the forward statistics: partial tiles hold
+// (mean, M2) of their rows (count from the row range: rpt rows each, the last
+// tile the remainder of M) and are merged with chan_merge in fp64 -- warp w
+// tiles t0+w, t0+w+8, ... in order, then warp 0 the eight warps in order; the
+// chunks likewise in the last CTA of the channel group.  Returns true on the
+// threads (warp 0, c < C) that hold the totals (count, mean, M2).
+__device__ __forceinline__ bool chunked_moments(const float* __restrict__ part, int C, int tiles, int64_t M, int rpt,
+                                                int cg, int chunk, int nchunk, double* scratch, int32_t* counter,
+                                                double& n_out, double& mean_out, double& m2_out) {
+  __shared__ double red[8][3][32];
+  __shared__ int is_last;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int c = cg * 32 + lane;
+  auto rows_of = [&](int64_t t0, int64_t t1) -> double {  // rows of tiles [t0, t1)
+    const int64_t a = t0 * rpt, b = t1 * rpt < M ? t1 * rpt : M;
+    return b > a ? (double)(b - a) : 0.0;
+  };
+  const int t0 = chunk * kFinTilesPerCta, t1 = min(tiles, t0 + kFinTilesPerCta);
+  double n = 0.0, mean = 0.0, m2 = 0.0;
+  if (c < C) {
+    float2 v[kFinTilesPerCta / 8];
+#pragma unroll
+    for (int k = 0; k < kFinTilesPerCta / 8; ++k) {
+      const int t = t0 + w + 8 * k;
+      v[k] = t < t1 ? *reinterpret_cast<const float2*>(part + ((int64_t)t * C + c) * 2) : make_float2(0.f, 0.f);
+    }
+#pragma unroll
+    for (int k = 0; k < kFinTilesPerCta / 8; ++k) {
+      const int t = t0 + w + 8 * k;
+      if (t < t1) chan_merge(n, mean, m2, rows_of(t, t + 1), (double)v[k].x, (double)v[k].y);
+    }
+  }
+  red[w][0][lane] = n;
+  red[w][1][lane] = mean;
+  red[w][2][lane] = m2;
+  __syncthreads();
+  n = mean = m2 = 0.0;
+  if (w == 0)
+    for (int k = 0; k < 8; ++k) chan_merge(n, mean, m2, red[k][0][lane], red[k][1][lane], red[k][2][lane]);
+  if (nchunk == 1) {
+    n_out = n; mean_out = mean; m2_out = m2;
+    return w == 0 && c < C;
+  }
+  if (w == 0 && c < C) {
+    scratch[((int64_t)chunk * C + c) * 2] = mean;
+    scratch[((int64_t)chunk * C + c) * 2 + 1] = m2;
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) is_last = atomicAdd(counter + cg, 1) == nchunk - 1;
+  __syncthreads();
+  if (!is_last) return false;
+  __threadfence();
+  n = mean = m2 = 0.0;
+  if (c < C)
+    for (int k = w; k < nchunk; k += 8) {
+      const int64_t a = (int64_t)k * kFinTilesPerCta, b = min((int64_t)tiles, a + kFinTilesPerCta);
+      chan_merge(n, mean, m2, rows_of(a, b), __ldcg(scratch + ((int64_t)k * C + c) * 2),
+                 __ldcg(scratch + ((int64_t)k * C + c) * 2 + 1));
+    }
+  __syncthreads();  // red[] of the chunk pass is read before it is rewritten
+  red[w][0][lane] = n;
+  red[w][1][lane] = mean;
+  red[w][2][lane] = m2;
+  __syncthreads();
+  n = mean = m2 = 0.0;
+  if (w == 0)
+    for (int k = 0; k < 8; ++k) chan_merge(n, mean, m2, red[k][0][lane], red[k][1][lane], red[k][2][lane]);
+  if (threadIdx.x == 0) counter[cg] = 0;  // ready for the next launch
+  n_out = n; mean_out = mean; m2_out = m2;
+  return w == 0 && c < C;
+}
+
 __global__ void __launch_bounds__(256) k_bn_fin(const BnFinDesc* __restrict__ tab, const int* __restrict__ tstart,
                                                 int n) {
   const int inst = find_instance(tstart, n, blockIdx.x);
@@ -497,10 +597,11 @@ __global__ void __launch_bounds__(256) k_bn_fin(const BnFinDesc* __restrict__ ta
     mean = d.run_mean[c];
     var = d.run_var[c];
   } else {
-    double s1, s2;
-    if (!chunked_sums(d.part, d.C, d.tiles, cg, chunk, d.nchunk, d.scratch, d.counter, s1, s2)) return;
-    mean = s1 / (double)d.count;
-    var = s2 / (double)d.count - mean * mean;
+    double cnt, m2;
+    if (!chunked_moments(d.part, d.C, d.tiles, d.count, d.rows_per_tile, cg, chunk, d.nchunk, d.scratch, d.counter,
+                         cnt, mean, m2))
+      return;
+    var = cnt > 0.0 ? m2 / cnt : 0.0;
     if (var < 0.0) var = 0.0;
     if (d.run_mean) {
       // running statistics follow the batch mean and the unbiased variance
@@ -978,6 +1079,38 @@ __global__ void k_copy_cast(const float* in, void* out, int32_t dt, int64_t n) {
 // ---------------------------------------------------------------- launchers
 static inline int cdiv64(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 
+namespace {
+constexpr int kMaxDevices = 64;
+std::atomic<int> g_sms[kMaxDevices];
+std::atomic<uint32_t> g_attr_done[kMaxDevices];
+std::mutex g_attr_mu;
+}  // namespace
+
+int device_sm_count() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 1;
+  int v = g_sms[dev].load(std::memory_order_acquire);
+  if (v > 0) return v;
+  int sms = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) return 1;
+  g_sms[dev].store(sms, std::memory_order_release);
+  return sms;
+}
+
+cudaError_t set_smem_attr_once(int slot, const void* kernel, int bytes) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices || slot < 0 || slot >= 32) return cudaErrorInvalidValue;
+  const uint32_t bit = 1u << slot;
+  if (g_attr_done[dev].load(std::memory_order_acquire) & bit) return cudaSuccess;
+  std::lock_guard<std::mutex> lk(g_attr_mu);
+  if (g_attr_done[dev].load(std::memory_order_acquire) & bit) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) g_attr_done[dev].fetch_or(bit, std::memory_order_release);
+  return e;
+}
+
 cudaError_t launch_conv_fwd_simt(const ConvDesc* tab, const int* tstart, int n, int total, int variant,
                                  cudaStream_t st) {
   if (total <= 0) return cudaSuccess;
@@ -1094,7 +1227,7 @@ cudaError_t launch_relu_mask(float* g, const float* pre, int64_t n, cudaStream_t
 cudaError_t launch_sgd(float* w, const float* g, float* v, void* shadow, int32_t shadow_dt, int64_t n, float lr,
                        float mu, float wd, int nesterov, int first, cudaStream_t st) {
   int blocks = cdiv64(n, 256);
-  if (blocks > 152 * 16) blocks = 152 * 16;
+  if (blocks > device_sm_count() * 16) blocks = device_sm_count() * 16;
   if (blocks < 1) blocks = 1;
   k_sgd<<<blocks, 256, 0, st>>>(w, g, v, shadow, shadow_dt, n, lr, mu, wd, nesterov, first);
   return cudaGetLastError();
@@ -1106,7 +1239,7 @@ cudaError_t launch_export(Src x, int B, int H, int W, int C, float* out, cudaStr
 }
 cudaError_t launch_copy_cast(const float* in, void* out, int32_t dt, int64_t n, cudaStream_t st) {
   int blocks = cdiv64(n, 256);
-  if (blocks > 152 * 16) blocks = 152 * 16;
+  if (blocks > device_sm_count() * 16) blocks = device_sm_count() * 16;
   if (blocks < 1) blocks = 1;
   k_copy_cast<<<blocks, 256, 0, st>>>(in, out, dt, n);
   return cudaGetLastError();

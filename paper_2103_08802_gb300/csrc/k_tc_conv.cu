@@ -29,6 +29,7 @@
 #include <stdint.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "pnn.h"
 #include "pnn_internal.h"
@@ -531,9 +532,8 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
           }
         }
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          if (nb + i < d.K) { s1[i] = v[i]; s2[i] = v[i] * v[i]; }
-        }
+        for (int i = 0; i < 16; ++i)
+          if (nb + i < d.K) s1[i] = v[i];
       }
       if (tstore) {
         // the store issued from this buffer two chunks ago must have read it
@@ -562,9 +562,20 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
       }
       RT(const unsigned long long c2 = clock64(); e1 += c2 - c1;)
       if (stats) {
-        const float a = warp_colsum16(s1, lane), b = warp_colsum16(s2, lane);
+        // (mean, M2) of the chunk's columns over this warp's valid rows: the
+        // column sums, the warp mean broadcast back, the squared deviations
+        const float nw = (float)__popc(__ballot_sync(0xffffffffu, mvalid));
+        const float a = warp_colsum16(s1, lane);
+        const float mw = nw > 0.f ? a / nw : 0.f;  // lane l: mean of column l >> 1
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float mi = __shfl_sync(0xffffffffu, mw, 2 * i);
+          const float dv = v[i] - mi;
+          s2[i] = mvalid && nb + i < d.K ? dv * dv : 0.f;
+        }
+        const float b = warp_colsum16(s2, lane);
         if ((lane & 1) == 0) {
-          red[q][j0 + (lane >> 1)][0] = a;
+          red[q][j0 + (lane >> 1)][0] = mw;
           red[q][j0 + (lane >> 1)][1] = b;
         }
       }
@@ -661,8 +672,22 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
     asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "r"(ethreads) : "memory");
     for (int j = etid; j < T.BN; j += ethreads) {
       if (T.n0 + j < T.Ncols) {
-        const float a = red[0][j][0] + red[1][j][0] + red[2][j][0] + red[3][j][0];
-        const float b = red[0][j][1] + red[1][j][1] + red[2][j][1] + red[3][j][1];
+        float a, b;
+        if (MODE == FWD) {
+          // the four warps' (mean, M2) merged in order; warp quarter qq holds
+          // the tile's rows 32 qq .. 32 qq + 31 that lie inside the layer
+          float n = 0.f;
+          a = 0.f;
+          b = 0.f;
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq) {
+            const int nq = min(32, max(0, T.Mrows - (T.m0 + 32 * qq)));
+            chan_merge(n, a, b, (float)nq, red[qq][j][0], red[qq][j][1]);
+          }
+        } else {
+          a = red[0][j][0] + red[1][j][0] + red[2][j][0] + red[3][j][0];
+          b = red[0][j][1] + red[1][j][1] + red[2][j][1] + red[3][j][1];
+        }
         const int scols = T.Ncols;
         spart[((int64_t)T.tm * scols + T.n0 + j) * 2] = a;
         spart[((int64_t)T.tm * scols + T.n0 + j) * 2 + 1] = b;
@@ -1508,17 +1533,9 @@ static cudaError_t launch_mode(ConvKernel kern, const ConvDesc* tab, const int* 
                                int32_t* status, cudaStream_t st, int max_ctas) {
   if (total <= 0) return cudaSuccess;
   if (bnmax < 16 || bnmax > 256 || (bnmax & 15)) return cudaErrorInvalidValue;
-  static bool attr = false;
-  static int sms = 0;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes(256));
-    if (e != cudaSuccess) return e;
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (sms <= 0) sms = 148;
-    attr = true;
-  }
+  cudaError_t e = set_smem_attr_once(MODE, reinterpret_cast<const void*>(kern), (int)smem_bytes(256));
+  if (e != cudaSuccess) return e;
+  const int sms = device_sm_count();
   int grid = total < sms ? total : sms;
   if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
   kern<<<grid, kThreads, smem_bytes(bnmax), st>>>(tab, tstart, n, total, bnmax, status);
@@ -1536,18 +1553,10 @@ cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, in
   if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || raw_bytes <= 0 || (raw_bytes & 1023) || mode < 0 || mode > 2)
     return cudaErrorInvalidValue;
   const int xw = mode == 2 ? 8 : 4;  // transform warps of the mode's kernel
-  static bool attr[3] = {false, false, false};
-  static int sms = 0;
   auto kern = mode == 0 ? k_conv_fwd_tma : (mode == 1 ? k_conv_dgrad_tma : k_conv_wgrad_tma);
-  if (!attr[mode]) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kTmaSmemBudget);
-    if (e != cudaSuccess) return e;
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (sms <= 0) sms = 148;
-    attr[mode] = true;
-  }
+  cudaError_t e = set_smem_attr_once(4 + mode, reinterpret_cast<const void*>(kern), kTmaSmemBudget);
+  if (e != cudaSuccess) return e;
+  const int sms = device_sm_count();
   const size_t smem = tma_smem_bytes(mode, bnmax, raw_bytes, tma_extra(mode, xw));
   if (smem > (size_t)kTmaSmemBudget) return cudaErrorInvalidValue;
   int grid = total < sms ? total : sms;
@@ -1664,27 +1673,31 @@ struct NoAllocSymbols {
   WReduceDesc* red = nullptr;
   int* ts = nullptr;
   int32_t* status = nullptr;
-  bool ready = false;
+  cudaError_t err = cudaSuccess;
 };
-NoAllocSymbols g_noalloc_syms[64];
+constexpr int kNoAllocDevices = 64;
+NoAllocSymbols g_noalloc_syms[kNoAllocDevices];
+std::once_flag g_noalloc_once[kNoAllocDevices];
 
-// Device addresses of the arrays for the current device (once per device).
-// The host-side names are stand-ins, not device addresses.
+// Device addresses of the arrays for the current device, looked up once per
+// device (std::call_once: concurrent first calls from several host threads
+// wait for one lookup).  The host-side names are stand-ins, not device
+// addresses.
 cudaError_t noalloc_symbols(NoAllocSymbols** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (dev < 0 || dev >= kNoAllocDevices) return cudaErrorInvalidDevice;
   NoAllocSymbols& s = g_noalloc_syms[dev];
-  if (!s.ready) {
-    e = cudaGetSymbolAddress((void**)&s.part, g_noalloc_part);
-    if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&s.conv, g_noalloc_conv);
-    if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&s.red, g_noalloc_red);
-    if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&s.ts, g_noalloc_ts);
-    if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&s.status, g_noalloc_status);
-    if (e != cudaSuccess) return e;
-    s.ready = true;
-  }
+  std::call_once(g_noalloc_once[dev], [&s]() {
+    cudaError_t r = cudaGetSymbolAddress((void**)&s.part, g_noalloc_part);
+    if (r == cudaSuccess) r = cudaGetSymbolAddress((void**)&s.conv, g_noalloc_conv);
+    if (r == cudaSuccess) r = cudaGetSymbolAddress((void**)&s.red, g_noalloc_red);
+    if (r == cudaSuccess) r = cudaGetSymbolAddress((void**)&s.ts, g_noalloc_ts);
+    if (r == cudaSuccess) r = cudaGetSymbolAddress((void**)&s.status, g_noalloc_status);
+    s.err = r;
+  });
+  if (s.err != cudaSuccess) return s.err;
   *out = &s;
   return cudaSuccess;
 }
@@ -1725,7 +1738,7 @@ extern "C" int pnn_conv_wgrad_noalloc(const float* x, const float* dy, float* dw
   cd.mtile_rows = kBM;
   cd.op_bf16 = 1;
   const int base = cd.mtiles * cd.ntiles;
-  int splits = (int)std::min<int64_t>((mp + 255) / 256, (2 * 152 + base - 1) / base);
+  int splits = (int)std::min<int64_t>((mp + 255) / 256, (2 * device_sm_count() + base - 1) / base);
   splits = std::max(1, std::min<int>(splits, (int)(kNoAllocFloats / nw)));
   cd.pix_per_split = (int)(((mp + splits - 1) / splits + 63) / 64 * 64);
   cd.splits = (int)((mp + cd.pix_per_split - 1) / cd.pix_per_split);

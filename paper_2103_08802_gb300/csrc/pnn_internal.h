@@ -33,7 +33,7 @@ struct ConvDesc {
   // forward epilogue
   void* y; int32_t y_dt;
   const void* res; int32_t res_dt;   // residual added to the output (or null)
-  float* stats;                       // per-tile BN partials [mtiles][K][2] or null
+  float* stats;                       // per-tile BN partials [mtiles][K][2] = (mean, M2) or null
   // dgrad: dx[B*H*W][C] (fp32) = (accumulate ? dx : 0) + W^T * dy
   float* dx; int32_t accumulate;
   // dgrad / wgrad operand dy[B*P*Q][K] (fp32)
@@ -71,7 +71,7 @@ struct EwDesc {
   int32_t nin;
   void* out; int32_t out_dt;
   int32_t relu;
-  float* stats;          // [tiles][C][2] or null
+  float* stats;          // [tiles][C][2] = (mean, M2) or null
   int64_t M;
   int32_t C;
   int32_t rows_per_tile;
@@ -92,9 +92,10 @@ struct EwBwdDesc {
 // BN statistics finalisation: partials[tiles][C][2] -> mean, rstd, scale, shift
 constexpr int kFinTilesPerCta = 64;  // BN finalize: partial tiles one CTA adds up (8 per warp)
 struct BnFinDesc {
-  const float* part;
+  const float* part;     // [tiles][C][2] = (mean, M2) of each tile's rows
   int32_t tiles, C;
   int64_t count;         // number of rows M
+  int32_t rows_per_tile; // rows of every partial tile but the last
   const float* gamma; const float* beta;
   float* mean; float* rstd; float* scale; float* shift;
   float* run_mean; float* run_var;  // running statistics of this BN layer
@@ -207,6 +208,12 @@ cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, in
 bool conv_tma_fits(int mode, int bnmax, int raw_bytes);
 // record a message for pnn_last_error(NULL) and return `code`
 int set_last_error(int code, const char* msg);
+// streaming multiprocessors of the current device, queried once per device
+// (thread-safe); 1 if the query fails, which keeps every grid valid
+int device_sm_count();
+// cudaFuncSetAttribute(MaxDynamicSharedMemorySize) once per (device, kernel
+// slot < 32); thread-safe
+cudaError_t set_smem_attr_once(int slot, const void* kernel, int bytes);
 
 // debug builds: first misaligned vector access of the tensor-core kernels (0 = none)
 unsigned long long conv_tc_debug_word();
@@ -235,6 +242,28 @@ constexpr int kEwRowsPerTile = 64;
 #else
 #define PNN_HD
 #endif
+// BN forward statistics are kept as (count, mean, M2 = sum of squared
+// deviations from the mean) and combined with the pairwise update of Chan,
+// Golub & LeVeque ("Updating formulae and a pairwise algorithm for computing
+// sample variances", 1979): for disjoint sets a and b with n = n_a + n_b and
+// delta = mean_b - mean_a,
+//   mean = mean_a + delta * n_b / n,   M2 = M2_a + M2_b + delta^2 * n_a * n_b / n,
+// which never subtracts two large sums (the one-pass sum(h^2) - n * mean^2
+// loses the variance when |mean| >> std).  Per-tile partials are
+// [tiles][C][2] = (mean, M2) of the tile's rows; a tile's count follows from
+// its row range.
+template <typename T>
+PNN_HD inline void chan_merge(T& n, T& mean, T& m2, T nb, T meanb, T m2b) {
+  if (nb <= T(0)) return;
+  if (n <= T(0)) { n = nb; mean = meanb; m2 = m2b; return; }
+  const T nn = n + nb;
+  const T delta = meanb - mean;
+  const T f = nb / nn;
+  mean = mean + delta * f;
+  m2 = m2 + m2b + delta * delta * n * f;
+  n = nn;
+}
+
 // TMA-fed weight gradient: the two boxes of a k-step (64 pixels) -- the
 // activation rows of every tap (halo of pad*W + pad rows each side) x cwx
 // channels, and the output-gradient rows x K -- and their raw-slot offsets
@@ -254,9 +283,46 @@ PNN_HD inline WgBoxes wg_boxes(int C, int K, int W, int pad, bool xbf) {
 }
 PNN_HD inline int wg_raw_bytes(const WgBoxes& b) { return (b.yoff + b.ybytes + 1023) & ~1023; }
 
+// ---------------------------------------------------------------- conv kernel choice
+// (mode 0 forward, 1 data gradient, 2 weight gradient; variant 1 = TMA-fed,
+// 0 = thread-gathered tensor-core kernel)
+// The TMA-fed forward / data gradient load each filter tap as one
+// [128 rows x min(channels, 64)] box: stride 1, same padding, and a channel
+// count (of the A source) that divides 64 or is a multiple of it.
+inline bool tma_shape_ok(int k, int stride, int pad, int ch) {
+  const bool geom = stride == 1 && ((k == 1 && pad == 0) || (k == 3 && pad == 1));
+  return geom && ch % 8 == 0 && (ch <= 64 ? 64 % ch == 0 : ch % 64 == 0);
+}
+// N columns of a tile when the layer needs several: 128 for the TMA-fed
+// forward and data gradient (a smaller operand slot leaves room for more
+// pipeline stages), 256 otherwise.
+inline int tc_ntile_cols(int mode, int variant) { return variant == 1 && mode != 2 ? 128 : 256; }
+// M rows of a tile: 256 for the TMA-fed weight gradient of a layer with at
+// most 128 input channels (two MMA halves share each B operand, so a layer
+// with up to 256 (r,s,c) rows makes one pass over the pixels; a tile then
+// holds whole taps, all inside the activation box), 128 otherwise.
+inline int tc_tile_rows(int mode, int variant, int C) { return mode == 2 && variant == 1 && C <= 128 ? 256 : kTcBM; }
+// 2-D tensor map (CUtensorMap, 128 bytes at `map`) over rows x inner elements
+// (bf16 or fp32, row pitch inner * element size) with box
+// [box_rows][box_inner]; swz: swizzle span in bytes (128, 64, 32 or 0).
+// Returns 0, or non-zero with a message in *why.
+int encode_tensor_map_2d(void* map, const void* base, bool bf16, int64_t inner, int64_t rows, int box_inner,
+                         int box_rows, int swz, const char** why);
+
 constexpr int kBnbRowsPerTile = 256;  // BN backward reduce/apply tiles: at least this many rows
 // rows of a BN-backward tile for C channels: about 32K elements a CTA
 inline int bnb_rows_per_tile(int C) { return C > 0 && 32768 / C > kBnbRowsPerTile ? 32768 / C : kBnbRowsPerTile; }
+// The TMA-fed weight gradient loads a k-step's activation rows for all taps
+// as one halo box and the output-gradient rows as another: channels 8..64
+// (dividing 64) or multiples of 128 up to 512, at most 128 output channels
+// (one N tile), a halo of at most 256 rows, and two stages in shared memory.
+inline bool tma_wgrad_ok(int k, int stride, int pad, int C, int K, int W, bool xbf) {
+  if (!(stride == 1 && ((k == 1 && pad == 0) || (k == 3 && pad == 1)))) return false;
+  if (!(C % 8 == 0 && ((C <= 64 && 64 % C == 0) || (C % 128 == 0 && C <= 512)))) return false;
+  if (K % 8 != 0 || K > 128) return false;
+  const WgBoxes b = wg_boxes(C, K, W, pad, xbf);
+  return b.hrows <= 256 && conv_tma_fits(2, 128, wg_raw_bytes(b));
+}
 struct ConvTile { int BM, BN; };
 inline ConvTile simt_tile(int variant) {
   return variant == 0 ? ConvTile{64, 64} : (variant == 1 ? ConvTile{128, 32} : ConvTile{256, 16});

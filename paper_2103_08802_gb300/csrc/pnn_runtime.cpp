@@ -64,6 +64,7 @@ struct Value {
 
 struct Norm {
   int fused_tiles = 0;                       // BN-backward partials written by a data-gradient epilogue: its m-tiles
+  int stat_rows = kEwRowsPerTile;            // rows of a forward-statistics partial tile
   int C = 0, h = -1, gamma = -1, beta = -1;  // gamma/beta: param ids
   int virt = -1;                             // the virtual BN(+ReLU) value
   int tiles = 0;
@@ -112,41 +113,11 @@ struct Launch {
   int block = -1;       // fine forward / backward: position of the layer in its segment
 };
 
-// The TMA-fed tensor-core conv (variant 1 of the TC forward / data-gradient
-// kinds) loads each filter tap as one [128 rows x min(channels, 64)] box:
-// stride 1, same padding, and a channel count that divides 64 or is a
-// multiple of it.
-static bool tma_shape_ok(int k, int stride, int pad, int ch) {
-  const bool geom = stride == 1 && ((k == 1 && pad == 0) || (k == 3 && pad == 1));
-  return geom && ch % 8 == 0 && (ch <= 64 ? 64 % ch == 0 : ch % 64 == 0);
-}
-
-// N columns of a tensor-core conv tile when the layer needs several: 128 for
-// the TMA-fed forward and data gradient (a smaller operand slot leaves room for
-// more pipeline stages), 256 otherwise.
-static int tc_ntile_w(int kind, int variant) {
-  return variant == 1 && (kind == K_CONV_FWD_TC || kind == K_DGRAD_TC) ? 128 : 256;
-}
-
-// M rows of a tensor-core conv tile: 256 for the TMA-fed weight gradient of a
-// layer with at most 128 input channels (two MMA halves share each B operand, so
-// a layer with up to 256 (r,s,c) rows makes one pass over the pixels; a tile
-// then holds whole taps, all inside the activation box), 128 otherwise.
-static int tc_mtile_rows(int kind, int variant, int C) {
-  return kind == K_WGRAD_TC && variant == 1 && C <= 128 ? 256 : kTcBM;
-}
-
-// The TMA-fed weight gradient loads a k-step's activation rows for all taps
-// as one halo box and the output-gradient rows as another: channels 8..64
-// (dividing 64) or multiples of 128 up to 512, at most 128 output channels
-// (one N tile), a halo of at most 256 rows, and two stages in shared memory.
-static bool tma_wgrad_ok(int k, int stride, int pad, int C, int K, int W, bool xbf) {
-  if (!(stride == 1 && ((k == 1 && pad == 0) || (k == 3 && pad == 1)))) return false;
-  if (!(C % 8 == 0 && ((C <= 64 && 64 % C == 0) || (C % 128 == 0 && C <= 512)))) return false;
-  if (K % 8 != 0 || K > 128) return false;
-  const WgBoxes b = wg_boxes(C, K, W, pad, xbf);
-  return b.hrows <= 256 && conv_tma_fits(2, 128, wg_raw_bytes(b));
-}
+// Tile and kernel-choice rules shared with the single-convolution entry
+// points (pnn_internal.h), in terms of this file's kinds.
+static int conv_mode(int kind) { return kind == K_DGRAD_TC ? 1 : (kind == K_WGRAD_TC ? 2 : 0); }
+static int tc_ntile_w(int kind, int variant) { return tc_ntile_cols(conv_mode(kind), variant); }
+static int tc_mtile_rows(int kind, int variant, int C) { return tc_tile_rows(conv_mode(kind), variant, C); }
 
 const char* kKindName[K_NKINDS] = {"conv_fwd", "conv_dgrad", "conv_wgrad", "wgrad_reduce", "elementwise",
                                    "elementwise_bwd", "bn_finalize", "bn_bwd_reduce", "bn_bwd_finalize",
@@ -293,6 +264,9 @@ struct pnn_net {
       if ((p.kind == K_CONV_FWD || p.kind == K_CONV_FWD_TC || (p.kind == K_EW && p.out == h)) && p.stats_norm < 0) {
         p.stats_norm = nid;
         norms[nid].tiles = p.tiles;
+        norms[nid].stat_rows = p.kind == K_CONV_FWD_TC ? kTcBM
+                               : p.kind == K_CONV_FWD  ? simt_tile(p.variant).BM
+                                                       : kEwRowsPerTile;
         return;
       }
     }
@@ -303,6 +277,7 @@ struct pnn_net {
     s.tiles = cdiv(rows(h), kEwRowsPerTile);
     s.key[0] = key0; s.key[1] = 90;
     norms[nid].tiles = s.tiles;
+    norms[nid].stat_rows = kEwRowsPerTile;
     new_op(list, s);
   }
   // virtual BN(+ReLU) of h with fresh or given gamma/beta params
@@ -543,7 +518,7 @@ struct pnn_net {
           wg.ntiles = cdiv(RSC, kWgradBN);
         }
         int base = wg.mtiles * wg.ntiles;
-        int splits = std::max(1, std::min(cdiv(Mp, 256), cdiv(2 * 152, base)));
+        int splits = std::max(1, std::min(cdiv(Mp, 256), cdiv(2 * (int64_t)device_sm_count(), base)));
         wg.pix_per_split = cdiv(cdiv(Mp, splits), pix_align) * pix_align;
         wg.splits = cdiv(Mp, wg.pix_per_split);
         wg.tiles = base * wg.splits;
@@ -680,28 +655,9 @@ struct pnn_net {
   // rows).  Loads read zeros outside the tensor; stores skip it.
   int encode_map(CUtensorMap* m, const void* base, bool bf16, int64_t inner, int64_t rows, int box_inner,
                  int box_rows, int swz) {
-    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
-    if (!encode) {
-      void* fn = nullptr;
-      cudaDriverEntryPointQueryResult q;
-      cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
-      if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
-        return fail(PNN_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
-      encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    }
-    const int esz = bf16 ? 2 : 4;
-    const cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)rows};
-    const cuuint64_t pitch[1] = {(cuuint64_t)inner * esz};
-    const cuuint32_t box[2] = {(cuuint32_t)box_inner, (cuuint32_t)box_rows};
-    const cuuint32_t estr[2] = {1, 1};
-    const CUresult r = encode(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
-                              const_cast<void*>(base), dims, pitch, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                              swz == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
-                              : swz == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
-                              : swz == 32 ? CU_TENSOR_MAP_SWIZZLE_32B
-                                          : CU_TENSOR_MAP_SWIZZLE_NONE,
-                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) return fail(PNN_ECUDA, "cuTensorMapEncodeTiled rejected a conv operand map");
+    const char* why = nullptr;
+    if (encode_tensor_map_2d(m, base, bf16, inner, rows, box_inner, box_rows, swz, &why) != 0)
+      return fail(PNN_ECUDA, why);
     return PNN_OK;
   }
   size_t put_table(const void* p, size_t n) {
@@ -979,7 +935,10 @@ int pnn_net::plan(const pnn_desc* d) {
     c.mtiles = cdiv(rows(c.out), t.BM);
     c.ntiles = cdiv(cout, t.BN);
     c.tiles = c.mtiles;
-    if (c.stats_norm >= 0) norms[c.stats_norm].tiles = c.tiles;
+    if (c.stats_norm >= 0) {
+      norms[c.stats_norm].tiles = c.tiles;
+      norms[c.stats_norm].stat_rows = t.BM;
+    }
   }
   // BN running statistics: one slot of 2C floats per BN layer, in the order of
   // its gamma in the parameter vector (the delta form's two evaluations of F^j
@@ -1347,6 +1306,7 @@ int pnn_net::build_tables() {
             const Norm& n = norms[o.norm];
             BnFinDesc f{};
             f.part = P<float>(n.part); f.tiles = n.tiles; f.C = n.C; f.count = n.count;
+            f.rows_per_tile = n.stat_rows;
             f.gamma = master + params[n.gamma].off; f.beta = master + params[n.beta].off;
             f.mean = P<float>(n.mean); f.rstd = P<float>(n.rstd); f.scale = P<float>(n.scale); f.shift = P<float>(n.shift);
             f.run_mean = P<float>(n.run); f.run_var = P<float>(n.run) + n.C;

@@ -54,6 +54,19 @@ class Options(C.Structure):
                 ("overlap", C.c_int32)]
 
 
+class ConvArgs(C.Structure):
+    _fields_ = [("batch", C.c_int32), ("h", C.c_int32), ("w", C.c_int32), ("c", C.c_int32),
+                ("k", C.c_int32), ("ksize", C.c_int32), ("stride", C.c_int32),
+                ("x", C.c_void_p), ("x_dtype", C.c_int32),
+                ("bn_scale", C.c_void_p), ("bn_shift", C.c_void_p), ("relu", C.c_int32),
+                ("wt", C.c_void_p), ("y", C.c_void_p), ("y_dtype", C.c_int32),
+                ("res", C.c_void_p), ("res_dtype", C.c_int32),
+                ("y_mean", C.c_void_p), ("y_rstd", C.c_void_p),
+                ("dy", C.c_void_p), ("dx", C.c_void_p), ("accumulate", C.c_int32),
+                ("bn_mean", C.c_void_p), ("bn_rstd", C.c_void_p), ("dgamma", C.c_void_p), ("dbeta", C.c_void_p),
+                ("dw", C.c_void_p)]
+
+
 class Trace(C.Structure):
     _fields_ = [("kind", C.c_int32), ("variant", C.c_int32), ("phase", C.c_int32), ("instances", C.c_int32),
                 ("tiles", C.c_int32),
@@ -113,6 +126,8 @@ def load():
         "pnn_kernel_kind_name": (C.c_char_p, [I32]),
         "pnn_conv_wgrad_noalloc": (C.c_int, [P, P, P, I32, I32, I32, I32, I32, I32, I32, P]),
         "pnn_selftest_wait_timeout": (C.c_int, [C.c_int64, P]),
+        "pnn_conv_workspace_bytes": (C.c_int, [I32, I32, I32, C.POINTER(ConvArgs), C.POINTER(SZ)]),
+        "pnn_conv_run": (C.c_int, [I32, I32, I32, C.POINTER(ConvArgs), P, SZ, P]),
         "pnn_last_error": (C.c_char_p, [P]),
         "pnn_status_string": (C.c_char_p, [C.c_int]),
     }
@@ -402,3 +417,45 @@ class ParaNet:
         c = (C.c_int32 * 3)()
         self._check(self.lib.pnn_launch_counts(self.h, c))
         return list(c)
+
+
+CONV_MODE = {"forward": 0, "dgrad": 1, "wgrad": 2}
+CONV_IMPL = {"auto": 0, "tma": 1, "gathered": 2}
+DTYPE = {"f32": 0, "bf16": 1}
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def _dt(t):
+    import torch
+    return DTYPE["bf16"] if t is not None and t.dtype == torch.bfloat16 else DTYPE["f32"]
+
+
+def conv_run(mode, instances, impl="auto", stream=None):
+    """One grouped convolution (pnn_conv_run) over `instances`, a list of dicts
+    with the geometry (batch, h, w, c, k, ksize, stride) and torch CUDA tensors
+    by the names of pnn_conv_args (x, bn_scale, bn_shift, relu, wt, y, res,
+    y_mean, y_rstd, dy, dx, accumulate, bn_mean, bn_rstd, dgamma, dbeta, dw).
+    The workspace comes from torch.  Raises PnnError on failure."""
+    import torch
+    lib = load()
+    n = len(instances)
+    arr = (ConvArgs * n)()
+    for i, g in enumerate(instances):
+        a = arr[i]
+        for key in ("batch", "h", "w", "c", "k", "ksize", "stride"):
+            setattr(a, key, int(g[key]))
+        a.relu = int(g.get("relu", 0))
+        a.accumulate = int(g.get("accumulate", 0))
+        for key in ("x", "bn_scale", "bn_shift", "wt", "y", "res", "y_mean", "y_rstd", "dy", "dx", "bn_mean",
+                    "bn_rstd", "dgamma", "dbeta", "dw"):
+            setattr(a, key, _ptr(g.get(key)))
+        a.x_dtype, a.y_dtype, a.res_dtype = _dt(g.get("x")), _dt(g.get("y")), _dt(g.get("res"))
+    m, im = CONV_MODE[mode], CONV_IMPL[impl]
+    nb = C.c_size_t()
+    _global_check(lib, lib.pnn_conv_workspace_bytes(m, im, n, arr, C.byref(nb)))
+    ws = torch.empty(max(256, nb.value), dtype=torch.uint8, device="cuda")
+    st = stream.cuda_stream if stream is not None else None
+    _global_check(lib, lib.pnn_conv_run(m, im, n, arr, ws.data_ptr(), ws.numel(), st))

@@ -146,3 +146,30 @@ def test_overlap_option_plans_the_last_subnetwork_apart(pnn):
     d1["segments"] = [4]
     d1["coarse"] = []
     assert counts(d1, overlap=32) == counts(d1)
+
+
+def test_single_conv_call_checks_its_arguments(pnn):
+    """pnn_conv_workspace_bytes / pnn_conv_run validate geometry and the kernel
+    choice on the host (no device memory is touched): the TMA-fed kernels take
+    stride 1 only, channel counts must be multiples of 8."""
+    lib = pnn.load()
+    fake = 256  # never dereferenced: the checks run before any device work
+
+    def args(**kw):
+        a = pnn.ConvArgs()
+        g = dict(batch=2, h=8, w=8, c=16, k=32, ksize=3, stride=1)
+        g.update(kw)
+        for key, v in g.items():
+            setattr(a, key, v)
+        a.x = a.wt = a.y = a.dy = a.dx = a.dw = fake
+        return (pnn.ConvArgs * 1)(a)
+
+    nb = C.c_size_t()
+    for mode in range(3):
+        assert lib.pnn_conv_workspace_bytes(mode, 0, 1, args(), C.byref(nb)) == 0 and nb.value > 0
+        assert lib.pnn_conv_workspace_bytes(mode, 1, 1, args(stride=2), C.byref(nb)) == 1   # TMA: stride 1 only
+        assert lib.pnn_conv_workspace_bytes(mode, 2, 1, args(stride=2), C.byref(nb)) == 0
+        assert lib.pnn_conv_workspace_bytes(mode, 0, 1, args(c=12), C.byref(nb)) == 1       # c % 8
+        assert lib.pnn_conv_workspace_bytes(mode, 0, 1, args(ksize=5), C.byref(nb)) == 1
+    # too small a workspace is refused before any launch
+    assert lib.pnn_conv_run(0, 0, 1, args(), C.c_void_p(256), 256, None) == 2

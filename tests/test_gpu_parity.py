@@ -5,21 +5,23 @@ through the C ABI.
 Tolerances.  The target bounds are 2e-2 (bf16 forward, max-relative),
 5e-2 (bf16 gradients, norm-relative) and 1e-4 (fp32 check mode).  They are
 applied as they stand wherever they are attainable: every forward tensor in
-bf16 and every quantity in fp32 check mode at small sizes.  Two effects make
-the gradient bounds unattainable for any implementation on the larger
-cases, and there the bound is measured instead of assumed:
+bf16 and every quantity in fp32 check mode at small sizes.  Beyond that, a
+floating-point decision (a ReLU mask, a maxpool argmax, the bf16 rounding of
+a stored value) flips when two correct computations differ by the last bits
+of an fp32 sum, and depth amplifies each flip.  How far the oracle's own
+result moves under differences of that size is measured and bounds the GPU:
 
-* decisions taken in floating point (ReLU masks, maxpool argmax) flip at
-  near-zero margins when two computations round differently; a flipped
-  fraction f of a layer's masks moves a gradient by ~sqrt(f), so the
-  oracle's own exact gradient changes by 10-30 % between its float64 and its
-  bf16 forward model.  A bf16 gradient passes when its error against the
-  bf16-model oracle is within 5e-2 or within 1.5x that measured noise;
-* in fp32 beyond the tiny config the same flips occur at the fp32
-  accumulation-order level (and amplify with depth); the bound is 3x the
-  oracle's own response to a 1e-5 relative perturbation of its parameters,
-  and never below the target bound.  The same measured bound covers
-  forward tensors where depth amplifies rounding past 2e-2 / 1e-4.
+* bf16: the oracle's bf16 model (forward values rounded where the library
+  stores them in bf16; every decision taken on those values) with each
+  convolution output perturbed by a relative 4e-6 (about sqrt(4608) * 2^-24,
+  the typical relative difference of two fp32 summation orders of the
+  longest contraction here, 3x3x512) before rounding; every quantity is held
+  to max(target bound, 3x the largest move over two draws).  Every bf16
+  forward tensor is also reported against the float64 oracle (bf16 weights and
+  inputs, no internal rounding) and held there to the 2e-2 bound.
+* fp32 check mode beyond the tiny config: 3x the oracle's response to a 1e-5
+  relative perturbation of its parameters (max of two draws), never below the
+  target bound.
 """
 import numpy as np
 import pytest
@@ -57,7 +59,9 @@ def _grad_keys(report):
 
 def _measured(desc, noise_fn, factor, floor):
     """Every key is bounded by max(target bound, factor * measured noise):
-    the forward bound for forward tensors, `floor` for D_j and gradients."""
+    the forward bound for forward tensors, `floor` for D_j and gradients.
+    bf16 runs also hold every forward tensor to the forward bound against
+    the float64 oracle."""
     onet, theta, x, labels = inputs(desc)
     g = run_gpu(desc, theta, x, labels)
     o = run_oracle(desc, theta, x, labels)
@@ -71,7 +75,9 @@ def _measured(desc, noise_fn, factor, floor):
         if k in ("grad_worst",):
             continue
         lo = floor if k in _grad_keys(err) else tol["fwd"]
-        if not e <= max(lo, factor * noise[k]):
+        b = max(lo, factor * noise[k])
+        print(f"  {k:10s} err {e:.2e}  bound {b:.2e}")
+        if not e <= b:
             bad.append((k, e, noise[k]))
     # per-tensor parameter gradients
     off = 0
@@ -82,6 +88,15 @@ def _measured(desc, noise_fn, factor, floor):
         if not e <= max(floor, factor * gn.get(i, 0.0)):
             bad.append((f"grad[{i}] {shape}", e, gn.get(i)))
         off += n
+    if desc["precision"] == "bf16":
+        o64 = run_oracle(desc, theta, x, labels, precision="fp64")
+        e64, _ = compare(desc, g, o64, LOOSE)
+        for k, e in e64.items():
+            if k.startswith("D") or k.startswith("grad"):
+                continue
+            print(f"  {k:10s} vs fp64 oracle {e:.2e}  bound {tol['fwd']:.0e}")
+            if not e <= tol["fwd"]:
+                bad.append((k + " vs fp64", e, tol["fwd"]))
     assert not bad, bad[:40]
 
 
@@ -94,13 +109,23 @@ def _per_tensor(onet, a, b):
     return out
 
 
-def bf16_decision_noise(desc, theta, x, labels, o):
-    """How far the oracle's exact gradient moves between its bf16 forward
-    model and float64."""
-    o64 = run_oracle(desc, theta, x, labels, precision="fp64")
-    r, _ = compare(desc, o, o64, LOOSE)
-    r["_per_tensor"] = _per_tensor(o["onet"], o["grad"], o64["grad"])
-    return r
+def bf16_accum_noise(desc, theta, x, labels, o, draws=2, rel=4e-6):
+    """How far the oracle's bf16 model moves when every convolution output
+    differs by a relative `rel` (fp32 summation-order size) before it is
+    rounded: the elementwise maximum over `draws` perturbations."""
+    from oracle import pnn_oracle as O
+    out = None
+    for k in range(draws):
+        with O.perturbed(np.random.default_rng(5 + k), rel):
+            o2 = run_oracle(desc, theta, x, labels)
+        r, _ = compare(desc, o2, o, LOOSE)
+        r["_per_tensor"] = _per_tensor(o["onet"], o2["grad"], o["grad"])
+        if out is None:
+            out = r
+        else:
+            for key, v in r.items():
+                out[key] = {i: max(a, v[i]) for i, a in out[key].items()} if key == "_per_tensor" else max(out[key], v)
+    return out
 
 
 def fp32_perturbation_noise(desc, theta, x, labels, o, draws=2, rel=1e-5):
@@ -187,11 +212,11 @@ def test_vgg_fp32_small_batch():
 # ------------------------------------------------------------------ measured bounds, full batch
 @pytest.mark.parametrize("idx", [1, 2, 3, 4])
 def test_bf16_full_batch(idx):
-    _measured(reduced(idx), bf16_decision_noise, 1.5, TOL["bf16"]["grad"])
+    _measured(reduced(idx), bf16_accum_noise, 3.0, TOL["bf16"]["grad"])
 
 
 def test_bf16_full_batch_delta_mode():
-    _measured(reduced(2, correction="delta"), bf16_decision_noise, 1.5, TOL["bf16"]["grad"])
+    _measured(reduced(2, correction="delta"), bf16_accum_noise, 3.0, TOL["bf16"]["grad"])
 
 
 @pytest.mark.parametrize("idx", [2, 4])
@@ -208,29 +233,37 @@ def test_paper_resnet_fp32_small_batch(n, mode):
 
 @pytest.mark.parametrize("n,batch", [(3, 128), (12, 32)])
 def test_paper_resnet_bf16(n, batch):
-    _measured(paper_reduced(n, batch=batch), bf16_decision_noise, 1.5, TOL["bf16"]["grad"])
+    _measured(paper_reduced(n, batch=batch), bf16_accum_noise, 3.0, TOL["bf16"]["grad"])
 
 
 def test_paper_vgg_coarse_fp32_small_batch():
-    """Batch 4.  At batch 2 the last subnetwork's BNs see 8 values per channel
-    and its ReLU decisions flip under relative perturbations of 3e-5 (the
-    oracle's own gradient of C^4 then moves by 12 %), below the difference
-    the fp32 one-pass variance leaves in x_4 (6e-5): no implementation can be
-    held to the fp32 bound there."""
-    d = W.parareal_vgg16(coarse="paper", precision="fp32", batch=4)
+    """Batch 2: the last subnetwork's BNs see 8 values per channel, where a
+    one-pass variance (sum h^2 - n mean^2) loses digits; the statistics are
+    combined as (count, mean, M2) partials (Chan's pairwise update) instead."""
+    d = W.parareal_vgg16(coarse="paper", precision="fp32", batch=2)
     _measured(d, fp32_perturbation_noise, 3.0, TOL["fp32"]["grad"])
 
 
 def test_paper_vgg_coarse_bf16():
-    _measured(W.parareal_vgg16(coarse="paper", batch=32), bf16_decision_noise, 1.5, TOL["bf16"]["grad"])
+    _measured(W.parareal_vgg16(coarse="paper", batch=32), bf16_accum_noise, 3.0, TOL["bf16"]["grad"])
 
 
 # ------------------------------------------------------------------ full depth
-@pytest.mark.parametrize("idx", [2, 4])
-def test_full_depth_fp32(idx):
-    desc = W.config(idx, batch=2)
+# Full-depth ResNet-1001 (333 bottlenecks): configurations 3 (N = 4), 4
+# (N = 16, 100 classes) and 5 (N = 8, 64x64 with the stride-2 stem, 200
+# classes) at small batches (the fp64 oracle holds every activation).
+@pytest.mark.parametrize("idx,batch", [(2, 2), (3, 2), (4, 2)])
+def test_full_depth_fp32(idx, batch):
+    desc = W.config(idx, batch=batch)
     desc["precision"] = "fp32"
     _measured(desc, fp32_perturbation_noise, 3.0, TOL["fp32"]["grad"])
+
+
+@pytest.mark.parametrize("idx,batch", [(2, 4), (3, 4), (4, 2)])
+def test_full_depth_bf16(idx, batch):
+    """The benchmarked path (tcgen05 kernels, bf16 storage) at full depth."""
+    desc = W.config(idx, batch=batch)
+    _measured(desc, bf16_accum_noise, 3.0, TOL["bf16"]["grad"])
 
 
 # ------------------------------------------------------------------ properties
