@@ -73,7 +73,105 @@ def parse():
                          "the step's work does not depend on it)")
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch (profiling a small case of the same network)")
+    ap.add_argument("--layer", default=None, choices=sorted(LAYERS),
+                    help="time one grouped convolution launch of the ResNet-1001 N=8 workload (pnn_conv_run) "
+                         "instead of the training step: a bottleneck conv (reduce = 1x1 out->mid, conv3x3 = "
+                         "mid->mid, expand = 1x1 mid->out with the residual add) and a mode (fwd, dgrad, "
+                         "wgrad), one instance per subnetwork at the stage its middle block sits in")
+    ap.add_argument("--layer-impl", default="auto", choices=["auto", "tma", "gathered"])
     return ap.parse_args()
+
+
+# grouped-launch microbenchmark: the same layer of the 8 subnetworks of the
+# 64x64 ResNet-1001 N=8 workload (batch 256; after the stride-2 stem the
+# stages run at 32x32 / 16x16 / 8x8 with widths 64 / 128 / 256 and bottleneck
+# widths 16 / 32 / 64); at the middle block of each subnetwork (uniform
+# tearing [42 x 7, 39] of 333 bottlenecks, 111 per stage) the stages are
+# [1, 1, 1, 2, 2, 3, 3, 3]
+LAYER_STAGES = [1, 1, 1, 2, 2, 3, 3, 3]
+STAGE_GEOM = {1: (32, 64, 16), 2: (16, 128, 32), 3: (8, 256, 64)}  # (hw, out, mid)
+LAYERS = {f"{conv}_{mode}": (conv, mode) for conv in ("reduce", "conv3x3", "expand")
+          for mode in ("fwd", "dgrad", "wgrad")}
+
+
+def layer_instances(name, batch, stream_dt):
+    """The instance list (host arrays and geometry) of a grouped layer launch."""
+    conv, mode = LAYERS[name]
+    rng = np.random.default_rng(7)
+    out = []
+    for st in LAYER_STAGES:
+        hw, wide, mid = STAGE_GEOM[st]
+        c, k, ks = {"reduce": (wide, mid, 1), "conv3x3": (mid, mid, 3), "expand": (mid, wide, 1)}[conv]
+        out.append(dict(batch=batch, h=hw, w=hw, c=c, k=k, ksize=ks, stride=1, relu=1,
+                        # the conv input: the stored BN input (the residual stream for reduce)
+                        x_dt=stream_dt if conv == "reduce" else "bf16", mode=mode, conv=conv))
+    return out
+
+
+def layer_arm(args, rank):
+    """Device time of one grouped conv launch of the training step, through
+    pnn_conv_time (CUDA events around repeated launches of the kernel alone),
+    with algorithmic bytes / FLOPs counted as the training step's profiler
+    counts them (each operand read once, each result written once)."""
+    import torch
+    from paper_2103_08802_gb300 import build, pnn
+    build.build()
+    if rank != 0:
+        return
+    torch.cuda.set_device(0)
+    B = args.batch or 256
+    sdt = "f32" if args.stream_fp32 else "bf16"
+    insts = layer_instances(args.layer, B, sdt)
+    conv, mode = LAYERS[args.layer]
+    dev, flops, nbytes = [], 0.0, 0.0
+    for g in insts:
+        M = B * g["h"] * g["w"]
+        xdt = torch.float32 if g["x_dt"] == "f32" else torch.bfloat16
+        xb = 4 if g["x_dt"] == "f32" else 2
+        d = {k: g[k] for k in ("batch", "h", "w", "c", "k", "ksize", "stride", "relu")}
+        d["wt"] = (torch.randn(g["k"] * g["ksize"] ** 2 * g["c"], device="cuda") * 0.1).to(torch.bfloat16)
+        d["x"] = torch.randn(M, g["c"], device="cuda").to(xdt)
+        d["bn_scale"] = torch.rand(g["c"], device="cuda") + 0.5
+        d["bn_shift"] = torch.randn(g["c"], device="cuda") * 0.1
+        w_bytes = g["k"] * g["ksize"] ** 2 * g["c"] * 2
+        macs = M * g["k"] * g["c"] * g["ksize"] ** 2
+        flops += 2.0 * macs
+        if mode == "fwd":
+            ydt = torch.float32 if (conv == "expand" and sdt == "f32") else torch.bfloat16
+            d["y"] = torch.empty(M, g["k"], device="cuda", dtype=ydt)
+            d["y_mean"] = torch.empty(g["k"], device="cuda")
+            d["y_rstd"] = torch.empty(g["k"], device="cuda")
+            nbytes += M * g["c"] * xb + w_bytes + M * g["k"] * d["y"].element_size()
+            if conv == "expand":
+                d["res"] = torch.randn(M, g["k"], device="cuda").to(ydt)
+                nbytes += M * g["k"] * d["res"].element_size()
+        elif mode == "dgrad":
+            d["dy"] = torch.randn(M, g["k"], device="cuda")
+            d["dx"] = torch.empty(M, g["c"], device="cuda")
+            nbytes += M * g["k"] * 4 + w_bytes + M * g["c"] * 4
+            # every input here is a BN+ReLU value: its backward sums ride along
+            d["bn_mean"] = torch.zeros(g["c"], device="cuda")
+            d["bn_rstd"] = torch.ones(g["c"], device="cuda")
+            d["dgamma"] = torch.empty(g["c"], device="cuda")
+            d["dbeta"] = torch.empty(g["c"], device="cuda")
+            nbytes += M * g["c"] * xb
+        else:
+            d["dy"] = torch.randn(M, g["k"], device="cuda")
+            d["dw"] = torch.empty(g["k"] * g["ksize"] ** 2 * g["c"], device="cuda")
+            nbytes += M * g["c"] * xb + M * g["k"] * 4 + g["k"] * g["ksize"] ** 2 * g["c"] * 4
+        dev.append(d)
+    pnn.conv_run({"fwd": "forward", "dgrad": "dgrad", "wgrad": "wgrad"}[mode], dev, impl=args.layer_impl)
+    ms = pnn.conv_run({"fwd": "forward", "dgrad": "dgrad", "wgrad": "wgrad"}[mode], dev, impl=args.layer_impl,
+                      repeat=max(1, args.steps))
+    pk, src = peaks()
+    gbs = nbytes / (ms / 1e3) / 1e9
+    print(json.dumps({
+        "metric": "grouped conv launch, algorithmic GB/s", "layer": args.layer, "impl": args.layer_impl,
+        "value": gbs, "unit": "GB/s", "ms_per_launch": ms, "tflops": flops / (ms / 1e3) / 1e12,
+        "frac_of_hbm": gbs / pk["hbm_gbs"], "frac_of_bf16_peak": flops / (ms / 1e3) / 1e12 / pk["bf16_tflops"],
+        "peak_source": src, "instances": [(g["c"], g["k"], g["ksize"], g["h"]) for g in insts], "batch": B,
+        "algorithmic_bytes": nbytes, "flops": flops, "residual_stream": sdt,
+        "l2": "operands larger than L2" if nbytes > 129e6 else "operands within L2"}), flush=True)
 
 
 def peaks():
@@ -509,6 +607,8 @@ def main():
         args.lr = 0.01 if desc["head"]["kind"] == "gap_mlp" else 0.1
     if args.impl == "reference":
         reference_arm(args, desc, rank)
+    elif args.layer:
+        layer_arm(args, rank)
     elif args.inference:
         infer_arm(args, desc, rank, local, world, dist)
     else:

@@ -385,6 +385,12 @@ typedef struct pnn_conv_args {
 int pnn_conv_workspace_bytes(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* args, size_t* bytes);
 int pnn_conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* args, void* workspace,
                  size_t workspace_bytes, void* stream);
+/* pnn_conv_run, then `repeat` (> 0) further launches of the convolution
+ * kernel alone between two CUDA events on `stream` (each rewrites what the
+ * first wrote; accumulate must be 0): *ms_per_launch = their mean device
+ * time.  A microbenchmark of one grouped launch; same errors as pnn_conv_run. */
+int pnn_conv_time(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* args, void* workspace,
+                  size_t workspace_bytes, void* stream, int32_t repeat, float* ms_per_launch);
 
 /* ---- allocation-free weight gradient of one convolution ----
  * The paper has no counterpart to this call.  It exists for callers that

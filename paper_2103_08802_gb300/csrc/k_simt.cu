@@ -510,25 +510,26 @@ __device__ __forceinline__ bool chunked_sums(const float* __restrict__ part, int
   return w == 0 && c < C;
 }
 
-// The same two-level reduction for the forward statistics: partial tiles hold
-// (mean, M2) of their rows (count from the row range: rpt rows each, the last
-// tile the remainder of M) and are merged with chan_merge in fp64 -- warp w
-// tiles t0+w, t0+w+8, ... in order, then warp 0 the eight warps in order; the
-// chunks likewise in the last CTA of the channel group.  Returns true on the
-// threads (warp 0, c < C) that hold the totals (count, mean, M2).
+// The same two-level reduction for the forward statistics.  Partial tiles
+// hold (mean_t, M2_t) of their rows (count n_t: rpt rows each, the last tile
+// the remainder of M).  They are combined as shifted sums around K = mean_0
+// (the first tile's mean, read by every CTA): with d_t = mean_t - K,
+//   S1 = sum n_t d_t,   S2 = sum (M2_t + n_t d_t^2),
+//   mean = K + S1 / M,  M2 = S2 - S1^2 / M,
+// which is Chan's pairwise update written for many sets at once (no term
+// subtracts two large sums: K lies within a few standard errors of the mean,
+// so S1^2 / M is a small part of S2).  Plain fp64 sums in the fixed order of
+// chunked_sums; returns true on the threads that hold (M, mean, M2).
 __device__ __forceinline__ bool chunked_moments(const float* __restrict__ part, int C, int tiles, int64_t M, int rpt,
                                                 int cg, int chunk, int nchunk, double* scratch, int32_t* counter,
                                                 double& n_out, double& mean_out, double& m2_out) {
-  __shared__ double red[8][3][32];
+  __shared__ double red[8][2][32];
   __shared__ int is_last;
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int c = cg * 32 + lane;
-  auto rows_of = [&](int64_t t0, int64_t t1) -> double {  // rows of tiles [t0, t1)
-    const int64_t a = t0 * rpt, b = t1 * rpt < M ? t1 * rpt : M;
-    return b > a ? (double)(b - a) : 0.0;
-  };
   const int t0 = chunk * kFinTilesPerCta, t1 = min(tiles, t0 + kFinTilesPerCta);
-  double n = 0.0, mean = 0.0, m2 = 0.0;
+  double a = 0.0, b = 0.0;
+  const double K = c < C && tiles > 0 ? (double)__ldg(part + (int64_t)c * 2) : 0.0;
   if (c < C) {
     float2 v[kFinTilesPerCta / 8];
 #pragma unroll
@@ -538,49 +539,63 @@ __device__ __forceinline__ bool chunked_moments(const float* __restrict__ part, 
     }
 #pragma unroll
     for (int k = 0; k < kFinTilesPerCta / 8; ++k) {
-      const int t = t0 + w + 8 * k;
-      if (t < t1) chan_merge(n, mean, m2, rows_of(t, t + 1), (double)v[k].x, (double)v[k].y);
+      const int64_t t = t0 + w + 8 * k;
+      if (t < t1) {
+        const int64_t r1 = (t + 1) * rpt < M ? (t + 1) * rpt : M;
+        const double n = (double)(r1 - t * rpt);
+        const double d = (double)v[k].x - K;
+        a += n * d;
+        b += (double)v[k].y + n * d * d;
+      }
     }
   }
-  red[w][0][lane] = n;
-  red[w][1][lane] = mean;
-  red[w][2][lane] = m2;
+  red[w][0][lane] = a;
+  red[w][1][lane] = b;
   __syncthreads();
-  n = mean = m2 = 0.0;
+  a = 0.0;
+  b = 0.0;
   if (w == 0)
-    for (int k = 0; k < 8; ++k) chan_merge(n, mean, m2, red[k][0][lane], red[k][1][lane], red[k][2][lane]);
-  if (nchunk == 1) {
-    n_out = n; mean_out = mean; m2_out = m2;
-    return w == 0 && c < C;
-  }
-  if (w == 0 && c < C) {
-    scratch[((int64_t)chunk * C + c) * 2] = mean;
-    scratch[((int64_t)chunk * C + c) * 2 + 1] = m2;
-  }
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) is_last = atomicAdd(counter + cg, 1) == nchunk - 1;
-  __syncthreads();
-  if (!is_last) return false;
-  __threadfence();
-  n = mean = m2 = 0.0;
-  if (c < C)
-    for (int k = w; k < nchunk; k += 8) {
-      const int64_t a = (int64_t)k * kFinTilesPerCta, b = min((int64_t)tiles, a + kFinTilesPerCta);
-      chan_merge(n, mean, m2, rows_of(a, b), __ldcg(scratch + ((int64_t)k * C + c) * 2),
-                 __ldcg(scratch + ((int64_t)k * C + c) * 2 + 1));
+    for (int k = 0; k < 8; ++k) {
+      a += red[k][0][lane];
+      b += red[k][1][lane];
     }
-  __syncthreads();  // red[] of the chunk pass is read before it is rewritten
-  red[w][0][lane] = n;
-  red[w][1][lane] = mean;
-  red[w][2][lane] = m2;
-  __syncthreads();
-  n = mean = m2 = 0.0;
-  if (w == 0)
-    for (int k = 0; k < 8; ++k) chan_merge(n, mean, m2, red[k][0][lane], red[k][1][lane], red[k][2][lane]);
-  if (threadIdx.x == 0) counter[cg] = 0;  // ready for the next launch
-  n_out = n; mean_out = mean; m2_out = m2;
-  return w == 0 && c < C;
+  bool have = w == 0 && c < C;
+  if (nchunk > 1) {
+    if (w == 0 && c < C) {
+      scratch[((int64_t)chunk * C + c) * 2] = a;
+      scratch[((int64_t)chunk * C + c) * 2 + 1] = b;
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) is_last = atomicAdd(counter + cg, 1) == nchunk - 1;
+    __syncthreads();
+    if (!is_last) return false;
+    __threadfence();
+    a = 0.0;
+    b = 0.0;
+    if (c < C)
+      for (int k = w; k < nchunk; k += 8) {
+        a += __ldcg(scratch + ((int64_t)k * C + c) * 2);
+        b += __ldcg(scratch + ((int64_t)k * C + c) * 2 + 1);
+      }
+    __syncthreads();  // warp 0 has read red[] of the chunk pass
+    red[w][0][lane] = a;
+    red[w][1][lane] = b;
+    __syncthreads();
+    a = 0.0;
+    b = 0.0;
+    if (w == 0)
+      for (int k = 0; k < 8; ++k) {
+        a += red[k][0][lane];
+        b += red[k][1][lane];
+      }
+    if (threadIdx.x == 0) counter[cg] = 0;  // ready for the next launch
+  }
+  const double n = (double)M;
+  n_out = n;
+  mean_out = K + a / n;
+  m2_out = b - a * a / n;
+  return have;
 }
 
 __global__ void __launch_bounds__(256) k_bn_fin(const BnFinDesc* __restrict__ tab, const int* __restrict__ tstart,

@@ -73,7 +73,7 @@ struct Plan {
   int bnmax = 16, raw = 0;
   int total = 0;
   size_t tab = 0, ts = 0, status = 0, aux_tab = 0, aux_ts = 0, fin_tab = 0, fin_ts = 0, red_tab = 0, red_ts = 0;
-  size_t bytes = 0;
+  size_t bytes = 0, init_bytes = 0;  // init_bytes: the prefix copied from the host
   std::vector<InstPlan> in;
 };
 
@@ -147,6 +147,8 @@ int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
   pl.bnmax = 16;
   pl.raw = 0;
   int esz = 2;
+  // pass 1: tile grids and the small regions that start from host values
+  // (tensor maps, gamma / beta, finalize counters); pass 2: device scratch
   for (int i = 0; i < n; ++i) {
     const pnn_conv_args& g = a[i];
     InstPlan& ip = pl.in[i];
@@ -165,28 +167,20 @@ int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
       ip.bn = g.y_mean != nullptr;
       if (ip.bn) {
         ip.stat_tiles = ip.mtiles;
-        ip.stats = take((size_t)ip.stat_tiles * g.k * 8);
-        ip.fscr = take((size_t)cdv(ip.stat_tiles, kFinTilesPerCta) * g.k * 16);
         ip.fcnt = take((size_t)cdv(g.k, 32) * 4);
         ip.gam = take((size_t)g.k * 4);
         ip.bet = take((size_t)g.k * 4);
-        ip.scl = take((size_t)g.k * 4);
-        ip.shf = take((size_t)g.k * 4);
       }
       pl.total += ip.mtiles * ip.ntiles;
     } else if (mode == 1) {
       ip.mtiles = cdv(Min, kTcBM);
       esz = 4;
-      ip.wt = take((size_t)g.k * rsc * 2);
       ip.bn = g.bn_mean != nullptr;
       if (ip.bn) {
         // the fused sums use 128-row tiles; the separate reduction its own
         ip.stat_tiles = std::max(ip.mtiles, cdv(Min, bnb_rows_per_tile(g.c)));
-        ip.stats = take((size_t)ip.stat_tiles * g.c * 8);
-        ip.fscr = take((size_t)cdv(ip.stat_tiles, kFinTilesPerCta) * g.c * 16);
         ip.fcnt = take((size_t)cdv(g.c, 32) * 4);
         ip.gam = take((size_t)g.c * 4);
-        ip.coef = take((size_t)g.c * 12);
       }
       pl.total += ip.mtiles * ip.ntiles;
     } else {
@@ -196,7 +190,6 @@ int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
       int splits = std::max(1, std::min(cdv(Mout, 256), cdv(2 * (int64_t)sms, base)));
       ip.pix_per_split = cdv(cdv(Mout, splits), 64) * 64;
       ip.splits = cdv(Mout, ip.pix_per_split);
-      ip.part = take((size_t)ip.splits * g.k * rsc * 4);
       if (pl.variant == 1) {
         const WgBoxes b = wg_boxes(g.c, g.k, g.w, ip.pad, g.x_dtype == PNN_DT_BF16);
         pl.raw = std::max(pl.raw, wg_raw_bytes(b));
@@ -204,6 +197,27 @@ int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
       pl.total += base * ip.splits;
     }
     if (pl.variant == 1) ip.maps = take(3 * 128);
+  }
+  pl.init_bytes = cur;
+  for (int i = 0; i < n; ++i) {
+    const pnn_conv_args& g = a[i];
+    InstPlan& ip = pl.in[i];
+    const int rsc = g.ksize * g.ksize * g.c;
+    if (mode == 0 && ip.bn) {
+      ip.stats = take((size_t)ip.stat_tiles * g.k * 8);
+      ip.fscr = take((size_t)cdv(ip.stat_tiles, kFinTilesPerCta) * g.k * 16);
+      ip.scl = take((size_t)g.k * 4);
+      ip.shf = take((size_t)g.k * 4);
+    } else if (mode == 1) {
+      ip.wt = take((size_t)g.k * rsc * 2);
+      if (ip.bn) {
+        ip.stats = take((size_t)ip.stat_tiles * g.c * 8);
+        ip.fscr = take((size_t)cdv(ip.stat_tiles, kFinTilesPerCta) * g.c * 16);
+        ip.coef = take((size_t)g.c * 12);
+      }
+    } else if (mode == 2) {
+      ip.part = take((size_t)ip.splits * g.k * rsc * 4);
+    }
   }
   if (pl.variant == 1 && mode != 2) pl.raw = kTcBM * 64 * esz;
   pl.bytes = cur;
@@ -224,8 +238,9 @@ extern "C" int pnn_conv_workspace_bytes(int32_t mode, int32_t impl, int32_t n, c
   return PNN_OK;
 }
 
-extern "C" int pnn_conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void* workspace,
-                            size_t workspace_bytes, void* stream) {
+namespace {
+int conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void* workspace, size_t workspace_bytes,
+             void* stream, int repeat, float* ms_out) {
   Plan pl;
   int r = make_plan(mode, impl, n, a, pl);
   if (r) return r;
@@ -235,7 +250,7 @@ extern "C" int pnn_conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_con
   char* ws = static_cast<char*>(workspace);
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
   // host images of every table, copied into the workspace before the launches
-  std::vector<uint8_t> img(pl.bytes, 0);
+  std::vector<uint8_t> img(pl.init_bytes, 0);
   auto at = [&](size_t off) { return img.data() + off; };
   std::vector<ConvDesc> cds(n);
   std::vector<int> ts(n + 1, 0);
@@ -374,21 +389,34 @@ extern "C" int pnn_conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_con
   if (!breds.empty()) memcpy(at(pl.red_tab), breds.data(), breds.size() * sizeof(BnBwdDesc));
   memcpy(at(pl.red_ts), red_ts.data(), red_ts.size() * sizeof(int));
   // (the image zero-fills the status word, the finalize counters and beta)
-  cudaError_t e = cudaMemcpyAsync(ws, img.data(), pl.bytes, cudaMemcpyHostToDevice, st);
+  cudaError_t e = cudaMemcpyAsync(ws, img.data(), pl.init_bytes, cudaMemcpyHostToDevice, st);
   const auto* tab = reinterpret_cast<const ConvDesc*>(ws + pl.tab);
   const int* tsd = reinterpret_cast<const int*>(ws + pl.ts);
   const int* auxts = reinterpret_cast<const int*>(ws + pl.aux_ts);
   if (e == cudaSuccess && mode == 1)
     e = launch_wtrans(reinterpret_cast<const WtDesc*>(ws + pl.aux_tab), auxts, n, aux_ts.back(), st);
-  if (e == cudaSuccess) {
-    if (pl.variant == 1)
-      e = launch_conv_tma(mode, tab, tsd, n, pl.total, pl.bnmax, pl.raw, status, st);
-    else if (mode == 0)
-      e = launch_conv_fwd_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
-    else if (mode == 1)
-      e = launch_conv_dgrad_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
-    else
-      e = launch_conv_wgrad_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
+  auto conv_launch = [&]() {
+    if (pl.variant == 1) return launch_conv_tma(mode, tab, tsd, n, pl.total, pl.bnmax, pl.raw, status, st);
+    if (mode == 0) return launch_conv_fwd_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
+    if (mode == 1) return launch_conv_dgrad_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
+    return launch_conv_wgrad_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
+  };
+  if (e == cudaSuccess) e = conv_launch();
+  if (e == cudaSuccess && repeat > 0) {
+    // device time of the conv kernel alone: `repeat` further launches (each
+    // rewrites what the first wrote) between two events on the stream
+    cudaEvent_t t0 = nullptr, t1 = nullptr;
+    e = cudaEventCreate(&t0);
+    if (e == cudaSuccess) e = cudaEventCreate(&t1);
+    if (e == cudaSuccess) e = cudaEventRecord(t0, st);
+    for (int r = 0; r < repeat && e == cudaSuccess; ++r) e = conv_launch();
+    if (e == cudaSuccess) e = cudaEventRecord(t1, st);
+    if (e == cudaSuccess) e = cudaEventSynchronize(t1);
+    float ms = 0.f;
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, t0, t1);
+    if (e == cudaSuccess) *ms_out = ms / (float)repeat;
+    if (t0) cudaEventDestroy(t0);
+    if (t1) cudaEventDestroy(t1);
   }
   if (e == cudaSuccess && mode == 2)
     e = launch_wreduce(reinterpret_cast<const WReduceDesc*>(ws + pl.aux_tab), auxts, n, aux_ts.back(), st);
@@ -407,4 +435,18 @@ extern "C" int pnn_conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_con
   if (e != cudaSuccess) return set_last_error(PNN_ECUDA, cudaGetErrorString(e));
   if (host_status == 3) return set_last_error(PNN_ETIMEOUT, "pnn_conv_run: a device wait timed out");
   return PNN_OK;
+}
+}  // namespace
+
+extern "C" int pnn_conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void* workspace,
+                            size_t workspace_bytes, void* stream) {
+  return conv_run(mode, impl, n, a, workspace, workspace_bytes, stream, 0, nullptr);
+}
+
+extern "C" int pnn_conv_time(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void* workspace,
+                             size_t workspace_bytes, void* stream, int32_t repeat, float* ms_per_launch) {
+  if (repeat <= 0 || !ms_per_launch) return set_last_error(PNN_EINVAL, "pnn_conv_time: repeat > 0 and an output");
+  for (int i = 0; i < n && a; ++i)
+    if (a[i].accumulate) return set_last_error(PNN_EINVAL, "pnn_conv_time: accumulating launches are not repeatable");
+  return conv_run(mode, impl, n, a, workspace, workspace_bytes, stream, repeat, ms_per_launch);
 }

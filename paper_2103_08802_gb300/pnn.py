@@ -128,6 +128,7 @@ def load():
         "pnn_selftest_wait_timeout": (C.c_int, [C.c_int64, P]),
         "pnn_conv_workspace_bytes": (C.c_int, [I32, I32, I32, C.POINTER(ConvArgs), C.POINTER(SZ)]),
         "pnn_conv_run": (C.c_int, [I32, I32, I32, C.POINTER(ConvArgs), P, SZ, P]),
+        "pnn_conv_time": (C.c_int, [I32, I32, I32, C.POINTER(ConvArgs), P, SZ, P, I32, C.POINTER(C.c_float)]),
         "pnn_last_error": (C.c_char_p, [P]),
         "pnn_status_string": (C.c_char_p, [C.c_int]),
     }
@@ -433,12 +434,14 @@ def _dt(t):
     return DTYPE["bf16"] if t is not None and t.dtype == torch.bfloat16 else DTYPE["f32"]
 
 
-def conv_run(mode, instances, impl="auto", stream=None):
+def conv_run(mode, instances, impl="auto", stream=None, repeat=0):
     """One grouped convolution (pnn_conv_run) over `instances`, a list of dicts
     with the geometry (batch, h, w, c, k, ksize, stride) and torch CUDA tensors
     by the names of pnn_conv_args (x, bn_scale, bn_shift, relu, wt, y, res,
     y_mean, y_rstd, dy, dx, accumulate, bn_mean, bn_rstd, dgamma, dbeta, dw).
-    The workspace comes from torch.  Raises PnnError on failure."""
+    The workspace comes from torch.  With repeat > 0 the kernel runs that many
+    more times between CUDA events (pnn_conv_time) and the mean device ms of
+    one launch is returned.  Raises PnnError on failure."""
     import torch
     lib = load()
     n = len(instances)
@@ -458,4 +461,9 @@ def conv_run(mode, instances, impl="auto", stream=None):
     _global_check(lib, lib.pnn_conv_workspace_bytes(m, im, n, arr, C.byref(nb)))
     ws = torch.empty(max(256, nb.value), dtype=torch.uint8, device="cuda")
     st = stream.cuda_stream if stream is not None else None
+    if repeat > 0:
+        ms = C.c_float()
+        _global_check(lib, lib.pnn_conv_time(m, im, n, arr, ws.data_ptr(), ws.numel(), st, repeat, C.byref(ms)))
+        return ms.value
     _global_check(lib, lib.pnn_conv_run(m, im, n, arr, ws.data_ptr(), ws.numel(), st))
+    return None

