@@ -529,7 +529,7 @@ __device__ __forceinline__ bool chunked_moments(const float* __restrict__ part, 
   const int c = cg * 32 + lane;
   const int t0 = chunk * kFinTilesPerCta, t1 = min(tiles, t0 + kFinTilesPerCta);
   double a = 0.0, b = 0.0;
-  const double K = c < C && tiles > 0 ? (double)__ldg(part + (int64_t)c * 2) : 0.0;
+  const float K = c < C && tiles > 0 ? __ldg(part + (int64_t)c * 2) : 0.f;
   if (c < C) {
     float2 v[kFinTilesPerCta / 8];
 #pragma unroll
@@ -537,17 +537,23 @@ __device__ __forceinline__ bool chunked_moments(const float* __restrict__ part, 
       const int t = t0 + w + 8 * k;
       v[k] = t < t1 ? *reinterpret_cast<const float2*>(part + ((int64_t)t * C + c) * 2) : make_float2(0.f, 0.f);
     }
+    // this thread's eight tiles in fp32 (d is a small difference of two
+    // close means; the S2 terms are all positive), then fp64 from here on
+    float fa = 0.f, fb = 0.f;
 #pragma unroll
     for (int k = 0; k < kFinTilesPerCta / 8; ++k) {
       const int64_t t = t0 + w + 8 * k;
       if (t < t1) {
         const int64_t r1 = (t + 1) * rpt < M ? (t + 1) * rpt : M;
-        const double n = (double)(r1 - t * rpt);
-        const double d = (double)v[k].x - K;
-        a += n * d;
-        b += (double)v[k].y + n * d * d;
+        const float n = (float)(r1 - t * rpt);
+        const float d = v[k].x - K;
+        const float nd = n * d;
+        fa += nd;
+        fb += v[k].y + nd * d;
       }
     }
+    a = fa;
+    b = fb;
   }
   red[w][0][lane] = a;
   red[w][1][lane] = b;
@@ -593,7 +599,7 @@ __device__ __forceinline__ bool chunked_moments(const float* __restrict__ part, 
   }
   const double n = (double)M;
   n_out = n;
-  mean_out = K + a / n;
+  mean_out = (double)K + a / n;
   m2_out = b - a * a / n;
   return have;
 }

@@ -111,9 +111,12 @@ class Case:
 
 
 def _check(name, got, exact, absbound, extra_rel, norm_tol, maxrel_tol=None):
+    """|got - exact| <= absbound * (1 + extra_rel) + extra_rel * |exact|: the
+    final rounding (relative extra_rel) applies to the computed value, which
+    is within absbound of exact."""
     got = np.asarray(got, np.float64)
     err = np.abs(got - exact)
-    bound = absbound + extra_rel * np.abs(exact) + 1e-30
+    bound = absbound * (1 + extra_rel) + extra_rel * np.abs(exact) + 1e-30
     worst = float((err / bound).max())
     nrel = float(np.linalg.norm(got - exact) / max(np.linalg.norm(exact), 1e-30))
     mrel = float(err.max() / max(np.abs(exact).max(), 1e-30))
@@ -193,15 +196,20 @@ def test_conv_forward(name, impl):
         M = cs.g["batch"] * cs.P * cs.Q
         rng = np.random.default_rng(100 + i)
         res = rng.standard_normal((cs.g["batch"], cs.P, cs.Q, cs.g["k"])).astype(np.float32)
-        ybf = (i + len(name)) % 2 == 0  # alternate bf16 and fp32 outputs (with a residual)
-        d["y"] = torch.full((M, cs.g["k"]), float("nan"), device="cuda",
-                            dtype=torch.bfloat16 if ybf else torch.float32)
-        if not ybf:
-            d["res"] = _t(res, torch.float32)
+        # three epilogues in turn: bf16 y; fp32 y + fp32 residual; bf16 y +
+        # bf16 residual (the residual stream's two storage precisions)
+        kind = (i + len(name)) % 3
+        ybf = kind != 1
         d["y_mean"] = torch.full((cs.g["k"],), float("nan"), device="cuda")
         d["y_rstd"] = torch.full((cs.g["k"],), float("nan"), device="cuda")
+        if kind == 2:
+            res = _bf16_round_f32(res).astype(np.float32)
+        d["y"] = torch.full((M, cs.g["k"]), float("nan"), device="cuda",
+                            dtype=torch.bfloat16 if ybf else torch.float32)
+        if kind:
+            d["res"] = _t(res, torch.float32 if kind == 1 else torch.bfloat16)
+        outs.append((cs, ybf, res if kind else None))
         insts.append(d)
-        outs.append((cs, ybf, res))
     pnn.conv_run("forward", insts, impl=impl)
     torch.cuda.synchronize()
     for (cs, ybf, res), d in zip(outs, insts):
@@ -211,12 +219,15 @@ def test_conv_forward(name, impl):
         mag = O.conv2d(np.abs(a), np.abs(w), cs.g["stride"], cs.pad)
         got = _nchw(d["y"].float().cpu().numpy().reshape(cs.g["batch"], cs.P, cs.Q, cs.g["k"]))
         absb = 2 * n * U * mag
-        if ybf:
-            _check(f"{name}/{impl} y(bf16)", got, exact, absb, 2.0 ** -8 + U, 4e-3, 8e-3)
-        else:
+        if res is not None:
             r = _nchw(res)
             exact = exact + r
-            _check(f"{name}/{impl} y(fp32)+res", got, exact, absb + U * np.abs(r), U, 1e-5)
+            absb = absb + U * np.abs(r)
+        if ybf:
+            _check(f"{name}/{impl} y(bf16){'+res' if res is not None else ''}", got, exact, absb, 2.0 ** -8 + U,
+                   4e-3, 8e-3)
+        else:
+            _check(f"{name}/{impl} y(fp32)+res", got, exact, absb, U, 1e-5)
         # batch statistics of the stored y (what the next BN normalises with)
         y = got
         mean = y.mean(axis=(0, 2, 3))
