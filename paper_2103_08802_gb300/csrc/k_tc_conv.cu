@@ -54,7 +54,7 @@ enum { FWD = 0, DGRAD = 1, WGRAD = 2 };
 // Diagnostic build only: forward epilogue phases (cycles, summed over the
 // first thread of each epilogue warp): TMEM load, residual + store, column
 // sums, statistics barrier + write; [4] chunks.
-__device__ unsigned long long g_epi_cycles[6];
+__device__ unsigned long long g_epi_cycles[2][8];
 #endif
 #ifdef PNN_ROLE_TIMING
 // Diagnostic build only: SM cycles each role spends waiting and working,
@@ -428,26 +428,6 @@ __device__ __forceinline__ void res_raw(const ConvDesc& d, int m, int nb, int nc
   }
 }
 
-// The epilogue operand in shared memory: boxes of 128 rows x rb bytes
-// (rb = 32, 64 or 128), box i holding tile bytes [128 i, 128 i + rb) of each
-// row, swizzled as TMA writes them (16-byte chunk c of row r at c ^ (r & 7),
-// c ^ ((r >> 1) & 3), c ^ ((r >> 2) & 1) for 128-, 64- and 32-byte rows), so
-// that the 32 rows of a warp read one chunk each without bank conflicts.
-__device__ __forceinline__ const uint8_t* eop_chunk(const uint8_t* slot, int row, int ch16, int rb) {
-  const int per = rb >> 4;
-  const int box = ch16 / per, c = ch16 - box * per;
-  const int sw = per == 8 ? (row & 7) : (per == 4 ? ((row >> 1) & 3) : ((row >> 2) & 1));
-  return slot + box * (128 * rb) + row * rb + ((c ^ sw) << 4);
-}
-// 16 elements of tile row `row` from column col0 (bf16: two 16-byte chunks,
-// fp32: four)
-__device__ __forceinline__ void eop_load(const uint8_t* slot, int row, int col0, bool bf, int rb, uint4 (&out)[4]) {
-  const int c0 = bf ? col0 >> 3 : col0 >> 2;
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-    if (i < (bf ? 2 : 4)) out[i] = *reinterpret_cast<const uint4*>(eop_chunk(slot, row, c0 + i, rb));
-}
-
 // One warp drains TMEM lanes 32q .. 32q+31 (its rows) for the 16-column
 // chunks j_first, j_first + j_step, ...; the ethreads epilogue threads
 // (etid = this thread's index among them) meet at named barrier 2.
@@ -457,7 +437,7 @@ __device__ __forceinline__ void eop_load(const uint8_t* slot, int row, int col0,
 template <int MODE>
 __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, int lane, float (&red)[4][256][2],
                                          int j_first, int j_step, int etid, int ethreads, uint8_t* ystage, int& ybuf,
-                                         int bar_id = 2, const uint8_t* eop = nullptr, int erb = 0) {
+                                         int bar_id = 2) {
   const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
   const int row = q * 32 + lane;
   const int m = T.m0 + row;
@@ -469,19 +449,16 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
   float* const spart = MODE == FWD ? d.stats : d.bnb_part;
   // forward residual: 16 columns a chunk, the next chunk's loads issued
   // before the current chunk is consumed
-  const bool rsm = MODE == FWD && d.res != nullptr && eop != nullptr;  // residual tile in shared memory
-  const bool rvec = MODE == FWD && d.res != nullptr && mvalid && (d.K % 8) == 0 && !rsm;
+  const bool rvec = MODE == FWD && d.res != nullptr && mvalid && (d.K % 8) == 0;
   uint4 rcur[4], rnext[4];
   if (rvec && j_first < T.BN) res_raw(d, m, T.n0 + j_first, T.Ncols, rcur);
-  RT(unsigned long long e0 = 0, e1 = 0, e2 = 0, e3 = 0, en = 0, e5 = 0;)
+  RT(unsigned long long e0 = 0, e1 = 0, e2 = 0, e3 = 0, en = 0, e5 = 0, e6 = 0, e7 = 0;)
   // fused data gradient: the chunk's BN input h (16 values of this row)
   const bool hload = MODE == DGRAD && stats && mvalid;
   for (int j0 = j_first; j0 < T.BN; j0 += j_step) {
     if (rvec && j0 + j_step < T.BN) res_raw(d, m, T.n0 + j0 + j_step, T.Ncols, rnext);
     uint4 hraw[4];
-    if (hload && eop) {
-      eop_load(eop, row, j0, d.x.dt == DT_BF16, erb, hraw);
-    } else if (hload) {
+    if (hload) {
       const bool hb = d.x.dt == DT_BF16;
       const int64_t o = (int64_t)m * d.C + T.n0 + j0;
       const uint4* src = hb ? reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(d.x.ptr) + o)
@@ -506,7 +483,6 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
         const int64_t o = (int64_t)m * d.K + nb;
         if (d.res) {
           if (vec) {
-            if (rsm) eop_load(eop, row, j0, d.res_dt == DT_BF16, erb, rcur);
             if (d.res_dt == DT_BF16) {
               const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(rcur);
 #pragma unroll
@@ -521,9 +497,13 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
               for (int i = 0; i < 16; ++i) v[i] += f[i];
             }
           } else {
-            for (int i = 0; i < 16 && nb + i < d.K; ++i)
-              v[i] += d.res_dt == DT_F32 ? reinterpret_cast<const float*>(d.res)[o + i]
-                                         : __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(d.res)[o + i]);
+            // (fully unrolled with a predicate: a loop with a run-time bound
+            // would make v[] addressable and move it to local memory)
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+              if (nb + i < d.K)
+                v[i] += d.res_dt == DT_F32 ? reinterpret_cast<const float*>(d.res)[o + i]
+                                           : __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(d.res)[o + i]);
           }
         }
         RT(if (true) { const unsigned long long cr = clock64(); e5 += cr - c1; })
@@ -550,7 +530,9 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
             }
           }
         } else {
-          for (int i = 0; i < 16 && nb + i < d.K; ++i) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            if (nb + i >= d.K) continue;
             if (d.y_dt == DT_BF16) reinterpret_cast<__nv_bfloat16*>(d.y)[o + i] = __float2bfloat16_rn(v[i]);
             else reinterpret_cast<float*>(d.y)[o + i] = v[i];
           }
@@ -561,8 +543,10 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
       }
       if (tstore) {
         // the store issued from this buffer two chunks ago must have read it
+        RT(const unsigned long long cw = clock64();)
         if (lane == 0) bulk_wait_read<1>();
         __syncwarp();
+        RT(e6 += clock64() - cw;)
         uint8_t* st = ystage + ybuf * 2048;
         if (d.y_dt == DT_BF16) {
           // 32-byte rows, 32-byte swizzle: 16-byte chunk c at c ^ ((row >> 2) & 1)
@@ -651,8 +635,10 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
         }
       }
       // staged chunk -> TMA store (fresh gradient) or TMA reduce-add (accumulate)
+      RT(const unsigned long long cw = clock64();)
       if (lane == 0) bulk_wait_read<1>();
       __syncwarp();
+      RT(e6 += clock64() - cw;)
       uint8_t* st = ystage + ybuf * 2048;
 #pragma unroll
       for (int c = 0; c < 4; ++c)
@@ -683,7 +669,9 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
           p[c] = a;
         }
       } else {
-        for (int i = 0; i < 16 && nb + i < T.Ncols; ++i) out[i] = acc ? out[i] + v[i] : v[i];
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          if (nb + i < T.Ncols) out[i] = acc ? out[i] + v[i] : v[i];
       }
     }
     if (rvec) {
@@ -720,9 +708,11 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
     asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "r"(ethreads) : "memory");  // red[] is reused by the next tile
   }
   RT(e3 += clock64() - c3;
-     if (MODE == FWD && lane == 0 && ethreads == 256) {
-       atomicAdd(&g_epi_cycles[0], e0); atomicAdd(&g_epi_cycles[1], e1); atomicAdd(&g_epi_cycles[2], e2);
-       atomicAdd(&g_epi_cycles[3], e3); atomicAdd(&g_epi_cycles[4], en); atomicAdd(&g_epi_cycles[5], e5);
+     if (MODE != WGRAD && lane == 0) {
+       unsigned long long* ec = g_epi_cycles[MODE == FWD ? 0 : 1];
+       atomicAdd(&ec[0], e0); atomicAdd(&ec[1], e1); atomicAdd(&ec[2], e2);
+       atomicAdd(&ec[3], e3); atomicAdd(&ec[4], en); atomicAdd(&ec[5], e5); atomicAdd(&ec[6], e6);
+       atomicAdd(&ec[7], e7);
      })
 }
 
@@ -942,8 +932,6 @@ struct TmaShared {
   uint64_t op_empty[kTmaMaxStages];
   uint64_t tfull[2];
   uint64_t tempty[2];
-  uint64_t efull[2];   // epilogue-operand slot b loaded (producer: expect_tx, or a plain arrive)
-  uint64_t eempty[2];  // slot b read by its epilogue group (128 arrivals)
   uint64_t drain;
   uint32_t tmem;
   int abort_flag;
@@ -961,9 +949,7 @@ __host__ __device__ constexpr int tma_op_bytes(int mode, int bnmax) { return tma
 // forward / data gradient: two 2 KB output staging tiles per epilogue warp
 // (12 - XW warps) after the rings
 constexpr int kTmaYStage = 8 * 2 * 2048;
-__host__ __device__ constexpr int tma_ystage(int mode, int xw) { return mode == 2 ? 0 : (12 - xw) * 2 * 2048; }
-// after the rings: the output staging tiles, then two epilogue-operand slots
-__host__ __device__ constexpr int tma_extra(int mode, int xw, int eslot) { return tma_ystage(mode, xw) + 2 * eslot; }
+__host__ __device__ constexpr int tma_extra(int mode, int xw) { return mode == 2 ? 0 : (12 - xw) * 2 * 2048; }
 __host__ __device__ inline int tma_stages(int mode, int bnmax, int raw_bytes, int extra) {
   const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - extra;
   int s = avail / (raw_bytes + tma_op_bytes(mode, bnmax));
@@ -1215,21 +1201,18 @@ __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDe
 
 template <int MODE, int XW>
 __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, const int* __restrict__ tstart,
-                                              int ninst, int total, int bnmax, int raw_bytes, int eslot,
-                                              int32_t* status) {
+                                              int ninst, int total, int bnmax, int raw_bytes, int32_t* status) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw0 = smem_u32(smem_raw);
   const uint32_t base = (raw0 + 1023u) & ~1023u;
   uint8_t* const gbase = smem_raw + (base - raw0);
-  if (MODE == WGRAD) eslot = 0;
-  const int S = tma_stages(MODE, bnmax, raw_bytes, tma_extra(MODE, XW, eslot));
+  const int S = tma_stages(MODE, bnmax, raw_bytes, tma_extra(MODE, XW));
   const int op_bytes = tma_op_bytes(MODE, bnmax);
   constexpr int kAMult = tma_amult(MODE);
   const uint32_t op_base = base + S * raw_bytes;
   RT(const unsigned long long rt_start = clock64();)
   uint8_t* const ystage0 = gbase + S * (raw_bytes + op_bytes);  // output staging (1024-aligned)
-  uint8_t* const eslot0 = ystage0 + tma_ystage(MODE, XW);       // epilogue-operand slots (1024-aligned)
-  TmaShared& sh = *reinterpret_cast<TmaShared*>(ystage0 + tma_extra(MODE, XW, eslot));
+  TmaShared& sh = *reinterpret_cast<TmaShared*>(ystage0 + tma_extra(MODE, XW));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   uint32_t colstride = 32;
   while ((int)colstride < bnmax) colstride <<= 1;
@@ -1245,8 +1228,6 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     for (int b = 0; b < 2; ++b) {
       mbar_init(smem_u32(&sh.tfull[b]), 1);
       mbar_init(smem_u32(&sh.tempty[b]), 128);  // one epilogue group drains a buffer
-      mbar_init(smem_u32(&sh.efull[b]), 1);
-      mbar_init(smem_u32(&sh.eempty[b]), 128);
     }
     mbar_init(smem_u32(&sh.drain), 1);
     sh.abort_flag = 0;
@@ -1263,33 +1244,11 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     // ================================================= TMA producer
     if (lane == 0) {
       uint32_t g = 0;
-      int li = 0;     // tiles of this CTA so far (epilogue-operand slot li & 1)
-      int armed = 0;  // tiles whose epilogue-operand slot phase has been armed
       bool ok = true;
       RT(unsigned long long rt_a = 0, rt_b = 0;)
-      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++li) {
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
         const Tile T = decode<MODE>(tab, tstart, ninst, tile);
         const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
-        if (MODE != WGRAD && eslot > 0) {
-          // the tile's epilogue operand into slot b, once its group has read
-          // the slot's previous tile; a tile without one still completes the
-          // slot's phase (a plain arrival), so every phase advances once a tile
-          const int b = li & 1;
-          if (!mbar_wait(smem_u32(&sh.eempty[b]), ((li >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
-          const uint32_t ef = smem_u32(&sh.efull[b]);
-          if (d.tma_e != nullptr) {
-            const int rb = d.e_rowbytes;
-            const bool ebf = MODE == FWD ? d.res_dt == DT_BF16 : d.x.dt == DT_BF16;
-            const int cpb = rb / (ebf ? 2 : 4);          // columns of one box
-            const int nbox = (T.BN + cpb - 1) / cpb;
-            mbar_expect_tx(ef, (uint32_t)(nbox * 128 * rb));
-            const uint32_t dst = smem_u32(eslot0) + b * eslot;
-            for (int i = 0; i < nbox; ++i) tma_load_2d(dst + i * 128 * rb, d.tma_e, T.n0 + i * cpb, T.m0, ef);
-          } else {
-            mbar_arrive(ef);
-          }
-          armed = li + 1;
-        }
         if constexpr (MODE == WGRAD) {
           // per k-step: the activation rows of all taps (a halo of pad*W+pad
           // rows each side) and the gradient rows of the k-step's 64 pixels
@@ -1339,11 +1298,6 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       // the copies of the last stages issued must land before the CTA exits
       for (uint32_t i = g > (uint32_t)S ? g - S : 0; i < g; ++i)
         mbar_wait_drain(smem_u32(&sh.tma_full[i % S]), (i / S) & 1);
-      // and those of the last two epilogue operands (each slot's last phase;
-      // a tile that stopped before its slot was armed is not counted)
-      if (MODE != WGRAD && eslot > 0)
-        for (int lj = armed > 2 ? armed - 2 : 0; lj < armed; ++lj)
-          mbar_wait_drain(smem_u32(&sh.efull[lj & 1]), (lj >> 1) & 1);
     }
     __syncwarp();
   } else if (warp < TmaRoles<MODE, XW>::kEpiWarp0) {
@@ -1507,9 +1461,6 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       const int b = li & 1;
       RT(const unsigned long long rt0 = clock64();)
       bool got = mbar_wait(smem_u32(&sh.tfull[b]), (li >> 1) & 1, abort_flag);
-      // and the slot's phase of this tile's epilogue operand (a tile without
-      // one completes it with a plain arrival); every thread reads the slot
-      if (got && MODE != WGRAD && eslot > 0) got = mbar_wait(smem_u32(&sh.efull[b]), (li >> 1) & 1, abort_flag);
       RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
       got = __all_sync(0xffffffffu, got);
       // the group's four warps decide together (they meet at its named barrier)
@@ -1519,10 +1470,8 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       asm volatile("bar.sync %0, 128;" ::"r"(bar) : "memory");
       if (!got) { ok = false; break; }
       fence_after();
-      const uint8_t* eop = MODE != WGRAD && eslot > 0 && T.d->tma_e != nullptr ? eslot0 + b * eslot : nullptr;
       epilogue<MODE>(T, tmem + b * bufcols, q, lane, sh.red[eg], 0, 16, (ew & 3) * 32 + lane, 128,
-                     MODE != WGRAD ? ystage0 + ew * 4096 : nullptr, ybuf, bar, eop, T.d->e_rowbytes);
-      if (MODE != WGRAD && eslot > 0) mbar_arrive(smem_u32(&sh.eempty[b]));
+                     MODE != WGRAD ? ystage0 + ew * 4096 : nullptr, ybuf, bar);
       if (kAMult == 2 && min(T.d->mtile_rows, T.Mrows - T.m0) > kBM) {
         // rows 128-255 of the tile, from the second accumulator half
         Tile T2 = T;
@@ -1557,22 +1506,19 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
 
 __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_fwd_tma(const ConvDesc* __restrict__ tab,
                                                                  const int* __restrict__ tstart, int ninst, int total,
-                                                                 int bnmax, int raw_bytes, int eslot,
-                                                                  int32_t* status) {
-  conv_tma_body<FWD, 4>(tab, tstart, ninst, total, bnmax, raw_bytes, eslot, status);
+                                                                 int bnmax, int raw_bytes, int32_t* status) {
+  conv_tma_body<FWD, 4>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
 
 __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_dgrad_tma(const ConvDesc* __restrict__ tab,
                                                                    const int* __restrict__ tstart, int ninst, int total,
-                                                                   int bnmax, int raw_bytes, int eslot,
-                                                                  int32_t* status) {
-  conv_tma_body<DGRAD, 4>(tab, tstart, ninst, total, bnmax, raw_bytes, eslot, status);
+                                                                   int bnmax, int raw_bytes, int32_t* status) {
+  conv_tma_body<DGRAD, 4>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
 __global__ void __launch_bounds__(kTmaThreads, 1) k_conv_wgrad_tma(const ConvDesc* __restrict__ tab,
                                                                    const int* __restrict__ tstart, int ninst, int total,
-                                                                   int bnmax, int raw_bytes, int eslot,
-                                                                  int32_t* status) {
-  conv_tma_body<WGRAD, 8>(tab, tstart, ninst, total, bnmax, raw_bytes, eslot, status);
+                                                                   int bnmax, int raw_bytes, int32_t* status) {
+  conv_tma_body<WGRAD, 8>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
 
 // one kernel name per mode (profiler filters and launch lists name the mode)
@@ -1615,30 +1561,21 @@ bool conv_tma_fits(int mode, int bnmax, int raw_bytes) {
   return avail / (raw_bytes + tma_op_bytes(mode, bnmax)) >= 2;
 }
 
-int conv_tma_stage_count(int mode, int bnmax, int raw_bytes, int eslot) {
-  const int xw = mode == 2 ? 8 : 4;
-  const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - tma_extra(mode, xw, mode == 2 ? 0 : eslot);
-  return avail / (raw_bytes + tma_op_bytes(mode, bnmax));
-}
-
 cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
-                            int raw_bytes, int eslot, int32_t* status, cudaStream_t st, int max_ctas) {
+                            int raw_bytes, int32_t* status, cudaStream_t st, int max_ctas) {
   if (total <= 0) return cudaSuccess;
-  if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || raw_bytes <= 0 || (raw_bytes & 1023) || mode < 0 || mode > 2 ||
-      eslot < 0 || (eslot & 1023))
+  if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || raw_bytes <= 0 || (raw_bytes & 1023) || mode < 0 || mode > 2)
     return cudaErrorInvalidValue;
-  if (mode == 2) eslot = 0;
   const int xw = mode == 2 ? 8 : 4;  // transform warps of the mode's kernel
   auto kern = mode == 0 ? k_conv_fwd_tma : (mode == 1 ? k_conv_dgrad_tma : k_conv_wgrad_tma);
   cudaError_t e = set_smem_attr_once(4 + mode, reinterpret_cast<const void*>(kern), kTmaSmemBudget);
   if (e != cudaSuccess) return e;
   const int sms = device_sm_count();
-  if (conv_tma_stage_count(mode, bnmax, raw_bytes, eslot) < 2) return cudaErrorInvalidValue;
-  const size_t smem = tma_smem_bytes(mode, bnmax, raw_bytes, tma_extra(mode, xw, eslot));
+  const size_t smem = tma_smem_bytes(mode, bnmax, raw_bytes, tma_extra(mode, xw));
   if (smem > (size_t)kTmaSmemBudget) return cudaErrorInvalidValue;
   int grid = total < sms ? total : sms;
   if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
-  kern<<<grid, kTmaThreads, smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, eslot, status);
+  kern<<<grid, kTmaThreads, smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, status);
   return cudaGetLastError();
 }
 
@@ -1673,7 +1610,7 @@ cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
 extern "C" int pnn_role_cycles(unsigned long long* out, int reset) {
   cudaError_t e = cudaMemcpyFromSymbol(out, pnn::g_role_cycles, sizeof(pnn::g_role_cycles));
   if (e == cudaSuccess) e = cudaMemcpyFromSymbol(out + 36, pnn::g_tma_cycles, sizeof(pnn::g_tma_cycles));  // 3 x 16
-  if (e == cudaSuccess) e = cudaMemcpyFromSymbol(out + 84, pnn::g_epi_cycles, sizeof(pnn::g_epi_cycles));
+  if (e == cudaSuccess) e = cudaMemcpyFromSymbol(out + 84, pnn::g_epi_cycles, sizeof(pnn::g_epi_cycles));  // 2 x 8
   if (e == cudaSuccess && reset) {
     static const unsigned long long zero[3][12] = {};
     e = cudaMemcpyToSymbol(pnn::g_role_cycles, zero, sizeof zero);

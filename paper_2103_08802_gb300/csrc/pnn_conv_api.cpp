@@ -65,12 +65,12 @@ struct InstPlan {
   int P = 0, Q = 0, pad = 0, mtiles = 0, ntiles = 0, splits = 1, pix_per_split = 0, rows = 0;
   size_t wt = 0, part = 0, stats = 0, fscr = 0, fcnt = 0, gam = 0, bet = 0, scl = 0, shf = 0, coef = 0;
   size_t maps = 0;
-  int stat_tiles = 0, ntw = 0, erb = 0;
+  int stat_tiles = 0;
   bool bn = false;  // forward statistics / data-gradient BN sums requested
 };
 struct Plan {
   int variant = 0;
-  int bnmax = 16, raw = 0, eslot = 0;
+  int bnmax = 16, raw = 0;
   int total = 0;
   size_t tab = 0, ts = 0, status = 0, aux_tab = 0, aux_ts = 0, fin_tab = 0, fin_ts = 0, red_tab = 0, red_ts = 0;
   size_t bytes = 0, init_bytes = 0;  // init_bytes: the prefix copied from the host
@@ -159,20 +159,8 @@ int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
     const int64_t Mout = (int64_t)g.batch * ip.P * ip.Q, Min = (int64_t)g.batch * g.h * g.w;
     const int rsc = g.ksize * g.ksize * g.c;
     const int ncols = mode == 1 ? g.c : g.k;
-    // the training step's rule: a TMA-fed data gradient that forms the BN
-    // sums of a bf16 BN input wider than 64 channels uses 64-column tiles
-    const bool fused = mode == 1 && pl.variant == 1 && g.bn_mean && !g.accumulate && g.c % 16 == 0;
-    ip.ntw = fused && g.c > 64 && g.x_dtype == PNN_DT_BF16 ? 64 : tc_ntile_cols(mode, pl.variant);
-    ip.ntiles = mode == 2 ? cdv(g.k, 256) : cdv(ncols, ip.ntw);
-    const int bn = ip.ntiles == 1 ? ((ncols + 15) & ~15) : ip.ntw;
-    pl.bnmax = std::max(pl.bnmax, bn);
-    // the epilogue's second operand in shared memory (forward residual,
-    // data-gradient BN input)
-    if (pl.variant == 1 && ((mode == 0 && g.res) || fused)) {
-      const int esz = mode == 0 ? (g.res_dtype == PNN_DT_BF16 ? 2 : 4) : (g.x_dtype == PNN_DT_BF16 ? 2 : 4);
-      ip.erb = eop_rowbytes(bn, esz);
-      if (ip.erb) pl.eslot = std::max(pl.eslot, eop_slot_bytes(bn, esz));
-    }
+    ip.ntiles = mode == 2 ? cdv(g.k, 256) : cdv(ncols, tc_ntile_cols(mode, pl.variant));
+    pl.bnmax = std::max(pl.bnmax, ip.ntiles == 1 ? ((ncols + 15) & ~15) : tc_ntile_cols(mode, pl.variant));
     if (mode == 0) {
       ip.mtiles = cdv(Mout, kTcBM);
       if (g.x_dtype == PNN_DT_F32) esz = 4;
@@ -208,7 +196,7 @@ int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
       }
       pl.total += base * ip.splits;
     }
-    if (pl.variant == 1) ip.maps = take(4 * 128);
+    if (pl.variant == 1) ip.maps = take(3 * 128);
   }
   pl.init_bytes = cur;
   for (int i = 0; i < n; ++i) {
@@ -232,10 +220,6 @@ int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
     }
   }
   if (pl.variant == 1 && mode != 2) pl.raw = kTcBM * 64 * esz;
-  if (pl.eslot > 0 && conv_tma_stage_count(mode, pl.bnmax, pl.raw, pl.eslot) < 2) {
-    pl.eslot = 0;  // no room for the slots: the epilogues read from global memory
-    for (auto& ip : pl.in) ip.erb = 0;
-  }
   pl.bytes = cur;
   return PNN_OK;
 }
@@ -287,7 +271,7 @@ int conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void
     c.B = g.batch; c.H = g.h; c.W = g.w; c.C = g.c; c.P = ip.P; c.Q = ip.Q; c.K = g.k;
     c.R = g.ksize; c.S = g.ksize; c.stride = g.stride; c.pad = ip.pad;
     c.mtiles = ip.mtiles; c.ntiles = ip.ntiles;
-    c.ntile_w = ip.ntw ? ip.ntw : tc_ntile_cols(mode, pl.variant);
+    c.ntile_w = tc_ntile_cols(mode, pl.variant);
     c.mtile_rows = tc_tile_rows(mode, pl.variant, g.c);
     c.op_bf16 = 1;
     const int64_t Mout = (int64_t)g.batch * ip.P * ip.Q, Min = (int64_t)g.batch * g.h * g.w;
@@ -321,13 +305,13 @@ int conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void
       uint8_t* m = at(ip.maps);
       int e = 0;
       if (mode == 0) {
-        const int bn = ip.ntiles == 1 ? ((g.k + 15) & ~15) : ip.ntw;
+        const int bn = ip.ntiles == 1 ? ((g.k + 15) & ~15) : tc_ntile_cols(0, 1);
         e = encode_tensor_map_2d(m, g.x, g.x_dtype == PNN_DT_BF16, g.c, Min, std::min(g.c, 64), kTcBM, 0, &why);
         if (!e) e = encode_tensor_map_2d(m + 128, g.wt, true, rsc, g.k, 64, bn, 128, &why);
         if (!e) e = encode_tensor_map_2d(m + 256, g.y, g.y_dtype == PNN_DT_BF16, g.k, Mout, 16, 32,
                                          g.y_dtype == PNN_DT_BF16 ? 32 : 64, &why);
       } else if (mode == 1) {
-        const int bn = ip.ntiles == 1 ? ((g.c + 15) & ~15) : ip.ntw;
+        const int bn = ip.ntiles == 1 ? ((g.c + 15) & ~15) : tc_ntile_cols(1, 1);
         e = encode_tensor_map_2d(m, g.dy, false, g.k, Mout, std::min(g.k, 64), kTcBM, 0, &why);
         if (!e) e = encode_tensor_map_2d(m + 128, ws + ip.wt, true, g.ksize * g.ksize * g.k, g.c, 64, bn, 128, &why);
         if (!e) e = encode_tensor_map_2d(m + 256, g.dx, false, g.c, Min, 16, 32, 64, &why);
@@ -335,15 +319,6 @@ int conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void
         const WgBoxes bx = wg_boxes(g.c, g.k, g.w, ip.pad, g.x_dtype == PNN_DT_BF16);
         e = encode_tensor_map_2d(m, g.x, g.x_dtype == PNN_DT_BF16, g.c, Min, bx.cwx, bx.hrows, 0, &why);
         if (!e) e = encode_tensor_map_2d(m + 128, g.dy, false, g.k, Mout, g.k, 64, 0, &why);
-      }
-      if (!e && ip.erb) {
-        const bool ebf = mode == 0 ? g.res_dtype == PNN_DT_BF16 : g.x_dtype == PNN_DT_BF16;
-        const int64_t rows = mode == 0 ? Mout : Min;
-        const int cols = mode == 0 ? g.k : g.c;
-        e = encode_tensor_map_2d(m + 384, mode == 0 ? g.res : g.x, ebf, cols, rows, ip.erb / (ebf ? 2 : 4), kTcBM,
-                                 ip.erb, &why);
-        c.tma_e = ws + ip.maps + 384;
-        c.e_rowbytes = ip.erb;
       }
       if (e) return set_last_error(PNN_ECUDA, why);
       c.tma_a = ws + ip.maps;
@@ -421,7 +396,7 @@ int conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void
   if (e == cudaSuccess && mode == 1)
     e = launch_wtrans(reinterpret_cast<const WtDesc*>(ws + pl.aux_tab), auxts, n, aux_ts.back(), st);
   auto conv_launch = [&]() {
-    if (pl.variant == 1) return launch_conv_tma(mode, tab, tsd, n, pl.total, pl.bnmax, pl.raw, pl.eslot, status, st);
+    if (pl.variant == 1) return launch_conv_tma(mode, tab, tsd, n, pl.total, pl.bnmax, pl.raw, status, st);
     if (mode == 0) return launch_conv_fwd_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
     if (mode == 1) return launch_conv_dgrad_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
     return launch_conv_wgrad_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);

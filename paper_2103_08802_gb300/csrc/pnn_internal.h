@@ -62,14 +62,6 @@ struct ConvDesc {
   const float* bn_mean;
   const float* bn_rstd;
   float* bnb_part;
-  // TMA-fed forward with a residual / data gradient with BN-backward sums:
-  // tensor map over the epilogue's second operand (the residual [pixels][K],
-  // or the BN input h [pixels][C]) with box [e_rowbytes / element size
-  // columns x 128 rows], swizzled over e_rowbytes (32, 64 or 128 bytes); the
-  // producer loads a tile's operand into shared memory ahead of its epilogue.
-  // Null: the epilogue reads the operand from global memory.
-  const void* tma_e;
-  int32_t e_rowbytes;
 };
 
 // out = act( sum_i coef_i * in_i ), optional BN partials of out, NHWC [M][C].
@@ -210,22 +202,10 @@ cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
 // TMA-fed stride-1 forward (mode 0), data-gradient (mode 1) or weight-gradient
 // (mode 2) tensor-core conv; raw_bytes: one pipeline stage's raw slot (the
 // largest over the launch's instances, a multiple of 1024)
-// eslot: bytes of one of the two epilogue-operand slots (a multiple of 1024;
-// 0 = no instance has an epilogue operand map)
 cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
-                            int raw_bytes, int eslot, int32_t* status, cudaStream_t st, int max_ctas = 0);
+                            int raw_bytes, int32_t* status, cudaStream_t st, int max_ctas = 0);
 // whether the TMA-fed kernel of `mode` holds at least two stages of this size
 bool conv_tma_fits(int mode, int bnmax, int raw_bytes);
-// pipeline stages that fit with two epilogue-operand slots of eslot bytes
-int conv_tma_stage_count(int mode, int bnmax, int raw_bytes, int eslot);
-// The epilogue operand of one instance: the box row bytes (32, 64 or 128;
-// 0 = not prefetched: the row of a BN-column tile is not 32 or 64 bytes nor a
-// multiple of 128) and the bytes of its slot (128 rows, 1024-aligned).
-inline int eop_rowbytes(int bn, int esz) {
-  const int b = bn * esz;
-  return (b == 32 || b == 64 || b == 128) ? b : (b % 128 == 0 ? 128 : 0);
-}
-inline int eop_slot_bytes(int bn, int esz) { return ((bn * esz * 128) + 1023) & ~1023; }
 // record a message for pnn_last_error(NULL) and return `code`
 int set_last_error(int code, const char* msg);
 // streaming multiprocessors of the current device, queried once per device

@@ -95,7 +95,6 @@ struct POp {
   int addv[2] = {-1, -1};                    // BNB_APPLY: extra gradients added into dh
   int splits = 1, pix_per_split = 0;
   int bn_fuse = -1;                          // TMA dgrad: norm whose BN-backward partials the epilogue writes
-  int ntw = 0;                               // tensor-core conv: N columns of a tile when not the default
   size_t scratch = 0;                        // wgrad partial buffer offset
   int tiles = 0, mtiles = 0, ntiles = 0;
   int head = 0;
@@ -111,7 +110,6 @@ struct Launch {
   int shape[6];         // first op: conv (C_in, C_out, k, stride, H_out, W_out); else (C, H, W, 0, 0, 0)
   int esz = 4;          // TMA-fed conv: largest element size of the A sources
   int raw = 0;          // TMA-fed conv: raw slot bytes of one stage
-  int eslot = 0;        // TMA-fed forward / data gradient: bytes of one epilogue-operand slot (0 = none)
   int block = -1;       // fine forward / backward: position of the layer in its segment
 };
 
@@ -608,14 +606,6 @@ struct pnn_net {
         if (fuse) {
           ops[wr].bn_fuse = f.norm;
           norms[f.norm].fused_tiles = ops[wr].mtiles;
-          // 64-column tiles when the BN input is bf16 and wider than that:
-          // the epilogue then prefetches a tile of it (128 rows x 64) into
-          // shared memory beside two pipeline stages
-          if (n.C > 64 && vals[n.h].dt == DT_BF16) {
-            ops[wr].ntw = 64;
-            ops[wr].ntiles = cdiv(n.C, 64);
-            ops[wr].tiles = ops[wr].mtiles * ops[wr].ntiles;
-          }
         } else {
           new_op(L, r);
         }
@@ -1170,7 +1160,6 @@ int pnn_net::build_tables() {
       std::vector<uint8_t> tab;
       std::vector<int> tstart;
       int total = 0;
-      int eslot_need = 0;  // largest epilogue-operand slot of the group's TMA-fed instances
       auto add = [&](const void* d, size_t sz, int tiles) {
         size_t o = tab.size();
         tab.resize(o + sz);
@@ -1195,7 +1184,7 @@ int pnn_net::build_tables() {
             c.B = B; c.H = iv.H; c.W = iv.W; c.C = iv.C; c.P = ov.H; c.Q = ov.W; c.K = ov.C;
             c.R = o.k; c.S = o.k; c.stride = o.stride; c.pad = o.pad;
             c.mtiles = o.mtiles; c.ntiles = o.ntiles;
-            c.ntile_w = o.ntw ? o.ntw : tc_ntile_w(o.kind, o.variant);
+            c.ntile_w = tc_ntile_w(o.kind, o.variant);
             c.mtile_rows = tc_mtile_rows(o.kind, o.variant, iv.C);
             c.op_bf16 = act_dt == DT_BF16 && ((o.kind != K_DGRAD && o.kind != K_WGRAD) || !opt.grad_fp32);
             if (o.kind == K_DGRAD_TC) c.w = (const char*)(ws + off_wt) + params[o.w].off * 2;
@@ -1207,25 +1196,9 @@ int pnn_net::build_tables() {
               const void* a_src = fwd ? c.x.ptr : (const void*)P<float>(gptr(o.out));
               const bool a_bf16 = fwd && c.x.dt == DT_BF16;
               const int64_t a_rows = fwd ? (int64_t)B * iv.H * iv.W : (int64_t)B * ov.H * ov.W;
-              const int bn = o.ntiles == 1 ? ((ncols + 15) & ~15) : c.ntile_w;
-              // a third map over the output for the epilogue's TMA stores; a
-              // fourth over the epilogue's second operand (forward: the
-              // residual; data gradient with the BN-backward sums: the BN input)
-              const void* e_src = nullptr;
-              bool e_bf = false, has_e = false;
-              int64_t e_rows = 0;
-              int e_cols = 0;
-              if (fwd && o.res >= 0) {
-                has_e = true;
-                e_src = ws ? ws + vals[o.res].off : nullptr; e_bf = vals[o.res].dt == DT_BF16;
-                e_rows = (int64_t)B * ov.H * ov.W; e_cols = ov.C;
-              } else if (!fwd && o.bn_fuse >= 0) {
-                has_e = true;
-                e_src = c.x.ptr; e_bf = vals[vals[o.in].virt ? vals[o.in].src : o.in].dt == DT_BF16;
-                e_rows = (int64_t)B * iv.H * iv.W; e_cols = iv.C;
-              }
-              const int erb = has_e ? eop_rowbytes(bn, e_bf ? 2 : 4) : 0;
-              CUtensorMap maps[4];
+              const int bn = o.ntiles == 1 ? ((ncols + 15) & ~15) : tc_ntile_w(o.kind, o.variant);
+              // a third map over the output for the epilogue's TMA stores
+              CUtensorMap maps[3];
               memset(maps, 0, sizeof maps);
               if (ws) {
                 int r = encode_map(&maps[0], a_src, a_bf16, ch, a_rows, std::min(ch, 64), kTcBM, 0);
@@ -1235,19 +1208,12 @@ int pnn_net::build_tables() {
                                  ov.dt == DT_BF16 ? 32 : 64);
                 if (!r && !fwd)  // data gradient: dx [pixels][C] fp32, stored or reduce-added
                   r = encode_map(&maps[2], P<float>(gptr(o.in)), false, iv.C, (int64_t)B * iv.H * iv.W, 16, 32, 64);
-                if (!r && erb)
-                  r = encode_map(&maps[3], e_src, e_bf, e_cols, e_rows, erb / (e_bf ? 2 : 4), kTcBM, erb);
                 if (r) return r;
               }
               const size_t mo = put(maps, sizeof maps);
               c.tma_a = ws ? ws + tables_off + mo : nullptr;
               c.tma_b = ws ? ws + tables_off + mo + sizeof(CUtensorMap) : nullptr;
               c.tma_y = ws ? ws + tables_off + mo + 2 * sizeof(CUtensorMap) : nullptr;
-              if (erb) {
-                c.tma_e = ws ? ws + tables_off + mo + 3 * sizeof(CUtensorMap) : nullptr;
-                c.e_rowbytes = erb;
-                eslot_need = std::max(eslot_need, eop_slot_bytes(bn, e_bf ? 2 : 4));
-              }
             }
             if (o.kind == K_WGRAD_TC && o.variant == 1) {
               // activation halo box [hrows][cwx] (its dtype), gradient box [64][K] fp32
@@ -1426,8 +1392,7 @@ int pnn_net::build_tables() {
       for (int id : g.ops)
         if (ops[id].kind == K_CONV_FWD_TC || ops[id].kind == K_DGRAD_TC || ops[id].kind == K_WGRAD_TC) {
           const int K = ops[id].kind == K_DGRAD_TC ? vals[ops[id].in].C : vals[ops[id].out].C;
-          L.aux = std::max(L.aux, ops[id].ntiles == 1 ? ((K + 15) & ~15)
-                                                     : (ops[id].ntw ? ops[id].ntw : tc_ntile_w(ops[id].kind, ops[id].variant)));
+          L.aux = std::max(L.aux, ops[id].ntiles == 1 ? ((K + 15) & ~15) : tc_ntile_w(ops[id].kind, ops[id].variant));
           if (ops[id].kind == K_DGRAD_TC) L.esz = 4;
           else if (ops[id].kind == K_CONV_FWD_TC) {
             const int src = vals[ops[id].in].virt ? vals[ops[id].in].src : ops[id].in;
@@ -1440,20 +1405,6 @@ int pnn_net::build_tables() {
           }
         }
       if (g.kind == K_CONV_FWD_TC || g.kind == K_DGRAD_TC) L.raw = kTcBM * 64 * L.esz;
-      if ((g.kind == K_CONV_FWD_TC || g.kind == K_DGRAD_TC) && g.variant == 1 && eslot_need > 0) {
-        // two epilogue-operand slots, if two pipeline stages still fit;
-        // otherwise every epilogue of the launch reads its operand from
-        // global memory
-        if (conv_tma_stage_count(g.kind == K_CONV_FWD_TC ? 0 : 1, L.aux, L.raw, eslot_need) >= 2) {
-          L.eslot = eslot_need;
-        } else {
-          for (size_t i = 0; i < g.ops.size(); ++i) {
-            ConvDesc* cd = reinterpret_cast<ConvDesc*>(tab.data() + i * sizeof(ConvDesc));
-            cd->tma_e = nullptr;
-            cd->e_rowbytes = 0;
-          }
-        }
-      }
       for (int id : g.ops) op_cost(ops[id], L.flops, L.bytes);
       tstart.push_back(total);
       L.table_off = put(tab.data(), tab.size());
@@ -1585,21 +1536,21 @@ int pnn_net::run_phase(int p, cudaStream_t st, int cap) {
       case K_CONV_FWD: e = launch_conv_fwd_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, st); break;
       case K_CONV_FWD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(0, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, L.eslot,
-                                  P<int32_t>(status_off), st, cap)
+                ? launch_conv_tma(0, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
+                                  st, cap)
                 : launch_conv_fwd_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), st, cap);
         break;
       case K_DGRAD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(1, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, L.eslot,
-                                  P<int32_t>(status_off), st, cap)
+                ? launch_conv_tma(1, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
+                                  st, cap)
                 : launch_conv_dgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
                                        st, cap);
         break;
       case K_WGRAD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(2, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, 0,
-                                  P<int32_t>(status_off), st, cap)
+                ? launch_conv_tma(2, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
+                                  st, cap)
                 : launch_conv_wgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
                                        st, cap);
         break;

@@ -46,16 +46,29 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 // A waiting thread may be suspended for up to kSuspendNs inside one try_wait
 // (it resumes as soon as the phase completes), so waiting warps leave the
 // issue slots to the working ones.
-constexpr uint32_t kSuspendNs = 20000;
+#ifndef PNN_SUSPEND_NS
+#define PNN_SUSPEND_NS 20000
+#endif
+constexpr uint32_t kSuspendNs = PNN_SUSPEND_NS;
 __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
   uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity), "r"(kSuspendNs)
-      : "memory");
+  if (kSuspendNs > 0) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(kSuspendNs)
+        : "memory");
+  } else {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+  }
   return ok != 0;
 }
 // bounded wait: false after limit_ns or when another thread of the CTA aborted
