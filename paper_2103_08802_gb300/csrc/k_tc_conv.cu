@@ -884,35 +884,48 @@ __device__ __forceinline__ void conv_tc_body(const ConvDesc* __restrict__ tab, c
 // data gradient: the negated offset), so one 2-D tensor-map box [128 rows x
 // min(channels, 64)] per tap brings a k-step's raw operand; rows that fall in
 // the zero padding are zeroed by the transform, which knows each row's
-// pixel.  Channel counts are 8, 16, 32, 64 or multiples of 64.  Roles (14
-// warps, one CTA per SM, persistent):
-//   warp 13     producer: waits for a free stage, issues the A boxes into the
+// pixel.  Channel counts are 8, 16, 32, 64 or multiples of 64.  Roles (one
+// CTA per SM, persistent; the warp counts below):
+//   producer    one thread: waits for a free stage, issues the A boxes into the
 //               stage's raw slot and the weight box (128-byte swizzle, the
 //               MMA's layout) into its operand slot, all completing on one
 //               transaction mbarrier;
-//   warps 0-3   transform: thread = A row; converts the row's 8 chunks of 8
-//               K elements -- BN scale/shift + ReLU of the producing layer
-//               (forward; staged in shared memory per instance), bf16,
-//               padding mask -- from the raw slot into the swizzled operand;
-//   warp 12     TMEM owner and MMA issuer;
-//   warps 4-11  epilogue: two groups of four warps (one per TMEM lane
-//               quarter); each group owns one of the two accumulators and
-//               drains every other tile, so two tiles drain at once.
+//   transform   converts each A row's chunks of 8 K elements -- BN
+//               scale/shift + ReLU of the producing layer (forward; staged in
+//               shared memory per instance), bf16, padding mask -- from the
+//               raw slot into the swizzled operand;
+//   MMA         TMEM owner and MMA issuer;
+//   epilogue    groups of four warps (one per TMEM lane quarter); each group
+//               owns one accumulator and drains every n-th tile.
 // Every wait is bounded; the producer drains its copies before the CTA exits.
-constexpr int kTmaThreads = 14 * 32;
-// transform / epilogue split of warps 0-11 (XW transform warps): the forward
-// (wide outputs) has the heavy epilogue (residual, statistics; 4 + 8 warps);
-// the gradients have the heavy transform (8 + 4 warps)
-template <int MODE, int XW>
+// Warp roles: XW transform warps, NE epilogue warps (NE / 4 groups, each
+// owning one TMEM accumulator and draining every (NE/4)-th tile), then the
+// MMA warp and the producer warp; at most 16 warps (four per SM
+// sub-partition, so that each thread keeps 128 registers).  Variant W = 0:
+// the forward and the data gradient 4 + 8 (two tiles drain at once), the
+// weight gradient (heavy transform, small epilogue) 8 + 4 with two
+// accumulators for its one group.  W = 1, for launches whose every tile is
+// one k-step (1x1 convs of at most 64 input channels, where the transform has
+// little to do and the epilogue -- residual, statistics, BN-backward sums,
+// the output -- bounds the kernel): 2 + 12, three tiles drain at once.
+__host__ __device__ constexpr int tma_xw(int mode, int w) { return mode == 2 ? 8 : (w ? 2 : 4); }
+__host__ __device__ constexpr int tma_ne(int mode, int w) { return mode == 2 ? 4 : (w ? 12 : 8); }
+__host__ __device__ constexpr int tma_warps(int mode, int w) { return tma_xw(mode, w) + tma_ne(mode, w) + 2; }
+template <int MODE, int W>
 struct TmaRoles {
-  static constexpr int kTransformWarps = XW;
-  static constexpr int kEpiWarps = 12 - kTransformWarps;
+  static constexpr int kTransformWarps = tma_xw(MODE, W);
+  static constexpr int kEpiWarps = tma_ne(MODE, W);
   static constexpr int kTransform = 32 * kTransformWarps;
   static constexpr int kEpilogue = 32 * kEpiWarps;
   static constexpr int kEpiWarp0 = kTransformWarps;
+  static constexpr int kMmaWarp = kTransformWarps + kEpiWarps;
+  static constexpr int kProducerWarp = kMmaWarp + 1;
+  static constexpr int kThreads = 32 * (kProducerWarp + 1);
+  static constexpr int kGroups = kEpiWarps / 4;
+  static constexpr int kAcc = kGroups > 1 ? kGroups : 2;  // TMEM accumulators
 };
-constexpr int kTmaMmaWarp = 12;
-constexpr int kTmaProducerWarp = 13;
+constexpr int kTmaMaxGroups = 3;
+constexpr int kTmaMaxAcc = 3;
 constexpr int kTmaMaxStages = 8;
 constexpr int kTmaMaxC = 512;         // channels of a BN-transformed source
 constexpr int kTmaSmemBudget = 227 * 1024;
@@ -930,13 +943,12 @@ struct TmaShared {
   uint64_t tma_full[kTmaMaxStages];
   uint64_t op_full[kTmaMaxStages];
   uint64_t op_empty[kTmaMaxStages];
-  uint64_t tfull[2];
-  uint64_t tempty[2];
+  uint64_t tfull[kTmaMaxAcc];
+  uint64_t tempty[kTmaMaxAcc];
   uint64_t drain;
   uint32_t tmem;
   int abort_flag;
-  int epi_ok[8];
-  float red[2][4][256][2];  // per epilogue group
+  int epi_ok[4 * kTmaMaxGroups];
   float scale[kTmaMaxC];
   float shift[kTmaMaxC];
 };
@@ -946,10 +958,14 @@ struct TmaShared {
 // then B (bnmax rows).
 __host__ __device__ constexpr int tma_amult(int mode) { return mode == 2 ? 2 : 1; }
 __host__ __device__ constexpr int tma_op_bytes(int mode, int bnmax) { return tma_amult(mode) * kABytes + bnmax * 128; }
-// forward / data gradient: two 2 KB output staging tiles per epilogue warp
-// (12 - XW warps) after the rings
-constexpr int kTmaYStage = 8 * 2 * 2048;
-__host__ __device__ constexpr int tma_extra(int mode, int xw) { return mode == 2 ? 0 : (12 - xw) * 2 * 2048; }
+// after the rings: (forward / data gradient) two 2 KB output staging tiles
+// per epilogue warp, then each epilogue group's column-reduction scratch
+// (float [4][256][2])
+constexpr int kTmaRedBytes = 4 * 256 * 2 * 4;
+__host__ __device__ constexpr int tma_ystage(int mode, int w) { return mode == 2 ? 0 : tma_ne(mode, w) * 2 * 2048; }
+__host__ __device__ constexpr int tma_extra(int mode, int w) {
+  return tma_ystage(mode, w) + (tma_ne(mode, w) / 4) * kTmaRedBytes;
+}
 __host__ __device__ inline int tma_stages(int mode, int bnmax, int raw_bytes, int extra) {
   const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - extra;
   int s = avail / (raw_bytes + tma_op_bytes(mode, bnmax));
@@ -1199,33 +1215,36 @@ __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDe
   }
 }
 
-template <int MODE, int XW>
+template <int MODE, int W>
 __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, const int* __restrict__ tstart,
                                               int ninst, int total, int bnmax, int raw_bytes, int32_t* status) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw0 = smem_u32(smem_raw);
   const uint32_t base = (raw0 + 1023u) & ~1023u;
   uint8_t* const gbase = smem_raw + (base - raw0);
-  const int S = tma_stages(MODE, bnmax, raw_bytes, tma_extra(MODE, XW));
+  using R = TmaRoles<MODE, W>;
+  const int S = tma_stages(MODE, bnmax, raw_bytes, tma_extra(MODE, W));
   const int op_bytes = tma_op_bytes(MODE, bnmax);
   constexpr int kAMult = tma_amult(MODE);
   const uint32_t op_base = base + S * raw_bytes;
   RT(const unsigned long long rt_start = clock64();)
   uint8_t* const ystage0 = gbase + S * (raw_bytes + op_bytes);  // output staging (1024-aligned)
-  TmaShared& sh = *reinterpret_cast<TmaShared*>(ystage0 + tma_extra(MODE, XW));
+  uint8_t* const red0 = ystage0 + tma_ystage(MODE, W);           // per-group reduction scratch
+  TmaShared& sh = *reinterpret_cast<TmaShared*>(ystage0 + tma_extra(MODE, W));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   uint32_t colstride = 32;
   while ((int)colstride < bnmax) colstride <<= 1;
   const uint32_t bufcols = kAMult * colstride;  // one accumulator buffer (two halves for 256-row tiles)
-  const uint32_t ncols = 2 * bufcols;
+  uint32_t ncols = 32;                           // TMEM columns: a power of two >= kAcc buffers
+  while (ncols < R::kAcc * bufcols) ncols <<= 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_u32(&sh.tma_full[s]), 1);
-      mbar_init(smem_u32(&sh.op_full[s]), TmaRoles<MODE, XW>::kTransform);
+      mbar_init(smem_u32(&sh.op_full[s]), R::kTransform);
       mbar_init(smem_u32(&sh.op_empty[s]), 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < R::kAcc; ++b) {
       mbar_init(smem_u32(&sh.tfull[b]), 1);
       mbar_init(smem_u32(&sh.tempty[b]), 128);  // one epilogue group drains a buffer
     }
@@ -1233,14 +1252,14 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     sh.abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == kTmaMmaWarp) tmem_alloc(smem_u32(&sh.tmem), ncols);
+  if (warp == R::kMmaWarp) tmem_alloc(smem_u32(&sh.tmem), ncols);
   fence_before();
   __syncthreads();
   fence_after();
   const uint32_t tmem = sh.tmem;
   volatile int* abort_flag = &sh.abort_flag;
 
-  if (warp == kTmaProducerWarp) {
+  if (warp == R::kProducerWarp) {
     // ================================================= TMA producer
     if (lane == 0) {
       uint32_t g = 0;
@@ -1300,15 +1319,17 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
         mbar_wait_drain(smem_u32(&sh.tma_full[i % S]), (i / S) & 1);
     }
     __syncwarp();
-  } else if (warp < TmaRoles<MODE, XW>::kEpiWarp0) {
+  } else if (warp < R::kEpiWarp0) {
     // ================================================= transform (thread = A row)
     // Control flow is the same for every transform thread (they meet at named
     // barrier 1): a thread whose wait fails raises the abort flag and walks
     // the remaining stages without waiting or working.  With 256 transform
     // threads two share a row (chunks 0-3 and 4-7).
-    const int row = threadIdx.x & 127;
-    constexpr int kRowSplit = TmaRoles<MODE, XW>::kTransform / 128;
-    const int jbeg = (threadIdx.x >> 7) * (8 / kRowSplit), jend = jbeg + 8 / kRowSplit;
+    // 256 threads: two per row; 128: one; 64: each thread two rows (row0, row0 + 64)
+    constexpr int kRowSplit = R::kTransform >= 128 ? R::kTransform / 128 : 1;
+    constexpr int kRPT = R::kTransform >= 128 ? 1 : 128 / R::kTransform;
+    const int row0 = R::kTransform >= 128 ? (threadIdx.x & 127) : threadIdx.x;
+    const int jbeg = R::kTransform >= 128 ? (threadIdx.x >> 7) * (8 / kRowSplit) : 0, jend = jbeg + 8 / kRowSplit;
     uint32_t g = 0;
     bool ok = true;
     const ConvDesc* staged = nullptr;  // instance whose scale/shift sit in shared memory
@@ -1323,37 +1344,44 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       const bool tr = MODE != DGRAD && d.x.scale != nullptr;
       if (tr && staged != T.d) {
         // all transform threads are past the previous tile's stages
-        asm volatile("bar.sync 1, %0;" ::"r"(TmaRoles<MODE, XW>::kTransform) : "memory");
-        for (int c = threadIdx.x; c < d.C; c += TmaRoles<MODE, XW>::kTransform) {
+        asm volatile("bar.sync 1, %0;" ::"r"(R::kTransform) : "memory");
+        for (int c = threadIdx.x; c < d.C; c += R::kTransform) {
           sh.scale[c] = __ldg(d.x.scale + c);
           sh.shift[c] = __ldg(d.x.shift + c);
         }
-        asm volatile("bar.sync 1, %0;" ::"r"(TmaRoles<MODE, XW>::kTransform) : "memory");
+        asm volatile("bar.sync 1, %0;" ::"r"(R::kTransform) : "memory");
         staged = T.d;
       }
       if constexpr (MODE == WGRAD) {
         wgrad_transform_tile(T, d, threadIdx.x, tr, g, ok, S, raw_bytes, op_bytes, gbase, sh RT(, rt_a, rt_b));
         continue;
       }
-      // this row's pixel and which of the R x S taps stay inside the image
-      const int m = T.m0 + row;
-      const bool mvalid = m < T.Mrows;
-      const int qx = m % d.W, py = (m / d.W) % d.H;
-      uint32_t tapok = 0;
-      for (int r = 0; r < d.R; ++r)
-        for (int sx = 0; sx < d.S; ++sx) {
-          const int dy = MODE == FWD ? r - d.pad : d.pad - r, dx = MODE == FWD ? sx - d.pad : d.pad - sx;
-          const bool in = py + dy >= 0 && py + dy < d.H && qx + dx >= 0 && qx + dx < d.W;
-          tapok |= (mvalid && in ? 1u : 0u) << (r * d.S + sx);
-        }
+      // each row's pixel and which of the R x S taps stay inside the image
+      uint32_t tapok[kRPT];
+      int hrow[kRPT];
+#pragma unroll
+      for (int ri = 0; ri < kRPT; ++ri) {
+        const int row = row0 + ri * (128 / kRPT);
+        const int m = T.m0 + row;
+        const bool mvalid = m < T.Mrows;
+        const int qx = m % d.W, py = (m / d.W) % d.H;
+        uint32_t ok_taps = 0;
+        for (int r = 0; r < d.R; ++r)
+          for (int sx = 0; sx < d.S; ++sx) {
+            const int dy = MODE == FWD ? r - d.pad : d.pad - r, dx = MODE == FWD ? sx - d.pad : d.pad - sx;
+            const bool in = py + dy >= 0 && py + dy < d.H && qx + dx >= 0 && qx + dx < d.W;
+            ok_taps |= (mvalid && in ? 1u : 0u) << (r * d.S + sx);
+          }
+        tapok[ri] = ok_taps;
+        // chunk order: cc = j ^ h(row & 7), h = multiplication by x in GF(8);
+        // h(u) and h(u) ^ u are both permutations, so the raw reads (bank
+        // group cc) and the swizzled stores (group cc ^ (row & 7)) of a warp
+        // each spread over all eight bank groups
+        hrow[ri] = (((row & 7) << 1) & 7) ^ ((row & 4) ? 3 : 0);
+      }
       const int taps = d.R * d.S;
       const int per_tap = big ? cdim / 64 : 1;      // k-steps per tap (big)
       const int relu = tr ? d.x.relu : 0;
-      // chunk order: cc = j ^ h(row & 7), h = multiplication by x in GF(8);
-      // h(u) and h(u) ^ u are both permutations, so the raw reads (bank
-      // group cc) and the swizzled stores (group cc ^ (row & 7)) of a warp
-      // each spread over all eight bank groups
-      const int hrow = (((row & 7) << 1) & 7) ^ ((row & 4) ? 3 : 0);
       for (int kt = 0; kt < T.nkt; ++kt, ++g) {
         const int s = g % S;
         RT(const unsigned long long rt0 = clock64();)
@@ -1370,13 +1398,17 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
         const int cb = big ? (kt - tapb * per_tap) * 64 : 0;
         // K elements of this stage the MMA reads (16-element steps)
         const int kread = min(kBK, (T.Kt - kt * kBK + 15) & ~15);
-        TStage st{row, hrow, kread, lg, cdim, tapb, cb, jbeg, jend, tapok, taps, tr, relu};
-        if (xbf) {
-          if (big) transform_stage<true, true>(rawp, A, sh.scale, sh.shift, st);
-          else transform_stage<true, false>(rawp, A, sh.scale, sh.shift, st);
-        } else {
-          if (big) transform_stage<false, true>(rawp, A, sh.scale, sh.shift, st);
-          else transform_stage<false, false>(rawp, A, sh.scale, sh.shift, st);
+#pragma unroll
+        for (int ri = 0; ri < kRPT; ++ri) {
+          const int row = row0 + ri * (128 / kRPT);
+          TStage st{row, hrow[ri], kread, lg, cdim, tapb, cb, jbeg, jend, tapok[ri], taps, tr, relu};
+          if (xbf) {
+            if (big) transform_stage<true, true>(rawp, A, sh.scale, sh.shift, st);
+            else transform_stage<true, false>(rawp, A, sh.scale, sh.shift, st);
+          } else {
+            if (big) transform_stage<false, true>(rawp, A, sh.scale, sh.shift, st);
+            else transform_stage<false, false>(rawp, A, sh.scale, sh.shift, st);
+          }
         }
         RT(const unsigned long long rt2 = clock64(); rt_c += rt2 - rt1;)
         fence_proxy_async();
@@ -1390,7 +1422,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       atomicAdd(&g_tma_cycles[MODE][12], rt_c); atomicAdd(&g_tma_cycles[MODE][13], rt_d);
     })
     if (!ok) { sh.abort_flag = 1; atomicExch(status, 3); }
-  } else if (warp == kTmaMmaWarp) {
+  } else if (warp == R::kMmaWarp) {
     // ================================================= MMA issuer
     if (lane == 0) {
       uint32_t g = 0;
@@ -1400,9 +1432,9 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       RT(unsigned long long rt_acc = 0, rt_full = 0, rt_issue = 0;)
       for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++li) {
         const Tile T = decode<MODE>(tab, tstart, ninst, tile);
-        const int b = li & 1;
+        const int b = li % R::kAcc;
         RT(unsigned long long rt0 = clock64();)
-        if (!mbar_wait(smem_u32(&sh.tempty[b]), ((li >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(smem_u32(&sh.tempty[b]), ((li / R::kAcc) & 1) ^ 1, abort_flag)) { ok = false; break; }
         RT(rt_acc += clock64() - rt0;)
         fence_after();
         const uint32_t tacc = tmem + b * bufcols;
@@ -1445,9 +1477,8 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     }
     __syncwarp();
   } else {
-    // ================================================= epilogue (warps 4-11)
-    using R = TmaRoles<MODE, XW>;
-    constexpr int kGroups = R::kEpiWarps / 4;
+    // ================================================= epilogue
+    constexpr int kGroups = R::kGroups;
     const int ew = warp - R::kEpiWarp0;   // 0 .. kEpiWarps-1
     const int q = warp & 3;               // TMEM lane quarter this warp may access
     const int eg = ew >> 2;               // epilogue group
@@ -1458,9 +1489,9 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     RT(unsigned long long rt_a = 0, rt_b = 0;)
     for (int tile = blockIdx.x + eg * gridDim.x; tile < total; tile += kGroups * gridDim.x, li += kGroups) {
       const Tile T = decode<MODE>(tab, tstart, ninst, tile);
-      const int b = li & 1;
+      const int b = li % R::kAcc;
       RT(const unsigned long long rt0 = clock64();)
-      bool got = mbar_wait(smem_u32(&sh.tfull[b]), (li >> 1) & 1, abort_flag);
+      bool got = mbar_wait(smem_u32(&sh.tfull[b]), (li / R::kAcc) & 1, abort_flag);
       RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
       got = __all_sync(0xffffffffu, got);
       // the group's four warps decide together (they meet at its named barrier)
@@ -1470,13 +1501,14 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       asm volatile("bar.sync %0, 128;" ::"r"(bar) : "memory");
       if (!got) { ok = false; break; }
       fence_after();
-      epilogue<MODE>(T, tmem + b * bufcols, q, lane, sh.red[eg], 0, 16, (ew & 3) * 32 + lane, 128,
+      float(&red)[4][256][2] = *reinterpret_cast<float(*)[4][256][2]>(red0 + eg * kTmaRedBytes);
+      epilogue<MODE>(T, tmem + b * bufcols, q, lane, red, 0, 16, (ew & 3) * 32 + lane, 128,
                      MODE != WGRAD ? ystage0 + ew * 4096 : nullptr, ybuf, bar);
       if (kAMult == 2 && min(T.d->mtile_rows, T.Mrows - T.m0) > kBM) {
         // rows 128-255 of the tile, from the second accumulator half
         Tile T2 = T;
         T2.m0 += kBM;
-        epilogue<MODE>(T2, tmem + b * bufcols + colstride, q, lane, sh.red[eg], 0, 16, (ew & 3) * 32 + lane, 128,
+        epilogue<MODE>(T2, tmem + b * bufcols + colstride, q, lane, red, 0, 16, (ew & 3) * 32 + lane, 128,
                        nullptr, ybuf, bar);
       }
       fence_before();
@@ -1494,7 +1526,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
   }
   fence_before();
   __syncthreads();
-  if (warp == kTmaMmaWarp) {
+  if (warp == R::kMmaWarp) {
     fence_after();
     tmem_dealloc(tmem, ncols);
   }
@@ -1504,21 +1536,32 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
   })
 }
 
-__global__ void __launch_bounds__(kTmaThreads, 1) k_conv_fwd_tma(const ConvDesc* __restrict__ tab,
-                                                                 const int* __restrict__ tstart, int ninst, int total,
-                                                                 int bnmax, int raw_bytes, int32_t* status) {
-  conv_tma_body<FWD, 4>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+__global__ void __launch_bounds__(TmaRoles<FWD, 0>::kThreads, 1) k_conv_fwd_tma(const ConvDesc* __restrict__ tab,
+                                                                         const int* __restrict__ tstart, int ninst,
+                                                                         int total, int bnmax, int raw_bytes,
+                                                                         int32_t* status) {
+  conv_tma_body<FWD, 0>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
-
-__global__ void __launch_bounds__(kTmaThreads, 1) k_conv_dgrad_tma(const ConvDesc* __restrict__ tab,
-                                                                   const int* __restrict__ tstart, int ninst, int total,
-                                                                   int bnmax, int raw_bytes, int32_t* status) {
-  conv_tma_body<DGRAD, 4>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+__global__ void __launch_bounds__(TmaRoles<FWD, 1>::kThreads, 1) k_conv_fwd_tma_w(const ConvDesc* __restrict__ tab,
+                                                                           const int* __restrict__ tstart, int ninst,
+                                                                           int total, int bnmax, int raw_bytes,
+                                                                           int32_t* status) {
+  conv_tma_body<FWD, 1>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
-__global__ void __launch_bounds__(kTmaThreads, 1) k_conv_wgrad_tma(const ConvDesc* __restrict__ tab,
-                                                                   const int* __restrict__ tstart, int ninst, int total,
-                                                                   int bnmax, int raw_bytes, int32_t* status) {
-  conv_tma_body<WGRAD, 8>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+__global__ void __launch_bounds__(TmaRoles<DGRAD, 0>::kThreads, 1) k_conv_dgrad_tma(
+    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes,
+    int32_t* status) {
+  conv_tma_body<DGRAD, 0>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+}
+__global__ void __launch_bounds__(TmaRoles<DGRAD, 1>::kThreads, 1) k_conv_dgrad_tma_w(
+    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes,
+    int32_t* status) {
+  conv_tma_body<DGRAD, 1>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+}
+__global__ void __launch_bounds__(TmaRoles<WGRAD, 0>::kThreads, 1) k_conv_wgrad_tma(
+    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes,
+    int32_t* status) {
+  conv_tma_body<WGRAD, 0>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
 }
 
 // one kernel name per mode (profiler filters and launch lists name the mode)
@@ -1557,25 +1600,27 @@ static cudaError_t launch_mode(ConvKernel kern, const ConvDesc* tab, const int* 
 }
 
 bool conv_tma_fits(int mode, int bnmax, int raw_bytes) {
-  const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - kTmaYStage;
+  const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - tma_extra(mode, 0);
   return avail / (raw_bytes + tma_op_bytes(mode, bnmax)) >= 2;
 }
 
-cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
+cudaError_t launch_conv_tma(int mode, int wide, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
                             int raw_bytes, int32_t* status, cudaStream_t st, int max_ctas) {
   if (total <= 0) return cudaSuccess;
   if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || raw_bytes <= 0 || (raw_bytes & 1023) || mode < 0 || mode > 2)
     return cudaErrorInvalidValue;
-  const int xw = mode == 2 ? 8 : 4;  // transform warps of the mode's kernel
-  auto kern = mode == 0 ? k_conv_fwd_tma : (mode == 1 ? k_conv_dgrad_tma : k_conv_wgrad_tma);
-  cudaError_t e = set_smem_attr_once(4 + mode, reinterpret_cast<const void*>(kern), kTmaSmemBudget);
+  const int w = mode != 2 && wide ? 1 : 0;
+  typedef void (*TmaKernel)(const ConvDesc*, const int*, int, int, int, int, int32_t*);
+  const TmaKernel kern = mode == 0 ? (w ? k_conv_fwd_tma_w : k_conv_fwd_tma)
+                                   : (mode == 1 ? (w ? k_conv_dgrad_tma_w : k_conv_dgrad_tma) : k_conv_wgrad_tma);
+  cudaError_t e = set_smem_attr_once(4 + 2 * mode + w, reinterpret_cast<const void*>(kern), kTmaSmemBudget);
   if (e != cudaSuccess) return e;
   const int sms = device_sm_count();
-  const size_t smem = tma_smem_bytes(mode, bnmax, raw_bytes, tma_extra(mode, xw));
+  const size_t smem = tma_smem_bytes(mode, bnmax, raw_bytes, tma_extra(mode, w));
   if (smem > (size_t)kTmaSmemBudget) return cudaErrorInvalidValue;
   int grid = total < sms ? total : sms;
   if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
-  kern<<<grid, kTmaThreads, smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, status);
+  kern<<<grid, 32 * tma_warps(mode, w), smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, status);
   return cudaGetLastError();
 }
 

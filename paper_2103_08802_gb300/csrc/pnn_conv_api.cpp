@@ -70,7 +70,7 @@ struct InstPlan {
 };
 struct Plan {
   int variant = 0;
-  int bnmax = 16, raw = 0;
+  int bnmax = 16, raw = 0, wide = 0;
   int total = 0;
   size_t tab = 0, ts = 0, status = 0, aux_tab = 0, aux_ts = 0, fin_tab = 0, fin_ts = 0, red_tab = 0, red_ts = 0;
   size_t bytes = 0, init_bytes = 0;  // init_bytes: the prefix copied from the host
@@ -220,6 +220,11 @@ int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
     }
   }
   if (pl.variant == 1 && mode != 2) pl.raw = kTcBM * 64 * esz;
+  // the training step's rule: the wide-epilogue variant when every tile is
+  // one k-step
+  pl.wide = pl.variant == 1 && mode != 2;
+  for (int i = 0; i < n; ++i)
+    if (a[i].ksize * a[i].ksize * (mode == 0 ? a[i].c : a[i].k) > 64) pl.wide = 0;
   pl.bytes = cur;
   return PNN_OK;
 }
@@ -396,7 +401,7 @@ int conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void
   if (e == cudaSuccess && mode == 1)
     e = launch_wtrans(reinterpret_cast<const WtDesc*>(ws + pl.aux_tab), auxts, n, aux_ts.back(), st);
   auto conv_launch = [&]() {
-    if (pl.variant == 1) return launch_conv_tma(mode, tab, tsd, n, pl.total, pl.bnmax, pl.raw, status, st);
+    if (pl.variant == 1) return launch_conv_tma(mode, pl.wide, tab, tsd, n, pl.total, pl.bnmax, pl.raw, status, st);
     if (mode == 0) return launch_conv_fwd_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
     if (mode == 1) return launch_conv_dgrad_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
     return launch_conv_wgrad_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);

@@ -202,7 +202,9 @@ cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
 // TMA-fed stride-1 forward (mode 0), data-gradient (mode 1) or weight-gradient
 // (mode 2) tensor-core conv; raw_bytes: one pipeline stage's raw slot (the
 // largest over the launch's instances, a multiple of 1024)
-cudaError_t launch_conv_tma(int mode, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
+// wide: every tile of the launch is one k-step (the epilogue bounds the
+// kernel): the variant with three epilogue groups and two transform warps
+cudaError_t launch_conv_tma(int mode, int wide, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
                             int raw_bytes, int32_t* status, cudaStream_t st, int max_ctas = 0);
 // whether the TMA-fed kernel of `mode` holds at least two stages of this size
 bool conv_tma_fits(int mode, int bnmax, int raw_bytes);

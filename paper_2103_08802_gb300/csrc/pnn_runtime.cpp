@@ -110,6 +110,7 @@ struct Launch {
   int shape[6];         // first op: conv (C_in, C_out, k, stride, H_out, W_out); else (C, H, W, 0, 0, 0)
   int esz = 4;          // TMA-fed conv: largest element size of the A sources
   int raw = 0;          // TMA-fed conv: raw slot bytes of one stage
+  int wide = 0;         // TMA-fed forward / data gradient: every tile one k-step (the wide-epilogue variant)
   int block = -1;       // fine forward / backward: position of the layer in its segment
 };
 
@@ -1405,6 +1406,14 @@ int pnn_net::build_tables() {
           }
         }
       if (g.kind == K_CONV_FWD_TC || g.kind == K_DGRAD_TC) L.raw = kTcBM * 64 * L.esz;
+      if ((g.kind == K_CONV_FWD_TC || g.kind == K_DGRAD_TC) && g.variant == 1) {
+        L.wide = 1;
+        for (int id : g.ops) {
+          const POp& o = ops[id];
+          const int ch = o.kind == K_CONV_FWD_TC ? vals[o.in].C : vals[o.out].C;  // channels of the A source
+          if (o.k * o.k * ch > 64) L.wide = 0;
+        }
+      }
       for (int id : g.ops) op_cost(ops[id], L.flops, L.bytes);
       tstart.push_back(total);
       L.table_off = put(tab.data(), tab.size());
@@ -1536,20 +1545,20 @@ int pnn_net::run_phase(int p, cudaStream_t st, int cap) {
       case K_CONV_FWD: e = launch_conv_fwd_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, st); break;
       case K_CONV_FWD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(0, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
+                ? launch_conv_tma(0, L.wide, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
                                   st, cap)
                 : launch_conv_fwd_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), st, cap);
         break;
       case K_DGRAD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(1, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
+                ? launch_conv_tma(1, L.wide, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
                                   st, cap)
                 : launch_conv_dgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
                                        st, cap);
         break;
       case K_WGRAD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(2, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
+                ? launch_conv_tma(2, L.wide, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
                                   st, cap)
                 : launch_conv_wgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
                                        st, cap);
