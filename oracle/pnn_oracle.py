@@ -39,7 +39,10 @@ operand (input activation, weight, and in the backward pass the output
 gradient), and every stored convolution / pooling output that is not
 followed by a residual add.  This makes the floating-point decisions of the
 forward pass (ReLU masks, maxpool argmax) use the kernel's precision; all
-arithmetic stays float64.
+arithmetic stays float64.  A description with "residual_stream": "bf16" also
+rounds the residual-stream values the library then stores in bf16: every
+residual block's output, r_j, rt_j, the delta form's x_{j+1} + rt_j, and
+ytilde.
 """
 from __future__ import annotations
 
@@ -299,9 +302,13 @@ class _Layer:
     linear = False
     bf16 = False      # precision model (see the module docstring)
     store_q = True    # this conv's output is stored (rounded) on its own
+    stream_q = False  # residual-stream values (block outputs) are stored in bf16
 
     def _q(self, a):
         return round_bf16(a) if self.bf16 else a
+
+    def _sq(self, a):
+        return round_bf16(a) if self.stream_q else a
 
     def _bn(self, h, g, b):
         if self.linear:
@@ -396,7 +403,7 @@ class Basic(_Layer):
         h2, k2 = self.c2.forward(a1, P[3:4])
         z2, b2 = self._bn(h2, P[4], P[5])
         s = z2 + x
-        return self._relu(s), (k1, z1, b1, k2, b2, s)
+        return self._sq(self._relu(s)), (k1, z1, b1, k2, b2, s)
 
     def backward(self, dout, P, cache, need_dx=True):
         k1, z1, b1, k2, b2, s = cache
@@ -446,7 +453,7 @@ class Bottleneck(_Layer):
             sc, kp = self.cp.forward(a1, P[9:10])
         else:
             sc, kp = x, None
-        return h3 + sc, (b1, z1, k1, b2, z2, k2, b3, z3, k3, kp)
+        return self._sq(h3 + sc), (b1, z1, k1, b2, z2, k2, b3, z3, k3, kp)
 
     def backward(self, dout, P, cache, need_dx=True):
         b1, z1, k1, b2, z2, k2, b3, z3, k3, kp = cache
@@ -497,7 +504,7 @@ class CoarseRU(_Layer):
             sc, kp = self.cp.forward(a1, P[6:7])
         else:
             sc, kp = x, None
-        return h2 + sc, (b1, z1, k1, b2, z2, k2, kp)
+        return self._sq(h2 + sc), (b1, z1, k1, b2, z2, k2, kp)
 
     def backward(self, dout, P, cache, need_dx=True):
         b1, z1, k1, b2, z2, k2, kp = cache
@@ -515,7 +522,7 @@ class CoarseRU(_Layer):
         return dx, [dg1, db1, dw1, dg2, db2, dw2] + grads_p
 
 
-def make_layer(spec, shape, linear=False, bf16=False):
+def make_layer(spec, shape, linear=False, bf16=False, stream_bf16=False):
     c, h, w = shape
     op = spec["op"]
     if op == "conv":
@@ -532,6 +539,7 @@ def make_layer(spec, shape, linear=False, bf16=False):
         raise ValueError(op)
     L.linear = linear
     L.bf16 = bf16
+    L.stream_q = bf16 and stream_bf16
     for sub in ("conv", "c1", "c2", "c3", "cp"):
         if getattr(L, sub, None) is not None:
             getattr(L, sub).linear = linear
@@ -542,11 +550,11 @@ def make_layer(spec, shape, linear=False, bf16=False):
 class Stack:
     """A sequence of layers with a contiguous slice of the parameter vector."""
 
-    def __init__(self, specs, shape, linear=False, bf16=False):
+    def __init__(self, specs, shape, linear=False, bf16=False, stream_bf16=False):
         self.layers = []
         self.in_shape = tuple(shape)
         for s in specs:
-            L = make_layer(s, shape, linear, bf16)
+            L = make_layer(s, shape, linear, bf16, stream_bf16)
             self.layers.append(L)
             shape = L.out_shape
         self.out_shape = tuple(shape)
@@ -680,6 +688,10 @@ class ParaNet:
         self.desc = desc
         self.mode = desc.get("correction", "residual")
         q = precision == "bf16"
+        # the residual stream (block outputs, correction tensors) stored in
+        # bf16 as well: a storage policy of the bf16 path
+        sq = q and desc.get("residual_stream", "fp32") == "bf16"
+        self.sq = (lambda a: round_bf16(a)) if sq else (lambda a: a)
         x_shape = (desc["in_c"], desc["in_h"], desc["in_w"])
         self.stem = Stack(desc["stem"], x_shape, bf16=q)
         segs = desc["segments"]
@@ -689,7 +701,7 @@ class ParaNet:
         shape = self.stem.out_shape
         start = 0
         for n in segs:
-            st = Stack(desc["body"][start:start + n], shape, linear_body, q)
+            st = Stack(desc["body"][start:start + n], shape, linear_body, q, sq)
             self.fine.append(st)
             shape = st.out_shape
             start += n
@@ -699,7 +711,7 @@ class ParaNet:
         assert len(desc["coarse"]) == self.N - 1
         self.coarse = []
         for j in range(self.N - 1):
-            st = Stack(desc["coarse"][j], self.X[j + 1], linear_body, q)
+            st = Stack(desc["coarse"][j], self.X[j + 1], linear_body, q, sq)
             assert st.out_shape == self.X[j + 2], (j, st.out_shape, self.X[j + 2])
             self.coarse.append(st)
         self.head = Head(desc["head"], self.X[self.N], desc["classes"])
@@ -777,23 +789,24 @@ class ParaNet:
             ys.append(yj)
             fc.append(c2)
         # coarse network, eq:correct
-        r = [ys[j] - xs[j + 1] for j in range(N - 1)] + [np.zeros_like(ys[N - 1])]
+        sq = self.sq  # storage rounding of residual-stream values (identity unless bf16)
+        r = [sq(ys[j] - xs[j + 1]) for j in range(N - 1)] + [np.zeros_like(ys[N - 1])]
         rt = [r[0]]
         cc, ccx = [], []
         for j in range(N - 1):
             if self.mode == "residual":
                 f, c = self.coarse[j].forward(rt[j], P[("coarse", j)])
                 cc.append(c)
-                rt.append(r[j + 1] + f)
+                rt.append(sq(r[j + 1] + f))
             else:
                 # F^j(x_{j+1}) first: with running statistics the order of the
                 # two evaluations matters, and this one does not depend on rt_j
                 f0, c0 = self.coarse[j].forward(xs[j + 1], P[("coarse", j)])
-                f1, c1 = self.coarse[j].forward(xs[j + 1] + rt[j], P[("coarse", j)])
+                f1, c1 = self.coarse[j].forward(sq(xs[j + 1] + rt[j]), P[("coarse", j)])
                 cc.append(c1)
                 ccx.append(c0)
-                rt.append(r[j + 1] + f1 - f0)
-        ytilde = ys[N - 1] + rt[N - 1]
+                rt.append(sq(r[j + 1] + f1 - f0))
+        ytilde = sq(ys[N - 1] + rt[N - 1])
         logits, hc = self.head.forward(ytilde, P[("head", 0)])
         loss, dz = softmax_cross_entropy(logits, st["labels"])
         st.update(x=x, xs=xs, ys=ys, r=r, rt=rt, ytilde=ytilde, logits=logits, loss=loss,

@@ -215,7 +215,7 @@ class ParaNet:
     uint8 tensor on `device`."""
 
     def __init__(self, desc, precision=None, correction=None, seed=0, lr=0.1, momentum=0.9,
-                 weight_decay=5e-4, nesterov=True, stream_fp32=True, conv_impl=0, grad_fp32=False, stream=None,
+                 weight_decay=5e-4, nesterov=True, stream_fp32=None, conv_impl=0, grad_fp32=False, stream=None,
                  device="cuda", bind=True, inference=False, bn_momentum=0.1, overlap=0):
         self.lib = load()
         self.desc = desc
@@ -225,6 +225,8 @@ class ParaNet:
         o.precision = PRECISION[precision or desc["precision"]]
         o.correction = CORRECTION[correction or desc.get("correction", "residual")]
         o.seed, o.lr, o.momentum, o.weight_decay = seed, lr, momentum, weight_decay
+        if stream_fp32 is None:  # the description's storage of the residual stream (fp32 if unstated)
+            stream_fp32 = desc.get("residual_stream", "fp32") == "fp32"
         o.nesterov, o.stream_fp32, o.conv_impl = int(nesterov), int(stream_fp32), int(conv_impl)
         o.grad_fp32 = int(grad_fp32)
         o.inference, o.bn_momentum, o.overlap = int(inference), bn_momentum, int(overlap)

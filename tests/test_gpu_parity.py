@@ -223,6 +223,15 @@ def test_bf16_full_batch(idx):
     _measured(reduced(idx), bf16_accum_noise, 3.0, TOL["bf16"]["grad"])
 
 
+@pytest.mark.parametrize("idx", [1, 2, 4])
+def test_bf16_full_batch_bf16_residual_stream(idx):
+    """The residual stream (block outputs, r_j, rt_j, ytilde) stored in bf16:
+    the oracle's bf16 model rounds the same values."""
+    d = reduced(idx)
+    d["residual_stream"] = "bf16"
+    _measured(d, bf16_accum_noise, 3.0, TOL["bf16"]["grad"])
+
+
 def test_bf16_full_batch_delta_mode():
     _measured(reduced(2, correction="delta"), bf16_accum_noise, 3.0, TOL["bf16"]["grad"])
 
@@ -267,10 +276,11 @@ def test_full_depth_fp32(idx, batch):
     _measured(desc, fp32_perturbation_noise, 3.0, TOL["fp32"]["grad"])
 
 
-@pytest.mark.parametrize("idx,batch", [(2, 4), (3, 4), (4, 2)])
-def test_full_depth_bf16(idx, batch):
+@pytest.mark.parametrize("idx,batch,stream", [(2, 4, "fp32"), (3, 4, "fp32"), (4, 2, "fp32"), (4, 2, "bf16")])
+def test_full_depth_bf16(idx, batch, stream):
     """The benchmarked path (tcgen05 kernels, bf16 storage) at full depth."""
     desc = W.config(idx, batch=batch)
+    desc["residual_stream"] = stream
     _measured(desc, bf16_accum_noise, 3.0, TOL["bf16"]["grad"])
 
 
