@@ -51,8 +51,9 @@ def parse():
     ap.add_argument("--config", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-batch", type=int, default=1)
-    ap.add_argument("--stream-fp32", type=int, default=1, choices=[0, 1],
-                    help="keep the residual stream and correction tensors in fp32 (1) or bf16 (0)")
+    ap.add_argument("--stream-fp32", type=int, default=None, choices=[0, 1],
+                    help="keep the residual stream and correction tensors in fp32 (1) or bf16 (0); default: "
+                         "the workload's (bf16 for the bf16 workloads)")
     ap.add_argument("--paper-net", default=None, choices=sorted(PAPER_NETS),
                     help="time one of the paper's own constructions instead of --config: Parareal "
                          "ResNet-N of Section 4.2 (batch 128, 3x32x32, 100 classes, the workload of "
@@ -120,7 +121,7 @@ def layer_arm(args, rank):
         return
     torch.cuda.set_device(0)
     B = args.batch or 256
-    sdt = "f32" if args.stream_fp32 else "bf16"
+    sdt = "f32" if args.stream_fp32 == 1 else "bf16"
     insts = layer_instances(args.layer, B, sdt)
     conv, mode = LAYERS[args.layer]
     dev, flops, nbytes = [], 0.0, 0.0
@@ -280,7 +281,7 @@ def config_of(args, desc, world=1, extra=None):
     c = {"workload": desc["name"] + "_b%d_%dpx_c%d" % (B, desc["in_h"], desc["classes"]),
          "batch": B, "input": "3x%dx%d" % (desc["in_h"], desc["in_w"]), "classes": desc["classes"],
          "subnetworks": len(desc["segments"]), "correction": desc.get("correction", "residual"),
-         "residual_stream": "fp32" if args.stream_fp32 else "bf16", "lr": args.lr,
+         "residual_stream": desc.get("residual_stream", "fp32"), "lr": args.lr,
          "tearing": "uniform" if args.tearing == "none" else args.tearing,
          "overlap_sms": args.overlap,
          "parallelism": "replicas" if world > 1 else "single-gpu"}
@@ -490,7 +491,7 @@ def our_arm(args, desc, rank, local, world, dist):
         if args.paper_net or args.config not in (2, 3, 4):
             raise SystemExit("--tearing applies to the ResNet-1001 configurations 2, 3 and 4")
         desc, tearing = retear(args, desc, stream)
-    net = pnn.ParaNet(desc, seed=0, stream=stream, stream_fp32=bool(args.stream_fp32), lr=args.lr,
+    net = pnn.ParaNet(desc, seed=0, stream=stream, lr=args.lr,
                       overlap=args.overlap)
     B = desc["batch"]
     x, labels = W.make_batch(desc, seed=1000 + desc.get("config_index", 0) + rank)
@@ -605,6 +606,8 @@ def main():
         desc = W.config(args.config, batch=args.batch)
     if args.lr is None:
         args.lr = 0.01 if desc["head"]["kind"] == "gap_mlp" else 0.1
+    if args.stream_fp32 is not None and desc["precision"] == "bf16":
+        desc["residual_stream"] = "fp32" if args.stream_fp32 else "bf16"
     if args.impl == "reference":
         reference_arm(args, desc, rank)
     elif args.layer:

@@ -224,11 +224,12 @@ def test_bf16_full_batch(idx):
 
 
 @pytest.mark.parametrize("idx", [1, 2, 4])
-def test_bf16_full_batch_bf16_residual_stream(idx):
-    """The residual stream (block outputs, r_j, rt_j, ytilde) stored in bf16:
-    the oracle's bf16 model rounds the same values."""
+def test_bf16_full_batch_fp32_residual_stream(idx):
+    """The residual stream (block outputs, r_j, rt_j, ytilde) kept in fp32
+    (the bf16 workloads store it in bf16 by default; the oracle's bf16 model
+    rounds whichever values the library stores in bf16)."""
     d = reduced(idx)
-    d["residual_stream"] = "bf16"
+    d["residual_stream"] = "fp32"
     _measured(d, bf16_accum_noise, 3.0, TOL["bf16"]["grad"])
 
 

@@ -65,7 +65,8 @@ def tiny_resnet(batch=8, precision="fp32", correction="residual"):
     2 basic blocks at 16 channels, one conv3x3+BN+ReLU coarse block."""
     return {
         "name": "tiny_resnet_n2", "batch": batch, "in_c": 3, "in_h": 32, "in_w": 32,
-        "classes": 10, "precision": precision, "correction": correction,
+        "classes": 10, "precision": precision,
+        "residual_stream": "bf16" if precision == "bf16" else "fp32", "correction": correction,
         "stem": [conv_bn_relu(16)],
         "body": [basic(16) for _ in range(4)],
         "segments": [2, 2],
@@ -89,7 +90,8 @@ def parareal_vgg16(batch=128, precision="bf16", correction="residual", classes=1
             conv_bn_relu(512), conv_bn_relu(512), conv_bn_relu(512, pool=2)]
     return {
         "name": "parareal_vgg16_n4", "batch": batch, "in_c": 3, "in_h": 32, "in_w": 32,
-        "classes": classes, "precision": precision, "correction": correction,
+        "classes": classes, "precision": precision,
+        "residual_stream": "bf16" if precision == "bf16" else "fp32", "correction": correction,
         "stem": [conv_bn_relu(64)],
         "body": body,
         "segments": [3, 3, 3, 3],
@@ -142,6 +144,7 @@ def parareal_resnet1001(n_seg=4, batch=128, classes=10, hw=32, precision="bf16",
     return {
         "name": f"parareal_resnet{9 * per_stage + 2}_n{n_seg}", "batch": batch, "in_c": 3,
         "in_h": hw, "in_w": hw, "classes": classes, "precision": precision,
+        "residual_stream": "bf16" if precision == "bf16" else "fp32",
         "correction": correction,
         "stem": stem, "body": body, "segments": segments, "coarse": coarse,
         "cj_post": "none",
@@ -184,7 +187,8 @@ def paper_parareal_resnet(n, batch=128, classes=100, hw=32, precision="bf16", co
     stem = [conv(16)] if hw == 32 else [conv_bn_relu(16), conv(16, stride=2)]
     return {
         "name": f"paper_parareal_resnet_n{n}", "batch": batch, "in_c": 3, "in_h": hw, "in_w": hw,
-        "classes": classes, "precision": precision, "correction": correction,
+        "classes": classes, "precision": precision,
+        "residual_stream": "bf16" if precision == "bf16" else "fp32", "correction": correction,
         "stem": stem, "body": body, "segments": [seg] * n, "coarse": coarse,
         "cj_post": "none",
         "head": {"kind": "bn_relu_gap_fc", "hidden": []},
