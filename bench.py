@@ -363,30 +363,85 @@ def retear(args, desc, stream):
     return desc, rec
 
 
-def roofline_of(prof, steps):
-    """Roofline record of the dominant kernel kind of a profiled window of
-    `steps` steps ({kind: (ms, launches, flops, bytes)})."""
+KERNEL_SYMBOL = {("conv_fwd_tc", 0): "k_conv_fwd_tc", ("conv_fwd_tc", 1): "k_conv_fwd_tma",
+                 ("conv_fwd_tc", 2): "k_conv_fwd_tma_w", ("conv_dgrad_tc", 0): "k_conv_dgrad_tc",
+                 ("conv_dgrad_tc", 1): "k_conv_dgrad_tma", ("conv_dgrad_tc", 2): "k_conv_dgrad_tma_w",
+                 ("conv_wgrad_tc", 0): "k_conv_wgrad_tc", ("conv_wgrad_tc", 1): "k_conv_wgrad_tma",
+                 ("bn_bwd_apply", 1): "k_bnb_apply8", ("bn_finalize", 0): "k_bn_fin"}
+
+
+def dram_traffic(symbol):
+    """The ncu record of `symbol` in profiles/dram_traffic.json, if it was taken
+    on the kernel source as it stands (the file names the sha256 of the
+    source file the kernel is built from); else None."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "dram_traffic.json")) as f:
+            rec = json.load(f).get(symbol)
+    except (OSError, ValueError):
+        return None
+    if not rec:
+        return None
+    src = os.path.join(ROOT, "paper_2103_08802_gb300", "csrc", rec["source"])
+    try:
+        with open(src, "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
+                return None
+    except OSError:
+        return None
+    return rec
+
+
+def roofline_of(prof, steps, trace=None):
+    """Roofline record of the dominant kernel: the launch group (kind,
+    variant, first-instance shape, instances) with the largest device time in
+    a profiled window of `steps` steps, from the per-launch trace; without a
+    trace, the dominant kind ({kind: (ms, launches, flops, bytes)})."""
     pk, src = peaks()
-    name, (kms, kn, kfl, kby) = max(prof.items(), key=lambda kv: kv[1][0])
+    if trace:
+        groups = {}
+        for r in trace:
+            k = (r["kind"], r["variant"], r["shape"], r["instances"])
+            g = groups.setdefault(k, [0.0, 0, 0.0, 0.0])
+            g[0] += r["ms"]; g[1] += 1; g[2] += r["flops"]; g[3] += r["bytes"]
+        (kind, variant, shape, inst), (kms, kn, kfl, kby) = max(groups.items(), key=lambda kv: kv[1][0])
+        name = KERNEL_SYMBOL.get((kind, variant), kind)
+        what = {"kind": kind, "variant": variant, "first_instance_shape": list(shape), "instances": inst}
+    else:
+        name, (kms, kn, kfl, kby) = max(prof.items(), key=lambda kv: kv[1][0])
+        kind, what = name, {"kind": name}
     per_launch_ms = kms / kn
     # the bound follows the kernel's algorithmic intensity: below the ridge point
     # (peak FLOP/s / peak B/s) the roof is HBM bandwidth
     ridge = pk["bf16_tflops_sustained"] * 1e12 / (pk["hbm_gbs"] * 1e9)
     intensity = kfl / kby if kby else float("inf")
-    if name.startswith("conv") and not name.endswith("_tc") and intensity >= FP32_ALU_TFLOPS * 1e3 / pk["hbm_gbs"]:
-        bound, peak, unit = "alu", FP32_ALU_TFLOPS, "TFLOP/s"
-        achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
-    elif name.endswith("_tc") and intensity >= ridge:
-        bound, peak, unit = "tensor", pk["bf16_tflops_sustained"], "TFLOP/s"
-        achieved = kfl / kn / (per_launch_ms / 1e3) / 1e12
+    tflops = kfl / kn / (per_launch_ms / 1e3) / 1e12
+    if kind.startswith("conv") and not kind.endswith("_tc") and intensity >= FP32_ALU_TFLOPS * 1e3 / pk["hbm_gbs"]:
+        bound, peak, unit, achieved = "alu", FP32_ALU_TFLOPS, "TFLOP/s", tflops
+    elif kind.endswith("_tc") and intensity >= ridge:
+        bound, peak, unit, achieved = "tensor", pk["bf16_tflops_sustained"], "TFLOP/s", tflops
     else:
         bound, peak, unit = "hbm", pk["hbm_gbs"], "GB/s"
         achieved = kby / kn / (per_launch_ms / 1e3) / 1e9
-    return {"kernel": name, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-            "frac": achieved / peak, "traffic": None, "intensity_flop_per_byte": intensity,
-            "peak_source": (src + (" (hbm_gbs)" if bound == "hbm" else " (bf16_tflops_sustained)"))
-            if bound != "alu" else "derived: 152 SM x 128 FP32 lanes x 2 x 2.07 GHz",
-            "launches_per_step": kn / steps}
+    out = {"kernel": name, **what, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+           "frac": achieved / peak, "traffic": None, "intensity_flop_per_byte": intensity,
+           "peak_source": (src + (" (hbm_gbs)" if bound == "hbm" else " (bf16_tflops_sustained)"))
+           if bound != "alu" else "derived: 152 SM x 128 FP32 lanes x 2 x 2.07 GHz",
+           "launches_per_step": kn / steps, "ms_per_launch": per_launch_ms,
+           "algorithmic_bytes_per_launch": kby / kn, "flops_per_launch": kfl / kn}
+    if kind.endswith("_tc"):
+        # the contraction against the dense bf16 tensor peak as well
+        out["tensor_tflops"] = tflops
+        out["tensor_frac_of_bf16_sustained"] = tflops / pk["bf16_tflops_sustained"]
+    rec = dram_traffic(name)
+    if rec:
+        # DRAM bytes / algorithmic bytes of the same grouped launch measured
+        # alone (bench.py --layer), scaled to this group's algorithmic bytes
+        ratio = rec["dram_bytes"] / rec["algorithmic_bytes"]
+        out["traffic"] = ratio * kby / kn
+        out["traffic_over_algorithmic"] = ratio
+        out["traffic_source"] = rec["command"]
+    return out
 
 
 def infer_arm(args, desc, rank, local, world, dist):
@@ -534,6 +589,7 @@ def our_arm(args, desc, rank, local, world, dist):
         net.backward()
         net.sgd_step()
     prof = net.profile_read()
+    trace = net.profile_trace()
     net.profile(False)
     fw, bw, up = net.launch_counts()
     launches_per_step = fw + bw + up
@@ -561,7 +617,7 @@ def our_arm(args, desc, rank, local, world, dist):
     conv_ms = sum(prof[k][0] for k in CONV_KINDS if k in prof)
     conv_flops = sum(prof[k][2] for k in CONV_KINDS if k in prof)
     total_prof_ms = sum(v[0] for v in prof.values())
-    roofline = roofline_of(prof, args.steps)
+    roofline = roofline_of(prof, args.steps, trace)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         b = args.cpu_sample_batch

@@ -294,8 +294,9 @@ int pnn_profile(pnn_net* net, int32_t enable);
 int pnn_profile_read(pnn_net* net, int32_t kind, double* ms, int64_t* launches, double* flops, double* bytes);
 
 /* One record per kernel launch bracketed since pnn_profile(net, 1), in launch
- * order: kind (as for pnn_kernel_kind_name), variant (tensor-core forward and
- * data-gradient convs: 1 = operands fed by TMA, 0 = gathered by threads),
+ * order: kind (as for pnn_kernel_kind_name), variant (tensor-core convs:
+ * 0 = operands gathered by threads, 1 = fed by TMA, 2 = fed by TMA with the
+ * wide epilogue of one-k-step tiles),
  * step phase (0 preprocessing
  * forward, 1 fine forward, 2 coarse forward, 3 head forward, 4 head backward,
  * 5 coarse backward, 6 correction backward, 7 fine backward, 8

@@ -2420,7 +2420,8 @@ int pnn_profile_trace(pnn_net* n, int32_t max, pnn_trace* out, int32_t* count) {
     pnn_trace& r = out[i];
     float t = 0.f;
     cudaEventElapsedTime(&t, n->pev[2 * i], n->pev[2 * i + 1]);
-    r.kind = L.kind; r.variant = L.variant; r.phase = L.phase; r.instances = L.count; r.tiles = L.total;
+    r.kind = L.kind; r.variant = L.variant + (L.wide ? 1 : 0); r.phase = L.phase; r.instances = L.count;
+    r.tiles = L.total;
     for (int j = 0; j < 6; ++j) r.shape[j] = L.shape[j];
     r.block = L.block;
     r.ms = t; r.flops = L.flops; r.bytes = L.bytes;
