@@ -121,6 +121,8 @@ __global__ void __launch_bounds__(256) k_conv_fwd(const ConvDesc* __restrict__ t
         const int64_t o = (int64_t)m * d.K + co;
         float v = acc[i][j];
         if (d.res) v += ldv(d.res, d.res_dt, o);
+        if (d.res2[0]) v = fmaf(d.res2_c[0], ldv(d.res2[0], d.res2_dt[0], o), v);
+        if (d.res2[1]) v = fmaf(d.res2_c[1], ldv(d.res2[1], d.res2_dt[1], o), v);
         v = rnd(d.y_dt, v);
         stv(d.y, d.y_dt, o, v);
         acc[i][j] = v;
@@ -715,8 +717,8 @@ __global__ void __launch_bounds__(256) k_bnb_apply(const BnBwdDesc* __restrict__
     if (d.relu && !(fmaf(d.scale[c], h, d.shift[c]) > 0.f)) dz = 0.f;
     const float xhat = (h - d.mean[c]) * d.rstd[c];
     float v = d.coef[c * 3] * (dz - d.coef[c * 3 + 1] - xhat * d.coef[c * 3 + 2]);
-    if (d.add0) v += d.add0[o];
-    if (d.add1) v += d.add1[o];
+    if (d.add0) v = fmaf(d.add_c[0], d.add0[o], v);
+    if (d.add1) v = fmaf(d.add_c[1], d.add1[o], v);
     d.dh[o] = d.accumulate ? d.dh[o] + v : v;
   }
 }
@@ -846,8 +848,8 @@ __global__ void __launch_bounds__(256) k_bnb_apply8(const BnBwdDesc* __restrict_
       if (d.relu && !(fmaf(sc[k], h[k], sh[k]) > 0.f)) dz[k] = 0.f;
       const float xhat = (h[k] - mean[k]) * rstd[k];
       out[k] = k0[k] * (dz[k] - k1[k] - xhat * k2[k]);
-      if (d.add0) out[k] += a0[k];
-      if (d.add1) out[k] += a1[k];
+      if (d.add0) out[k] = fmaf(d.add_c[0], a0[k], out[k]);
+      if (d.add1) out[k] = fmaf(d.add_c[1], a1[k], out[k]);
       if (d.accumulate) out[k] += ac[k];
     }
     st8f(d.dh + o, out);

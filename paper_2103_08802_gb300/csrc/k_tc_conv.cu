@@ -428,6 +428,31 @@ __device__ __forceinline__ void res_raw(const ConvDesc& d, int m, int nb, int nc
   }
 }
 
+// The extra addends of a forward epilogue (the parareal correction folded
+// into the conv): v[i] += c_e * res2_e[row m, column nb + i]
+__device__ __forceinline__ void add_extra(const ConvDesc& d, int64_t o, int nb, bool vec, float (&v)[16]) {
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    if (d.res2[e] == nullptr) continue;
+    const float c = d.res2_c[e];
+    if (vec) {
+      float x[16];
+      load8(d.res2[e], d.res2_dt[e], o, x);
+      load8(d.res2[e], d.res2_dt[e], o + 8, x + 8);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) v[i] = fmaf(c, x[i], v[i]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        if (nb + i < d.K)
+          v[i] = fmaf(c,
+                      d.res2_dt[e] == DT_F32 ? reinterpret_cast<const float*>(d.res2[e])[o + i]
+                                             : __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(d.res2[e])[o + i]),
+                      v[i]);
+    }
+  }
+}
+
 // One warp drains TMEM lanes 32q .. 32q+31 (its rows) for the 16-column
 // chunks j_first, j_first + j_step, ...; the ethreads epilogue threads
 // (etid = this thread's index among them) meet at named barrier 2.
@@ -506,6 +531,7 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
                                            : __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(d.res)[o + i]);
           }
         }
+        add_extra(d, o, nb, vec, v);
         RT(if (true) { const unsigned long long cr = clock64(); e5 += cr - c1; })
         if (d.y_dt == DT_BF16) {
 #pragma unroll

@@ -33,6 +33,10 @@ struct ConvDesc {
   // forward epilogue
   void* y; int32_t y_dt;
   const void* res; int32_t res_dt;   // residual added to the output (or null)
+  // up to two more addends, out += res2_c[e] * res2[e] (null: none): the
+  // parareal correction folded into the conv that produces its operand
+  // (r_j = y_j - x_{j+1}, rt_{j+1} = r_{j+1} + F^j(rt_j), ytilde = y_N + rt_N)
+  const void* res2[2]; int32_t res2_dt[2]; float res2_c[2];
   float* stats;                       // per-tile BN partials [mtiles][K][2] = (mean, M2) or null
   // dgrad: dx[B*H*W][C] (fp32) = (accumulate ? dx : 0) + W^T * dy
   float* dx; int32_t accumulate;
@@ -122,6 +126,7 @@ struct BnBwdDesc {
   float* coef;           // [C][3]
   float* dh; int32_t accumulate;     // apply: accumulate into dh; fin: into dgamma/dbeta
   const float* add0; const float* add1;  // apply: extra gradients added into dh (residual paths)
+  float add_c[2];                          // their coefficients
   int64_t M; int32_t C;
   int32_t rows_per_tile, tiles;
   double* scratch; int32_t* counter; int32_t cgroups, nchunk;  // fin: as for BnFinDesc

@@ -59,7 +59,8 @@ struct Value {
   bool grad_written = false;
   int gwrites = 0;           // ops that wrote (stored or accumulated) this gradient
   int gwriter_dgrad = -1;    // the last data-gradient op among them
-  std::vector<int> pending;  // values whose gradient is to be added into this one's
+  // values whose gradient, times a coefficient, is to be added into this one's
+  std::vector<std::pair<int, float>> pending;
 };
 
 struct Norm {
@@ -93,6 +94,9 @@ struct POp {
   int acc = 0;                               // accumulate into the written gradient
   int acc_in[3] = {0, 0, 0};
   int addv[2] = {-1, -1};                    // BNB_APPLY: extra gradients added into dh
+  float addc[2] = {1.f, 1.f};                // ... with these coefficients
+  int res2[2] = {-1, -1};                    // conv forward: more addends of the output
+  float rcoef[2] = {0.f, 0.f};               // ... with these coefficients
   int splits = 1, pix_per_split = 0;
   int bn_fuse = -1;                          // TMA dgrad: norm whose BN-backward partials the epilogue writes
   size_t scratch = 0;                        // wgrad partial buffer offset
@@ -158,6 +162,11 @@ struct pnn_net {
   int x_in = -1;
   std::vector<int> xs, ys, rs, rts;
   int ytilde = -1;
+  // the correction folded into conv epilogues: y_j (j < N) not stored (the
+  // value ys[j] holds r_j = y_j - x_{j+1}), rt_N not stored (rts[N-1] is
+  // ytilde = y_N + rt_N)
+  std::vector<char> y_is_r;
+  bool rtN_in_ytilde = false;
   // head
   int head_in = -1, head_norm = -1;
   std::vector<int> fc_w, fc_b;
@@ -451,12 +460,13 @@ struct pnn_net {
   }
   void flush_pending(std::vector<int>& L, int v, const int* key) {
     // add pending residual gradients of v as plain accumulate ops
-    for (int src : vals[v].pending) {
+    for (const auto& pc : vals[v].pending) {
+      const int src = pc.first;
       POp e;
       e.kind = K_EW_BWD;
       e.in = src;  // dout = grad(src)
       e.out = -1;
-      e.nin = 1; e.ins[0] = v; e.coef[0] = 1.f; e.acc_in[0] = grad_acc(v);
+      e.nin = 1; e.ins[0] = v; e.coef[0] = pc.second; e.acc_in[0] = grad_acc(v);
       e.tiles = cdiv(rows(v), kEwRowsPerTile);
       e.key[0] = key[0]; e.key[1] = key[1]; e.key[2] = 9;
       new_op(L, e);
@@ -469,8 +479,8 @@ struct pnn_net {
   void resolve(std::vector<int>& L, int v, const int* key) {
     Value& x = vals[v];
     if (x.pending.empty()) return;
-    if (!x.grad_written && x.pending.size() == 1) {
-      x.galias = x.pending[0];
+    if (!x.grad_written && x.pending.size() == 1 && x.pending[0].second == 1.f) {
+      x.galias = x.pending[0].first;
       x.grad_written = true;
       x.pending.clear();
       return;
@@ -494,7 +504,9 @@ struct pnn_net {
       case K_CONV_FWD:
       case K_CONV_FWD_TC: {
         const Value& ov = vals[f.out];
-        if (f.res >= 0 && vals[f.res].need_grad) vals[f.res].pending.push_back(f.out);
+        if (f.res >= 0 && vals[f.res].need_grad) vals[f.res].pending.push_back({f.out, 1.f});
+        for (int e = 0; e < 2; ++e)
+          if (f.res2[e] >= 0 && vals[f.res2[e]].need_grad) vals[f.res2[e]].pending.push_back({f.out, f.rcoef[e]});
         POp wg;
         wg.kind = K_WGRAD; wg.in = f.in; wg.out = f.out; wg.w = f.w; wg.k = f.k; wg.stride = f.stride; wg.pad = f.pad;
         const int RSC = f.k * f.k * vals[f.in].C;
@@ -624,7 +636,8 @@ struct pnn_net {
           key(ap, 2);
           // residual gradients pending on h are folded into this apply
           for (int i = 0; i < 2 && !vals[n.h].pending.empty(); ++i) {
-            ap.addv[i] = vals[n.h].pending.back();
+            ap.addv[i] = vals[n.h].pending.back().first;
+            ap.addc[i] = vals[n.h].pending.back().second;
             vals[n.h].pending.pop_back();
           }
           new_op(L, ap);
@@ -693,6 +706,8 @@ struct pnn_net {
           const POp& o = ops[id];
           reads(o.in, li);
           reads(o.res, li);
+          reads(o.res2[0], li);
+          reads(o.res2[1], li);
           for (int i = 0; i < o.nin; ++i) reads(o.ins[i], li);
           if (o.out >= 0 && !vals[o.out].virt && def[o.out] < 0) def[o.out] = li;
         }
@@ -739,7 +754,9 @@ struct pnn_net {
         flops += 2 * macs;
         const double wbytes = (double)ov.C * iv.C * o.k * o.k * wsz;
         if (o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC)
-          bytes += elems(o.in) * esz(o.in) + wbytes + elems(o.out) * esz(o.out) + (o.res >= 0 ? elems(o.res) * esz(o.res) : 0);
+          bytes += elems(o.in) * esz(o.in) + wbytes + elems(o.out) * esz(o.out) + (o.res >= 0 ? elems(o.res) * esz(o.res) : 0) +
+                   (o.res2[0] >= 0 ? elems(o.res2[0]) * esz(o.res2[0]) : 0) +
+                   (o.res2[1] >= 0 ? elems(o.res2[1]) * esz(o.res2[1]) : 0);
         else if (o.kind == K_DGRAD || o.kind == K_DGRAD_TC)
           bytes += elems(o.out) * 4 + wbytes + elems(o.in) * 4 * (o.acc ? 2 : 1);
         else
@@ -848,8 +865,38 @@ int pnn_net::plan(const pnn_desc* d) {
   int cofs = 0;
   rs.assign(std::max(0, N - 1), -1);
   rts.assign(N, -1);
-  for (int j = 0; j + 1 < N; ++j)
-    rs[j] = ew(coarse_f, {ys[j], xs[j + 1]}, {1.f, -1.f}, false, stream_dt, 1000, j);
+  y_is_r.assign(N, 0);
+  rtN_in_ytilde = false;
+  // The correction's sums go into the epilogue of the conv that produces
+  // their first operand when that conv already adds a residual (a
+  // pre-activation bottleneck or coarse RU output) and has room for more
+  // addends: r_j = y_j - x_{j+1} into the last conv of g^j, rt_{j+1} = r_{j+1}
+  // + F^j(rt_j) (delta form: - F^j(x_{j+1})) into the last conv of F^j,
+  // ytilde = y_N + rt_N into the last conv of F^{N-1}.  (Not with the
+  // coarse/fine overlap, which defers a term of the r_{N-1} backward.)
+  const bool fuse = !(opt.overlap > 0 && opt.correction == PNN_CORR_RESIDUAL) && N > 1;
+  auto free_slots = [&](int v) -> int {
+    const int p = v >= 0 ? vals[v].producer : -1;
+    if (!fuse || p < 0) return 0;
+    const POp& o = ops[p];
+    if (!((o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC) && o.out == v && o.res >= 0)) return 0;
+    return (o.res2[0] < 0) + (o.res2[1] < 0);
+  };
+  auto fuse_add = [&](int v, int addend, float c) {
+    POp& o = ops[vals[v].producer];
+    const int e = o.res2[0] < 0 ? 0 : 1;
+    o.res2[e] = addend;
+    o.rcoef[e] = c;
+  };
+  for (int j = 0; j + 1 < N; ++j) {
+    if (free_slots(ys[j]) >= 1) {
+      fuse_add(ys[j], xs[j + 1], -1.f);
+      rs[j] = ys[j];
+      y_is_r[j] = 1;
+    } else {
+      rs[j] = ew(coarse_f, {ys[j], xs[j + 1]}, {1.f, -1.f}, false, stream_dt, 1000, j);
+    }
+  }
   std::vector<int> f0(std::max(0, N - 1), -1);
   if (N > 1) rts[0] = rs[0];
   std::vector<int> coarse_start(N, 0);
@@ -874,18 +921,40 @@ int pnn_net::plan(const pnn_desc* d) {
     if (vals[out].C != std::get<0>(Xshape[j + 2]) || vals[out].H != std::get<1>(Xshape[j + 2]))
       return fail(PNN_EINVAL, "coarse block output is not X_{j+1}");
     if (!delta) {
-      rts[j + 1] = (j + 1 < N - 1) ? ew(coarse_f, {rs[j + 1], out}, {1.f, 1.f}, false, stream_dt, 2000 + 100 * j, 98)
-                                   : out;
+      if (j + 1 == N - 1) {
+        rts[j + 1] = out;
+      } else if (free_slots(out) >= 1) {
+        fuse_add(out, rs[j + 1], 1.f);
+        rts[j + 1] = out;
+      } else {
+        rts[j + 1] = ew(coarse_f, {rs[j + 1], out}, {1.f, 1.f}, false, stream_dt, 2000 + 100 * j, 98);
+      }
     } else {
-      if (j + 1 < N - 1)
-        rts[j + 1] = ew(coarse_f, {rs[j + 1], out, f0[j]}, {1.f, 1.f, -1.f}, false, stream_dt, 2000 + 100 * j, 98);
-      else
+      if (j + 1 < N - 1) {
+        if (free_slots(out) >= 2) {
+          fuse_add(out, rs[j + 1], 1.f);
+          fuse_add(out, f0[j], -1.f);
+          rts[j + 1] = out;
+        } else {
+          rts[j + 1] = ew(coarse_f, {rs[j + 1], out, f0[j]}, {1.f, 1.f, -1.f}, false, stream_dt, 2000 + 100 * j, 98);
+        }
+      } else if (free_slots(out) >= 1) {
+        fuse_add(out, f0[j], -1.f);
+        rts[j + 1] = out;
+      } else {
         rts[j + 1] = ew(coarse_f, {out, f0[j]}, {1.f, -1.f}, false, stream_dt, 2000 + 100 * j, 98);
+      }
     }
   }
   // ytilde joins the post phase, so that its backward (which writes dL/dy_N =
   // D_N) is complete when the head's backward is
-  ytilde = N > 1 ? ew(head_f, {ys[N - 1], rts[N - 1]}, {1.f, 1.f}, false, stream_dt, 9000, 0) : ys[0];
+  if (N > 1 && free_slots(rts[N - 1]) >= 1) {
+    fuse_add(rts[N - 1], ys[N - 1], 1.f);
+    ytilde = rts[N - 1];
+    rtN_in_ytilde = true;
+  } else {
+    ytilde = N > 1 ? ew(head_f, {ys[N - 1], rts[N - 1]}, {1.f, 1.f}, false, stream_dt, 9000, 0) : ys[0];
+  }
   if (N == 1) rts[0] = ytilde;
   // head h
   std::vector<int> head_ids;
@@ -1235,6 +1304,12 @@ int pnn_net::build_tables() {
             if (o.kind == K_CONV_FWD || o.kind == K_CONV_FWD_TC) {
               c.y = ws + ov.off; c.y_dt = ov.dt;
               if (o.res >= 0) { c.res = ws + vals[o.res].off; c.res_dt = vals[o.res].dt; }
+              for (int e = 0; e < 2; ++e)
+                if (o.res2[e] >= 0) {
+                  c.res2[e] = ws + vals[o.res2[e]].off;
+                  c.res2_dt[e] = vals[o.res2[e]].dt;
+                  c.res2_c[e] = o.rcoef[e];
+                }
               if (o.stats_norm >= 0) c.stats = P<float>(norms[o.stats_norm].part);
               add(&c, sizeof c, o.mtiles * o.ntiles);
             } else if (o.kind == K_DGRAD || o.kind == K_DGRAD_TC) {
@@ -1344,6 +1419,8 @@ int pnn_net::build_tables() {
               b.accumulate = o.acc;
               b.add0 = o.addv[0] >= 0 ? P<float>(gptr(o.addv[0])) : nullptr;
               b.add1 = o.addv[1] >= 0 ? P<float>(gptr(o.addv[1])) : nullptr;
+              b.add_c[0] = o.addc[0];
+              b.add_c[1] = o.addc[1];
             }
             add(&b, sizeof b, o.kind == K_BNB_FIN ? b.cgroups * b.nchunk : o.tiles);
             break;
@@ -2317,6 +2394,26 @@ int pnn_get_tensor(pnn_net* n, int32_t which, int32_t j, float* host, size_t cou
   size_t want;
   pnn_tensor_size(n, which, j, &want);
   if (!host || count != want) return n->fail(PNN_EINVAL, "length must equal pnn_tensor_size");
+  // values the step does not store (the correction folded into conv
+  // epilogues): y_j = r_j + x_{j+1}, rt_N = ytilde - y_N, from what it stores
+  int a = -1, b = -1;
+  float cb = 0.f;
+  if (which == PNN_T_Y && j >= 1 && j < n->N && n->y_is_r[j - 1]) { a = n->ys[j - 1]; b = n->xs[j]; cb = 1.f; }
+  if (which == PNN_T_RTILDE && j == n->N && n->rtN_in_ytilde) { a = n->ytilde; b = n->ys[n->N - 1]; cb = -1.f; }
+  if (a >= 0) {
+    const Value& va = n->vals[a];
+    std::vector<float> tmp(want);
+    cudaError_t e = launch_export(make_src(*n, a), n->B, va.H, va.W, va.C, n->P<float>(n->export_off), n->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(n->stream);
+    if (e == cudaSuccess) e = cudaMemcpy(host, n->ws + n->export_off, want * 4, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess)
+      e = launch_export(make_src(*n, b), n->B, va.H, va.W, va.C, n->P<float>(n->export_off), n->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(n->stream);
+    if (e == cudaSuccess) e = cudaMemcpy(tmp.data(), n->ws + n->export_off, want * 4, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess)
+      for (size_t i = 0; i < want; ++i) host[i] += cb * tmp[i];
+    return n->cuda_check(e, "export tensor");
+  }
   cudaError_t e = cudaSuccess;
   if (v == -2) {
     const int nfc = (int)n->fc_width.size() - 1;

@@ -126,8 +126,10 @@ def test_running_stats_layout_and_inference_plan(pnn, idx):
 
 def test_overlap_option_plans_the_last_subnetwork_apart(pnn):
     """opts.overlap moves the last subnetwork's backward out of the grouped
-    launches (more backward launches, the same forward) in the residual form
-    with N > 1, and leaves the delta form and N = 1 as they are."""
+    launches (more backward launches) in the residual form with N > 1, and
+    leaves the delta form and N = 1 as they are.  It also keeps the
+    correction's sums as launches of their own (r_j, rt_{j+1} and ytilde:
+    (N-1) + (N-2) + 1 of them) instead of folding them into conv epilogues."""
     import ctypes as C
 
     def counts(d, **kw):
@@ -137,8 +139,9 @@ def test_overlap_option_plans_the_last_subnetwork_apart(pnn):
         return list(c)
 
     d = W.config(2)
+    N = len(d["segments"])
     seq, ov = counts(d), counts(d, overlap=32)
-    assert ov[0] == seq[0] and ov[1] > seq[1] and ov[2] == seq[2]
+    assert ov[0] == seq[0] + (N - 1) + (N - 2) + 1 and ov[1] > seq[1] and ov[2] == seq[2]
     dd = W.config(2)
     dd["correction"] = "delta"
     assert counts(dd, overlap=32) == counts(dd)
