@@ -135,11 +135,18 @@ typedef struct {
                             stream, its persistent kernels capped to leave
                             `overlap` SMs to the chain; the chain's term of
                             dL/dx_N is added after both.  0 = phases in sequence */
+  int32_t fuse_correction; /* 1 (default): the correction's sums r_j, rt_{j+1},
+                            ytilde are formed in the epilogue of the conv that
+                            produces their first operand wherever that conv adds
+                            a residual (y_j for j < N and rt_N are then not
+                            stored; pnn_get_tensor derives them); 0 = launches of
+                            their own.  The residual form with overlap > 0 always
+                            uses launches of their own. */
 } pnn_options;
 
 /* Fill o with the defaults: bf16, residual correction, seed 0, lr 0.1,
  * momentum 0.9, weight decay 5e-4, Nesterov (Section 4), stream_fp32 1,
- * bn_momentum 0.1, inference 0, overlap 0. */
+ * bn_momentum 0.1, inference 0, overlap 0, fuse_correction 1. */
 void pnn_default_options(pnn_options* o);
 
 /* Plan the network from a description.  Host only: no GPU work, no device

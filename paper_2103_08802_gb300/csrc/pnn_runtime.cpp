@@ -874,7 +874,7 @@ int pnn_net::plan(const pnn_desc* d) {
   // + F^j(rt_j) (delta form: - F^j(x_{j+1})) into the last conv of F^j,
   // ytilde = y_N + rt_N into the last conv of F^{N-1}.  (Not with the
   // coarse/fine overlap, which defers a term of the r_{N-1} backward.)
-  const bool fuse = !(opt.overlap > 0 && opt.correction == PNN_CORR_RESIDUAL) && N > 1;
+  const bool fuse = opt.fuse_correction && !(opt.overlap > 0 && opt.correction == PNN_CORR_RESIDUAL) && N > 1;
   auto free_slots = [&](int v) -> int {
     const int p = v >= 0 ? vals[v].producer : -1;
     if (!fuse || p < 0) return 0;
@@ -1884,6 +1884,7 @@ void pnn_default_options(pnn_options* o) {
   o->bn_momentum = 0.1f;
   o->inference = 0;
   o->overlap = 0;
+  o->fuse_correction = 1;
 }
 
 int pnn_create(const pnn_desc* desc, const pnn_options* opts, pnn_net** out) {

@@ -51,7 +51,7 @@ class Options(C.Structure):
                 ("nesterov", C.c_int32), ("stream_fp32", C.c_int32), ("conv_impl", C.c_int32),
                 ("grad_fp32", C.c_int32),
                 ("stream", C.c_void_p), ("bn_momentum", C.c_float), ("inference", C.c_int32),
-                ("overlap", C.c_int32)]
+                ("overlap", C.c_int32), ("fuse_correction", C.c_int32)]
 
 
 class ConvArgs(C.Structure):
@@ -216,7 +216,7 @@ class ParaNet:
 
     def __init__(self, desc, precision=None, correction=None, seed=0, lr=0.1, momentum=0.9,
                  weight_decay=5e-4, nesterov=True, stream_fp32=None, conv_impl=0, grad_fp32=False, stream=None,
-                 device="cuda", bind=True, inference=False, bn_momentum=0.1, overlap=0):
+                 device="cuda", bind=True, inference=False, bn_momentum=0.1, overlap=0, fuse_correction=True):
         self.lib = load()
         self.desc = desc
         d, self._keep = _make_desc(desc)
@@ -230,6 +230,7 @@ class ParaNet:
         o.nesterov, o.stream_fp32, o.conv_impl = int(nesterov), int(stream_fp32), int(conv_impl)
         o.grad_fp32 = int(grad_fp32)
         o.inference, o.bn_momentum, o.overlap = int(inference), bn_momentum, int(overlap)
+        o.fuse_correction = int(fuse_correction)
         self.stream = stream
         o.stream = None if stream is None else C.c_void_p(stream.cuda_stream)
         self.h = C.c_void_p()

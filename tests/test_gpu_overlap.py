@@ -1,6 +1,8 @@
 """Coarse/fine overlap (opts.overlap): the last subnetwork's backward needs
 only D_N (Algorithm 2), so it runs on a second stream beside the coarse
-chain's backward, and the chain's term of dL/dx_N is added after both.  The
+chain's backward, and the chain's term of dL/dx_N is added after both.  (The
+correction's sums then keep launches of their own; the sequential schedule
+they are compared with is planned the same way, fuse_correction=False.)  The
 step computes the same quantities as the sequential schedule: everything but
 dL/dx_N is accumulated in the same order and agrees bit for bit; dL/dx_N
 sums the same two terms in the other order, so only the gradients of C^N
@@ -39,7 +41,7 @@ def test_overlap_matches_sequential(name):
     else:
         desc = W.paper_parareal_resnet(6, batch=128, per_stage=2)
     onet, theta, x, labels = inputs(desc)
-    a = run_gpu(desc, theta, x, labels)
+    a = run_gpu(desc, theta, x, labels, fuse_correction=False)
     b = run_gpu(desc, theta, x, labels, overlap=32)
     for k in a:
         if k in ("net", "onet", "grad", "theta_new", "momentum"):
