@@ -167,6 +167,9 @@ struct pnn_net {
   // ytilde = y_N + rt_N)
   std::vector<char> y_is_r;
   bool rtN_in_ytilde = false;
+  // interface tensors the step does not store, exported as a + c * b of two
+  // stored values: (which, j) -> (a, b, c)
+  std::map<std::pair<int, int>, std::tuple<int, int, float>> derived;
   // head
   int head_in = -1, head_norm = -1;
   std::vector<int> fc_w, fc_b;
@@ -888,17 +891,32 @@ int pnn_net::plan(const pnn_desc* d) {
     o.res2[e] = addend;
     o.rcoef[e] = c;
   };
-  for (int j = 0; j + 1 < N; ++j) {
-    if (free_slots(ys[j]) >= 1) {
-      fuse_add(ys[j], xs[j + 1], -1.f);
-      rs[j] = ys[j];
-      y_is_r[j] = 1;
-    } else {
-      rs[j] = ew(coarse_f, {ys[j], xs[j + 1]}, {1.f, -1.f}, false, stream_dt, 1000, j);
+  derived.clear();
+  // The delta form as a chain of states s_j = x_{j+1} + rt_j: s_1 = y_1,
+  // s_{j+1} = y_{j+1} + F^j(s_j) - F^j(x_{j+1}), ytilde = s_N -- the same
+  // values (r_{j+1} + x_{j+2} = y_{j+1}) without r_j or a separate state sum;
+  // rt_j = s_j - x_{j+1} and r_j = y_j - x_{j+1} are exported from them.
+  const bool chain = fuse && delta;
+  std::vector<int> f0(std::max(0, N - 1), -1);
+  if (!chain) {
+    for (int j = 0; j + 1 < N; ++j) {
+      if (free_slots(ys[j]) >= 1) {
+        fuse_add(ys[j], xs[j + 1], -1.f);
+        rs[j] = ys[j];
+        y_is_r[j] = 1;
+        derived[{PNN_T_Y, j + 1}] = std::make_tuple(ys[j], xs[j + 1], 1.f);
+      } else {
+        rs[j] = ew(coarse_f, {ys[j], xs[j + 1]}, {1.f, -1.f}, false, stream_dt, 1000, j);
+      }
+    }
+    if (N > 1) rts[0] = rs[0];
+  } else {
+    rts[0] = ys[0];  // s_1 = y_1
+    for (int j = 0; j + 1 < N; ++j) {
+      derived[{PNN_T_R, j + 1}] = std::make_tuple(ys[j], xs[j + 1], -1.f);
+      derived[{PNN_T_RTILDE, j + 1}] = std::make_tuple(-1, xs[j + 1], -1.f);  // a = s_{j+1}, filled below
     }
   }
-  std::vector<int> f0(std::max(0, N - 1), -1);
-  if (N > 1) rts[0] = rs[0];
   std::vector<int> coarse_start(N, 0);
   for (int j = 0; j + 1 < N; ++j) { coarse_start[j] = cofs; cofs += d->coarse_len[j]; }
   for (int j = 0; j + 1 < N; ++j) {
@@ -907,8 +925,13 @@ int pnn_net::plan(const pnn_desc* d) {
     if (!check_layers(F, nF) || nF <= 0) return fail(PNN_EINVAL, "bad coarse layer");
     int out;
     PCur pc{&coarse_ids[j], 0, false};
-    if (!delta) {
+    if (!delta || chain) {
       out = stack(coarse_f, F, nF, rts[j], pc, 2000 + 100 * j, true);
+      if (chain) {
+        PCur pr{&coarse_ids[j], 0, true};
+        delta_f.emplace_back();
+        f0[j] = stack(delta_f.back(), F, nF, xs[j + 1], pr, 0, true);
+      }
     } else {
       int state = ew(coarse_f, {xs[j + 1], rts[j]}, {1.f, 1.f}, false, stream_dt, 2000 + 100 * j, 99);
       out = stack(coarse_f, F, nF, state, pc, 2000 + 100 * j, true);
@@ -920,7 +943,16 @@ int pnn_net::plan(const pnn_desc* d) {
     }
     if (vals[out].C != std::get<0>(Xshape[j + 2]) || vals[out].H != std::get<1>(Xshape[j + 2]))
       return fail(PNN_EINVAL, "coarse block output is not X_{j+1}");
-    if (!delta) {
+    if (chain) {
+      // s_{j+1} = y_{j+1} + F^j(s_j) - F^j(x_{j+1})
+      if (free_slots(out) >= 2) {
+        fuse_add(out, ys[j + 1], 1.f);
+        fuse_add(out, f0[j], -1.f);
+        rts[j + 1] = out;
+      } else {
+        rts[j + 1] = ew(coarse_f, {ys[j + 1], out, f0[j]}, {1.f, 1.f, -1.f}, false, stream_dt, 2000 + 100 * j, 98);
+      }
+    } else if (!delta) {
       if (j + 1 == N - 1) {
         rts[j + 1] = out;
       } else if (free_slots(out) >= 1) {
@@ -948,10 +980,15 @@ int pnn_net::plan(const pnn_desc* d) {
   }
   // ytilde joins the post phase, so that its backward (which writes dL/dy_N =
   // D_N) is complete when the head's backward is
-  if (N > 1 && free_slots(rts[N - 1]) >= 1) {
+  if (chain) {
+    ytilde = rts[N - 1];  // s_N
+    for (int j = 0; j + 1 < N; ++j) std::get<0>(derived[{PNN_T_RTILDE, j + 1}]) = rts[j];
+    derived[{PNN_T_RTILDE, N}] = std::make_tuple(ytilde, ys[N - 1], -1.f);
+  } else if (N > 1 && free_slots(rts[N - 1]) >= 1) {
     fuse_add(rts[N - 1], ys[N - 1], 1.f);
     ytilde = rts[N - 1];
     rtN_in_ytilde = true;
+    derived[{PNN_T_RTILDE, N}] = std::make_tuple(ytilde, ys[N - 1], -1.f);
   } else {
     ytilde = N > 1 ? ew(head_f, {ys[N - 1], rts[N - 1]}, {1.f, 1.f}, false, stream_dt, 9000, 0) : ys[0];
   }
@@ -2363,6 +2400,11 @@ static int tensor_value(const pnn_net* n, int which, int j, int* v, bool* grad) 
   const int N = n->N;
   *grad = false;
   *v = -1;
+  const auto it = n->derived.find({which, j});
+  if (it != n->derived.end()) {  // not stored: same shape as its first operand
+    *v = std::get<0>(it->second);
+    return PNN_OK;
+  }
   switch (which) {
     case PNN_T_X: if (j >= 1 && j <= N) *v = n->xs[j - 1]; break;
     case PNN_T_Y: if (j >= 1 && j <= N) *v = n->ys[j - 1]; break;
@@ -2399,8 +2441,8 @@ int pnn_get_tensor(pnn_net* n, int32_t which, int32_t j, float* host, size_t cou
   // epilogues): y_j = r_j + x_{j+1}, rt_N = ytilde - y_N, from what it stores
   int a = -1, b = -1;
   float cb = 0.f;
-  if (which == PNN_T_Y && j >= 1 && j < n->N && n->y_is_r[j - 1]) { a = n->ys[j - 1]; b = n->xs[j]; cb = 1.f; }
-  if (which == PNN_T_RTILDE && j == n->N && n->rtN_in_ytilde) { a = n->ytilde; b = n->ys[n->N - 1]; cb = -1.f; }
+  const auto it = n->derived.find({which, j});
+  if (it != n->derived.end()) std::tie(a, b, cb) = it->second;
   if (a >= 0) {
     const Value& va = n->vals[a];
     std::vector<float> tmp(want);

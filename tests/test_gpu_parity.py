@@ -363,17 +363,19 @@ def test_step_is_deterministic():
     np.testing.assert_array_equal(a["theta_new"], b["theta_new"])
 
 
-@pytest.mark.parametrize("paper", [False, True])
-def test_correction_folded_into_conv_epilogues(paper):
-    """The correction's sums (r_j, rt_{j+1}, ytilde; residual form) ride in the
+@pytest.mark.parametrize("paper,mode", [(False, "residual"), (True, "residual"), (False, "delta")])
+def test_correction_folded_into_conv_epilogues(paper, mode):
+    """The correction's sums (residual form: r_j, rt_{j+1}, ytilde; delta form:
+    the states s_{j+1} = y_{j+1} + F^j(s_j) - F^j(x_{j+1})) ride in the
     epilogues of the convs that produce their operands, and their backward
     scatter (dL/dy_j = D_j, dL/dx_{j+1} -= D_j) in gradient aliases and the
     BN-backward apply of x_{j+1}: no elementwise launch in the coarse phases
-    of a step.  (Values the step no longer stores -- y_j for j < N, rt_N --
-    are still exported exactly; the parity tests above compare them.)"""
+    of a step.  (Values the step no longer stores -- y_j for j < N, rt_N, the
+    delta form's r_j and rt_j -- are still exported exactly; the parity tests
+    above compare them.)"""
     import torch
     from paper_2103_08802_gb300 import pnn
-    desc = paper_reduced(3) if paper else reduced(2)
+    desc = paper_reduced(3) if paper else reduced(2, correction=mode)
     onet, theta, x, labels = inputs(desc)
     net = pnn.ParaNet(desc)
     net.set_params(theta)
