@@ -301,6 +301,87 @@ __global__ void __launch_bounds__(256) k_conv_wgrad(const ConvDesc* __restrict__
   }
 }
 
+// Weight gradient of a conv with few input channels (the 3-channel stem and
+// C^j convs, R*S*C <= 64): the same tiles, splits and partial layout as
+// k_conv_wgrad, but each 64-pixel step stages dY [64 px][64 k_out] and the
+// im2col operand [64 px][R*S*C] once in shared memory (pixel and (r,s,c)
+// coordinates from per-CTA tables instead of divisions per element), and
+// thread t accumulates outputs (k, j) = t, t + 256, ... of the tile over the
+// step's pixels in order.
+__global__ void __launch_bounds__(256) k_conv_wgrad_small(const ConvDesc* __restrict__ tab,
+                                                          const int* __restrict__ tstart, int n) {
+  constexpr int BM = kWgradBM, BN = kWgradBN, BP = 64, MAXO = (BM * BN) / 256;
+  __shared__ float As[BP][BM + 1];  // dY[pixel][k_out]
+  __shared__ float Bs[BP][BN + 1];  // im2col[pixel][j]
+  __shared__ int jr[BN], js[BN], jc[BN];
+  __shared__ int pn[BP], ph[BP], pw[BP];
+  const int inst = find_instance(tstart, n, blockIdx.x);
+  const ConvDesc& d = tab[inst];
+  int t = blockIdx.x - tstart[inst];
+  const int tm = t % d.mtiles;
+  t /= d.mtiles;
+  const int tn = t % d.ntiles, split = t / d.ntiles;
+  const int RSC = d.R * d.S * d.C, Mp = d.B * d.P * d.Q;
+  const int m0 = tm * BM, n0 = tn * BN;
+  const int km = min(BM, d.K - m0), jn = min(BN, RSC - n0);
+  const int p_begin = split * d.pix_per_split;
+  const int p_end = min(Mp, p_begin + d.pix_per_split);
+  const int tid = threadIdx.x;
+  for (int j = tid; j < jn; j += 256) {
+    const int jj = n0 + j, c = jj % d.C, rs = jj / d.C;
+    jr[j] = rs / d.S - d.pad;
+    js[j] = rs % d.S - d.pad;
+    jc[j] = c;
+  }
+  float acc[MAXO];
+#pragma unroll
+  for (int i = 0; i < MAXO; ++i) acc[i] = 0.f;
+  for (int k0 = p_begin; k0 < p_end; k0 += BP) {
+    __syncthreads();  // the previous step's tiles are consumed
+    if (tid < BP) {
+      const int pix = k0 + tid;
+      const int q = pix % d.Q, tmp = pix / d.Q, pp = tmp % d.P;
+      pn[tid] = pix < p_end ? tmp / d.P : -1;
+      ph[tid] = pp * d.stride;
+      pw[tid] = q * d.stride;
+    }
+    __syncthreads();
+    for (int e = tid; e < BP * BM; e += 256) {
+      const int kk = e % BM, px = e / BM;
+      const float v = (kk < km && pn[px] >= 0) ? __ldg(d.dy + (int64_t)(k0 + px) * d.K + m0 + kk) : 0.f;
+      As[px][kk] = d.op_bf16 ? rnd(DT_BF16, v) : v;
+    }
+    for (int e = tid; e < BP * BN; e += 256) {
+      const int j = e % BN, px = e / BN;
+      float v = 0.f;
+      if (j < jn && pn[px] >= 0) {
+        const int h = ph[px] + jr[j], w = pw[px] + js[j];
+        if (h >= 0 && h < d.H && w >= 0 && w < d.W)
+          v = ld_src(d.x, ((int64_t)(pn[px] * d.H + h) * d.W + w) * d.C + jc[j], jc[j]);
+      }
+      Bs[px][j] = d.op_bf16 ? rnd(DT_BF16, v) : v;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < MAXO; ++i) {
+      const int o = tid + 256 * i;
+      if (o >= km * jn) break;
+      const int k = o / jn, j = o - k * jn;
+      float a = acc[i];
+      for (int px = 0; px < BP; ++px) a = fmaf(As[px][k], Bs[px][j], a);
+      acc[i] = a;
+    }
+  }
+  float* out = d.dw_part + (int64_t)split * d.K * RSC;
+#pragma unroll
+  for (int i = 0; i < MAXO; ++i) {
+    const int o = tid + 256 * i;
+    if (o >= km * jn) break;
+    const int k = o / jn, j = o - k * jn;
+    out[(int64_t)(m0 + k) * RSC + n0 + j] = acc[i];
+  }
+}
+
 // 32 elements per CTA, 8 lanes per element: lane l sums splits l, l+8, ...
 // in order, then a fixed xor-shuffle tree combines the 8 lanes.
 // 32 consecutive partial positions e per CTA; warp w sums splits w, w+8, ..
@@ -1150,9 +1231,11 @@ cudaError_t launch_conv_dgrad_simt(const ConvDesc* tab, const int* tstart, int n
   else k_conv_dgrad<256, 16><<<total, 256, 0, st>>>(tab, tstart, n);
   return cudaGetLastError();
 }
-cudaError_t launch_conv_wgrad_simt(const ConvDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {
+cudaError_t launch_conv_wgrad_simt(const ConvDesc* tab, const int* tstart, int n, int total, int variant,
+                                   cudaStream_t st) {
   if (total <= 0) return cudaSuccess;
-  k_conv_wgrad<<<total, 256, 0, st>>>(tab, tstart, n);
+  if (variant == 1) k_conv_wgrad_small<<<total, 256, 0, st>>>(tab, tstart, n);
+  else k_conv_wgrad<<<total, 256, 0, st>>>(tab, tstart, n);
   return cudaGetLastError();
 }
 cudaError_t launch_wreduce(const WReduceDesc* tab, const int* tstart, int n, int total, cudaStream_t st) {

@@ -179,7 +179,8 @@ cudaError_t launch_conv_fwd_simt(const ConvDesc* tab, const int* tstart, int n, 
                                  int variant, cudaStream_t st);
 cudaError_t launch_conv_dgrad_simt(const ConvDesc* tab, const int* tstart, int n, int total_tiles,
                                    int variant, cudaStream_t st);
-cudaError_t launch_conv_wgrad_simt(const ConvDesc* tab, const int* tstart, int n, int total_tiles,
+// variant 1: few input channels (R*S*C <= 64), im2col staged per 64-pixel step
+cudaError_t launch_conv_wgrad_simt(const ConvDesc* tab, const int* tstart, int n, int total_tiles, int variant,
                                    cudaStream_t st);
 cudaError_t launch_wreduce(const WReduceDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);
 cudaError_t launch_ew(const EwDesc* tab, const int* tstart, int n, int total_tiles, cudaStream_t st);

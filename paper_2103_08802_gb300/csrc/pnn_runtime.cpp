@@ -532,6 +532,9 @@ struct pnn_net {
         } else {
           wg.mtiles = cdiv(ov.C, kWgradBM);
           wg.ntiles = cdiv(RSC, kWgradBN);
+          // few input channels (the 3-channel stem and C^j convs): the
+          // kernel that stages the im2col operand once per pixel step
+          wg.variant = vals[f.in].C < 8 && RSC <= kWgradBN ? 1 : 0;
         }
         int base = wg.mtiles * wg.ntiles;
         int splits = std::max(1, std::min(cdiv(Mp, 256), cdiv(2 * (int64_t)device_sm_count(), base)));
@@ -1678,7 +1681,7 @@ int pnn_net::run_phase(int p, cudaStream_t st, int cap) {
                                        st, cap);
         break;
       case K_DGRAD: e = launch_conv_dgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, st); break;
-      case K_WGRAD: e = launch_conv_wgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, st); break;
+      case K_WGRAD: e = launch_conv_wgrad_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, st); break;
       case K_WREDUCE: e = launch_wreduce((const WReduceDesc*)tab, ts, L.count, L.total, st); break;
       case K_EW: e = launch_ew((const EwDesc*)tab, ts, L.count, L.total, st); break;
       case K_EW_BWD: e = launch_ew_bwd((const EwBwdDesc*)tab, ts, L.count, L.total, st); break;
