@@ -79,7 +79,7 @@ def parse():
                          "instead of the training step: a bottleneck conv (reduce = 1x1 out->mid, conv3x3 = "
                          "mid->mid, expand = 1x1 mid->out with the residual add) and a mode (fwd, dgrad, "
                          "wgrad), one instance per subnetwork at the stage its middle block sits in")
-    ap.add_argument("--layer-impl", default="auto", choices=["auto", "tma", "gathered"])
+    ap.add_argument("--layer-impl", default="auto", choices=["auto", "tma", "gathered", "tma_tap"])
     return ap.parse_args()
 
 
@@ -366,6 +366,7 @@ def retear(args, desc, stream):
 KERNEL_SYMBOL = {("conv_fwd_tc", 0): "k_conv_fwd_tc", ("conv_fwd_tc", 1): "k_conv_fwd_tma",
                  ("conv_fwd_tc", 2): "k_conv_fwd_tma_w", ("conv_dgrad_tc", 0): "k_conv_dgrad_tc",
                  ("conv_dgrad_tc", 1): "k_conv_dgrad_tma", ("conv_dgrad_tc", 2): "k_conv_dgrad_tma_w",
+                 ("conv_fwd_tc", 3): "k_conv_fwd_tma_h", ("conv_dgrad_tc", 3): "k_conv_dgrad_tma_h",
                  ("conv_wgrad_tc", 0): "k_conv_wgrad_tc", ("conv_wgrad_tc", 1): "k_conv_wgrad_tma",
                  ("bn_bwd_apply", 1): "k_bnb_apply8", ("bn_finalize", 0): "k_bn_fin"}
 

@@ -119,7 +119,9 @@ typedef struct {
                             forward and data-gradient convs fed by TMA), 1 = CUDA-core
                             kernels only, 2 = CUDA-core forward + tensor-core gradients,
                             3 = tensor cores with every operand gathered by threads
-                            (no TMA producer; same results as 0) */
+                            (no TMA producer; same results as 0), 4 = as 0 but the
+                            TMA-fed 3x3 convs load one box per tap (no halo tiles;
+                            same results as 0) */
   int32_t grad_fp32;     /* bf16 mode: contract gradients (dgrad, wgrad) with fp32
                             operands instead of bf16 ones */
   void* stream;          /* cudaStream_t; NULL = legacy default stream */
@@ -303,7 +305,7 @@ int pnn_profile_read(pnn_net* net, int32_t kind, double* ms, int64_t* launches, 
 /* One record per kernel launch bracketed since pnn_profile(net, 1), in launch
  * order: kind (as for pnn_kernel_kind_name), variant (tensor-core convs:
  * 0 = operands gathered by threads, 1 = fed by TMA, 2 = fed by TMA with the
- * wide epilogue of one-k-step tiles),
+ * wide epilogue of one-k-step tiles, 3 = fed by TMA with halo tiles),
  * step phase (0 preprocessing
  * forward, 1 fine forward, 2 coarse forward, 3 head forward, 4 head backward,
  * 5 coarse backward, 6 correction backward, 7 fine backward, 8
@@ -357,7 +359,9 @@ uint64_t pnn_debug_word(void);
  *   mode PNN_CONV_WGRAD    dw[kk][r][s][cc] = sum_{n,p,q} dy[n][p][q][kk] * v(x)[n][p*stride+r-pad][q*stride+s-pad][cc]
  * impl: 0 = the kernel a training step would choose, 1 = the TMA-fed kernel
  * (stride 1 only; PNN_EINVAL where the shape does not allow it), 2 = the
- * thread-gathered kernel.  c and k multiples of 8.  All pointers are device
+ * thread-gathered kernel, 3 = the TMA-fed kernel with one box per 3x3 tap
+ * (1 and 0 use one halo box per 128-pixel tile where the tile lies inside
+ * one image: 3x3, 128 | h*w, w <= 63, 16 | the A source's channels <= 64).  c and k multiples of 8.  All pointers are device
  * memory of the current device, NHWC with the batch folded into the rows;
  * w is bf16 [k][ksize][ksize][c].  The caller owns every buffer and a
  * workspace of pnn_conv_workspace_bytes bytes (256-byte aligned); the call

@@ -86,9 +86,10 @@ struct Tile {
   const ConvDesc* d;
   int tm, tn, split;
   int Mrows, Ncols, Kt, pbeg, pend, nkt, BN, n0, m0;
+  bool halo;  // TMA-fed 3x3 tile inside one image: one stage holds all nine taps
 };
 
-template <int MODE>
+template <int MODE, bool HALO = false>
 __device__ __forceinline__ Tile decode(const ConvDesc* tab, const int* tstart, int ninst, int tile) {
   Tile t;
   int lo = 0, hi = ninst - 1;
@@ -112,6 +113,8 @@ __device__ __forceinline__ Tile decode(const ConvDesc* tab, const int* tstart, i
   t.BN = d.ntiles == 1 ? ((t.Ncols + 15) & ~15) : d.ntile_w;
   t.n0 = t.tn * d.ntile_w;
   t.m0 = t.tm * (d.mtile_rows > 0 ? d.mtile_rows : kBM);
+  t.halo = HALO && MODE != WGRAD && d.tma_h != nullptr;
+  if (t.halo) t.nkt = 1;
   return t;
 }
 
@@ -992,14 +995,13 @@ __host__ __device__ constexpr int tma_ystage(int mode, int w) { return mode == 2
 __host__ __device__ constexpr int tma_extra(int mode, int w) {
   return tma_ystage(mode, w) + (tma_ne(mode, w) / 4) * kTmaRedBytes;
 }
-__host__ __device__ inline int tma_stages(int mode, int bnmax, int raw_bytes, int extra) {
+__host__ __device__ inline int tma_stages(int op_bytes, int raw_bytes, int extra) {
   const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - extra;
-  int s = avail / (raw_bytes + tma_op_bytes(mode, bnmax));
+  int s = avail / (raw_bytes + op_bytes);
   return s < 2 ? 2 : (s > kTmaMaxStages ? kTmaMaxStages : s);
 }
-__host__ __device__ inline size_t tma_smem_bytes(int mode, int bnmax, int raw_bytes, int extra) {
-  return 1024 + (size_t)tma_stages(mode, bnmax, raw_bytes, extra) * (raw_bytes + tma_op_bytes(mode, bnmax)) + extra +
-         sizeof(TmaShared);
+__host__ __device__ inline size_t tma_smem_bytes(int op_bytes, int raw_bytes, int extra) {
+  return 1024 + (size_t)tma_stages(op_bytes, raw_bytes, extra) * (raw_bytes + op_bytes) + extra + sizeof(TmaShared);
 }
 
 // One transform thread's share of a stage: row `row` of the A operand, its
@@ -1075,6 +1077,93 @@ __device__ __forceinline__ void transform_stage(const uint8_t* __restrict__ rawp
     }
     *reinterpret_cast<uint4*>(A + swz(t.row, cc)) = valid ? pack8(v) : make_uint4(0, 0, 0, 0);
   }
+  }
+}
+
+// One halo tile's transform (halo_ok): raw box row u = 0 .. halo_rows(W) - 1
+// holds pixel m0 - W - 1 + u (cdim channels, as loaded); each 8-channel
+// chunk is transformed once (BN + ReLU of the source, bf16) and stored to the
+// three column-offset copies: copy sp (s' = sp - 1) row j = u - sp, zero where
+// the pixel lies outside the tile's image or its output column x - s' leaves
+// the row.  Thread tid of nthreads takes whole rows (one division per row);
+// a row's chunks are read in groups of four, all loads first, starting at
+// chunk u mod nch so that the lanes' raw reads spread over the banks.
+template <bool XBF>
+__device__ __forceinline__ void halo_transform(const uint8_t* __restrict__ rawp, uint8_t* __restrict__ A,
+                                               const float* __restrict__ scs, const float* __restrict__ sfs,
+                                               const Tile& T, const ConvDesc& d, int cdim, bool tr, int relu,
+                                               int tid, int nthreads) {
+  const int W = d.W, HW = d.H * d.W;
+  const int hr = halo_rows(W), prow = kBM + 2 * W;
+  const int plane = halo_plane_bytes(W), copy = halo_copy_bytes(W, cdim);
+  const int img0 = T.m0 - T.m0 % HW;
+  const int lq0 = T.m0 - W - 1 - img0;  // raw row 0, as a pixel index within the tile's image
+  const int nch = cdim >> 3;
+  constexpr int EW = XBF ? 1 : 2;       // 16-byte words per 8-channel chunk
+  for (int u = tid; u < hr; u += nthreads) {
+    const int lq = lq0 + u;
+    const bool in = lq >= 0 && lq < HW;
+    const int xq = in ? lq % W : 0;
+    bool okc[3];
+#pragma unroll
+    for (int sp = 0; sp < 3; ++sp) {
+      const int j = u - sp, xo = xq - (sp - 1);  // the output column that reads this pixel through copy sp
+      okc[sp] = in && xo >= 0 && xo < W && j >= 0 && j < prow;
+    }
+    const int rot = u % nch;
+    const uint8_t* row = rawp + u * cdim * (XBF ? 2 : 4);
+    uint8_t* dst = A + u * 16;
+    for (int p0 = 0; p0 < nch; p0 += 2) {
+      // two chunks: both loads first
+      const int pa = p0 + rot >= nch ? p0 + rot - nch : p0 + rot;
+      const int pb = pa + 1 >= nch ? pa + 1 - nch : pa + 1;
+      const bool two = p0 + 1 < nch;
+      uint4 ra[EW], rb[EW];
+#pragma unroll
+      for (int e = 0; e < EW; ++e) {
+        ra[e] = *reinterpret_cast<const uint4*>(row + pa * 16 * EW + e * 16);
+        if (two) rb[e] = *reinterpret_cast<const uint4*>(row + pb * 16 * EW + e * 16);
+      }
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        if (i == 1 && !two) break;
+        const int pc = i ? pb : pa;
+        const uint4* r = i ? rb : ra;
+        float v[8];
+        if (XBF) {
+          const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&r[0]);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(hh[e]);
+            v[2 * e] = f.x;
+            v[2 * e + 1] = f.y;
+          }
+        } else {
+          const float* f0 = reinterpret_cast<const float*>(&r[0]);
+          const float* f1 = reinterpret_cast<const float*>(&r[EW - 1]);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) { v[e] = f0[e]; v[4 + e] = f1[e]; }
+        }
+        if (tr) {
+          const int c = pc * 8;
+          const float4 s0 = *reinterpret_cast<const float4*>(scs + c);
+          const float4 s1 = *reinterpret_cast<const float4*>(scs + c + 4);
+          const float4 f0 = *reinterpret_cast<const float4*>(sfs + c);
+          const float4 f1 = *reinterpret_cast<const float4*>(sfs + c + 4);
+          const float sc[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+          const float sf[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+          act8(v, sc, sf, relu);
+        }
+        const uint4 pk = pack8(v);
+#pragma unroll
+        for (int sp = 0; sp < 3; ++sp) {
+          // row j = u - sp of copy sp; rows outside the copy are skipped
+          const int j = u - sp;
+          if (j < 0 || j >= prow) continue;
+          *reinterpret_cast<uint4*>(dst + sp * (copy - 16) + pc * plane) = okc[sp] ? pk : make_uint4(0, 0, 0, 0);
+        }
+      }
+    }
   }
 }
 
@@ -1241,16 +1330,19 @@ __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDe
   }
 }
 
-template <int MODE, int W>
+// HALO: the launch may hold halo tiles (a separate instantiation, so that
+// the code of the other variants is unchanged by it)
+template <int MODE, int W, bool HALO>
 __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, const int* __restrict__ tstart,
-                                              int ninst, int total, int bnmax, int raw_bytes, int32_t* status) {
+                                              int ninst, int total, int bnmax, int raw_bytes, int op_bytes_arg,
+                                              int32_t* status) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw0 = smem_u32(smem_raw);
   const uint32_t base = (raw0 + 1023u) & ~1023u;
   uint8_t* const gbase = smem_raw + (base - raw0);
   using R = TmaRoles<MODE, W>;
-  const int S = tma_stages(MODE, bnmax, raw_bytes, tma_extra(MODE, W));
-  const int op_bytes = tma_op_bytes(MODE, bnmax);
+  const int op_bytes = op_bytes_arg > 0 ? op_bytes_arg : tma_op_bytes(MODE, bnmax);
+  const int S = tma_stages(op_bytes, raw_bytes, tma_extra(MODE, W));
   constexpr int kAMult = tma_amult(MODE);
   const uint32_t op_base = base + S * raw_bytes;
   RT(const unsigned long long rt_start = clock64();)
@@ -1292,7 +1384,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       bool ok = true;
       RT(unsigned long long rt_a = 0, rt_b = 0;)
       for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
-        const Tile T = decode<MODE>(tab, tstart, ninst, tile);
+        const Tile T = decode<MODE, HALO>(tab, tstart, ninst, tile);
         const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
         if constexpr (MODE == WGRAD) {
           // per k-step: the activation rows of all taps (a halo of pad*W+pad
@@ -1316,6 +1408,22 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
         const int cdim = MODE == FWD ? d.C : d.K;
         const int cw = cdim < 64 ? cdim : 64;
         const int esz = (MODE == FWD && d.x.dt == DT_BF16) ? 2 : 4;
+        if (T.halo) {
+          // one stage: the halo box (all nine taps) and the tile's weight boxes
+          const int s = g % S;
+          RT(const unsigned long long rt0 = clock64();)
+          if (!mbar_wait(smem_u32(&sh.op_empty[s]), ((g / S) & 1) ^ 1, abort_flag)) { ok = false; break; }
+          RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
+          const int nbox = halo_nbox(cdim);
+          const uint32_t full = smem_u32(&sh.tma_full[s]);
+          mbar_expect_tx(full, (uint32_t)(halo_rows(d.W) * cdim * esz) + (uint32_t)(nbox * T.BN * 128));
+          tma_load_2d(base + s * raw_bytes, d.tma_h, 0, T.m0 - d.W - 1, full);
+          for (int bx = 0; bx < nbox; ++bx)
+            tma_load_2d(op_base + s * op_bytes + bx * T.BN * 128, d.tma_b, bx * 64, T.n0, full);
+          RT(rt_b += clock64() - rt1;)
+          ++g;
+          continue;
+        }
         const uint32_t box = (uint32_t)(kBM * cw * esz);
         const int taps = d.R * d.S;
         for (int kt = 0; kt < T.nkt; ++kt, ++g) {
@@ -1361,7 +1469,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     const ConvDesc* staged = nullptr;  // instance whose scale/shift sit in shared memory
     RT(unsigned long long rt_a = 0, rt_b = 0, rt_c = 0, rt_d = 0;)
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
-      const Tile T = decode<MODE>(tab, tstart, ninst, tile);
+      const Tile T = decode<MODE, HALO>(tab, tstart, ninst, tile);
       const ConvDesc d = *T.d;  // a private copy: stores through other pointers cannot force reloads
       const int cdim = MODE == FWD ? d.C : d.K;
       const bool big = cdim >= 64;                  // one tap per k-step, 64 channels
@@ -1381,6 +1489,34 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       if constexpr (MODE == WGRAD) {
         wgrad_transform_tile(T, d, threadIdx.x, tr, g, ok, S, raw_bytes, op_bytes, gbase, sh RT(, rt_a, rt_b));
         continue;
+      }
+      if (MODE != WGRAD && T.halo) {
+        {
+          const int s = g % S;
+          RT(const unsigned long long rt0 = clock64();)
+          if (ok && !mbar_wait(smem_u32(&sh.tma_full[s]), (g / S) & 1, abort_flag)) {
+            ok = false;
+            sh.abort_flag = 1;
+          }
+          RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
+          if (ok) {
+            const int cdim = MODE == FWD ? d.C : d.K;
+            const uint8_t* rawp = gbase + s * raw_bytes;
+            uint8_t* A = gbase + S * raw_bytes + s * op_bytes + halo_nbox(cdim) * T.BN * 128;
+            if (MODE == FWD && d.x.dt == DT_BF16)
+              halo_transform<true>(rawp, A, sh.scale, sh.shift, T, d, cdim, tr, tr ? d.x.relu : 0, threadIdx.x,
+                                   R::kTransform);
+            else
+              halo_transform<false>(rawp, A, sh.scale, sh.shift, T, d, cdim, tr, tr ? d.x.relu : 0, threadIdx.x,
+                                    R::kTransform);
+            RT(const unsigned long long rt2 = clock64(); rt_c += rt2 - rt1;)
+            fence_proxy_async();
+            mbar_arrive(smem_u32(&sh.op_full[s]));
+            RT(rt_b += clock64() - rt1;)
+          }
+          ++g;
+          continue;
+        }
       }
       // each row's pixel and which of the R x S taps stay inside the image
       uint32_t tapok[kRPT];
@@ -1457,7 +1593,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       bool issued = false;
       RT(unsigned long long rt_acc = 0, rt_full = 0, rt_issue = 0;)
       for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++li) {
-        const Tile T = decode<MODE>(tab, tstart, ninst, tile);
+        const Tile T = decode<MODE, HALO>(tab, tstart, ninst, tile);
         const int b = li % R::kAcc;
         RT(unsigned long long rt0 = clock64();)
         if (!mbar_wait(smem_u32(&sh.tempty[b]), ((li / R::kAcc) & 1) ^ 1, abort_flag)) { ok = false; break; }
@@ -1467,7 +1603,37 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
         const uint32_t idesc = idesc_bf16(kBM, T.BN);
         // a second 128-row half: only in a 256-row tile that has more than 128 rows
         const bool two = kAMult == 2 && min(T.d->mtile_rows, T.Mrows - T.m0) > kBM;
-        for (int kt = 0; kt < T.nkt; ++kt, ++g) {
+        if (T.halo) {
+          // tap (r, s) reads copy s' from row (r' + 1) W (forward: r' = r - 1,
+          // s' = s - 1; data gradient: r' = 1 - r, s' = 1 - s), K = 16 channels
+          // an MMA, the weight K index tap * cdim + 16 kc
+          const int s = g % S;
+          RT(rt0 = clock64();)
+          if (!mbar_wait(smem_u32(&sh.op_full[s]), (g / S) & 1, abort_flag)) { ok = false; break; }
+          RT(const unsigned long long rt1 = clock64(); rt_full += rt1 - rt0;)
+          fence_after();
+          const int cdim = MODE == FWD ? T.d->C : T.d->K;
+          const int Wd = T.d->W;
+          const uint32_t b_addr = op_base + s * op_bytes;
+          const uint32_t a_addr = b_addr + halo_nbox(cdim) * T.BN * 128;
+          const uint32_t plane = halo_plane_bytes(Wd), copy = halo_copy_bytes(Wd, cdim);
+          for (int tap = 0; tap < 9; ++tap) {
+            const int r = tap / 3, sx = tap - 3 * r;
+            const int dr = MODE == FWD ? r - 1 : 1 - r, ds = MODE == FWD ? sx - 1 : 1 - sx;
+            const uint32_t a_tap = a_addr + (ds + 1) * copy + (dr + 1) * Wd * 16;
+            for (int kc = 0; kc < (cdim >> 4); ++kc) {
+              const int k = tap * cdim + kc * 16;
+              mma_bf16(tacc, nosw_desc(a_tap + 2 * kc * plane, plane, 128),
+                       sw128_desc(b_addr + (k >> 6) * T.BN * 128 + ((k & 63) >> 4) * 32), idesc,
+                       (tap | kc) ? 1u : 0u);
+            }
+          }
+          issued = true;
+          mma_commit(smem_u32(&sh.op_empty[s]));
+          RT(rt_issue += clock64() - rt1;)
+          ++g;
+        }
+        for (int kt = 0; kt < (T.halo ? 0 : T.nkt); ++kt, ++g) {
           const int s = g % S;
           RT(rt0 = clock64();)
           if (!mbar_wait(smem_u32(&sh.op_full[s]), (g / S) & 1, abort_flag)) { ok = false; break; }
@@ -1514,7 +1680,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
     bool ok = true;
     RT(unsigned long long rt_a = 0, rt_b = 0;)
     for (int tile = blockIdx.x + eg * gridDim.x; tile < total; tile += kGroups * gridDim.x, li += kGroups) {
-      const Tile T = decode<MODE>(tab, tstart, ninst, tile);
+      const Tile T = decode<MODE, HALO>(tab, tstart, ninst, tile);
       const int b = li % R::kAcc;
       RT(const unsigned long long rt0 = clock64();)
       bool got = mbar_wait(smem_u32(&sh.tfull[b]), (li / R::kAcc) & 1, abort_flag);
@@ -1564,30 +1730,41 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
 
 __global__ void __launch_bounds__(TmaRoles<FWD, 0>::kThreads, 1) k_conv_fwd_tma(const ConvDesc* __restrict__ tab,
                                                                          const int* __restrict__ tstart, int ninst,
-                                                                         int total, int bnmax, int raw_bytes,
+                                                                         int total, int bnmax, int raw_bytes, int op_bytes,
                                                                          int32_t* status) {
-  conv_tma_body<FWD, 0>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+  conv_tma_body<FWD, 0, false>(tab, tstart, ninst, total, bnmax, raw_bytes, op_bytes, status);
 }
 __global__ void __launch_bounds__(TmaRoles<FWD, 1>::kThreads, 1) k_conv_fwd_tma_w(const ConvDesc* __restrict__ tab,
                                                                            const int* __restrict__ tstart, int ninst,
-                                                                           int total, int bnmax, int raw_bytes,
+                                                                           int total, int bnmax, int raw_bytes, int op_bytes,
                                                                            int32_t* status) {
-  conv_tma_body<FWD, 1>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+  conv_tma_body<FWD, 1, false>(tab, tstart, ninst, total, bnmax, raw_bytes, op_bytes, status);
 }
 __global__ void __launch_bounds__(TmaRoles<DGRAD, 0>::kThreads, 1) k_conv_dgrad_tma(
-    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes,
+    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes, int op_bytes,
     int32_t* status) {
-  conv_tma_body<DGRAD, 0>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+  conv_tma_body<DGRAD, 0, false>(tab, tstart, ninst, total, bnmax, raw_bytes, op_bytes, status);
 }
 __global__ void __launch_bounds__(TmaRoles<DGRAD, 1>::kThreads, 1) k_conv_dgrad_tma_w(
-    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes,
+    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes, int op_bytes,
     int32_t* status) {
-  conv_tma_body<DGRAD, 1>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+  conv_tma_body<DGRAD, 1, false>(tab, tstart, ninst, total, bnmax, raw_bytes, op_bytes, status);
 }
 __global__ void __launch_bounds__(TmaRoles<WGRAD, 0>::kThreads, 1) k_conv_wgrad_tma(
-    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes,
+    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes, int op_bytes,
     int32_t* status) {
-  conv_tma_body<WGRAD, 0>(tab, tstart, ninst, total, bnmax, raw_bytes, status);
+  conv_tma_body<WGRAD, 0, false>(tab, tstart, ninst, total, bnmax, raw_bytes, op_bytes, status);
+}
+// with halo tiles (3x3 launches)
+__global__ void __launch_bounds__(TmaRoles<FWD, 0>::kThreads, 1) k_conv_fwd_tma_h(
+    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes,
+    int op_bytes, int32_t* status) {
+  conv_tma_body<FWD, 0, true>(tab, tstart, ninst, total, bnmax, raw_bytes, op_bytes, status);
+}
+__global__ void __launch_bounds__(TmaRoles<DGRAD, 0>::kThreads, 1) k_conv_dgrad_tma_h(
+    const ConvDesc* __restrict__ tab, const int* __restrict__ tstart, int ninst, int total, int bnmax, int raw_bytes,
+    int op_bytes, int32_t* status) {
+  conv_tma_body<DGRAD, 0, true>(tab, tstart, ninst, total, bnmax, raw_bytes, op_bytes, status);
 }
 
 // one kernel name per mode (profiler filters and launch lists name the mode)
@@ -1625,28 +1802,44 @@ static cudaError_t launch_mode(ConvKernel kern, const ConvDesc* tab, const int* 
   return cudaGetLastError();
 }
 
-bool conv_tma_fits(int mode, int bnmax, int raw_bytes) {
+int conv_tma_op_bytes(int mode, int bnmax) { return tma_op_bytes(mode, bnmax); }
+
+bool conv_halo_fits(int mode, int W, int ch, int bn) {
+  // against the largest per-tap stage a launch can mix in (fp32 source, 128-column tiles)
+  const int raw = std::max(kBM * 64 * 4, halo_raw_bytes(W, ch, 4));
+  const int op = std::max(tma_op_bytes(mode, 128), halo_op_bytes(W, ch, bn));
+  return conv_tma_fits(mode, 128, raw, op);
+}
+
+bool conv_tma_fits(int mode, int bnmax, int raw_bytes, int op_bytes) {
   const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - tma_extra(mode, 0);
-  return avail / (raw_bytes + tma_op_bytes(mode, bnmax)) >= 2;
+  return avail / (raw_bytes + (op_bytes > 0 ? op_bytes : tma_op_bytes(mode, bnmax))) >= 2;
 }
 
 cudaError_t launch_conv_tma(int mode, int wide, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
-                            int raw_bytes, int32_t* status, cudaStream_t st, int max_ctas) {
+                            int raw_bytes, int op_bytes, int32_t* status, cudaStream_t st, int max_ctas) {
   if (total <= 0) return cudaSuccess;
   if (bnmax < 16 || bnmax > 256 || (bnmax & 15) || raw_bytes <= 0 || (raw_bytes & 1023) || mode < 0 || mode > 2)
     return cudaErrorInvalidValue;
-  const int w = mode != 2 && wide ? 1 : 0;
-  typedef void (*TmaKernel)(const ConvDesc*, const int*, int, int, int, int, int32_t*);
-  const TmaKernel kern = mode == 0 ? (w ? k_conv_fwd_tma_w : k_conv_fwd_tma)
-                                   : (mode == 1 ? (w ? k_conv_dgrad_tma_w : k_conv_dgrad_tma) : k_conv_wgrad_tma);
-  cudaError_t e = set_smem_attr_once(4 + 2 * mode + w, reinterpret_cast<const void*>(kern), kTmaSmemBudget);
+  if (op_bytes < 0 || (op_bytes & 1023) || (op_bytes > 0 && op_bytes < tma_op_bytes(mode, bnmax)))
+    return cudaErrorInvalidValue;
+  const int opb = op_bytes > 0 ? op_bytes : tma_op_bytes(mode, bnmax);
+  // an operand slot of its own marks a launch with halo tiles (never wide: 3x3)
+  const bool halo = op_bytes > 0 && mode != 2;
+  const int w = mode != 2 && wide && !halo ? 1 : 0;
+  typedef void (*TmaKernel)(const ConvDesc*, const int*, int, int, int, int, int, int32_t*);
+  const TmaKernel kern = halo ? (mode == 0 ? k_conv_fwd_tma_h : k_conv_dgrad_tma_h)
+                              : (mode == 0 ? (w ? k_conv_fwd_tma_w : k_conv_fwd_tma)
+                                           : (mode == 1 ? (w ? k_conv_dgrad_tma_w : k_conv_dgrad_tma) : k_conv_wgrad_tma));
+  cudaError_t e = set_smem_attr_once(halo ? 10 + mode : 4 + 2 * mode + w, reinterpret_cast<const void*>(kern),
+                                     kTmaSmemBudget);
   if (e != cudaSuccess) return e;
   const int sms = device_sm_count();
-  const size_t smem = tma_smem_bytes(mode, bnmax, raw_bytes, tma_extra(mode, w));
+  const size_t smem = tma_smem_bytes(opb, raw_bytes, tma_extra(mode, w));
   if (smem > (size_t)kTmaSmemBudget) return cudaErrorInvalidValue;
   int grid = total < sms ? total : sms;
   if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
-  kern<<<grid, 32 * tma_warps(mode, w), smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, status);
+  kern<<<grid, 32 * tma_warps(mode, w), smem, st>>>(tab, tstart, n, total, bnmax, raw_bytes, opb, status);
   return cudaGetLastError();
 }
 

@@ -66,11 +66,12 @@ struct InstPlan {
   size_t wt = 0, part = 0, stats = 0, fscr = 0, fcnt = 0, gam = 0, bet = 0, scl = 0, shf = 0, coef = 0;
   size_t maps = 0;
   int stat_tiles = 0;
-  bool bn = false;  // forward statistics / data-gradient BN sums requested
+  bool bn = false;    // forward statistics / data-gradient BN sums requested
+  bool halo = false;  // TMA-fed 3x3 forward / data gradient with halo tiles
 };
 struct Plan {
   int variant = 0;
-  int bnmax = 16, raw = 0, wide = 0;
+  int bnmax = 16, raw = 0, op = 0, wide = 0;
   int total = 0;
   size_t tab = 0, ts = 0, status = 0, aux_tab = 0, aux_ts = 0, fin_tab = 0, fin_ts = 0, red_tab = 0, red_ts = 0;
   size_t bytes = 0, init_bytes = 0;  // init_bytes: the prefix copied from the host
@@ -78,7 +79,7 @@ struct Plan {
 };
 
 int check_args(int mode, int impl, int n, const pnn_conv_args* a) {
-  if (mode < 0 || mode > 2 || impl < 0 || impl > 2 || n <= 0 || n > 4096 || !a)
+  if (mode < 0 || mode > 2 || impl < 0 || impl > 3 || n <= 0 || n > 4096 || !a)
     return set_last_error(PNN_EINVAL, "pnn_conv_run: bad mode, impl or instance count");
   for (int i = 0; i < n; ++i) {
     const pnn_conv_args& g = a[i];
@@ -114,22 +115,31 @@ bool tma_ok(int mode, const pnn_conv_args& g) {
   return tma_wgrad_ok(g.ksize, g.stride, pad, g.c, g.k, g.w, g.x_dtype == PNN_DT_BF16);
 }
 
+// whether instance g of a TMA-fed forward / data-gradient launch takes halo tiles
+bool halo_inst(int mode, const pnn_conv_args& g) {
+  if (mode == 2) return false;
+  const int ncols = mode == 1 ? g.c : g.k, ch = mode == 1 ? g.k : g.c;
+  const int bn = ncols <= tc_ntile_cols(mode, 1) ? ((ncols + 15) & ~15) : tc_ntile_cols(mode, 1);
+  return halo_ok(g.ksize, g.stride, g.ksize / 2, g.h, g.w, ch) && conv_halo_fits(mode, g.w, ch, bn);
+}
+
 int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
   int r = check_args(mode, impl, n, a);
   if (r) return r;
-  bool all_tma = true, any_tma = false;
+  // (an instance with halo tiles needs no per-tap boxes)
+  bool all_tma = true, all_tap = true;
   for (int i = 0; i < n; ++i) {
-    const bool t = tma_ok(mode, a[i]);
-    all_tma = all_tma && t;
-    any_tma = any_tma || t;
+    all_tap = all_tap && tma_ok(mode, a[i]);
+    all_tma = all_tma && (tma_ok(mode, a[i]) || halo_inst(mode, a[i]));
   }
-  if (impl == 1 && !all_tma) return set_last_error(PNN_EINVAL, "pnn_conv_run: the TMA-fed kernel does not take this shape");
+  if ((impl == 1 && !all_tma) || (impl == 3 && !all_tap))
+    return set_last_error(PNN_EINVAL, "pnn_conv_run: the TMA-fed kernel does not take this shape");
   // the training step's rule: TMA-fed where the shape allows (the forward only
-  // for at least 64 output channels)
+  // for at least 64 output channels or with halo tiles)
   bool auto_tma = all_tma;
   if (mode == 0)
-    for (int i = 0; i < n; ++i) auto_tma = auto_tma && a[i].k >= 64;
-  pl.variant = impl == 1 ? 1 : (impl == 2 ? 0 : (auto_tma ? 1 : 0));
+    for (int i = 0; i < n; ++i) auto_tma = auto_tma && ((a[i].k >= 64 && tma_ok(mode, a[i])) || halo_inst(mode, a[i]));
+  pl.variant = (impl == 1 || impl == 3) ? 1 : (impl == 2 ? 0 : (auto_tma ? 1 : 0));
   size_t cur = 0;
   auto take = [&](size_t b) { size_t o = cur; cur = al256(cur + b); return o; };
   pl.tab = take((size_t)n * sizeof(ConvDesc));
@@ -196,7 +206,8 @@ int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
       }
       pl.total += base * ip.splits;
     }
-    if (pl.variant == 1) ip.maps = take(3 * 128);
+    ip.halo = pl.variant == 1 && impl != 3 && halo_inst(mode, g);
+    if (pl.variant == 1) ip.maps = take(4 * 128);
   }
   pl.init_bytes = cur;
   for (int i = 0; i < n; ++i) {
@@ -219,7 +230,22 @@ int make_plan(int mode, int impl, int n, const pnn_conv_args* a, Plan& pl) {
       ip.part = take((size_t)ip.splits * g.k * rsc * 4);
     }
   }
-  if (pl.variant == 1 && mode != 2) pl.raw = kTcBM * 64 * esz;
+  if (pl.variant == 1 && mode != 2) {
+    // per instance: one tap box per k-step, or (halo tiles) one halo box per tile
+    pl.raw = 1024;
+    for (int i = 0; i < n; ++i) {
+      const pnn_conv_args& g = a[i];
+      const int ch = mode == 1 ? g.k : g.c, ncols = mode == 1 ? g.c : g.k;
+      if (pl.in[i].halo) {
+        const int bn = pl.in[i].ntiles == 1 ? ((ncols + 15) & ~15) : tc_ntile_cols(mode, 1);
+        pl.raw = std::max(pl.raw, halo_raw_bytes(g.w, ch, esz));
+        pl.op = std::max(pl.op, halo_op_bytes(g.w, ch, bn));
+      } else {
+        pl.raw = std::max(pl.raw, kTcBM * 64 * esz);
+      }
+    }
+    if (pl.op > 0) pl.op = std::max(pl.op, conv_tma_op_bytes(mode, pl.bnmax));
+  }
   // the training step's rule: the wide-epilogue variant when every tile is
   // one k-step
   pl.wide = pl.variant == 1 && mode != 2;
@@ -315,11 +341,14 @@ int conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void
         if (!e) e = encode_tensor_map_2d(m + 128, g.wt, true, rsc, g.k, 64, bn, 128, &why);
         if (!e) e = encode_tensor_map_2d(m + 256, g.y, g.y_dtype == PNN_DT_BF16, g.k, Mout, 16, 32,
                                          g.y_dtype == PNN_DT_BF16 ? 32 : 64, &why);
+        if (!e && ip.halo)
+          e = encode_tensor_map_2d(m + 384, g.x, g.x_dtype == PNN_DT_BF16, g.c, Min, g.c, halo_rows(g.w), 0, &why);
       } else if (mode == 1) {
         const int bn = ip.ntiles == 1 ? ((g.c + 15) & ~15) : tc_ntile_cols(1, 1);
         e = encode_tensor_map_2d(m, g.dy, false, g.k, Mout, std::min(g.k, 64), kTcBM, 0, &why);
         if (!e) e = encode_tensor_map_2d(m + 128, ws + ip.wt, true, g.ksize * g.ksize * g.k, g.c, 64, bn, 128, &why);
         if (!e) e = encode_tensor_map_2d(m + 256, g.dx, false, g.c, Min, 16, 32, 64, &why);
+        if (!e && ip.halo) e = encode_tensor_map_2d(m + 384, g.dy, false, g.k, Mout, g.k, halo_rows(g.w), 0, &why);
       } else {
         const WgBoxes bx = wg_boxes(g.c, g.k, g.w, ip.pad, g.x_dtype == PNN_DT_BF16);
         e = encode_tensor_map_2d(m, g.x, g.x_dtype == PNN_DT_BF16, g.c, Min, bx.cwx, bx.hrows, 0, &why);
@@ -329,6 +358,7 @@ int conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void
       c.tma_a = ws + ip.maps;
       c.tma_b = ws + ip.maps + 128;
       c.tma_y = mode == 2 ? nullptr : ws + ip.maps + 256;
+      c.tma_h = ip.halo ? ws + ip.maps + 384 : nullptr;
     }
     if (ip.bn && mode == 0) {
       // forward statistics: the epilogue's per-tile partials, then the
@@ -401,7 +431,8 @@ int conv_run(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* a, void
   if (e == cudaSuccess && mode == 1)
     e = launch_wtrans(reinterpret_cast<const WtDesc*>(ws + pl.aux_tab), auxts, n, aux_ts.back(), st);
   auto conv_launch = [&]() {
-    if (pl.variant == 1) return launch_conv_tma(mode, pl.wide, tab, tsd, n, pl.total, pl.bnmax, pl.raw, status, st);
+    if (pl.variant == 1)
+      return launch_conv_tma(mode, pl.wide, tab, tsd, n, pl.total, pl.bnmax, pl.raw, pl.op, status, st);
     if (mode == 0) return launch_conv_fwd_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
     if (mode == 1) return launch_conv_dgrad_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);
     return launch_conv_wgrad_tc(tab, tsd, n, pl.total, pl.bnmax, status, st);

@@ -56,6 +56,11 @@ struct ConvDesc {
   // 128-byte swizzle)
   const void* tma_a;
   const void* tma_b;
+  // TMA-fed 3x3 forward / data gradient whose tiles lie inside one image
+  // (halo_ok): tensor map over the same A source rows with box [halo_rows(W)
+  // rows x channels] (no swizzle) -- one box per tile covers all nine taps
+  // (null: one box per tap)
+  const void* tma_h;
   // TMA-fed forward: tensor map over the output y [pixels][K] (box 16
   // columns x 32 rows, 64-byte swizzle for fp32, 32-byte for bf16), or null
   const void* tma_y;
@@ -207,13 +212,20 @@ cudaError_t launch_conv_wgrad_tc(const ConvDesc* tab, const int* tstart, int n, 
                                  int32_t* status, cudaStream_t st, int max_ctas = 0);
 // TMA-fed stride-1 forward (mode 0), data-gradient (mode 1) or weight-gradient
 // (mode 2) tensor-core conv; raw_bytes: one pipeline stage's raw slot (the
-// largest over the launch's instances, a multiple of 1024)
+// largest over the launch's instances, a multiple of 1024); op_bytes: one
+// stage's operand slot when the launch has halo tiles (the larger of
+// halo_op_bytes and the default slot), 0 for the default slot
 // wide: every tile of the launch is one k-step (the epilogue bounds the
 // kernel): the variant with three epilogue groups and two transform warps
 cudaError_t launch_conv_tma(int mode, int wide, const ConvDesc* tab, const int* tstart, int n, int total, int bnmax,
-                            int raw_bytes, int32_t* status, cudaStream_t st, int max_ctas = 0);
+                            int raw_bytes, int op_bytes, int32_t* status, cudaStream_t st, int max_ctas = 0);
 // whether the TMA-fed kernel of `mode` holds at least two stages of this size
-bool conv_tma_fits(int mode, int bnmax, int raw_bytes);
+bool conv_tma_fits(int mode, int bnmax, int raw_bytes, int op_bytes = 0);
+// the default operand slot of a TMA-fed stage (A then bnmax weight rows)
+int conv_tma_op_bytes(int mode, int bnmax);
+// whether a halo instance (mode 0 or 1; A source W x ch, N tile bn) leaves
+// two stages even beside per-tap instances of the same launch
+bool conv_halo_fits(int mode, int W, int ch, int bn);
 // record a message for pnn_last_error(NULL) and return `code`
 int set_last_error(int code, const char* msg);
 // streaming multiprocessors of the current device, queried once per device
@@ -290,6 +302,31 @@ PNN_HD inline WgBoxes wg_boxes(int C, int K, int W, int pad, bool xbf) {
   return b;
 }
 PNN_HD inline int wg_raw_bytes(const WgBoxes& b) { return (b.yoff + b.ybytes + 1023) & ~1023; }
+
+// TMA-fed 3x3 forward / data gradient, halo tiles.  A 128-pixel tile that
+// lies inside one image reads input pixels m0 - W - 1 .. m0 + 128 + W: one
+// box of halo_rows(W) rows.  The transform forms three copies of it, one per
+// column offset s' in {-1, 0, 1}, each of 128 + 2W rows (copy s' row j =
+// pixel m0 - W + s' + j, zero where that pixel lies outside the tile's image
+// or where the output column x - s' would leave the row), in the
+// no-swizzle K-major layout: one plane of 16-byte rows per 8 channels.  Tap
+// (r', s') is then copy s' from row (r' + 1) W: a descriptor offset, for any
+// W.  Needs 128 | H*W (no tile crosses an image), W <= 63 (a TMA box holds
+// at most 256 rows) and 16 | channels <= 64.
+PNN_HD inline bool halo_ok(int k, int stride, int pad, int H, int W, int ch) {
+  return k == 3 && stride == 1 && pad == 1 && W > 0 && (H * W) % kTcBM == 0 && kTcBM + 2 * W + 2 <= 256 &&
+         ch % 16 == 0 && ch <= 64;
+}
+PNN_HD inline int halo_rows(int W) { return kTcBM + 2 * W + 2; }
+PNN_HD inline int halo_plane_bytes(int W) { return (kTcBM + 2 * W) * 16; }
+PNN_HD inline int halo_copy_bytes(int W, int ch) { return (ch / 8) * halo_plane_bytes(W); }
+// weight boxes of a halo tile: the tile's whole K = 9 * ch in boxes of 64
+PNN_HD inline int halo_nbox(int ch) { return (9 * ch + 63) / 64; }
+PNN_HD inline int halo_raw_bytes(int W, int ch, int esz) { return (halo_rows(W) * ch * esz + 1023) & ~1023; }
+// operand slot of a halo tile: the weight boxes (bn rows each), then the three copies
+PNN_HD inline int halo_op_bytes(int W, int ch, int bn) {
+  return (halo_nbox(ch) * bn * 128 + 3 * halo_copy_bytes(W, ch) + 1023) & ~1023;
+}
 
 // ---------------------------------------------------------------- conv kernel choice
 // (mode 0 forward, 1 data gradient, 2 weight gradient; variant 1 = TMA-fed,

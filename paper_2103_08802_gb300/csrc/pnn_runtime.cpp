@@ -114,6 +114,7 @@ struct Launch {
   int shape[6];         // first op: conv (C_in, C_out, k, stride, H_out, W_out); else (C, H, W, 0, 0, 0)
   int esz = 4;          // TMA-fed conv: largest element size of the A sources
   int raw = 0;          // TMA-fed conv: raw slot bytes of one stage
+  int op = 0;           // TMA-fed conv with halo tiles: operand slot bytes of one stage (0: default)
   int wide = 0;         // TMA-fed forward / data gradient: every tile one k-step (the wide-epilogue variant)
   int block = -1;       // fine forward / backward: position of the layer in its segment
 };
@@ -123,6 +124,16 @@ struct Launch {
 static int conv_mode(int kind) { return kind == K_DGRAD_TC ? 1 : (kind == K_WGRAD_TC ? 2 : 0); }
 static int tc_ntile_w(int kind, int variant) { return tc_ntile_cols(conv_mode(kind), variant); }
 static int tc_mtile_rows(int kind, int variant, int C) { return tc_tile_rows(conv_mode(kind), variant, C); }
+// conv_impl values with the TMA-fed kernels (4: without halo tiles)
+static bool tma_impl(int conv_impl) { return conv_impl == 0 || conv_impl == 4; }
+// a TMA-fed 3x3 forward / data gradient instance that takes halo tiles:
+// A source H x W x ch, N tile bn
+static bool use_halo(int conv_impl, int mode, int k, int stride, int pad, int H, int W, int ch, int bn) {
+  return conv_impl == 0 && halo_ok(k, stride, pad, H, W, ch) && conv_halo_fits(mode, W, ch, bn);
+}
+static int tma_bn(int mode, int ncols) {
+  return ncols <= tc_ntile_cols(mode, 1) ? ((ncols + 15) & ~15) : tc_ntile_cols(mode, 1);
+}
 
 const char* kKindName[K_NKINDS] = {"conv_fwd", "conv_dgrad", "conv_wgrad", "wgrad_reduce", "elementwise",
                                    "elementwise_bwd", "bn_finalize", "bn_bwd_reduce", "bn_bwd_finalize",
@@ -322,13 +333,15 @@ struct pnn_net {
     c.in = in; c.out = out; c.res = res; c.w = w; c.k = k; c.stride = stride; c.pad = k / 2;
     c.key[0] = key0; c.key[1] = slot;
     int M = B * P * Q;
-    if (act_dt == DT_BF16 && (opt.conv_impl == 0 || opt.conv_impl == 3) && iv.C % 8 == 0 && cout % 8 == 0) {
+    if (act_dt == DT_BF16 && (tma_impl(opt.conv_impl) || opt.conv_impl == 3) && iv.C % 8 == 0 && cout % 8 == 0) {
       // tcgen05 path: 128-pixel tiles, all output channels (<= 256) per tile
       c.kind = K_CONV_FWD_TC;
       // the TMA-fed forward (eight epilogue warps) pays off when the epilogue
-      // is wide (measured: 2x on 16->64 with the residual); narrow outputs keep
-      // the thread-gathered kernel, which is faster there
-      c.variant = opt.conv_impl == 0 && cout >= 64 && tma_shape_ok(k, stride, k / 2, iv.C) ? 1 : 0;
+      // is wide (measured: 2x on 16->64 with the residual) or when the 3x3
+      // taps come from one halo box; other narrow outputs keep the
+      // thread-gathered kernel, which is faster there
+      const bool halo = use_halo(opt.conv_impl, 0, k, stride, k / 2, iv.H, iv.W, iv.C, tma_bn(0, cout));
+      c.variant = tma_impl(opt.conv_impl) && ((cout >= 64 && tma_shape_ok(k, stride, k / 2, iv.C)) || halo) ? 1 : 0;
       c.mtiles = cdiv(M, kTcBM);
       c.ntiles = cdiv(cout, tc_ntile_w(c.kind, c.variant));
     } else {
@@ -521,7 +534,7 @@ struct pnn_net {
           wg.kind = K_WGRAD_TC;
           {
             const int src = vals[f.in].virt ? vals[f.in].src : f.in;
-            wg.variant = opt.conv_impl == 0 && tma_wgrad_ok(f.k, f.stride, f.pad, vals[f.in].C, ov.C, vals[f.in].W,
+            wg.variant = tma_impl(opt.conv_impl) && tma_wgrad_ok(f.k, f.stride, f.pad, vals[f.in].C, ov.C, vals[f.in].W,
                                                              vals[src].dt == DT_BF16)
                              ? 1
                              : 0;
@@ -556,7 +569,11 @@ struct pnn_net {
           const Value& iv = vals[f.in];
           if (act_dt == DT_BF16 && opt.conv_impl != 1 && iv.C % 8 == 0 && ov.C % 8 == 0 && params[f.w].off % 8 == 0) {
             dg.kind = K_DGRAD_TC;
-            dg.variant = opt.conv_impl == 0 && tma_shape_ok(f.k, f.stride, f.pad, ov.C) ? 1 : 0;
+            const int bn = tma_bn(1, iv.C);
+            dg.variant = tma_impl(opt.conv_impl) && (tma_shape_ok(f.k, f.stride, f.pad, ov.C) ||
+                                                     use_halo(opt.conv_impl, 1, f.k, f.stride, f.pad, ov.H, ov.W, ov.C, bn))
+                             ? 1
+                             : 0;
             dg.mtiles = cdiv((int64_t)B * iv.H * iv.W, kTcBM);
             dg.ntiles = cdiv(iv.C, tc_ntile_w(dg.kind, dg.variant));
           } else {
@@ -1307,8 +1324,11 @@ int pnn_net::build_tables() {
               const bool a_bf16 = fwd && c.x.dt == DT_BF16;
               const int64_t a_rows = fwd ? (int64_t)B * iv.H * iv.W : (int64_t)B * ov.H * ov.W;
               const int bn = o.ntiles == 1 ? ((ncols + 15) & ~15) : tc_ntile_w(o.kind, o.variant);
-              // a third map over the output for the epilogue's TMA stores
-              CUtensorMap maps[3];
+              // a third map over the output for the epilogue's TMA stores, a
+              // fourth (halo tiles) over the A source with one box per tile
+              const int aW = fwd ? iv.W : ov.W, aH = fwd ? iv.H : ov.H;
+              const bool halo = use_halo(opt.conv_impl, fwd ? 0 : 1, o.k, o.stride, o.pad, aH, aW, ch, bn);
+              CUtensorMap maps[4];
               memset(maps, 0, sizeof maps);
               if (ws) {
                 int r = encode_map(&maps[0], a_src, a_bf16, ch, a_rows, std::min(ch, 64), kTcBM, 0);
@@ -1318,12 +1338,14 @@ int pnn_net::build_tables() {
                                  ov.dt == DT_BF16 ? 32 : 64);
                 if (!r && !fwd)  // data gradient: dx [pixels][C] fp32, stored or reduce-added
                   r = encode_map(&maps[2], P<float>(gptr(o.in)), false, iv.C, (int64_t)B * iv.H * iv.W, 16, 32, 64);
+                if (!r && halo) r = encode_map(&maps[3], a_src, a_bf16, ch, a_rows, ch, halo_rows(aW), 0);
                 if (r) return r;
               }
               const size_t mo = put(maps, sizeof maps);
               c.tma_a = ws ? ws + tables_off + mo : nullptr;
               c.tma_b = ws ? ws + tables_off + mo + sizeof(CUtensorMap) : nullptr;
               c.tma_y = ws ? ws + tables_off + mo + 2 * sizeof(CUtensorMap) : nullptr;
+              c.tma_h = ws && halo ? ws + tables_off + mo + 3 * sizeof(CUtensorMap) : nullptr;
             }
             if (o.kind == K_WGRAD_TC && o.variant == 1) {
               // activation halo box [hrows][cwx] (its dtype), gradient box [64][K] fp32
@@ -1522,7 +1544,24 @@ int pnn_net::build_tables() {
             L.raw = std::max(L.raw, wg_raw_bytes(b));
           }
         }
-      if (g.kind == K_CONV_FWD_TC || g.kind == K_DGRAD_TC) L.raw = kTcBM * 64 * L.esz;
+      if (g.kind == K_CONV_FWD_TC || g.kind == K_DGRAD_TC) {
+        // per instance: one tap box per k-step, or (halo tiles) one halo box per tile
+        L.raw = 1024;
+        for (int id : g.ops) {
+          const POp& o = ops[id];
+          const bool fwd = o.kind == K_CONV_FWD_TC;
+          const Value& av = fwd ? vals[o.in] : vals[o.out];  // the A source
+          const int ncols = fwd ? vals[o.out].C : vals[o.in].C;
+          const int bn = o.ntiles == 1 ? ((ncols + 15) & ~15) : tc_ntile_w(o.kind, o.variant);
+          if (g.variant == 1 && use_halo(opt.conv_impl, fwd ? 0 : 1, o.k, o.stride, o.pad, av.H, av.W, av.C, bn)) {
+            L.raw = std::max(L.raw, halo_raw_bytes(av.W, av.C, L.esz));
+            L.op = std::max(L.op, halo_op_bytes(av.W, av.C, bn));
+          } else {
+            L.raw = std::max(L.raw, kTcBM * 64 * L.esz);
+          }
+        }
+        if (L.op > 0) L.op = std::max(L.op, conv_tma_op_bytes(conv_mode(g.kind), L.aux));
+      }
       if ((g.kind == K_CONV_FWD_TC || g.kind == K_DGRAD_TC) && g.variant == 1) {
         L.wide = 1;
         for (int id : g.ops) {
@@ -1662,21 +1701,21 @@ int pnn_net::run_phase(int p, cudaStream_t st, int cap) {
       case K_CONV_FWD: e = launch_conv_fwd_simt((const ConvDesc*)tab, ts, L.count, L.total, L.variant, st); break;
       case K_CONV_FWD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(0, L.wide, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
-                                  st, cap)
+                ? launch_conv_tma(0, L.wide, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, L.op,
+                                  P<int32_t>(status_off), st, cap)
                 : launch_conv_fwd_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off), st, cap);
         break;
       case K_DGRAD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(1, L.wide, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
-                                  st, cap)
+                ? launch_conv_tma(1, L.wide, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, L.op,
+                                  P<int32_t>(status_off), st, cap)
                 : launch_conv_dgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
                                        st, cap);
         break;
       case K_WGRAD_TC:
         e = L.variant == 1
-                ? launch_conv_tma(2, L.wide, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, P<int32_t>(status_off),
-                                  st, cap)
+                ? launch_conv_tma(2, L.wide, (const ConvDesc*)tab, ts, L.count, L.total, L.aux, L.raw, L.op,
+                                  P<int32_t>(status_off), st, cap)
                 : launch_conv_wgrad_tc((const ConvDesc*)tab, ts, L.count, L.total, L.aux, P<int32_t>(status_off),
                                        st, cap);
         break;
@@ -2563,7 +2602,7 @@ int pnn_profile_trace(pnn_net* n, int32_t max, pnn_trace* out, int32_t* count) {
     pnn_trace& r = out[i];
     float t = 0.f;
     cudaEventElapsedTime(&t, n->pev[2 * i], n->pev[2 * i + 1]);
-    r.kind = L.kind; r.variant = L.variant + (L.wide ? 1 : 0); r.phase = L.phase; r.instances = L.count;
+    r.kind = L.kind; r.variant = L.variant + (L.wide ? 1 : (L.op > 0 ? 2 : 0)); r.phase = L.phase; r.instances = L.count;
     r.tiles = L.total;
     for (int j = 0; j < 6; ++j) r.shape[j] = L.shape[j];
     r.block = L.block;

@@ -112,6 +112,19 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
   d |= (uint64_t)2 << 61;                  // swizzle mode: 128 B
   return d;
 }
+// shared-memory matrix descriptor: K-major, no swizzle.  Core matrices of 8
+// rows x 16 bytes (rows 16 bytes apart, 128 contiguous bytes); lbo = bytes
+// between core matrices adjacent in K, sbo = bytes between adjacent 8-row
+// groups.  The start needs only 16-byte alignment, so a window that starts
+// at any row of a row-contiguous plane is a valid operand.
+__device__ __forceinline__ uint64_t nosw_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((addr & 0x3FFFF) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFF) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
+  d |= (uint64_t)1 << 46;                  // descriptor version (sm_100 family); swizzle mode 0: none
+  return d;
+}
 // instruction descriptor: kind::f16, A = B = bf16, D = f32, both K-major, M x N
 __device__ __forceinline__ uint32_t idesc_bf16(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);

@@ -424,7 +424,7 @@ class ParaNet:
 
 
 CONV_MODE = {"forward": 0, "dgrad": 1, "wgrad": 2}
-CONV_IMPL = {"auto": 0, "tma": 1, "gathered": 2}
+CONV_IMPL = {"auto": 0, "tma": 1, "gathered": 2, "tma_tap": 3}
 DTYPE = {"f32": 0, "bf16": 1}
 
 

@@ -142,6 +142,14 @@ CASES = {
     "1x1_c512_k256_fp32x": dict(batch=2, h=7, w=7, c=512, k=256, ksize=1, stride=1, bn=True, x_fp32=True),
     "3x3_c8_k24_raw": dict(batch=2, h=9, w=10, c=8, k=24, ksize=3, stride=1, bn=False),
     "3x3_c64_k64_norelu": dict(batch=2, h=8, w=8, c=64, k=64, ksize=3, stride=1, bn=True, relu=False),
+    # halo tiles (128 | h*w, w <= 63): one tile per image, a wide image, a
+    # narrow one, A sources of 16, 32 and 48 channels (forward c, data
+    # gradient k); 64 channels at w = 16 exceed two stages of shared memory
+    # and keep one box per tap
+    "3x3_c32_k16_halo_hw128": dict(batch=3, h=16, w=8, c=32, k=16, ksize=3, stride=1, bn=True),
+    "3x3_c16_k32_halo_w32": dict(batch=2, h=8, w=32, c=16, k=32, ksize=3, stride=1, bn=True),
+    "3x3_c48_k16_halo_w4": dict(batch=2, h=32, w=4, c=48, k=16, ksize=3, stride=1, bn=False),
+    "3x3_c64_k64_w16_tap": dict(batch=2, h=16, w=16, c=64, k=64, ksize=3, stride=1, bn=True),
 }
 # grouped: instances of different stages in one launch, as the N subnetworks'
 # same layer in a step (stage 1 / 2 / 3 bottleneck 3x3 and 1x1 convs)
@@ -149,6 +157,10 @@ GROUPS = {
     "group_3x3": [dict(batch=2, h=16, w=16, c=16, k=16, ksize=3, stride=1, bn=True),
                   dict(batch=2, h=8, w=8, c=32, k=32, ksize=3, stride=1, bn=True),
                   dict(batch=2, h=4, w=4, c=64, k=64, ksize=3, stride=1, bn=True)],
+    # halo instances (16x16, 16x8) beside per-tap ones (8x8: 128 does not divide h*w)
+    "group_3x3_halo": [dict(batch=2, h=16, w=16, c=16, k=16, ksize=3, stride=1, bn=True),
+                       dict(batch=2, h=16, w=8, c=32, k=32, ksize=3, stride=1, bn=True),
+                       dict(batch=3, h=8, w=8, c=64, k=64, ksize=3, stride=1, bn=True)],
     "group_1x1_expand": [dict(batch=2, h=16, w=16, c=16, k=64, ksize=1, stride=1, bn=True),
                          dict(batch=2, h=8, w=8, c=32, k=128, ksize=1, stride=1, bn=True),
                          dict(batch=2, h=4, w=4, c=64, k=256, ksize=1, stride=1, bn=True)],
@@ -158,6 +170,13 @@ GROUPS = {
 def _cases(name, seed=0):
     specs = GROUPS[name] if name in GROUPS else [CASES[name]]
     return [Case(seed + 17 * i, **s) for i, s in enumerate(specs)]
+
+
+def _halo(mode, s):
+    """Whether the TMA-fed kernel takes halo tiles for this instance."""
+    ch = s["c"] if mode == "forward" else s["k"]
+    return (mode != "wgrad" and s["ksize"] == 3 and s["stride"] == 1 and (s["h"] * s["w"]) % 128 == 0
+            and 128 + 2 * s["w"] + 2 <= 256 and ch % 16 == 0 and ch <= 64)
 
 
 def _tma_ok(mode, s):
@@ -178,8 +197,10 @@ def _params(mode):
     for name in list(CASES) + list(GROUPS):
         specs = GROUPS[name] if name in GROUPS else [CASES[name]]
         impls = ["gathered"]
-        if all(_tma_ok(mode, s) for s in specs):
+        if all(_tma_ok(mode, s) or _halo(mode, s) for s in specs):
             impls.append("tma")
+            if any(_halo(mode, s) for s in specs) and all(_tma_ok(mode, s) for s in specs):
+                impls.append("tma_tap")  # the same launch with one box per tap
         out += [(name, impl) for impl in impls]
     return out
 
