@@ -393,6 +393,25 @@ def dram_traffic(symbol):
     return rec
 
 
+def launch_groups(trace, steps, n=14):
+    """The n launch groups (kind, variant, first-instance shape, instances)
+    with the most device time per step, with their algorithmic GB/s against
+    the measured HBM peak."""
+    pk, _ = peaks()
+    groups = {}
+    for r in trace or []:
+        k = (r["kind"], r["variant"], r["shape"], r["instances"])
+        g = groups.setdefault(k, [0.0, 0, 0.0])
+        g[0] += r["ms"]; g[1] += 1; g[2] += r["bytes"]
+    out = []
+    for (kind, variant, shape, inst), (ms, cnt, by) in sorted(groups.items(), key=lambda kv: -kv[1][0])[:n]:
+        gbs = by / (ms / 1e3) / 1e9 if ms else 0.0
+        out.append({"kernel": KERNEL_SYMBOL.get((kind, variant), kind), "shape": list(shape), "instances": inst,
+                    "launches_per_step": cnt / steps, "ms_per_step": ms / steps, "us_per_launch": 1e3 * ms / cnt,
+                    "gbs": gbs, "frac_of_hbm": gbs / pk["hbm_gbs"]})
+    return out
+
+
 def roofline_of(prof, steps, trace=None):
     """Roofline record of the dominant kernel: the launch group (kind,
     variant, first-instance shape, instances) with the largest device time in
@@ -637,6 +656,7 @@ def our_arm(args, desc, rank, local, world, dist):
         "conv_frac_of_bf16_peak": (conv_flops / (conv_ms / 1e3) / 1e12) / pk["bf16_tflops_sustained"] if conv_ms else None,
         "conv_share_of_device_time": conv_ms / total_prof_ms if total_prof_ms else None,
         "roofline": roofline,
+        "launch_groups": launch_groups(trace, args.steps),
         "kernels": {k: {"ms_per_step": v[0] / args.steps, "launches_per_step": v[1] / args.steps,
                         "gflop_per_step": v[2] / args.steps / 1e9, "gb_per_step": v[3] / args.steps / 1e9}
                     for k, v in sorted(prof.items(), key=lambda kv: -kv[1][0])},

@@ -1022,14 +1022,20 @@ __device__ __forceinline__ void transform_stage(const uint8_t* __restrict__ rawp
                                                 const float* __restrict__ scs, const float* __restrict__ sfs,
                                                 const TStage& t) {
   constexpr int G = XBF ? 4 : 2;  // chunks per group (fp32 raw: two 16-byte words a chunk)
+  // only the stage's kread / 8 chunks are visited (a warp-uniform count);
+  // the per-row order is a permutation of them: j ^ h(row) when the count
+  // is a power of two, else j
+  const int nv = t.kread >> 3;
+  const int pm = (nv & (nv - 1)) == 0 ? nv - 1 : 0;
 #pragma unroll
   for (int h = 0; h < 8; h += G) {
-  if (h < t.jbeg || h >= t.jend) continue;
+  if (h >= nv || h < t.jbeg || h >= t.jend) continue;
   uint4 raw[G][XBF ? 1 : 2];
 #pragma unroll
   for (int jj = 0; jj < G; ++jj) {
     const int j = h + jj;
-    const int cc = j ^ t.hrow;
+    if (j >= nv) continue;
+    const int cc = pm ? (j ^ t.hrow) & pm : j;
     const int e8 = cc * 8;
     if (e8 >= t.kread) continue;
     const int ti = BIG ? 0 : e8 >> t.lg;
@@ -1044,7 +1050,8 @@ __device__ __forceinline__ void transform_stage(const uint8_t* __restrict__ rawp
 #pragma unroll
   for (int jj = 0; jj < G; ++jj) {
     const int j = h + jj;
-    const int cc = j ^ t.hrow;
+    if (j >= nv) continue;
+    const int cc = pm ? (j ^ t.hrow) & pm : j;
     const int e8 = cc * 8;
     if (e8 >= t.kread) continue;
     const int ti = BIG ? 0 : e8 >> t.lg;
