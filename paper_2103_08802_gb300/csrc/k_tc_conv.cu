@@ -1174,110 +1174,113 @@ __device__ __forceinline__ void halo_transform(const uint8_t* __restrict__ rawp,
   }
 }
 
-// one A half-unit of the weight-gradient transform (constants for a tile)
-struct WgA {
-  bool on;
-  int jg, pg, hf;         // row group (of the up to 256 tile rows), pixel group, half
-  int c0, cl, hoff, dyr, dxs;
-  Pix px;                 // pixel of K position 8*pg + 4*hf (3x3 only)
-};
-__device__ __forceinline__ WgA wg_aunit(const Tile& T, const ConvDesc& d, int a, int nA, int cbase) {
-  WgA u;
-  u.on = a < nA;
-  const int au = a >> 1;
-  u.hf = a & 1;
-  u.jg = au >> 3;
-  u.pg = au & 7;
-  const int j0 = T.m0 + u.jg * 8;
-  const int tap = j0 / d.C;
-  u.c0 = j0 - tap * d.C;
-  const int r = tap / d.S, sx = tap - r * d.S;
-  u.hoff = r * d.W + sx;
-  u.dyr = r - d.pad;
-  u.dxs = sx - d.pad;
-  u.cl = u.c0 - cbase;
-  if (u.on && !(d.R == 1 && d.S == 1)) u.px.init(T.pbeg + u.pg + 32 * u.hf, d.P, d.Q);
-  return u;
-}
+// Weight-gradient operands in the MN-major no-swizzle layout (the
+// contraction runs over pixels, so both operands keep the channels of a
+// pixel together, as they arrive, and no transposes are needed): a plane of
+// 64 pixel rows x 16 bytes (8 channels) per 8-row M group of A -- rows
+// (tap, c) of the tile -- and per 8-column N group of B -- output channels;
+// planes 1 KB apart (the descriptors' MN-group stride), 8-pixel groups 128
+// bytes apart (their K-group stride).
+constexpr int kWgPlane = kBK * 16;
 
-// Weight-gradient transform of one tile (256 threads, up to 256 rows).  The
-// operands are built in half-units of 8 rows x 4 pixels: A half-unit (rows
-// jg*8 .. jg*8+7 = (tap, c .. c+7) of the tile; BN scale/shift + ReLU of the
-// producing layer; zero outside the image or the split) from the halo box,
-// B half-unit (k_out kg*8 .. +7) from the gradient box.  Unit (g, pg) holds
-// the k-step pixels pg, pg+8, .., pg+56 at K positions 8*pg .. 8*pg+7, half
-// `hf` the pixels pg + 8*(4*hf + i), i < 4, at K bytes 8*hf of chunk pg.  The
-// contraction sums over pixels, so a K permutation shared by A and B leaves it
-// unchanged; this one makes the lanes of a warp read consecutive raw rows.
-// Thread t takes A half-units t and t + 256 and B half-unit 255 - t (those
-// that exist); rows 128-255 go to the second 16 KB half of A; rows past the
-// layer's M are not written (the MMA rows are independent and the epilogue
-// does not store them).
-__device__ __forceinline__ void store_half8x4(const uint32_t (&w)[4][4], uint8_t* base, int row0, int chunk,
-                                              int hf) {
-  // w[pixel][pair of rows] -> rows row0 + c, 4 pixels each (8 bytes)
+// One k-step of the weight-gradient transform (256 threads).  A units are
+// (activation box row u, 8-channel chunk jb): the chunk is transformed once
+// (BN scale/shift + ReLU of the producing layer, bf16) and stored to every
+// (tap, chunk) plane of the tile that reads it, at pixel row k = u - halo -
+// off(tap), zero where that output pixel's tap leaves the image or the
+// pixel lies past the split.  B units (pixel k, 8-channel group n) convert
+// the output gradient to bf16.  Units are spread evenly over the threads;
+// consecutive threads take consecutive rows, each starting at a chunk
+// rotated by its row so that the raw reads of a warp spread over the banks
+// (the stores, one row apart, are conflict-free in any plane).
+template <int KS, typename Sh>
+__device__ __forceinline__ void wg_stage_mn(const Tile& T, const ConvDesc& d, const WgBoxes& bx, int t, bool tr,
+                                            int relu, int cbase, int pix0, const uint8_t* __restrict__ rawx,
+                                            const uint8_t* __restrict__ rawy, uint8_t* __restrict__ A,
+                                            uint8_t* __restrict__ Bt, const Sh& sh) {
+  const bool xbf = d.x.dt == DT_BF16;
+  const int arows = min(d.mtile_rows > 0 ? d.mtile_rows : kBM, T.Mrows - T.m0);
+  const int ng = arows >> 3, g0 = T.m0 >> 3, cg = d.C >> 3;
+  const int nxc = bx.cwx >> 3;  // a power of two (1 .. 16)
+  const int hr = KS == 1 ? kBK : bx.hrows;
+  const int nA = hr * nxc, nbp = T.BN >> 3, nB = kBK * nbp;
+  const bool bpow2 = (nbp & (nbp - 1)) == 0;
+  const float inv_hr = 1.f / (float)hr;  // unit -> (rotation, row) without an integer division (units < 2^12)
+  const int W = d.W, H = d.H;
+  const int Mtot = d.B * H * W;
+  for (int i = t; i < nA + nB; i += 256) {
+    if (i < nA) {
+      const int jr = (int)(((float)i + 0.5f) * inv_hr);
+      const int u = i - jr * hr;
+      const int jb = (jr + u) & (nxc - 1);
+      const int gch = (cbase >> 3) + jb - g0;  // plane of tap 0 for this chunk
+      const int c = cbase + jb * 8;
+      float v[8];
+      if (xbf) {
+        const uint4 q = *reinterpret_cast<const uint4*>(rawx + (u * bx.cwx + jb * 8) * 2);
+        const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&q);
 #pragma unroll
-  for (int c = 0; c < 8; ++c) {
-    const uint32_t sel = (c & 1) ? 0x7632 : 0x5410;
-    const uint2 o = make_uint2(__byte_perm(w[0][c / 2], w[1][c / 2], sel), __byte_perm(w[2][c / 2], w[3][c / 2], sel));
-    *reinterpret_cast<uint2*>(base + swz(row0 + c, chunk) + 8 * hf) = o;
-  }
-}
-template <typename Sh>
-__device__ __forceinline__ void wg_a_stage(const ConvDesc& d, const Tile& T, WgA& u, bool one, bool xbf, bool tr,
-                                           int relu, int pix0, const WgBoxes& bx, const uint8_t* __restrict__ rawx,
-                                           uint8_t* __restrict__ A, const Sh& sh) {
-  // validity of the 4 pixels pix0 + pg + 8 * (4 * hf + i)
-  unsigned xin = 0;
-  if (one) {
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __bfloat1622float2(hh[e]);
+          v[2 * e] = f.x;
+          v[2 * e + 1] = f.y;
+        }
+      } else {
+        const float4 a = *reinterpret_cast<const float4*>(rawx + (u * bx.cwx + jb * 8) * 4);
+        const float4 b = *reinterpret_cast<const float4*>(rawx + (u * bx.cwx + jb * 8) * 4 + 16);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+      }
+      if (tr) {
+        const float4 s0 = *reinterpret_cast<const float4*>(&sh.scale[c]);
+        const float4 s1 = *reinterpret_cast<const float4*>(&sh.scale[c + 4]);
+        const float4 f0 = *reinterpret_cast<const float4*>(&sh.shift[c]);
+        const float4 f1 = *reinterpret_cast<const float4*>(&sh.shift[c + 4]);
+        const float sc[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+        const float sf[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+        act8(v, sc, sf, relu);
+      }
+      const uint4 pk = pack8(v);
+      const uint4 zero = make_uint4(0, 0, 0, 0);
+      if constexpr (KS == 1) {
+        // 1x1: one tap, pixel row u
+        if (gch >= 0 && gch < ng)
+          *reinterpret_cast<uint4*>(A + gch * kWgPlane + u * 16) = pix0 + u < T.pend ? pk : zero;
+      } else {
+        // 3x3, pad 1: the box row is pixel q; it is tap (r, s) of output
+        // pixel q - ((r-1) W + (s-1)) when that pixel's row and column
+        // stay in the image, i.e. x(q) - (s-1) and y(q) - (r-1) do
+        const int q = pix0 - bx.halo + u;
+        const bool qin = q >= 0 && q < Mtot;
+        const int qy = qin ? q / W : 0;
+        const int xq = q - qy * W;
+        const int yq = qin ? qy % H : 0;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) xin |= (pix0 + u.pg + 8 * (4 * u.hf + i) < T.pend ? 1u : 0u) << i;
-  } else {
-    Pix px = u.px;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      if (i) px.step(8, d.P, d.Q);
-      const bool in = pix0 + u.pg + 8 * (4 * u.hf + i) < T.pend && px.y + u.dyr >= 0 && px.y + u.dyr < d.H &&
-                      px.x + u.dxs >= 0 && px.x + u.dxs < d.W;
-      xin |= (in ? 1u : 0u) << i;
-    }
-    u.px.step(kBK, d.P, d.Q);
-  }
-  float sc[8], sf[8];
-  if (tr) {
-    const float4 s0 = *reinterpret_cast<const float4*>(&sh.scale[u.c0]);
-    const float4 s1 = *reinterpret_cast<const float4*>(&sh.scale[u.c0 + 4]);
-    const float4 f0 = *reinterpret_cast<const float4*>(&sh.shift[u.c0]);
-    const float4 f1 = *reinterpret_cast<const float4*>(&sh.shift[u.c0 + 4]);
-    sc[0] = s0.x; sc[1] = s0.y; sc[2] = s0.z; sc[3] = s0.w; sc[4] = s1.x; sc[5] = s1.y; sc[6] = s1.z; sc[7] = s1.w;
-    sf[0] = f0.x; sf[1] = f0.y; sf[2] = f0.z; sf[3] = f0.w; sf[4] = f1.x; sf[5] = f1.y; sf[6] = f1.z; sf[7] = f1.w;
-  }
-  uint32_t w[4][4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int row = u.pg + 8 * (4 * u.hf + i) + u.hoff;
-    float v[8];
-    if (xbf) {
-      const uint4 q = *reinterpret_cast<const uint4*>(rawx + (row * bx.cwx + u.cl) * 2);
-      const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&q);
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float2 f = __bfloat1622float2(hh[e]);
-        v[2 * e] = f.x;
-        v[2 * e + 1] = f.y;
+        for (int tap = 0; tap < 9; ++tap) {
+          const int rp = tap / 3 - 1, sp = tap % 3 - 1;
+          const int gp = gch + tap * cg;
+          const int k = u - bx.halo - (rp * W + sp);
+          if (gp < 0 || gp >= ng || k < 0 || k >= kBK) continue;
+          const bool ok = qin && xq - sp >= 0 && xq - sp < W && yq - rp >= 0 && yq - rp < H && pix0 + k < T.pend;
+          *reinterpret_cast<uint4*>(A + gp * kWgPlane + k * 16) = ok ? pk : zero;
+        }
       }
     } else {
-      const float4 a = *reinterpret_cast<const float4*>(rawx + (row * bx.cwx + u.cl) * 4);
-      const float4 b = *reinterpret_cast<const float4*>(rawx + (row * bx.cwx + u.cl) * 4 + 16);
-      v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-      v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+      const int ib = i - nA;
+      const int nr = ib >> 6, k = ib & (kBK - 1);
+      const int nn = nr + k;
+      const int n = bpow2 ? (nn & (nbp - 1)) : nn % nbp;
+      const bool ok = pix0 + k < T.pend && T.n0 + n * 8 < d.K;
+      uint4 o = make_uint4(0, 0, 0, 0);
+      if (ok) {
+        const float* src = reinterpret_cast<const float*>(rawy) + k * d.K + T.n0 + n * 8;
+        const float4 a = *reinterpret_cast<const float4*>(src);
+        const float4 b = *reinterpret_cast<const float4*>(src + 4);
+        o = make_uint4(pack_bf16(a.x, a.y), pack_bf16(a.z, a.w), pack_bf16(b.x, b.y), pack_bf16(b.z, b.w));
+      }
+      *reinterpret_cast<uint4*>(Bt + n * kWgPlane + k * 16) = o;
     }
-    if (tr) act8(v, sc, sf, relu);
-    const bool in = (xin >> i) & 1;
-#pragma unroll
-    for (int e = 0; e < 4; ++e) w[i][e] = in ? pack_bf16(v[2 * e], v[2 * e + 1]) : 0u;
   }
-  store_half8x4(w, A + (u.jg >> 4) * kABytes, (u.jg & 15) * 8, u.pg, u.hf);
 }
 template <typename Sh>
 __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDesc& d, int t, bool tr, uint32_t& g,
@@ -1285,20 +1288,9 @@ __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDe
                                                      Sh& sh RT(, unsigned long long& rt_a, unsigned long long& rt_b)) {
   const bool xbf = d.x.dt == DT_BF16;
   const WgBoxes bx = wg_boxes(d.C, d.K, d.W, d.pad, xbf);
-  const int tile_rows = d.mtile_rows > 0 ? d.mtile_rows : kBM;
   const int cbase = d.C <= 64 ? 0 : T.m0 % d.C;
   const bool one = d.R == 1 && d.S == 1;
   const int relu = tr ? d.x.relu : 0;
-  const int arows = min(tile_rows, T.Mrows - T.m0);       // rows of the tile in the layer (multiple of 8)
-  const int nA = (arows >> 3) * 16;
-  WgA u0 = wg_aunit(T, d, t, nA, cbase);
-  WgA u1 = wg_aunit(T, d, t + 256, nA, cbase);
-  // B half-unit of this thread
-  const int bh = 255 - t;
-  const bool bside = bh < 2 * T.BN;
-  const int bu = bh >> 1, bhf = bh & 1;
-  const int kg = bu >> 3, bpg = bu & 7;
-  const bool bcols = bside && T.n0 + kg * 8 < d.K;
   for (int kt = 0; kt < T.nkt; ++kt, ++g) {
     const int s = g % S;
     RT(const unsigned long long rt0 = clock64();)
@@ -1313,24 +1305,8 @@ __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDe
     uint8_t* __restrict__ A = gbase + S * raw_bytes + s * op_bytes;
     uint8_t* __restrict__ Bt = A + 2 * kABytes;
     const int pix0 = T.pbeg + kt * kBK;
-    if (u0.on) wg_a_stage(d, T, u0, one, xbf, tr, relu, pix0, bx, rawx, A, sh);
-    if (u1.on) wg_a_stage(d, T, u1, one, xbf, tr, relu, pix0, bx, rawx, A, sh);
-    if (bside) {
-      uint32_t w[4][4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int row = bpg + 8 * (4 * bhf + i);
-        const float* src = reinterpret_cast<const float*>(rawy) + row * d.K + kg * 8;
-        const float4 a = *reinterpret_cast<const float4*>(src);
-        const float4 b = *reinterpret_cast<const float4*>(src + 4);
-        const bool in = bcols && pix0 + row < T.pend;
-        w[i][0] = in ? pack_bf16(a.x, a.y) : 0u;
-        w[i][1] = in ? pack_bf16(a.z, a.w) : 0u;
-        w[i][2] = in ? pack_bf16(b.x, b.y) : 0u;
-        w[i][3] = in ? pack_bf16(b.z, b.w) : 0u;
-      }
-      store_half8x4(w, Bt, kg * 8, bpg, bhf);
-    }
+    if (one) wg_stage_mn<1>(T, d, bx, t, tr, relu, cbase, pix0, rawx, rawy, A, Bt, sh);
+    else wg_stage_mn<3>(T, d, bx, t, tr, relu, cbase, pix0, rawx, rawy, A, Bt, sh);
     fence_proxy_async();
     mbar_arrive(smem_u32(&sh.op_full[s]));
     RT(rt_b += clock64() - rt1;)
@@ -1651,11 +1627,19 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
           // (weight gradient: pixels sit at permuted K positions, all 64 are read)
           const int krem = MODE == WGRAD ? kBK : T.Kt - kt * kBK;
           const int ksub = min(4, (krem + 15) / 16);
-          for (int kk = 0; kk < ksub; ++kk) {
-            mma_bf16(tacc, sw128_desc(a_addr + kk * 32), sw128_desc(b_addr + kk * 32), idesc, (kt | kk) ? 1u : 0u);
-            if (two)
-              mma_bf16(tacc + colstride, sw128_desc(a_addr + kABytes + kk * 32), sw128_desc(b_addr + kk * 32), idesc,
-                       (kt | kk) ? 1u : 0u);
+          if constexpr (MODE == WGRAD) {
+            // MN-major planes: 16 pixels a K step (256 bytes), M/N groups 1 KB apart
+            const uint32_t idesc_mn = idesc | (1u << 15) | (1u << 16);
+            for (int kk = 0; kk < ksub; ++kk) {
+              mma_bf16(tacc, nosw_desc(a_addr + kk * 256, 128, kWgPlane), nosw_desc(b_addr + kk * 256, 128, kWgPlane),
+                       idesc_mn, (kt | kk) ? 1u : 0u);
+              if (two)
+                mma_bf16(tacc + colstride, nosw_desc(a_addr + kABytes + kk * 256, 128, kWgPlane),
+                         nosw_desc(b_addr + kk * 256, 128, kWgPlane), idesc_mn, (kt | kk) ? 1u : 0u);
+            }
+          } else {
+            for (int kk = 0; kk < ksub; ++kk)
+              mma_bf16(tacc, sw128_desc(a_addr + kk * 32), sw128_desc(b_addr + kk * 32), idesc, (kt | kk) ? 1u : 0u);
           }
           issued = true;
           mma_commit(smem_u32(&sh.op_empty[s]));
