@@ -50,7 +50,10 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-sample-batch", type=int, default=1)
+    ap.add_argument("--cpu-sample-batch", type=int, default=1,
+                    help="images per step of the reference arm (the CPU oracle)")
+    ap.add_argument("--cpu-baseline-batch", type=int, default=12,
+                    help="images of the cpu_baseline sample (about 15 s of oracle work on 16 cores)")
     ap.add_argument("--stream-fp32", type=int, default=None, choices=[0, 1],
                     help="keep the residual stream and correction tensors in fp32 (1) or bf16 (0); default: "
                          "the workload's (bf16 for the bf16 workloads)")
@@ -520,7 +523,7 @@ def infer_arm(args, desc, rank, local, world, dist):
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         from oracle import pnn_oracle as O
-        d1 = W.with_batch(desc, args.cpu_sample_batch)
+        d1 = W.with_batch(desc, args.cpu_baseline_batch)
         onet = O.ParaNet(d1, precision="bf16" if d1["precision"] == "bf16" else "fp64")
         theta = W.init_params(onet.spec, seed=0, bf16=d1["precision"] == "bf16")
         x1, _ = W.make_batch(d1)
@@ -640,7 +643,7 @@ def our_arm(args, desc, rank, local, world, dist):
     roofline = roofline_of(prof, args.steps, trace)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        b = args.cpu_sample_batch
+        b = args.cpu_baseline_batch
         t = oracle_sample(desc, b)
         cpu = {"value": b / t, "unit": "images/s", "cores": cores(), "kind": "oracle",
                "sample": f"{b} image(s) of the same network, one forward+backward+SGD step of the CPU "
