@@ -427,11 +427,15 @@ def roofline_of(prof, steps, trace=None):
             k = (r["kind"], r["variant"], r["shape"], r["instances"])
             g = groups.setdefault(k, [0.0, 0, 0.0, 0.0])
             g[0] += r["ms"]; g[1] += 1; g[2] += r["flops"]; g[3] += r["bytes"]
-        (kind, variant, shape, inst), (kms, kn, kfl, kby) = max(groups.items(), key=lambda kv: kv[1][0])
+        # (a group with no algorithmic bytes or FLOPs -- the per-channel BN
+        # finalisation, the head -- has no roof to be measured against)
+        cand = {k: g for k, g in groups.items() if g[2] > 0 or g[3] > 0} or groups
+        (kind, variant, shape, inst), (kms, kn, kfl, kby) = max(cand.items(), key=lambda kv: kv[1][0])
         name = KERNEL_SYMBOL.get((kind, variant), kind)
         what = {"kind": kind, "variant": variant, "first_instance_shape": list(shape), "instances": inst}
     else:
-        name, (kms, kn, kfl, kby) = max(prof.items(), key=lambda kv: kv[1][0])
+        cand = {k: v for k, v in prof.items() if v[2] > 0 or v[3] > 0} or prof
+        name, (kms, kn, kfl, kby) = max(cand.items(), key=lambda kv: kv[1][0])
         kind, what = name, {"kind": name}
     per_launch_ms = kms / kn
     # the bound follows the kernel's algorithmic intensity: below the ridge point
