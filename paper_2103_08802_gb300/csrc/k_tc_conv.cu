@@ -992,8 +992,12 @@ __host__ __device__ constexpr int tma_op_bytes(int mode, int bnmax) { return tma
 // (float [4][256][2])
 constexpr int kTmaRedBytes = 4 * 256 * 2 * 4;
 __host__ __device__ constexpr int tma_ystage(int mode, int w) { return mode == 2 ? 0 : tma_ne(mode, w) * 2 * 2048; }
+// (weight gradient) then the two-pass 3x3 transform's bf16 halo (8-channel
+// planes of box rows) and its per-row tap masks
+constexpr int kWgHaloBytes = 16384;
+constexpr int kWgMaskBytes = 512;
 __host__ __device__ constexpr int tma_extra(int mode, int w) {
-  return tma_ystage(mode, w) + (tma_ne(mode, w) / 4) * kTmaRedBytes;
+  return tma_ystage(mode, w) + (tma_ne(mode, w) / 4) * kTmaRedBytes + (mode == 2 ? kWgHaloBytes + kWgMaskBytes : 0);
 }
 __host__ __device__ inline int tma_stages(int op_bytes, int raw_bytes, int extra) {
   const int avail = kTmaSmemBudget - 1024 - (int)sizeof(TmaShared) - extra;
@@ -1282,21 +1286,143 @@ __device__ __forceinline__ void wg_stage_mn(const Tile& T, const ConvDesc& d, co
     }
   }
 }
+// Two-pass weight-gradient transform of a 3x3 k-step (C <= 64, the box's
+// 8-channel planes of hr rows fit kWgHaloBytes).  Pass 1 (units = box row u
+// x chunk jb, and the B units): the chunk transformed once into the bf16 halo
+// hb[jb][u]; the unit with rotation 0 of each row also stores the row's tap
+// mask (bit t: the pixel is tap t of an output pixel inside the image).
+// Pass 2 (units = A plane gp x pixel row k): plane gp = (tap, jb) row k is
+// hb[jb][k + halo + off(tap)] or zero.  The 256 transform threads meet at
+// named barrier 1 before and between the passes -- every thread, also one
+// whose wait failed, so that none waits at a barrier the others skip.
+template <typename Sh>
+__device__ __forceinline__ void wg_stage_two_pass(const Tile& T, const ConvDesc& d, const WgBoxes& bx, int t, bool tr,
+                                                  int relu, int pix0, bool work, const uint8_t* __restrict__ rawx,
+                                                  const uint8_t* __restrict__ rawy, uint8_t* __restrict__ A,
+                                                  uint8_t* __restrict__ Bt, uint8_t* __restrict__ hb,
+                                                  uint16_t* __restrict__ hmask, const Sh& sh) {
+  const bool xbf = d.x.dt == DT_BF16;
+  const int arows = min(d.mtile_rows > 0 ? d.mtile_rows : kBM, T.Mrows - T.m0);
+  const int ng = arows >> 3, g0 = T.m0 >> 3, cg = d.C >> 3;
+  const int lcg = 31 - __clz(cg);  // cg is a power of two (1 .. 8)
+  const int nxc = bx.cwx >> 3, hr = bx.hrows;
+  const int nA = hr * nxc, nbp = T.BN >> 3, nB = kBK * nbp;
+  const bool bpow2 = (nbp & (nbp - 1)) == 0;
+  const float inv_hr = 1.f / (float)hr;
+  const int W = d.W, H = d.H;
+  const int Mtot = d.B * H * W;
+  asm volatile("bar.sync 1, 256;" ::: "memory");  // the previous k-step's pass 2 has read hb
+  if (work) {
+    for (int i = t; i < nA + nB; i += 256) {
+      if (i < nA) {
+        const int jr = (int)(((float)i + 0.5f) * inv_hr);
+        const int u = i - jr * hr;
+        const int jb = (jr + u) & (nxc - 1);
+        const int c = jb * 8;
+        float v[8];
+        if (xbf) {
+          const uint4 q = *reinterpret_cast<const uint4*>(rawx + (u * bx.cwx + c) * 2);
+          const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&q);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(hh[e]);
+            v[2 * e] = f.x;
+            v[2 * e + 1] = f.y;
+          }
+        } else {
+          const float4 a = *reinterpret_cast<const float4*>(rawx + (u * bx.cwx + c) * 4);
+          const float4 b = *reinterpret_cast<const float4*>(rawx + (u * bx.cwx + c) * 4 + 16);
+          v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+          v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+        }
+        if (tr) {
+          const float4 s0 = *reinterpret_cast<const float4*>(&sh.scale[c]);
+          const float4 s1 = *reinterpret_cast<const float4*>(&sh.scale[c + 4]);
+          const float4 f0 = *reinterpret_cast<const float4*>(&sh.shift[c]);
+          const float4 f1 = *reinterpret_cast<const float4*>(&sh.shift[c + 4]);
+          const float sc[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+          const float sf[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+          act8(v, sc, sf, relu);
+        }
+        *reinterpret_cast<uint4*>(hb + (jb * hr + u) * 16) = pack8(v);
+        if (jr == 0) {
+          // box row u is pixel q; tap (r, s) of output pixel q - ((r-1) W + (s-1))
+          // when x(q) - (s-1) and y(q) - (r-1) stay in the image
+          const int q = pix0 - bx.halo + u;
+          uint32_t m = 0;
+          if (q >= 0 && q < Mtot) {
+            const int qy = q / W;
+            const int xq = q - qy * W, yq = qy % H;
+#pragma unroll
+            for (int tap = 0; tap < 9; ++tap) {
+              const int rp = tap / 3 - 1, sp = tap % 3 - 1;
+              m |= (xq - sp >= 0 && xq - sp < W && yq - rp >= 0 && yq - rp < H ? 1u : 0u) << tap;
+            }
+          }
+          hmask[u] = (uint16_t)m;
+        }
+      } else {
+        const int ib = i - nA;
+        const int nr = ib >> 6, k = ib & (kBK - 1);
+        const int nn = nr + k;
+        const int n = bpow2 ? (nn & (nbp - 1)) : nn % nbp;
+        const bool ok = pix0 + k < T.pend && T.n0 + n * 8 < d.K;
+        uint4 o = make_uint4(0, 0, 0, 0);
+        if (ok) {
+          const float* src = reinterpret_cast<const float*>(rawy) + k * d.K + T.n0 + n * 8;
+          const float4 a = *reinterpret_cast<const float4*>(src);
+          const float4 b = *reinterpret_cast<const float4*>(src + 4);
+          o = make_uint4(pack_bf16(a.x, a.y), pack_bf16(a.z, a.w), pack_bf16(b.x, b.y), pack_bf16(b.z, b.w));
+        }
+        *reinterpret_cast<uint4*>(Bt + n * kWgPlane + k * 16) = o;
+      }
+    }
+  }
+  asm volatile("bar.sync 1, 256;" ::: "memory");  // hb and the masks are complete
+  if (work) {
+    for (int i = t; i < ng * kBK; i += 256) {
+      const int gp = i >> 6, k = i & (kBK - 1);
+      const int gg = g0 + gp;
+      const int tap = gg >> lcg, jb = gg & (cg - 1);
+      const int u = k + bx.halo + (tap / 3 - 1) * W + (tap % 3 - 1);
+      const uint4 v = *reinterpret_cast<const uint4*>(hb + (jb * hr + u) * 16);
+      const bool ok = ((hmask[u] >> tap) & 1) && pix0 + k < T.pend;
+      *reinterpret_cast<uint4*>(A + gp * kWgPlane + k * 16) = ok ? v : make_uint4(0, 0, 0, 0);
+    }
+  }
+}
 template <typename Sh>
 __device__ __forceinline__ void wgrad_transform_tile(const Tile& T, const ConvDesc& d, int t, bool tr, uint32_t& g,
                                                      bool& ok, int S, int raw_bytes, int op_bytes, uint8_t* gbase,
-                                                     Sh& sh RT(, unsigned long long& rt_a, unsigned long long& rt_b)) {
+                                                     uint8_t* hb, Sh& sh
+                                                     RT(, unsigned long long& rt_a, unsigned long long& rt_b)) {
   const bool xbf = d.x.dt == DT_BF16;
   const WgBoxes bx = wg_boxes(d.C, d.K, d.W, d.pad, xbf);
   const int cbase = d.C <= 64 ? 0 : T.m0 % d.C;
   const bool one = d.R == 1 && d.S == 1;
   const int relu = tr ? d.x.relu : 0;
+  // 3x3 with C <= 64 whose bf16 halo fits: two passes (the same decision on
+  // every transform thread: it depends on the instance alone)
+  const bool two = !one && d.C <= 64 && (bx.cwx >> 3) * bx.hrows * 16 <= kWgHaloBytes && bx.hrows * 2 <= kWgMaskBytes;
   for (int kt = 0; kt < T.nkt; ++kt, ++g) {
     const int s = g % S;
     RT(const unsigned long long rt0 = clock64();)
     if (ok && !mbar_wait(smem_u32(&sh.tma_full[s]), (g / S) & 1, &sh.abort_flag)) {
       ok = false;
       sh.abort_flag = 1;
+    }
+    if (two) {
+      RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
+      const uint8_t* __restrict__ rawx = gbase + s * raw_bytes;
+      uint8_t* __restrict__ A = gbase + S * raw_bytes + s * op_bytes;
+      wg_stage_two_pass(T, d, bx, t, tr, relu, T.pbeg + kt * kBK, ok, rawx, rawx + bx.yoff, A, A + 2 * kABytes, hb,
+                        reinterpret_cast<uint16_t*>(hb + kWgHaloBytes), sh);
+      if (ok) {
+        fence_proxy_async();
+        mbar_arrive(smem_u32(&sh.op_full[s]));
+      }
+      RT(rt_b += clock64() - rt1;)
+      continue;
     }
     if (!ok) continue;
     RT(const unsigned long long rt1 = clock64(); rt_a += rt1 - rt0;)
@@ -1470,7 +1596,8 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
         staged = T.d;
       }
       if constexpr (MODE == WGRAD) {
-        wgrad_transform_tile(T, d, threadIdx.x, tr, g, ok, S, raw_bytes, op_bytes, gbase, sh RT(, rt_a, rt_b));
+        wgrad_transform_tile(T, d, threadIdx.x, tr, g, ok, S, raw_bytes, op_bytes, gbase,
+                             red0 + R::kGroups * kTmaRedBytes, sh RT(, rt_a, rt_b));
         continue;
       }
       if (MODE != WGRAD && T.halo) {
