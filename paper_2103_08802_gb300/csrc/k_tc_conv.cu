@@ -462,7 +462,9 @@ __device__ __forceinline__ void add_extra(const ConvDesc& d, int64_t o, int nb, 
 // ystage (forward, may be null): this warp's two 2 KB staging tiles for TMA
 // stores of the output (box 32 rows x 16 columns, swizzled as the output map
 // says); ybuf alternates between them across chunks and tiles.
-template <int MODE>
+// SSTATS: a forward chunk staged in bf16 takes its statistics from the
+// staging tile (the values stored) instead of warp shuffle trees
+template <int MODE, bool SSTATS = false>
 __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, int lane, float (&red)[4][256][2],
                                          int j_first, int j_step, int etid, int ethreads, uint8_t* ystage, int& ybuf,
                                          int bar_id = 2) {
@@ -507,6 +509,8 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
       for (int i = 0; i < 16; ++i) { s1[i] = 0.f; s2[i] = 0.f; }
       const bool vec = full && (d.K % 8) == 0;
       const bool tstore = vec && ystage != nullptr && d.tma_y != nullptr;
+      const bool sstats = SSTATS && stats && tstore && d.y_dt == DT_BF16;
+      uint8_t* staged = nullptr;
       if (mvalid) {
         const int64_t o = (int64_t)m * d.K + nb;
         if (d.res) {
@@ -536,7 +540,9 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
         }
         add_extra(d, o, nb, vec, v);
         RT(if (true) { const unsigned long long cr = clock64(); e5 += cr - c1; })
-        if (d.y_dt == DT_BF16) {
+        // (the packing for a store rounds to bf16 itself; the register
+        // statistics need the rounded values)
+        if (d.y_dt == DT_BF16 && !sstats) {
 #pragma unroll
           for (int i = 0; i < 16; ++i) v[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
         }
@@ -566,9 +572,11 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
             else reinterpret_cast<float*>(d.y)[o + i] = v[i];
           }
         }
+        if (!sstats) {
 #pragma unroll
-        for (int i = 0; i < 16; ++i)
-          if (nb + i < d.K) s1[i] = v[i];
+          for (int i = 0; i < 16; ++i)
+            if (nb + i < d.K) s1[i] = v[i];
+        }
       }
       if (tstore) {
         // the store issued from this buffer two chunks ago must have read it
@@ -577,6 +585,7 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
         __syncwarp();
         RT(e6 += clock64() - cw;)
         uint8_t* st = ystage + ybuf * 2048;
+        staged = st;
         if (d.y_dt == DT_BF16) {
           // 32-byte rows, 32-byte swizzle: 16-byte chunk c at c ^ ((row >> 2) & 1)
 #pragma unroll
@@ -598,7 +607,37 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
         ybuf ^= 1;
       }
       RT(const unsigned long long c2 = clock64(); e1 += c2 - c1;)
-      if (stats) {
+      if (sstats) {
+        // (mean, M2) of the chunk's 16 columns over this warp's valid rows from
+        // the staged tile: lane l reads column l & 15 of rows (l >> 4) + 2i
+        // (the two lanes of a column cover the 32 rows), two passes
+        const int col = lane & 15;
+        const int nvalid = min(32, max(0, T.Mrows - (T.m0 + q * 32)));
+        float vv[16];
+        float a = 0.f;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int r = (lane >> 4) + 2 * i;
+          const int off = r * 32 + ((((col >> 3) ^ (r >> 2)) & 1) << 4) + (col & 7) * 2;
+          const uint32_t bits = *reinterpret_cast<const unsigned short*>(staged + off);
+          vv[i] = r < nvalid ? __uint_as_float(bits << 16) : 0.f;
+          a += vv[i];
+        }
+        a += __shfl_xor_sync(0xffffffffu, a, 16);
+        const float mw = nvalid > 0 ? a / (float)nvalid : 0.f;
+        float b = 0.f;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int r = (lane >> 4) + 2 * i;
+          const float dv = vv[i] - mw;
+          b += r < nvalid ? dv * dv : 0.f;
+        }
+        b += __shfl_xor_sync(0xffffffffu, b, 16);
+        if (lane < 16) {
+          red[q][j0 + lane][0] = mw;
+          red[q][j0 + lane][1] = b;
+        }
+      } else if (stats) {
         // (mean, M2) of the chunk's columns over this warp's valid rows: the
         // column sums, the warp mean broadcast back, the squared deviations
         const float nw = (float)__popc(__ballot_sync(0xffffffffu, mvalid));
@@ -1812,8 +1851,8 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       if (!got) { ok = false; break; }
       fence_after();
       float(&red)[4][256][2] = *reinterpret_cast<float(*)[4][256][2]>(red0 + eg * kTmaRedBytes);
-      epilogue<MODE>(T, tmem + b * bufcols, q, lane, red, 0, 16, (ew & 3) * 32 + lane, 128,
-                     MODE != WGRAD ? ystage0 + ew * 4096 : nullptr, ybuf, bar);
+      epilogue<MODE, W == 1>(T, tmem + b * bufcols, q, lane, red, 0, 16, (ew & 3) * 32 + lane, 128,
+                             MODE != WGRAD ? ystage0 + ew * 4096 : nullptr, ybuf, bar);
       if (kAMult == 2 && min(T.d->mtile_rows, T.Mrows - T.m0) > kBM) {
         // rows 128-255 of the tile, from the second accumulator half
         Tile T2 = T;
