@@ -60,13 +60,13 @@ def _grad_keys(report):
     return [k for k in report if k.startswith("D") or k.startswith("grad")]
 
 
-def _measured(desc, noise_fn, factor, floor):
+def _measured(desc, noise_fn, factor, floor, conv_impl=0):
     """Every key is bounded by max(target bound, factor * measured noise):
     the forward bound for forward tensors, `floor` for D_j and gradients.
     bf16 runs also hold every forward tensor to the forward bound against
-    the float64 oracle."""
+    the float64 oracle.  conv_impl: the library's kernel choice (options)."""
     onet, theta, x, labels = inputs(desc)
-    g = run_gpu(desc, theta, x, labels)
+    g = run_gpu(desc, theta, x, labels, conv_impl=conv_impl)
     o = run_oracle(desc, theta, x, labels)
     err, _ = compare(desc, g, o, LOOSE)
     noise = noise_fn(desc, theta, x, labels, o)
@@ -316,41 +316,26 @@ def _conv_variants(desc, theta, x, labels, conv_impl):
 
 
 @pytest.mark.parametrize("idx", [1, 2, 4, "paper_n3"])
-def test_tma_fed_convs_match_thread_gathered(idx):
-    """The TMA-fed stride-1 convolutions (the default) and the thread-gathered
-    tensor-core convolutions (conv_impl=3) build the same bf16 operands, and the
-    forward kernels accumulate them in the same K order with the same
-    epilogue: every activation, correction tensor, logit and the loss agree bit
-    for bit.  The backward differs only in fp32 summation order -- the TMA-fed
-    weight gradient sums each 64-pixel k-step in a permuted order, and the
-    TMA-fed data gradient of a BN(+ReLU) value also forms that BN's backward
-    sums over its 128-row tiles (the thread-gathered path runs the separate
-    reduction kernel).  A last-bit change of a BN-backward sum can flip the
-    bf16 rounding of gradient operands further down (one bf16 ulp is 4e-3
-    relative), so D_j, the gradients and the SGD update agree to the level of
-    such flips: norm-relative 2e-2, the bound the tensor-core / CUDA-core
-    backward comparison uses; correctness of each path against the oracle is
-    what the parity tests above check.  (VGG-16's 3x3 convs with 64..512
-    channels, ResNet's 1x1 and 3x3 bottleneck convs, the coarse RUs' 3x3 convs
-    at 128 and 256 channels; stride-2 convs take the gathered kernel on both
-    sides.)"""
+def test_thread_gathered_convs_match_oracle(idx):
+    """The thread-gathered tensor-core convolutions (conv_impl=3: no TMA
+    producer) against the oracle's bf16 model within the same measured bound
+    as the default path (test_bf16_full_batch, test_paper_resnet_bf16), on
+    workloads whose default plan does use the TMA-fed forward, data- and
+    weight-gradient kernels.  The two paths build the same bf16 operands; the
+    epilogues differ in fp32 summation orders (the wide-epilogue forward sums
+    a staged chunk's BN-statistics columns per lane, the other kernels by
+    shuffle trees; the TMA-fed data gradient forms the BN-backward sums over
+    its 128-row tiles), and these deep networks respond to such rounding-level
+    changes far beyond them, so each path is held to the oracle rather than
+    to the other.  (VGG-16's 3x3 convs with 64..512 channels, ResNet's 1x1
+    and 3x3 bottleneck convs, the coarse RUs' 3x3 convs at 128 and 256
+    channels; stride-2 convs take the gathered kernel on both paths.)"""
     desc = paper_reduced(3) if idx == "paper_n3" else reduced(idx)
     onet, theta, x, labels = inputs(desc)
     tma = _conv_variants(desc, theta, x, labels, 0)
     assert ("conv_fwd_tc", 1) in tma and ("conv_dgrad_tc", 1) in tma and ("conv_wgrad_tc", 1) in tma, tma
     assert all(v == 0 for _, v in _conv_variants(desc, theta, x, labels, 3))
-    a = run_gpu(desc, theta, x, labels)
-    b = run_gpu(desc, theta, x, labels, conv_impl=3)
-    backward = ("grad", "theta_new", "momentum")
-    for k in a:
-        if k in ("net", "onet"):
-            continue
-        ak, bk = np.asarray(a[k]), np.asarray(b[k])
-        if k in backward or k.startswith("D"):
-            err = np.linalg.norm(ak - bk) / max(np.linalg.norm(bk), 1e-30)
-            assert err <= 2e-2, (k, err)
-        else:
-            np.testing.assert_array_equal(ak, bk, err_msg=k)
+    _measured(desc, bf16_accum_noise, 3.0, TOL["bf16"]["grad"], conv_impl=3)
 
 
 def test_step_is_deterministic():
