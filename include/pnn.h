@@ -423,8 +423,7 @@ int pnn_conv_time(int32_t mode, int32_t impl, int32_t n, const pnn_conv_args* ar
  *   c and k multiples of 8; ksize 1 or 3; stride 1 or 2; stream NULL = legacy default.
  * Every GPU that loads the library keeps these arrays until the process ends.
  * The first call on a device looks up their device addresses (once per
- * device); make that first call before capturing a stream into a CUDA graph.
- * All calls share the arrays and each call overwrites them: calls that
+ * device, thread-safe).  All calls share the arrays and each call overwrites them: calls that
  * overlap on the GPU (other streams, other threads) race.  Synchronises.
  * Errors: PNN_EINVAL (arguments), PNN_ECUDA, PNN_ETIMEOUT; message in
  * pnn_last_error(NULL). */
