@@ -39,7 +39,15 @@ __device__ __forceinline__ float ld_src(const Src& s, int64_t i, int c) {
   return v;
 }
 // index of the instance that owns CTA b: the largest i with tstart[i] <= b
+// (every thread of the block calls it with the same b: up to 32 instances
+// the warp reads the starts at once and counts those <= b -- one dependent
+// load instead of log2(n) -- else a binary search)
 __device__ __forceinline__ int find_instance(const int* tstart, int n, int b) {
+  if (n <= 32) {
+    const int lane = threadIdx.x & 31;
+    const bool le = lane < n && __ldg(tstart + lane) <= b;
+    return __popc(__ballot_sync(0xffffffffu, le)) - 1;
+  }
   int lo = 0, hi = n - 1;
   while (lo < hi) {
     int mid = (lo + hi + 1) >> 1;
@@ -680,10 +688,13 @@ __device__ __forceinline__ bool chunked_moments(const float* __restrict__ part, 
       }
     if (threadIdx.x == 0) counter[cg] = 0;  // ready for the next launch
   }
+  // one fp64 division (the reciprocal of the count); this part's fp64 units
+  // are slow, and the callers finish in fp32
   const double n = (double)M;
+  const double rn = 1.0 / n;
   n_out = n;
-  mean_out = (double)K + a / n;
-  m2_out = b - a * a / n;
+  mean_out = (double)K + a * rn;
+  m2_out = b - a * a * rn;
   return have;
 }
 
@@ -694,33 +705,35 @@ __global__ void __launch_bounds__(256) k_bn_fin(const BnFinDesc* __restrict__ ta
   const int local = blockIdx.x - tstart[inst];
   const int cg = local % d.cgroups, chunk = local / d.cgroups;
   const int c = cg * 32 + (threadIdx.x & 31);
-  double mean, var;
+  float mean, var;
   if (d.eval) {
     // eval mode: the running statistics stand in for the batch's
     if (threadIdx.x >= 32 || c >= d.C) return;
     mean = d.run_mean[c];
     var = d.run_var[c];
   } else {
-    double cnt, m2;
+    double cnt, mean64, m2;
     if (!chunked_moments(d.part, d.C, d.tiles, d.count, d.rows_per_tile, cg, chunk, d.nchunk, d.scratch, d.counter,
-                         cnt, mean, m2))
+                         cnt, mean64, m2))
       return;
-    var = cnt > 0.0 ? m2 / cnt : 0.0;
-    if (var < 0.0) var = 0.0;
+    // (the sums were fp64; from here fp32 holds every quantity to 2^-24)
+    mean = (float)mean64;
+    var = cnt > 0.0 ? (float)m2 / (float)cnt : 0.f;
+    if (var < 0.f) var = 0.f;
     if (d.run_mean) {
       // running statistics follow the batch mean and the unbiased variance
-      const double m = d.momentum;
-      const double unbiased = d.count > 1 ? var * (double)d.count / (double)(d.count - 1) : var;
-      d.run_mean[c] = (float)((1.0 - m) * (double)d.run_mean[c] + m * mean);
-      d.run_var[c] = (float)((1.0 - m) * (double)d.run_var[c] + m * unbiased);
+      const float m = d.momentum;
+      const float unbiased = d.count > 1 ? var * ((float)d.count / (float)(d.count - 1)) : var;
+      d.run_mean[c] = (1.f - m) * d.run_mean[c] + m * mean;
+      d.run_var[c] = (1.f - m) * d.run_var[c] + m * unbiased;
     }
   }
-  const double rstd = 1.0 / sqrt(var + 1e-5);
-  const double sc = (double)d.gamma[c] * rstd;
-  d.mean[c] = (float)mean;
-  d.rstd[c] = (float)rstd;
-  d.scale[c] = (float)sc;
-  d.shift[c] = (float)((double)d.beta[c] - mean * sc);
+  const float rstd = 1.f / sqrtf(var + 1e-5f);
+  const float sc = d.gamma[c] * rstd;
+  d.mean[c] = mean;
+  d.rstd[c] = rstd;
+  d.scale[c] = sc;
+  d.shift[c] = fmaf(-mean, sc, d.beta[c]);
 }
 
 __global__ void __launch_bounds__(256) k_bnb_reduce(const BnBwdDesc* __restrict__ tab,
@@ -779,8 +792,9 @@ __global__ void __launch_bounds__(256) k_bnb_fin(const BnBwdDesc* __restrict__ t
   d.dbeta[c] = d.accumulate ? d.dbeta[c] + (float)s1 : (float)s1;
   d.dgamma[c] = d.accumulate ? d.dgamma[c] + (float)s2 : (float)s2;
   d.coef[c * 3 + 0] = d.gamma[c] * d.rstd[c];
-  d.coef[c * 3 + 1] = (float)(s1 / (double)d.M);
-  d.coef[c * 3 + 2] = (float)(s2 / (double)d.M);
+  const double rm = 1.0 / (double)d.M;
+  d.coef[c * 3 + 1] = (float)(s1 * rm);
+  d.coef[c * 3 + 2] = (float)(s2 * rm);
 }
 
 __global__ void __launch_bounds__(256) k_bnb_apply(const BnBwdDesc* __restrict__ tab,
