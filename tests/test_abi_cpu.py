@@ -176,3 +176,58 @@ def test_single_conv_call_checks_its_arguments(pnn):
         assert lib.pnn_conv_workspace_bytes(mode, 0, 1, args(ksize=5), C.byref(nb)) == 1
     # too small a workspace is refused before any launch
     assert lib.pnn_conv_run(0, 0, 1, args(), C.c_void_p(256), 256, None) == 2
+
+
+def test_halo_tiles_kernel_choice(pnn):
+    """The TMA-fed 3x3 forward / data gradient take halo tiles (one box per
+    128-pixel tile) where 128 divides h*w, w <= 63 and the A source has 16 |
+    channels <= 64, and two pipeline stages fit: impl 1 accepts such a
+    source even when its channel count rules out one box per tap (48), impl
+    3 (one box per tap) refuses it; the workspace holds a fourth tensor map
+    per instance either way."""
+    lib = pnn.load()
+    fake = 256
+
+    def args(**kw):
+        a = pnn.ConvArgs()
+        g = dict(batch=2, h=32, w=4, c=48, k=16, ksize=3, stride=1)
+        g.update(kw)
+        for key, v in g.items():
+            setattr(a, key, v)
+        a.x = a.wt = a.y = a.dy = a.dx = a.dw = fake
+        return (pnn.ConvArgs * 1)(a)
+
+    nb = C.c_size_t()
+    # forward, A source c = 48: halo tiles only
+    assert lib.pnn_conv_workspace_bytes(0, 1, 1, args(), C.byref(nb)) == 0
+    assert lib.pnn_conv_workspace_bytes(0, 3, 1, args(), C.byref(nb)) == 1
+    # 8x8 images: 128 does not divide h*w, no halo tiles, and 48 channels take no per-tap box
+    assert lib.pnn_conv_workspace_bytes(0, 1, 1, args(h=8, w=8), C.byref(nb)) == 1
+    # a 64-wide image needs a box of 128 + 2*64 + 2 > 256 rows
+    assert lib.pnn_conv_workspace_bytes(0, 1, 1, args(h=8, w=64), C.byref(nb)) == 1
+    # 16 channels: both layouts
+    for impl in (1, 3):
+        assert lib.pnn_conv_workspace_bytes(0, impl, 1, args(c=16), C.byref(nb)) == 0
+    # data gradient: the A source is dy (k channels)
+    assert lib.pnn_conv_workspace_bytes(1, 1, 1, args(c=16, k=48), C.byref(nb)) == 0
+    assert lib.pnn_conv_workspace_bytes(1, 3, 1, args(c=16, k=48), C.byref(nb)) == 1
+
+
+def test_roofline_group_has_algorithmic_work():
+    """bench.py's roofline record takes the launch group with the most device
+    time among those with algorithmic bytes or FLOPs: per-layer BN
+    finalisations (no bytes counted, one trace shape for all layers) can sum
+    to more time in an untorn network without being a roofline candidate."""
+    import bench
+    conv = {"kind": "conv_fwd_tc", "variant": 2, "shape": (16, 64, 1, 1, 32, 32), "instances": 8,
+            "ms": 0.2, "flops": 4.3e9, "bytes": 3.5e8}
+    fin = {"kind": "bn_finalize", "variant": 0, "shape": (0, 0, 0, 0, 0, 0), "instances": 8,
+           "ms": 0.05, "flops": 0.0, "bytes": 0.0}
+    trace = [dict(conv) for _ in range(3)] + [dict(fin) for _ in range(20)]
+    r = bench.roofline_of({}, 1, trace)
+    assert r["kernel"] == "k_conv_fwd_tma_w" and r["kind"] == "conv_fwd_tc", r
+    assert r["launches_per_step"] == 3 and abs(r["ms_per_launch"] - 0.2) < 1e-12
+    assert abs(r["achieved"] - 3.5e8 / 0.2e-3 / 1e9) < 1e-6 and r["bound"] == "hbm"
+    groups = bench.launch_groups(trace, 1)
+    assert [g["kernel"] for g in groups] == ["k_bn_fin", "k_conv_fwd_tma_w"]  # by time, bytes or not
+    assert groups[0]["launches_per_step"] == 20 and groups[1]["gbs"] > 0
