@@ -657,7 +657,10 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
       }
       RT(e2 += clock64() - c2;)
     } else if (MODE == DGRAD && ystage != nullptr && d.tma_y != nullptr) {
-      if (stats) {
+      // SSTATS with a bf16 BN input: the BN-backward sums come from the staged
+      // dX chunk and this warp's staged h rows after the store is issued (below)
+      const bool sst = SSTATS && stats && d.x.dt == DT_BF16;
+      if (stats && !sst) {
         // BN-backward partial sums of the input's BN: g = dA masked by the
         // ReLU of the forward BN output, xhat = (h - mean) * rstd
         float s1[16], s2[16];
@@ -712,12 +715,49 @@ __device__ __forceinline__ void epilogue(const Tile& T, uint32_t tacc, int q, in
       for (int c = 0; c < 4; ++c)
         *reinterpret_cast<float4*>(st + lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4)) =
             make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+      if (sst && mvalid) {
+        // this row's 16 BN inputs, bf16, 32-byte rows
+        uint4* hs = reinterpret_cast<uint4*>(ystage + 4096 + lane * 32);
+        hs[0] = hraw[0];
+        hs[1] = hraw[1];
+      }
       fence_proxy_async();
       __syncwarp();
       if (lane == 0 && T.m0 + q * 32 < T.Mrows) {
         if (d.accumulate) tma_reduce_add_2d(d.tma_y, nb, T.m0 + q * 32, smem_u32(st));
         else tma_store_2d(d.tma_y, nb, T.m0 + q * 32, smem_u32(st));
         bulk_commit();
+      }
+      if (sst) {
+        // sums over this warp's valid rows: lane l takes column l & 15 of rows
+        // (l >> 4) + 2i (two lanes a column), g = dA masked by the ReLU of the
+        // forward BN output, xhat = (h - mean) * rstd
+        const int col = lane & 15;
+        const int nvalid = min(32, max(0, T.Mrows - (T.m0 + q * 32)));
+        const float scv = __ldg(d.x.scale + nb + col), shv = __ldg(d.x.shift + nb + col);
+        const float muv = __ldg(d.bn_mean + nb + col), rsv = __ldg(d.bn_rstd + nb + col);
+        float a = 0.f, b = 0.f;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int r = (lane >> 4) + 2 * i;
+          const float g = *reinterpret_cast<const float*>(st + r * 64 + ((((col >> 2) ^ (r >> 1)) & 3) << 4) +
+                                                          (col & 3) * 4);
+          const float h =
+              __uint_as_float((uint32_t)*reinterpret_cast<const unsigned short*>(ystage + 4096 + r * 32 + col * 2)
+                              << 16);
+          float gv = g;
+          if (d.x.relu && !(fmaf(scv, h, shv) > 0.f)) gv = 0.f;
+          const bool ok = r < nvalid;
+          a += ok ? gv : 0.f;
+          b += ok ? gv * ((h - muv) * rsv) : 0.f;
+        }
+        a += __shfl_xor_sync(0xffffffffu, a, 16);
+        b += __shfl_xor_sync(0xffffffffu, b, 16);
+        if (lane < 16) {
+          red[q][j0 + lane][0] = a;
+          red[q][j0 + lane][1] = b;
+        }
+        __syncwarp();  // every lane has read the staged h before the next chunk rewrites it
       }
       ybuf ^= 1;
     } else if (mvalid) {
@@ -1030,7 +1070,12 @@ __host__ __device__ constexpr int tma_op_bytes(int mode, int bnmax) { return tma
 // per epilogue warp, then each epilogue group's column-reduction scratch
 // (float [4][256][2])
 constexpr int kTmaRedBytes = 4 * 256 * 2 * 4;
-__host__ __device__ constexpr int tma_ystage(int mode, int w) { return mode == 2 ? 0 : tma_ne(mode, w) * 2 * 2048; }
+// (the wide data gradient also stages a chunk's BN input h, 1 KB a warp, for
+// its BN-backward sums)
+__host__ __device__ constexpr int tma_ystage_warp(int mode, int w) {
+  return mode == 2 ? 0 : 2 * 2048 + (mode == 1 && w == 1 ? 1024 : 0);
+}
+__host__ __device__ constexpr int tma_ystage(int mode, int w) { return tma_ne(mode, w) * tma_ystage_warp(mode, w); }
 // (weight gradient) then the two-pass 3x3 transform's bf16 halo (8-channel
 // planes of box rows) and its per-row tap masks
 constexpr int kWgHaloBytes = 16384;
@@ -1852,7 +1897,7 @@ __device__ __forceinline__ void conv_tma_body(const ConvDesc* __restrict__ tab, 
       fence_after();
       float(&red)[4][256][2] = *reinterpret_cast<float(*)[4][256][2]>(red0 + eg * kTmaRedBytes);
       epilogue<MODE, W == 1>(T, tmem + b * bufcols, q, lane, red, 0, 16, (ew & 3) * 32 + lane, 128,
-                             MODE != WGRAD ? ystage0 + ew * 4096 : nullptr, ybuf, bar);
+                             MODE != WGRAD ? ystage0 + ew * tma_ystage_warp(MODE, W) : nullptr, ybuf, bar);
       if (kAMult == 2 && min(T.d->mtile_rows, T.Mrows - T.m0) > kBM) {
         // rows 128-255 of the tile, from the second accumulator half
         Tile T2 = T;
